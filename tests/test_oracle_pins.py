@@ -1,0 +1,360 @@
+"""Pins of the oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: special
+cases the paper states, closed forms computed with a different routine, a
+library optimiser (torch.optim.Adam), the paper's printed numbers, and a
+loop-only twin on tiny inputs.
+"""
+
+import math
+import os
+
+import numpy as np
+import pytest
+
+from oracle import moara_ref as o
+from oracle import brute
+import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+# ---------------------------------------------------------------- decompose
+
+@pytest.mark.parametrize("m,n,B", [(5, 12, 4), (7, 10, 3), (3, 16, 16), (6, 9, 1)])
+def test_recomposition_exact_without_eps(m, n, B):
+    """§3.1: G_pad = Rep_B(M) (.) V_pad exactly as eps -> 0."""
+    G = _rng(1).standard_normal((m, n))
+    M, V = o.decompose(G, B, eps=0.0)
+    np.testing.assert_allclose(o.rep_b(M, B, n) * V, G, rtol=1e-14, atol=1e-15)
+
+
+def test_recomposition_with_eps_closed_form():
+    """App. B.1: m*v = ||g|| / (||g|| + eps) * g for finite eps."""
+    eps = 1e-3
+    G = _rng(2).standard_normal((4, 10)) * 1e-2
+    B = 4
+    M, V = o.decompose(G, B, eps=eps)
+    Gp = np.zeros((4, 12))
+    Gp[:, :10] = G
+    norms = np.linalg.norm(Gp.reshape(4, 3, 4), axis=2)
+    factor = np.repeat(norms / (norms + eps), 4, axis=1)[:, :10]
+    np.testing.assert_allclose(o.rep_b(M, B, 10) * V, factor * G, rtol=1e-13)
+
+
+def test_zero_block_gives_zero_direction():
+    """App. B.3: a zero block has v = 0 (automatic with eps > 0)."""
+    G = _rng(3).standard_normal((3, 8))
+    G[1, 4:8] = 0.0
+    M, V = o.decompose(G, 4)
+    assert M[1, 1] == 0.0
+    assert np.all(V[1, 4:8] == 0.0)
+    Mz, Vz = o.decompose(np.zeros((2, 5)), 2)
+    assert np.all(Mz == 0) and np.all(Vz == 0)
+
+
+def test_block_size_one_is_sign():
+    """App. B.3 small-B regime: B = 1 gives M = |G| and V = sign(G)."""
+    G = _rng(4).standard_normal((6, 7))
+    G[2, 3] = 0.0
+    with np.errstate(invalid="ignore"):
+        M, V = o.decompose(G, 1, eps=0.0)
+    np.testing.assert_array_equal(M, np.abs(G))
+    np.testing.assert_array_equal(np.nan_to_num(V), np.sign(G))
+    M, V = o.decompose(G, 1)
+    np.testing.assert_array_equal(M, np.abs(G))
+    dev = np.abs(V - np.sign(G))
+    assert np.all(dev <= 1e-12 / np.maximum(np.abs(G), 1e-300) + 1e-15)
+
+
+def test_block_size_n_is_row_normalisation():
+    """§3.1: a single block per row is the row-wise decomposition."""
+    G = _rng(5).standard_normal((5, 11))
+    M, V = o.decompose(G, 11)
+    rn = np.linalg.norm(G, axis=1)
+    np.testing.assert_allclose(M[:, 0], rn, rtol=1e-14)
+    np.testing.assert_allclose(V, G / rn[:, None], rtol=1e-11)
+
+
+def test_blocks_run_along_columns():
+    """§3.1 / App. B.1: rows are kept, blocks are contiguous column ranges."""
+    G = _rng(6).standard_normal((3, 12))
+    M, _ = o.decompose(G, 4)
+    assert M.shape == (3, 3)
+    for i in range(3):
+        for b in range(3):
+            assert M[i, b] == pytest.approx(np.linalg.norm(G[i, 4 * b:4 * b + 4]), rel=1e-14)
+
+
+@pytest.mark.parametrize("n,B", [(10, 4), (2736, 32), (13, 5), (7, 8)])
+def test_padding_invariance(n, B):
+    """App. B.1: zero padding does not change the last block's magnitude;
+    decomposing G equals decomposing the explicitly padded G, then cropping."""
+    m = 3
+    G = _rng(7).standard_normal((m, n))
+    k = -(-n // B)
+    Gp = np.zeros((m, k * B))
+    Gp[:, :n] = G
+    M1, V1 = o.decompose(G, B)
+    M2, V2 = o.decompose(Gp, B)
+    np.testing.assert_array_equal(M1, M2)
+    np.testing.assert_array_equal(V1, V2[:, :n])
+    last = np.linalg.norm(G[:, (k - 1) * B:], axis=1)
+    np.testing.assert_allclose(M1[:, -1], last, rtol=1e-14)
+
+
+def test_proposition_1_block_cosine():
+    """App. B.3, Proposition 1: cos(G_b, m_b * vt_b) = cos(v_b, vt_b)."""
+    m, n, B, r = 16, 24, 6, 5
+    G = _rng(8).standard_normal((m, n))
+    M, V = o.decompose(G, B)
+    P = synth.random_orthonormal(m, r, seed=3)
+    Vt = P @ (P.T @ V)
+    for i in range(m):
+        for b in range(n // B):
+            gb = G[i, b * B:(b + 1) * B]
+            vb = V[i, b * B:(b + 1) * B]
+            tb = Vt[i, b * B:(b + 1) * B]
+            c1 = gb @ (M[i, b] * tb) / (np.linalg.norm(gb) * np.linalg.norm(M[i, b] * tb))
+            c2 = vb @ tb / (np.linalg.norm(vb) * np.linalg.norm(tb))
+            assert c1 == pytest.approx(c2, rel=1e-12, abs=1e-14)
+
+
+# ------------------------------------------------- Adam reductions (library)
+
+def _torch_adam_trajectory(W0, grads, lr, beta1, beta2, eps):
+    torch = pytest.importorskip("torch")
+    p = torch.nn.Parameter(torch.tensor(W0, dtype=torch.float64))
+    opt = torch.optim.Adam([p], lr=lr, betas=(beta1, beta2), eps=eps,
+                           weight_decay=0.0)
+    for G in grads:
+        p.grad = torch.tensor(G, dtype=torch.float64)
+        opt.step()
+    return p.detach().numpy()
+
+
+@pytest.mark.parametrize("m,n", [(6, 9), (8, 8)])
+def test_galore_full_rank_signed_permutation_is_adam(m, n):
+    """Decomposition off, P a signed permutation with r = m <= n: the GaLore
+    step is plain Adam (torch.optim.Adam with lr * alpha)."""
+    hp = o.Hparams(decompose=False, scale=0.25, adam_eps=1e-8, block_size=3)
+    lr = 1e-2
+    P = synth.signed_permutation(m, m, seed=11)
+    grads = [_rng(20 + t).standard_normal((m, n)) for t in range(10)]
+    W0 = _rng(19).standard_normal((m, n)) * 0.02
+    st = o.run(o.init_state(W0, m, 3, P=P), grads, lr, hp, auto_refresh=False)
+    ref = _torch_adam_trajectory(W0, grads, lr * hp.scale, hp.beta1, hp.beta2, hp.adam_eps)
+    np.testing.assert_allclose(st.W, ref, rtol=1e-12, atol=1e-15)
+
+
+def test_galore_partial_permutation_updates_selected_rows_only():
+    """r < m with P = r columns of a signed permutation: selected rows follow
+    Adam, the other rows are untouched."""
+    m, n, r = 7, 5, 3
+    hp = o.Hparams(decompose=False, scale=1.0, adam_eps=1e-8, block_size=5)
+    P = synth.signed_permutation(m, r, seed=4)
+    rows = [int(np.flatnonzero(P[:, j])[0]) for j in range(r)]
+    grads = [_rng(40 + t).standard_normal((m, n)) for t in range(6)]
+    W0 = _rng(39).standard_normal((m, n))
+    st = o.run(o.init_state(W0, r, 5, P=P), grads, 1e-2, hp, auto_refresh=False)
+    ref = _torch_adam_trajectory(W0, grads, 1e-2, hp.beta1, hp.beta2, hp.adam_eps)
+    other = [i for i in range(m) if i not in rows]
+    np.testing.assert_allclose(st.W[rows], ref[rows], rtol=1e-12)
+    np.testing.assert_array_equal(st.W[other], W0[other])
+
+
+def test_identity_projector_is_adam_of_v_times_adam_of_m():
+    """Decomposition on and P = I: the update is Rep_B(Adam(M)) (.) Adam(V),
+    with both Adams run by torch.optim.Adam and M, V from np.linalg.norm."""
+    torch = pytest.importorskip("torch")
+    m, n, B = 5, 10, 4
+    k = 3
+    hp = o.Hparams(decompose=True, scale=0.25, adam_eps=1e-6, block_size=B)
+    lr = 3e-3
+    grads = [_rng(60 + t).standard_normal((m, n)) for t in range(8)]
+    W0 = _rng(59).standard_normal((m, n)) * 0.02
+    st = o.run(o.init_state(W0, m, B, P=np.eye(m)), grads, lr, hp, auto_refresh=False)
+
+    pv = torch.nn.Parameter(torch.zeros(m, n, dtype=torch.float64))
+    pm = torch.nn.Parameter(torch.zeros(m, k, dtype=torch.float64))
+    ov = torch.optim.Adam([pv], lr=1.0, betas=(hp.beta1, hp.beta2), eps=hp.adam_eps)
+    om = torch.optim.Adam([pm], lr=1.0, betas=(hp.beta1, hp.beta2), eps=hp.adam_eps)
+    W = W0.copy()
+    for G in grads:
+        Gp = np.zeros((m, k * B))
+        Gp[:, :n] = G
+        Mg = np.linalg.norm(Gp.reshape(m, k, B), axis=2)
+        Vg = G / (np.repeat(Mg, B, axis=1)[:, :n] + hp.decomp_eps)
+        before_v, before_m = pv.detach().clone(), pm.detach().clone()
+        pv.grad = torch.tensor(Vg)
+        pm.grad = torch.tensor(Mg)
+        ov.step()
+        om.step()
+        dV = (before_v - pv.detach()).numpy()
+        dM = (before_m - pm.detach()).numpy()
+        W = W - lr * hp.scale * np.repeat(dM, B, axis=1)[:, :n] * dV
+    np.testing.assert_allclose(st.W, W, rtol=1e-11, atol=1e-14)
+
+
+def test_projector_column_sign_flip_invariance():
+    """Flipping the sign of projector columns leaves the trajectory unchanged."""
+    m, n, r, B = 12, 16, 4, 4
+    hp = o.Hparams(block_size=B, adam_eps=1e-8)
+    P = synth.random_orthonormal(m, r, seed=9)
+    Pf = P * np.array([1, -1, -1, 1])
+    grads = [_rng(80 + t).standard_normal((m, n)) for t in range(5)]
+    W0 = _rng(79).standard_normal((m, n))
+    a = o.run(o.init_state(W0, r, B, P=P), grads, 1e-3, hp, auto_refresh=False)
+    b = o.run(o.init_state(W0, r, B, P=Pf), grads, 1e-3, hp, auto_refresh=False)
+    np.testing.assert_allclose(a.W, b.W, rtol=1e-13, atol=1e-16)
+
+
+def test_projector_rotation_changes_update():
+    """Adam is elementwise, so a general rotation of P does change the step:
+    the P = I reduction above needs a signed permutation."""
+    m, n = 6, 6
+    hp = o.Hparams(decompose=False, block_size=3)
+    Q = synth.random_orthonormal(m, m, seed=2)
+    G = _rng(90).standard_normal((m, n))
+    W0 = np.zeros((m, n))
+    a = o.step(o.init_state(W0, m, 3, P=np.eye(m)), G, 1, 1e-2, hp, refresh=False)
+    b = o.step(o.init_state(W0, m, 3, P=Q), G, 1, 1e-2, hp, refresh=False)
+    assert np.max(np.abs(a.W - b.W)) > 1e-4
+
+
+# ---------------------------------------------------------------- refresh
+
+def test_refresh_orthonormal_and_eckart_young():
+    """TruncatedSVD: P^T P = I, and the captured energy ||P^T V||_F^2 equals
+    the sum of the top-r squared singular values (Eckart-Young), more than
+    any other orthonormal P."""
+    m, n, r = 30, 40, 6
+    G = synth.lowrank_grad(m, n, 8, 10.0, 0.01, 1, seed=1)
+    _, V = o.decompose(G, 8)
+    P, S = o.truncated_svd(V, r)
+    np.testing.assert_allclose(P.T @ P, np.eye(r), atol=1e-12)
+    e = np.sum((P.T @ V) ** 2)
+    assert e == pytest.approx(np.sum(S[:r] ** 2), rel=1e-12)
+    for s in range(5):
+        Q = synth.random_orthonormal(m, r, seed=100 + s)
+        assert np.sum((Q.T @ V) ** 2) < e
+
+
+def test_refresh_step_index():
+    """Algorithm 1 refreshes at s mod T == 0 with s = t - 1."""
+    assert o.is_refresh_step(1, 200)
+    assert not o.is_refresh_step(200, 200)
+    assert o.is_refresh_step(201, 200)
+    assert [t for t in range(1, 11) if o.is_refresh_step(t, 3)] == [1, 4, 7, 10]
+
+
+# -------------------------------------------------- brute-force twin on 8x8
+
+def _gap_ok(X, r, rel=1e-6):
+    S = np.linalg.svd(np.asarray(X), compute_uv=False)
+    if r >= len(S):
+        return S[-1] > rel * S[0]
+    return (S[r - 1] - S[r]) > rel * S[0]
+
+
+CASES = [
+    # (m, n, B, r, decompose, src)
+    (8, 8, 1, 3, True, "V"), (8, 8, 2, 5, True, "V"), (8, 8, 3, 4, True, "V"),
+    (8, 8, 4, 8, True, "V"), (8, 8, 8, 1, True, "V"), (8, 8, 4, 2, True, "G"),
+    (8, 8, 2, 6, False, "V"), (8, 11, 3, 7, True, "V"), (6, 8, 4, 6, True, "V"),
+    (8, 5, 2, 5, True, "V"),
+]
+
+
+@pytest.mark.parametrize("m,n,B,r,dec,src", CASES)
+def test_oracle_matches_loop_twin(m, n, B, r, dec, src):
+    T = 3
+    grads = [list(map(list, _rng(300 + t).standard_normal((m, n)))) for t in range(10)]
+    W0 = _rng(299).standard_normal((m, n)) * 0.02
+    hp = o.Hparams(block_size=B, refresh_interval=T, decompose=dec,
+                   refresh_src=src, adam_eps=1e-6, scale=0.25)
+    for t in range(1, 11):
+        if o.is_refresh_step(t, T):
+            Gt = np.array(grads[t - 1])
+            X = o.decompose(Gt, B)[1] if (dec and src == "V") else Gt
+            if not _gap_ok(X, r):
+                pytest.skip("degenerate spectrum at the truncation rank")
+    st = o.run(o.init_state(W0, r, B), [np.array(g) for g in grads], 1e-2, hp)
+    Wb, Pb = brute.run([list(row) for row in W0], grads, r, 1e-2, B, T,
+                       decompose_on=dec, refresh_src=src, adam_eps=1e-6,
+                       scale=0.25)
+    np.testing.assert_allclose(np.array(Pb), st.P, atol=1e-9)
+    np.testing.assert_allclose(np.array(Wb), st.W, rtol=1e-9, atol=1e-12)
+
+
+# ------------------------------------------------------- rank table (Phase 3)
+
+def _golden_rows(name):
+    rows = {}
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                p = line.split()
+                rows[p[0]] = p[1:]
+    return rows
+
+
+def test_rank_table_matches_final_allocation():
+    """App. C: D = {q, k}, R = {down}, delta_r = r_base/2 at r_base = 256."""
+    ours = [int(x) for x in _golden_rows("rank_allocations.txt")["Ours"]]
+    got = o.rank_table(256, ["q", "k"], ["down"], 128)
+    assert [got[t] for t in o.MODULE_TYPES] == ours
+
+
+def test_rank_tables_preserve_budget():
+    """Every allocation in the paper's table (and every output of the rule,
+    including uneven splits) keeps sum_tau r_tau = 7 r_base."""
+    for run, vals in _golden_rows("rank_allocations.txt").items():
+        assert sum(int(v) for v in vals) == 7 * 256, run
+    for donors, recv, dr in [(["q", "k", "v"], ["up", "down"], 100),
+                             (["q"], ["gate", "up", "down"], 64),
+                             ([], [], 0), (["o", "k"], ["q"], 255)]:
+        got = o.rank_table(512, donors, recv, dr)
+        assert sum(got.values()) == 7 * 512
+    uneven = o.rank_table(512, ["q", "k", "v"], ["up", "down"], 101)
+    assert (uneven["up"], uneven["down"]) == (512 + 152, 512 + 151)
+
+
+# ------------------------------------------------ memory model (Appendix G)
+
+@pytest.mark.parametrize("model", ["350M", "1B", "7B"])
+def test_memory_model_reproduces_printed_table(model):
+    """Appendix G: 2 b_V r d_W + 2 b_M m ceil(n/B) summed over the target
+    matrices reproduces all printed optimizer-state MiB values, with
+    b_V = 2, b_M = 4 (fp32 magnitude branch, App. D.2), d_W = max(m, n),
+    plus untied 32000-token embedding/head with full Adam in 2-byte states
+    and fp32 norm weights."""
+    row = _golden_rows("memory_table.txt")[model]
+    h, f, L, B, rb = (int(x) for x in row[:5])
+    printed = [float(x) for x in row[5:]]
+    shp = {"q": (h, h), "k": (h, h), "v": (h, h), "o": (h, h),
+           "gate": (f, h), "up": (f, h), "down": (h, f)}
+    uni = {t: rb for t in shp}
+    aware = o.rank_table(rb, ["q", "k"], ["down"], rb // 2)
+    other = 2 * 32000 * h * 2 * 2 + (2 * L + 1) * h * 4
+
+    def total(ranks, dec):
+        return L * sum(o.moment_bytes(m, n, ranks[t], B, 2, 4, "max", dec)
+                       for t, (m, n) in shp.items()) + other
+
+    got = [total(uni, False), total(uni, True), total(aware, False), total(aware, True)]
+    for g, p in zip(got, printed):
+        assert round(g / 2 ** 20, 2) == pytest.approx(p, abs=1e-9)
+
+
+def test_alignment_full_rank_projection_is_one():
+    """§3.2: with P spanning the whole column space, G_recon = Rep_B(M) (.) V,
+    so S(W, t) = 1 up to the eps of the decomposition."""
+    G = _rng(12).standard_normal((6, 9))
+    assert o.alignment(G, np.eye(6), 3) == pytest.approx(1.0, abs=1e-12)
+    P = synth.random_orthonormal(6, 2, seed=1)
+    assert o.alignment(G, P, 3) < 0.99
