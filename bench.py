@@ -1,0 +1,421 @@
+"""Benchmark: ms per full-model projected-Adam step on one GB300.
+
+Workload: the 224 target matrices of a 32-layer Llama-2-7B-shaped model
+(hidden 4096, MLP 11008) with the module-aware rank table q/k 512,
+v/o/gate/up 1024, down 2048 (r_base 1024), block size 128, bf16 gradients,
+fp32 weights and optimizer states; synthetic inputs (low-rank-plus-noise
+gradients, random-normal weights).  One step is one moara_step_grouped call
+over all 224 modules; the every-200-steps projector refresh is timed once and
+added amortised (refresh_ms / 200).
+
+value: device-timed ms per step (CUDA events on the launching stream, inputs
+resident in HBM); e2e: the same step through the C ABI with the gradients
+copied from pinned host memory each step and the device status word read
+back.  roofline: the kernel with the largest share of step time, its
+algorithmic bytes or flops per launch over its event-timed average launch.
+
+`--impl reference` times the float64 oracle on the host cores instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "llama2_7b_full_module_aware"
+METRIC = "ms per full-model projected-Adam step"
+LR = 1e-3
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return pk["hbm_gbs"], pk["bf16_tflops"], pk["bf16_tflops_sustained"], "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def _dist():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        import tempfile
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            p = [x.strip() for x in line.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                mx.append(float(p[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, p[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        os.unlink(self.path)
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2] if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def _algorithmic(mods, B):
+    """Algorithmic bytes and flops of one step over `mods` (Module list)."""
+    tot_b = tot_f = 0
+    per = {"project": [0, 0], "backproject": [0, 0]}
+    for md in mods:
+        m, n, r = md.m, md.n, md.r
+        k = -(-n // B)
+        # minimum traffic of one fused pass: G read (bf16), W read+write,
+        # direction moments read+write, P read once (bf16), magnitude moments
+        tot_b += 2 * m * n + 8 * m * n + 16 * r * n + 2 * m * r + 16 * m * k
+        tot_f += 4 * m * r * n
+        per["project"][1] += 2 * m * r * n
+        per["backproject"][1] += 2 * m * r * n
+    return tot_b, tot_f, per
+
+
+def _kernel_bytes(mods, B, tc):
+    """Algorithmic bytes per launch of the projection and back-projection
+    kernels as built (tc: bf16 N hand-off; otherwise fp32 N, fp32 P)."""
+    pb = bb = 0
+    for md in mods:
+        m, n, r = md.m, md.n, md.r
+        k = -(-n // B)
+        nb = 2 if tc else 4
+        pbytes = 2 if tc else 4
+        # projection: G read, moments read+write, N write, P read, magnitude
+        # moments read+write and dM write
+        pb += 2 * m * n + 16 * r * n + nb * r * n + pbytes * m * r + 20 * m * k
+        # back-projection: W read+write, N read, P read, dM read
+        bb += 8 * m * n + nb * r * n + pbytes * m * r + 4 * m * k
+    return pb, bb
+
+
+def run_gpu(args):
+    import torch
+    import paper_2609_15037_gb300 as M
+    import synth
+
+    rank, world, local = _dist()
+    torch.cuda.set_device(local)
+    dev = torch.device(f"cuda:{local}")
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    wl = synth.workload(args.workload)
+    mods = wl["modules"]
+    B = wl["block_size"]
+    hp = M.moara_default_hparams()
+    hp.block_size = B
+    hp.adam_eps = wl["adam_eps"]
+    g = M.MoaraGroup(hp, device=local)
+    stream = torch.cuda.current_stream(dev)
+    grads = []
+    for i, md in enumerate(mods):
+        g.add(md.m, md.n, md.r, "bf16")
+        with torch.no_grad():
+            g.modules[i].W.normal_(0.0, 0.02)
+        grads.append(synth.lowrank_grad_torch(md.m, md.n, wl["signal_rank"], wl["sigma0"],
+                                              wl["noise"], 1, seed=0, module=i,
+                                              noise_rel=wl["noise_rel"], device=dev))
+    torch.cuda.synchronize()
+    ids = list(g.ids)
+    gptr = [x.data_ptr() for x in grads]
+    cs = stream.cuda_stream
+
+    # projector refresh (once, timed; amortised over T = 200 steps)
+    g.ensure_refresh_workspace()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    M.moara_refresh_projector(g.ctx, ids, gptr, cs)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    refresh_ms = t0.elapsed_time(t1)
+
+    # warm-up
+    step = 1
+    for _ in range(args.warmup):
+        M.moara_step_grouped(g.ctx, ids, gptr, step, LR, False, cs)
+        step += 1
+    torch.cuda.synchronize()
+
+    # timed region (device time, CUDA events on the launching stream)
+    M.moara_profile_read(g.ctx)
+    M.moara_profile_enable(g.ctx, True)
+    launches0 = M.moara_launch_count(g.ctx)
+    clocks = Clocks(local)
+    clocks.start()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        M.moara_step_grouped(g.ctx, ids, gptr, step, LR, False, cs)
+        step += 1
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    launches = M.moara_launch_count(g.ctx) - launches0
+    M.moara_profile_enable(g.ctx, False)
+    prof = M.moara_profile_read(g.ctx)
+    elapsed = ev0.elapsed_time(ev1)
+    if world > 1:
+        t = torch.tensor([elapsed], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        elapsed = float(t.item())
+    step_ms = elapsed / args.steps
+    status = M.moara_get_device_status(g.ctx, cs)
+
+    # end to end through the C ABI with host buffers
+    host = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for x in grads]
+    for h, x in zip(host, grads):
+        h.copy_(x)
+    st_host = torch.empty(1, dtype=torch.int32, pin_memory=True)
+    st_dev = torch.zeros(1, dtype=torch.int32, device=dev)
+    e2e_steps = max(1, min(args.steps, 5))
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        for h, x in zip(host, grads):
+            x.copy_(h, non_blocking=True)
+        M.moara_step_grouped(g.ctx, ids, gptr, step, LR, False, cs)
+        step += 1
+        st_host.copy_(st_dev, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    h2d = sum(x.numel() * x.element_size() for x in grads)
+
+    hbm, bf16_peak, bf16_sus, peak_src = _peaks()
+    alg_bytes, alg_flops, _ = _algorithmic(mods, B)
+    total_ms = step_ms + refresh_ms / 200.0
+    roof_ms = max(alg_bytes / (hbm * 1e9), alg_flops / (bf16_sus * 1e12)) * 1e3
+
+    # dominant kernel
+    used_tc = prof["tc_project"][1] > 0
+    pbytes, bbytes = _kernel_bytes(mods, B, used_tc)
+    names = ["decompose", "project", "backproject", "tc_project", "tc_backproject"]
+    dom = max(names, key=lambda k: prof[k][0])
+    dom_ms = prof[dom][0] / max(prof[dom][1], 1)
+    n_launch_per_step = max(prof[dom][1] // args.steps, 1)
+    flops_dom = alg_flops / 2 / n_launch_per_step
+    if dom in ("project", "backproject"):
+        # fp32 SIMT GEMM: bound by the FP32 FMA pipes
+        alu_peak = 152 * 128 * 2 * 2.07e9 / 1e12
+        achieved = flops_dom / (dom_ms * 1e-3) / 1e12
+        roof = {"bound": "alu", "achieved": round(achieved, 2), "peak": round(alu_peak, 1),
+                "unit": "TFLOP/s", "frac": round(achieved / alu_peak, 4), "traffic": None,
+                "kernel": dom, "peak_source": "152 SMs x 128 FP32 lanes x 2 x 2.07 GHz"}
+    elif dom == "tc_project":
+        achieved = flops_dom / (dom_ms * 1e-3) / 1e12
+        roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": bf16_sus,
+                "unit": "TFLOP/s", "frac": round(achieved / bf16_sus, 4), "traffic": None,
+                "kernel": dom, "peak_source": f"bf16_tflops_sustained ({peak_src})"}
+    else:
+        by = (bbytes if dom in ("backproject", "tc_backproject") else pbytes) / n_launch_per_step
+        achieved = by / (dom_ms * 1e-3) / 1e9
+        roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
+                "frac": round(achieved / hbm, 4), "traffic": None, "kernel": dom,
+                "peak_source": f"hbm_gbs ({peak_src})"}
+
+    kernels = {k: {"ms_per_step": round(prof[k][0] / args.steps, 4),
+                   "launches_per_step": prof[k][1] / args.steps,
+                   "share": round(prof[k][0] / max(sum(prof[x][0] for x in names), 1e-9), 4)}
+               for k in names if prof[k][1] > 0}
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(args, budget_s=args.cpu_seconds)
+    out = {
+        "metric": METRIC, "value": round(total_ms / world, 4), "unit": "ms",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(total_ms, 4), "higher_is_better": False, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 G, fp32 W/states" if used_tc else "fp32 (bf16 G)",
+        "data": "synthetic",
+        "config": {"workload": args.workload, "modules": len(mods), "block_size": B,
+                   "ranks": "q/k 512, v/o/gate/up 1024, down 2048",
+                   "l2": "inputs larger than L2 (no flush needed)",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "step_ms_no_refresh": round(step_ms, 4),
+        "refresh_ms": round(refresh_ms, 2), "refresh_amortised_ms": round(refresh_ms / 200.0, 4),
+        "hbm_gbs_algorithmic": round(alg_bytes / (step_ms * 1e-3) / 1e9, 1),
+        "step_roofline": {"alg_bytes": alg_bytes, "alg_flops": alg_flops,
+                          "roofline_ms": round(roof_ms, 3),
+                          "frac": round(roof_ms / step_ms, 4),
+                          "peaks": f"hbm {hbm} GB/s, bf16 {bf16_sus} TFLOP/s sustained ({peak_src})"},
+        "roofline": roof,
+        "kernels": kernels,
+        "e2e": {"value": round(e2e_ms + refresh_ms / 200.0, 4), "unit": "ms",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4},
+        "gpu_launches": int(launches),
+        "device_status": status,
+        "clocks": clk,
+    }
+    if cpu is not None:
+        out["cpu_baseline"] = cpu
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    g.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def _oracle_layer_sample(wl, layer_modules, seed=0):
+    """Oracle step on the seven modules of one decoder layer (float64)."""
+    import numpy as np
+    from oracle import moara_ref as o
+    hp = o.Hparams(block_size=wl["block_size"], adam_eps=wl["adam_eps"])
+    rng = np.random.default_rng(seed)
+    states, grads = [], []
+    for md in layer_modules:
+        W = rng.standard_normal((md.m, md.n)) * 0.02
+        P = np.linalg.qr(rng.standard_normal((md.m, md.r)))[0]
+        states.append(o.init_state(W, md.r, wl["block_size"], P=P))
+        grads.append(rng.standard_normal((md.m, md.n)) * 1e-3)
+    return states, grads, hp
+
+
+def cpu_baseline(args, budget_s=20.0):
+    """The oracle as it stands, one 7B decoder layer per sample, scaled to the
+    full model (x layers).  Runs in this process on the host cores."""
+    import numpy as np
+    from oracle import moara_ref as o
+    import synth
+    wl = synth.workload(args.workload)
+    layer = [md for md in wl["modules"] if md.name.startswith("layer0.")]
+    layers = len(wl["modules"]) // len(layer)
+    states, grads, hp = _oracle_layer_sample(wl, layer)
+    times = []
+    t_start = time.time()
+    t = 1
+    while True:
+        t0 = time.perf_counter()
+        for i in range(len(layer)):
+            states[i] = o.step(states[i], grads[i], t, LR, hp, refresh=False)
+        times.append(time.perf_counter() - t0)
+        t += 1
+        if time.time() - t_start > budget_s or len(times) >= 3:
+            break
+    per_layer = min(times)
+    try:
+        cores = len(os.sched_getaffinity(0))
+    except Exception:
+        cores = os.cpu_count()
+    threads = os.environ.get("OMP_NUM_THREADS") or os.environ.get("OPENBLAS_NUM_THREADS") or str(cores)
+    return {"value": round(per_layer * layers * 1e3, 1), "unit": "ms", "cores": int(threads),
+            "kind": "oracle",
+            "sample": f"one decoder layer (7 modules) of the {len(wl['modules'])}-matrix model, "
+                      f"float64 NumPy step without refresh, best of {len(times)}, x{layers} layers"}
+
+
+def run_reference(args):
+    """Times the oracle on the host cores (rank 0 only)."""
+    rank, world, _ = _dist()
+    if rank != 0:
+        return
+    import synth
+    from oracle import moara_ref as o
+    wl = synth.workload(args.workload)
+    layer = [md for md in wl["modules"] if md.name.startswith("layer0.")]
+    layers = len(wl["modules"]) // len(layer)
+    states, grads, hp = _oracle_layer_sample(wl, layer)
+    t = 1
+    for _ in range(args.warmup):
+        for i in range(len(layer)):
+            states[i] = o.step(states[i], grads[i], t, LR, hp, refresh=False)
+        t += 1
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        for i in range(len(layer)):
+            states[i] = o.step(states[i], grads[i], t, LR, hp, refresh=False)
+        t += 1
+    per_layer = (time.perf_counter() - t0) / args.steps
+    val = per_layer * layers * 1e3
+    try:
+        cores = len(os.sched_getaffinity(0))
+    except Exception:
+        cores = os.cpu_count()
+    out = {"impl": "reference", "metric": METRIC, "value": round(val, 1), "unit": "ms",
+           "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(val, 1), "higher_is_better": False, "scaling": "weak",
+           "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": args.workload, "modules": len(wl["modules"]),
+                      "block_size": wl["block_size"]},
+           "cpu_baseline": {"value": round(val, 1), "unit": "ms", "cores": cores,
+                            "kind": "oracle",
+                            "sample": f"each step: one decoder layer (7 modules) in float64 "
+                                      f"NumPy, x{layers} layers, no refresh"},
+           "e2e": {"value": round(val, 1), "unit": "ms", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--cpu-seconds", type=float, default=20.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

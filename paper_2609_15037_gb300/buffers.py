@@ -1,0 +1,133 @@
+"""Device-memory plumbing for libmoara: torch tensors that back one module's
+buffers, and a small driver that owns a context.  Every computation happens in
+the library's kernels; torch only allocates and holds memory.
+"""
+
+from __future__ import annotations
+
+import torch
+
+from . import binding as B
+
+
+def _bf16_bits(t):
+    return t.to(torch.bfloat16).view(torch.int16)
+
+
+class ModuleBuffers:
+    """Caller-owned buffers of one registered weight (layouts of moara.h)."""
+
+    def __init__(self, m, n, r, block_size, grad_dtype="bf16", device="cuda",
+                 W0=None, with_bf16=True):
+        self.m, self.n, self.r, self.block_size = m, n, r, block_size
+        self.kb = -(-n // block_size)
+        self.grad_dtype = grad_dtype
+        dev = torch.device(device)
+        f32 = dict(dtype=torch.float32, device=dev)
+        if W0 is None:
+            self.W = torch.zeros(m, n, **f32)
+        else:
+            self.W = torch.as_tensor(W0).to(**f32).contiguous().clone()
+        self.P = torch.zeros(m, r, **f32)
+        self.P_bf16 = torch.zeros(m, r, dtype=torch.int16, device=dev) if with_bf16 else None
+        self.exp_avg = torch.zeros(r, n, **f32)
+        self.exp_avg_sq = torch.zeros(r, n, **f32)
+        self.mag_avg = torch.zeros(m, self.kb, **f32)
+        self.mag_avg_sq = torch.zeros(m, self.kb, **f32)
+        nbytes = B.moara_workspace_bytes(m, n, r, block_size)
+        self.workspace = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+
+    def desc(self):
+        d = B.moara_module_desc()
+        d.m, d.n, d.r = self.m, self.n, self.r
+        d.grad_dtype = B.MOARA_DTYPE_BF16 if self.grad_dtype == "bf16" else B.MOARA_DTYPE_F32
+        d.W = self.W.data_ptr()
+        d.P = self.P.data_ptr()
+        d.P_bf16 = self.P_bf16.data_ptr() if self.P_bf16 is not None else None
+        d.exp_avg = self.exp_avg.data_ptr()
+        d.exp_avg_sq = self.exp_avg_sq.data_ptr()
+        d.mag_avg = self.mag_avg.data_ptr()
+        d.mag_avg_sq = self.mag_avg_sq.data_ptr()
+        d.workspace = self.workspace.data_ptr()
+        d.workspace_bytes = self.workspace.numel()
+        return d
+
+    def state_tensors(self):
+        return {"W": self.W, "P": self.P, "exp_avg": self.exp_avg,
+                "exp_avg_sq": self.exp_avg_sq, "mag_avg": self.mag_avg,
+                "mag_avg_sq": self.mag_avg_sq}
+
+    def state_dict(self):
+        sd = {k: v.detach().clone() for k, v in self.state_tensors().items()}
+        if self.P_bf16 is not None:
+            sd["P_bf16"] = self.P_bf16.clone()
+        return sd
+
+    def load_state_dict(self, sd):
+        for k, v in self.state_tensors().items():
+            v.copy_(sd[k])
+        if self.P_bf16 is not None and "P_bf16" in sd:
+            self.P_bf16.copy_(sd["P_bf16"])
+
+
+class MoaraGroup:
+    """A context plus the modules registered in it."""
+
+    def __init__(self, hp=None, device=0, refresh_workspace_bytes=None, **overrides):
+        self.hp = hp if hp is not None else B.moara_default_hparams()
+        for k, v in overrides.items():
+            setattr(self.hp, k, v)
+        self.device = device
+        self.ctx = B.moara_create(self.hp, device)
+        self.modules = []
+        self.ids = []
+        self._refresh_ws = None
+        self._refresh_ws_request = refresh_workspace_bytes
+
+    def add(self, m, n, r, grad_dtype="bf16", W0=None):
+        buf = ModuleBuffers(m, n, r, self.hp.block_size, grad_dtype,
+                            f"cuda:{self.device}", W0=W0,
+                            with_bf16=True)
+        mid = B.moara_init_module(self.ctx, buf.desc())
+        self.modules.append(buf)
+        self.ids.append(mid)
+        return mid
+
+    def ensure_refresh_workspace(self):
+        need = max(B.moara_refresh_workspace_bytes(self.ctx, b.m, b.n, b.r) for b in self.modules)
+        want = max(need, self._refresh_ws_request or 0)
+        if self._refresh_ws is None or self._refresh_ws.numel() < want:
+            self._refresh_ws = torch.empty(want, dtype=torch.uint8,
+                                           device=f"cuda:{self.device}")
+            B.moara_set_refresh_workspace(self.ctx, self._refresh_ws.data_ptr(), want)
+
+    def load_projector(self, mid, P, stream=0):
+        src = torch.as_tensor(P, dtype=torch.float32).to(f"cuda:{self.device}").contiguous()
+        B.moara_load_projector(self.ctx, mid, src.data_ptr(), stream)
+        torch.cuda.current_stream(self.device).synchronize() if stream == 0 else None
+
+    def refresh(self, grads, ids=None, stream=0):
+        self.ensure_refresh_workspace()
+        ids = self.ids if ids is None else ids
+        B.moara_refresh_projector(self.ctx, ids, [g.data_ptr() for g in grads], stream)
+
+    def step(self, grads, t, lr, auto_refresh=False, ids=None, stream=0):
+        ids = self.ids if ids is None else ids
+        if auto_refresh:
+            self.ensure_refresh_workspace()
+        B.moara_step_grouped(self.ctx, ids, [g.data_ptr() for g in grads], t, lr,
+                             auto_refresh, stream)
+
+    def status(self, stream=0):
+        return B.moara_get_device_status(self.ctx, stream)
+
+    def close(self):
+        if self.ctx:
+            B.moara_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,902 @@
+// Host side of libmoara: argument validation, the context and its device
+// module table, the memory model and rank table helpers, and the sequencing of
+// the step and refresh kernels.  Declarations and contracts are in moara.h.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <limits>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "internal.h"
+#include "tc.h"
+
+struct moara_ctx {
+    int device = 0;
+    moara_hparams hp{};
+    std::vector<moara_module_desc> mods;
+    std::vector<moara::ModDev> moddev;
+    std::vector<int64_t> refresh_count;
+    moara::ModDev* d_mods = nullptr;
+    int cap = 0;
+    int* d_status = nullptr;
+    int* h_status = nullptr;
+    void* refresh_ws = nullptr;
+    size_t refresh_ws_bytes = 0;
+    std::string last_error;
+    int64_t launches = 0;
+    moara::TcState* tc = nullptr;
+    // per-kernel CUDA-event timing (moara_profile_enable)
+    bool prof = false;
+    struct Rec { int phase; cudaEvent_t a, b; };
+    std::vector<Rec> recs;
+    std::vector<cudaEvent_t> free_events;
+    double prof_ms[MOARA_NUM_PHASES] = {0};
+    int64_t prof_n[MOARA_NUM_PHASES] = {0};
+};
+
+namespace {
+
+constexpr int kMaxModules = 65536;
+
+int fail(moara_ctx* ctx, int code, const char* fmt, ...) {
+    if (ctx != nullptr) {
+        char buf[512];
+        va_list ap;
+        va_start(ap, fmt);
+        std::vsnprintf(buf, sizeof(buf), fmt, ap);
+        va_end(ap);
+        ctx->last_error = buf;
+    }
+    return code;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int blocks_of(int n, int B) { return (n + B - 1) / B; }
+
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) cudaSetDevice(dev);
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+int check_hparams(moara_ctx* ctx, const moara_hparams* hp) {
+    if (hp == nullptr) return fail(ctx, MOARA_ERR_INVALID_ARG, "hparams is NULL");
+    if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f) || !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f))
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "betas must lie in [0, 1)");
+    if (!(hp->adam_eps >= 0.0f) || !std::isfinite(hp->adam_eps))
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "adam_eps must be finite and >= 0");
+    if (!(hp->decomp_eps >= 0.0f) || !std::isfinite(hp->decomp_eps))
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "decomp_eps must be finite and >= 0");
+    if (!std::isfinite(hp->scale)) return fail(ctx, MOARA_ERR_INVALID_ARG, "scale must be finite");
+    if (hp->block_size < 1) return fail(ctx, MOARA_ERR_SHAPE, "block_size must be >= 1");
+    if (hp->refresh_interval < 1) return fail(ctx, MOARA_ERR_SHAPE, "refresh_interval must be >= 1");
+    if (hp->decompose != 0 && hp->decompose != 1)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "decompose must be 0 or 1");
+    if (hp->refresh_src != MOARA_REFRESH_SRC_V && hp->refresh_src != MOARA_REFRESH_SRC_G)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "unknown refresh_src");
+    if (hp->oversample < 0 || hp->power_iters < 0 || hp->ritz_iters < 0)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "oversample, power_iters, ritz_iters must be >= 0");
+    if (hp->oversample > 4096 || hp->power_iters > 64 || hp->ritz_iters > 256)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "refresh parameters out of range");
+    if (hp->precision != MOARA_PREC_AUTO && hp->precision != MOARA_PREC_FP32 &&
+        hp->precision != MOARA_PREC_BF16_TC)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "unknown precision");
+    return MOARA_OK;
+}
+
+int cuda_fail(moara_ctx* ctx, cudaError_t e, const char* what) {
+    return fail(ctx, MOARA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+cudaEvent_t take_event(moara_ctx* ctx) {
+    if (!ctx->free_events.empty()) {
+        cudaEvent_t e = ctx->free_events.back();
+        ctx->free_events.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+}
+
+// Records an event pair around the launches made in its scope when profiling.
+struct ProfScope {
+    moara_ctx* ctx;
+    int phase;
+    cudaStream_t s;
+    cudaEvent_t a = nullptr;
+    ProfScope(moara_ctx* c, int ph, cudaStream_t st) : ctx(c), phase(ph), s(st) {
+        if (ctx->prof) {
+            a = take_event(ctx);
+            cudaEventRecord(a, s);
+        }
+    }
+    ~ProfScope() {
+        if (a != nullptr) {
+            cudaEvent_t b = take_event(ctx);
+            cudaEventRecord(b, s);
+            ctx->recs.push_back({phase, a, b});
+        }
+    }
+};
+
+// Whether module `mi` runs its step on tensor cores.
+bool use_tc(const moara_ctx* ctx, int mi) {
+    const moara_module_desc& d = ctx->mods[mi];
+    if (ctx->hp.precision == MOARA_PREC_FP32) return false;
+    if (ctx->hp.precision == MOARA_PREC_AUTO && d.grad_dtype != MOARA_DTYPE_BF16) return false;
+    return moara::tc_supported(d.m, d.n, d.r, ctx->hp.block_size, d.grad_dtype, ctx->hp.decompose) &&
+           d.P_bf16 != nullptr && ctx->tc != nullptr;
+}
+
+}  // namespace
+
+namespace moara {
+
+WsLayout workspace_layout(int m, int n, int r, int B) {
+    const int kb = blocks_of(n, B);
+    WsLayout w{};
+    size_t off = 0;
+    w.off_N = off;   off = align_up(off + sizeof(float) * (size_t)r * n, 256);
+    w.off_dM = off;  off = align_up(off + sizeof(float) * (size_t)m * kb, 256);
+    w.off_inv = off; off = align_up(off + sizeof(float) * (size_t)m * kb, 256);
+    w.total = off;
+    return w;
+}
+
+size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v) {
+    (void)r;
+    const int kb = blocks_of(n, B);
+    size_t off = 0;
+    auto add = [&](size_t bytes) { off = align_up(off + bytes, 256); };
+    if (src_v) add(sizeof(float) * (size_t)m * kb);
+    add(sizeof(float) * (size_t)n * l);  // Za (also Omega)
+    add(sizeof(float) * (size_t)n * l);  // Zb
+    add(sizeof(float) * (size_t)m * l);  // Qa
+    add(sizeof(float) * (size_t)m * l);  // Qb
+    for (int i = 0; i < 5; ++i) add(sizeof(float) * (size_t)l * l);
+    add(sizeof(float) * (size_t)l);
+    add(sizeof(int) * (size_t)l);
+    add(sizeof(int) * 4);
+    return off;
+}
+
+void refresh_carve(RefreshItem& it, void* base, int m, int n, int r, int l, int B, int src_v) {
+    (void)r;
+    const int kb = blocks_of(n, B);
+    char* p = static_cast<char*>(base);
+    size_t off = 0;
+    auto take = [&](size_t bytes) { char* q = p + off; off = align_up(off + bytes, 256); return q; };
+    it.inv = src_v ? reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * kb)) : nullptr;
+    it.Za = reinterpret_cast<float*>(take(sizeof(float) * (size_t)n * l));
+    it.Omega = it.Za;
+    it.Zb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)n * l));
+    it.Qa = reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * l));
+    it.Qb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * l));
+    it.Cg = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
+    it.Linv = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
+    it.Cr = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
+    it.Xa = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
+    it.Xb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
+    it.ritz = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l));
+    it.perm = reinterpret_cast<int*>(take(sizeof(int) * (size_t)l));
+    it.fail = reinterpret_cast<int*>(take(sizeof(int) * 4));
+}
+
+}  // namespace moara
+
+namespace {
+
+int refresh_l(const moara_ctx* ctx, int m, int n, int r) {
+    long long l = (long long)r + ctx->hp.oversample;
+    l = std::min<long long>(l, std::min(m, n));
+    return static_cast<int>(std::max<long long>(l, r));
+}
+
+// ------------------------------------------------------------------ refresh
+struct RefreshRunner {
+    moara_ctx* ctx;
+    cudaStream_t s;
+    std::vector<moara::RefreshItem> it;
+    int src_v;
+    cudaError_t err = cudaSuccess;
+
+    void chk(cudaError_t e) { if (err == cudaSuccess && e != cudaSuccess) err = e; }
+
+    template <class F>
+    void gemm(const moara::GemmKind& kind, F fill) {
+        moara::GemmBatch b{};
+        b.count = static_cast<int>(it.size());
+        b.B = ctx->hp.block_size;
+        for (int i = 0; i < b.count; ++i) {
+            b.p[i] = moara::GemmProb{};
+            fill(i, b.p[i]);
+        }
+        chk(moara::launch_gemm(kind, b, s, &ctx->launches));
+    }
+
+    moara::SmallBatch small() {
+        moara::SmallBatch b{};
+        b.count = static_cast<int>(it.size());
+        return b;
+    }
+
+    // X_out = X_in * chol(X_in^T X_in + shift)^-T for every item (rows(i) x l).
+    void cholqr_pass(std::vector<float*>& Xin, std::vector<float*>& Xout,
+                     const std::vector<int>& rows, float shift_rel) {
+        moara::GemmKind gram{moara::A_MCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
+        gemm(gram, [&](int i, moara::GemmProb& p) {
+            const int l = it[i].l;
+            p.A = Xin[i]; p.Bm = Xin[i]; p.C = it[i].Cg;
+            p.M = l; p.N = l; p.K = rows[i]; p.lda = l; p.ldb = l; p.ldc = l;
+        });
+        moara::SmallBatch sb = small();
+        sb.shift_rel = shift_rel;
+        for (size_t i = 0; i < it.size(); ++i) {
+            sb.l[i] = it[i].l; sb.rows[i] = rows[i]; sb.a[i] = it[i].Cg; sb.c[i] = it[i].Linv;
+            sb.fail[i] = it[i].fail;
+        }
+        chk(moara::launch_cholesky(sb, s, &ctx->launches));
+        chk(moara::launch_tri_inverse(sb, s, &ctx->launches));
+        moara::GemmKind apply{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
+        gemm(apply, [&](int i, moara::GemmProb& p) {
+            const int l = it[i].l;
+            p.A = Xin[i]; p.Bm = it[i].Linv; p.C = Xout[i];
+            p.M = rows[i]; p.N = l; p.K = l; p.lda = l; p.ldb = l; p.ldc = l;
+        });
+    }
+
+    // Shifted CholeskyQR followed by CholeskyQR2; result lands in `b`.
+    void cholqr3(std::vector<float*>& a, std::vector<float*>& b, const std::vector<int>& rows) {
+        const float u = 5.9604645e-08f;   // fp32 unit roundoff
+        cholqr_pass(a, b, rows, 2.0f * u);
+        cholqr_pass(b, a, rows, 0.0f);
+        cholqr_pass(a, b, rows, 0.0f);
+    }
+
+    void run() {
+        const int n_it = static_cast<int>(it.size());
+        const moara_hparams& hp = ctx->hp;
+        for (auto& x : it) chk(cudaMemsetAsync(x.fail, 0, sizeof(int), s));
+        // block scales of Decompose(G, B) when the source is V
+        if (src_v) {
+            moara::DecompBatch db{};
+            db.count = n_it; db.B = hp.block_size; db.do_mag = 0; db.decomp_eps = hp.decomp_eps;
+            long long acc = 0;
+            for (int i = 0; i < n_it; ++i) {
+                db.item_start[i] = acc;
+                db.p[i] = moara::DecompItem{it[i].G, it[i].inv, nullptr, nullptr, nullptr,
+                                            it[i].m, it[i].n, it[i].kb, it[i].dtype};
+                acc += (long long)it[i].m * it[i].kb;
+            }
+            db.item_start[n_it] = acc;
+            chk(moara::launch_decompose(db, s, &ctx->launches));
+        }
+        // Gaussian test matrix Omega (n x l)
+        {
+            moara::SmallBatch sb = small();
+            for (int i = 0; i < n_it; ++i) {
+                sb.a[i] = it[i].Omega; sb.rows[i] = it[i].n; sb.l[i] = it[i].l; sb.key[i] = it[i].key;
+            }
+            chk(moara::launch_philox_gaussian(sb, s, &ctx->launches));
+        }
+        std::vector<float*> Qa(n_it), Qb(n_it), Za(n_it), Zb(n_it), Xa(n_it), Xb(n_it);
+        std::vector<int> rows_m(n_it), rows_n(n_it), rows_l(n_it);
+        for (int i = 0; i < n_it; ++i) {
+            Qa[i] = it[i].Qa; Qb[i] = it[i].Qb; Za[i] = it[i].Za; Zb[i] = it[i].Zb;
+            Xa[i] = it[i].Xa; Xb[i] = it[i].Xb;
+            rows_m[i] = it[i].m; rows_n[i] = it[i].n; rows_l[i] = it[i].l;
+        }
+        const int bf = it.empty() ? 0 : (it[0].dtype == MOARA_DTYPE_BF16);
+        // Y = V * Omega  (m x l)
+        auto v_times = [&](std::vector<float*>& rhs, std::vector<float*>& out) {
+            for (int d = 0; d < 2; ++d) {  // per-dtype sub-batches
+                std::vector<int> sel;
+                for (int i = 0; i < n_it; ++i) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
+                if (sel.empty()) continue;
+                moara::GemmKind k{moara::A_KCONTIG, moara::B_NCONTIG, src_v, 0, d, 0, moara::EPI_STORE};
+                moara::GemmBatch b{};
+                b.count = static_cast<int>(sel.size());
+                b.B = hp.block_size;
+                for (int q = 0; q < b.count; ++q) {
+                    const auto& x = it[sel[q]];
+                    moara::GemmProb& p = b.p[q];
+                    p = moara::GemmProb{};
+                    p.A = x.G; p.a_inv = x.inv; p.Bm = rhs[sel[q]]; p.C = out[sel[q]];
+                    p.M = x.m; p.N = x.l; p.K = x.n; p.lda = x.n; p.ldb = x.l; p.ldc = x.l; p.kb = x.kb;
+                    p.a_bf16 = d;
+                }
+                chk(moara::launch_gemm(k, b, s, &ctx->launches));
+            }
+        };
+        // Z = V^T * Q  (n x l)
+        auto vt_times = [&](std::vector<float*>& rhs, std::vector<float*>& out) {
+            for (int d = 0; d < 2; ++d) {
+                std::vector<int> sel;
+                for (int i = 0; i < n_it; ++i) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
+                if (sel.empty()) continue;
+                moara::GemmKind k{moara::A_MCONTIG, moara::B_NCONTIG, src_v, 0, d, 0, moara::EPI_STORE};
+                moara::GemmBatch b{};
+                b.count = static_cast<int>(sel.size());
+                b.B = hp.block_size;
+                for (int q = 0; q < b.count; ++q) {
+                    const auto& x = it[sel[q]];
+                    moara::GemmProb& p = b.p[q];
+                    p = moara::GemmProb{};
+                    p.A = x.G; p.a_inv = x.inv; p.Bm = rhs[sel[q]]; p.C = out[sel[q]];
+                    p.M = x.n; p.N = x.l; p.K = x.m; p.lda = x.n; p.ldb = x.l; p.ldc = x.l; p.kb = x.kb;
+                    p.a_bf16 = d;
+                }
+                chk(moara::launch_gemm(k, b, s, &ctx->launches));
+            }
+        };
+        (void)bf;
+        v_times(Za, Qa);
+        cholqr3(Qa, Qb, rows_m);          // Q in Qb
+        for (int q = 0; q < hp.power_iters; ++q) {
+            vt_times(Qb, Za);
+            cholqr3(Za, Zb, rows_n);      // Z in Zb
+            v_times(Zb, Qa);
+            cholqr3(Qa, Qb, rows_m);      // Q in Qb
+        }
+        // Rayleigh-Ritz on span(Q): C = (V^T Q)^T (V^T Q), eigenvectors of C by
+        // orthogonal iteration with CholeskyQR, ordered by Ritz value.
+        vt_times(Qb, Za);
+        {
+            moara::GemmKind gram{moara::A_MCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
+            gemm(gram, [&](int i, moara::GemmProb& p) {
+                const int l = it[i].l;
+                p.A = Za[i]; p.Bm = Za[i]; p.C = it[i].Cr;
+                p.M = l; p.N = l; p.K = it[i].n; p.lda = l; p.ldb = l; p.ldc = l;
+            });
+        }
+        {
+            moara::SmallBatch sb = small();
+            for (int i = 0; i < n_it; ++i) { sb.a[i] = Xa[i]; sb.l[i] = it[i].l; }
+            chk(moara::launch_set_identity(sb, s, &ctx->launches));
+        }
+        moara::GemmKind prod{moara::A_KCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
+        for (int q = 0; q < hp.ritz_iters; ++q) {
+            gemm(prod, [&](int i, moara::GemmProb& p) {
+                const int l = it[i].l;
+                p.A = it[i].Cr; p.Bm = Xa[i]; p.C = Xb[i];
+                p.M = l; p.N = l; p.K = l; p.lda = l; p.ldb = l; p.ldc = l;
+            });
+            cholqr3(Xb, Xa, rows_l);      // X in Xa
+        }
+        // Ritz values and order: W = C X into Xb
+        gemm(prod, [&](int i, moara::GemmProb& p) {
+            const int l = it[i].l;
+            p.A = it[i].Cr; p.Bm = Xa[i]; p.C = Xb[i];
+            p.M = l; p.N = l; p.K = l; p.lda = l; p.ldb = l; p.ldc = l;
+        });
+        {
+            moara::SmallBatch sb = small();
+            for (int i = 0; i < n_it; ++i) {
+                sb.a[i] = Xa[i]; sb.b[i] = Xb[i]; sb.c[i] = it[i].ritz; sb.iaux[i] = it[i].perm;
+                sb.l[i] = it[i].l;
+            }
+            chk(moara::launch_ritz_sort(sb, s, &ctx->launches));
+        }
+        {   // Xs (l x r) = X[:, perm[:r]] into Linv
+            moara::SmallBatch sb = small();
+            for (int i = 0; i < n_it; ++i) {
+                sb.a[i] = Xa[i]; sb.c[i] = it[i].Linv; sb.iaux[i] = it[i].perm;
+                sb.l[i] = it[i].l; sb.rows[i] = it[i].r;
+            }
+            chk(moara::launch_gather_cols(sb, s, &ctx->launches));
+        }
+        // P_tmp (m x r) = Q * Xs into Qa
+        gemm(prod, [&](int i, moara::GemmProb& p) {
+            p.A = Qb[i]; p.Bm = it[i].Linv; p.C = Qa[i];
+            p.M = it[i].m; p.N = it[i].r; p.K = it[i].l; p.lda = it[i].l; p.ldb = it[i].r; p.ldc = it[i].r;
+        });
+        {
+            moara::SmallBatch sb = small();
+            for (int i = 0; i < n_it; ++i) {
+                sb.a[i] = Qa[i]; sb.c[i] = it[i].P; sb.h[i] = it[i].Pb; sb.fail[i] = it[i].fail;
+                sb.rows[i] = it[i].m; sb.l[i] = it[i].r;
+            }
+            chk(moara::launch_sign_fix_store(sb, s, &ctx->launches));
+        }
+    }
+};
+
+int do_refresh(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, cudaStream_t s) {
+    const moara_hparams& hp = ctx->hp;
+    const int src_v = (hp.refresh_src == MOARA_REFRESH_SRC_V && hp.decompose) ? 1 : 0;
+    // group modules so that each group fits the refresh workspace
+    int start = 0;
+    while (start < n_mod) {
+        RefreshRunner rr{ctx, s, {}, src_v};
+        size_t used = 0;
+        int end = start;
+        while (end < n_mod && static_cast<int>(rr.it.size()) < moara::kMaxGroup) {
+            const int id = ids[end];
+            const moara_module_desc& d = ctx->mods[id];
+            const int l = refresh_l(ctx, d.m, d.n, d.r);
+            const size_t need = align_up(moara::refresh_ws_bytes(d.m, d.n, d.r, l, hp.block_size, src_v), 256);
+            if (used + need > ctx->refresh_ws_bytes) {
+                if (rr.it.empty())
+                    return fail(ctx, MOARA_ERR_WORKSPACE,
+                                "refresh workspace of %zu bytes is smaller than the %zu bytes module %d needs",
+                                ctx->refresh_ws_bytes, need, id);
+                break;
+            }
+            moara::RefreshItem x{};
+            x.m = d.m; x.n = d.n; x.r = d.r; x.l = l; x.kb = blocks_of(d.n, hp.block_size);
+            x.dtype = d.grad_dtype; x.G = G[end];
+            moara::refresh_carve(x, static_cast<char*>(ctx->refresh_ws) + used, d.m, d.n, d.r, l,
+                                 hp.block_size, src_v);
+            x.P = d.P; x.Pb = d.P_bf16;
+            const uint64_t cnt = static_cast<uint64_t>(ctx->refresh_count[id]++);
+            x.key = hp.seed ^ (0x9E3779B97F4A7C15ull * (static_cast<uint64_t>(id) + 1)) ^
+                    (cnt * 0xD1B54A32D192ED03ull);
+            rr.it.push_back(x);
+            used += need;
+            ++end;
+        }
+        rr.run();
+        if (rr.err != cudaSuccess) return cuda_fail(ctx, rr.err, "refresh launch");
+        start = end;
+    }
+    return MOARA_OK;
+}
+
+// ------------------------------------------------------------------ step
+int do_step_simt(moara_ctx* ctx, const std::vector<int>& sel, const int* ids, const void* const* G,
+                 int64_t t, float lr, cudaStream_t s) {
+    const moara_hparams& hp = ctx->hp;
+    const double bc1 = 1.0 - std::pow((double)hp.beta1, (double)t);
+    const double bc2 = 1.0 - std::pow((double)hp.beta2, (double)t);
+    // longest K (= m for the projection) first
+    std::vector<int> order(sel);
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) {
+        return ctx->mods[ids[a]].m > ctx->mods[ids[b]].m;
+    });
+    for (size_t c0 = 0; c0 < order.size(); c0 += moara::kMaxGroup) {
+        const int cnt = static_cast<int>(std::min<size_t>(moara::kMaxGroup, order.size() - c0));
+        if (hp.decompose) {
+            moara::DecompBatch db{};
+            db.count = cnt; db.B = hp.block_size; db.do_mag = 1; db.decomp_eps = hp.decomp_eps;
+            db.beta1 = hp.beta1; db.beta2 = hp.beta2; db.adam_eps = hp.adam_eps;
+            db.bc1 = static_cast<float>(bc1); db.bc2 = static_cast<float>(bc2);
+            long long acc = 0;
+            for (int q = 0; q < cnt; ++q) {
+                const int i = order[c0 + q];
+                const moara::ModDev& md = ctx->moddev[ids[i]];
+                db.item_start[q] = acc;
+                db.p[q] = moara::DecompItem{G[i], md.ws_inv, md.mag_avg, md.mag_avg_sq, md.ws_dM,
+                                            md.m, md.n, md.kb, md.dtype};
+                acc += (long long)md.m * md.kb;
+            }
+            db.item_start[cnt] = acc;
+            cudaError_t e;
+            {
+                ProfScope ps(ctx, MOARA_PHASE_DECOMPOSE, s);
+                e = moara::launch_decompose(db, s, &ctx->launches);
+            }
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "decompose launch");
+        }
+        // projection + direction Adam, split by gradient dtype
+        for (int d = 0; d < 2; ++d) {
+            moara::GemmBatch b{};
+            b.B = hp.block_size; b.beta1 = hp.beta1; b.beta2 = hp.beta2; b.adam_eps = hp.adam_eps;
+            b.bc1 = static_cast<float>(bc1); b.bc2 = static_cast<float>(bc2);
+            for (int q = 0; q < cnt; ++q) {
+                const int i = order[c0 + q];
+                const moara::ModDev& md = ctx->moddev[ids[i]];
+                if ((md.dtype == MOARA_DTYPE_BF16) != (d == 1)) continue;
+                moara::GemmProb& p = b.p[b.count++];
+                p = moara::GemmProb{};
+                p.A = md.P; p.Bm = G[i]; p.b_inv = hp.decompose ? md.ws_inv : nullptr;
+                p.C = md.ws_N; p.aux0 = md.exp_avg; p.aux1 = md.exp_avg_sq;
+                p.M = md.r; p.N = md.n; p.K = md.m; p.lda = md.r; p.ldb = md.n; p.ldc = md.n;
+                p.kb = md.kb; p.b_bf16 = d;
+            }
+            moara::GemmKind k{moara::A_MCONTIG, moara::B_NCONTIG, 0, hp.decompose, 0, d, moara::EPI_ADAM};
+            if (b.count == 0) continue;
+            cudaError_t e;
+            {
+                ProfScope ps(ctx, MOARA_PHASE_PROJECT, s);
+                e = moara::launch_gemm(k, b, s, &ctx->launches);
+            }
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "projection launch");
+        }
+        // back-projection + weight update
+        {
+            moara::GemmBatch b{};
+            b.B = hp.block_size;
+            b.step_scale = lr * hp.scale;
+            for (int q = 0; q < cnt; ++q) {
+                const int i = order[c0 + q];
+                const moara::ModDev& md = ctx->moddev[ids[i]];
+                moara::GemmProb& p = b.p[b.count++];
+                p = moara::GemmProb{};
+                p.A = md.P; p.Bm = md.ws_N; p.aux0 = md.W; p.aux2 = hp.decompose ? md.ws_dM : nullptr;
+                p.M = md.m; p.N = md.n; p.K = md.r; p.lda = md.r; p.ldb = md.n; p.ldc = md.n; p.kb = md.kb;
+            }
+            moara::GemmKind k{moara::A_KCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_UPDATE};
+            cudaError_t e;
+            {
+                ProfScope ps(ctx, MOARA_PHASE_BACKPROJECT, s);
+                e = moara::launch_gemm(k, b, s, &ctx->launches);
+            }
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "back-projection launch");
+        }
+    }
+    return MOARA_OK;
+}
+
+int check_ids(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G) {
+    if (n_mod < 0) return fail(ctx, MOARA_ERR_INVALID_ARG, "n_mod must be >= 0");
+    if (n_mod > 0 && (ids == nullptr || G == nullptr))
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "ids and G must not be NULL");
+    std::vector<char> seen(ctx->mods.size(), 0);
+    for (int i = 0; i < n_mod; ++i) {
+        if (ids[i] < 0 || ids[i] >= static_cast<int>(ctx->mods.size()))
+            return fail(ctx, MOARA_ERR_UNKNOWN_MODULE, "module id %d is not registered", ids[i]);
+        if (seen[ids[i]]) return fail(ctx, MOARA_ERR_INVALID_ARG, "module id %d listed twice", ids[i]);
+        seen[ids[i]] = 1;
+        if (G[i] == nullptr) return fail(ctx, MOARA_ERR_INVALID_ARG, "G[%d] is NULL", i);
+        if (!aligned16(G[i])) return fail(ctx, MOARA_ERR_ALIGN, "G[%d] is not 16-byte aligned", i);
+    }
+    return MOARA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int moara_default_hparams(moara_hparams* out) {
+    if (out == nullptr) return MOARA_ERR_INVALID_ARG;
+    std::memset(out, 0, sizeof(*out));
+    out->beta1 = 0.9f;
+    out->beta2 = 0.999f;
+    out->adam_eps = 1e-6f;
+    out->decomp_eps = 1e-12f;
+    out->scale = 0.25f;
+    out->block_size = 128;
+    out->refresh_interval = 200;
+    out->decompose = 1;
+    out->refresh_src = MOARA_REFRESH_SRC_V;
+    out->oversample = 0;
+    out->power_iters = 2;
+    out->ritz_iters = 16;
+    out->precision = MOARA_PREC_AUTO;
+    out->seed = 0;
+    return MOARA_OK;
+}
+
+int moara_create(moara_ctx** out, const moara_hparams* hp, int device) {
+    if (out == nullptr) return MOARA_ERR_INVALID_ARG;
+    *out = nullptr;
+    moara_ctx tmp;
+    int rc = check_hparams(&tmp, hp);
+    if (rc != MOARA_OK) return rc;
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) return MOARA_ERR_CUDA;
+    moara_ctx* ctx = new (std::nothrow) moara_ctx();
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    ctx->device = device;
+    ctx->hp = *hp;
+    DeviceGuard g(device);
+    ctx->cap = 1024;
+    if (cudaMalloc(&ctx->d_mods, sizeof(moara::ModDev) * ctx->cap) != cudaSuccess ||
+        cudaMalloc(&ctx->d_status, sizeof(int) * 4) != cudaSuccess ||
+        cudaMallocHost(&ctx->h_status, sizeof(int) * 4) != cudaSuccess ||
+        cudaMemset(ctx->d_status, 0, sizeof(int) * 4) != cudaSuccess) {
+        moara_destroy(ctx);
+        return MOARA_ERR_CUDA;
+    }
+    ctx->tc = moara::tc_create(device, ctx->d_status);
+    *out = ctx;
+    return MOARA_OK;
+}
+
+void moara_destroy(moara_ctx* ctx) {
+    if (ctx == nullptr) return;
+    DeviceGuard g(ctx->device);
+    if (ctx->tc) moara::tc_destroy(ctx->tc);
+    for (auto& r : ctx->recs) { cudaEventDestroy(r.a); cudaEventDestroy(r.b); }
+    for (auto e : ctx->free_events) cudaEventDestroy(e);
+    if (ctx->d_mods) cudaFree(ctx->d_mods);
+    if (ctx->d_status) cudaFree(ctx->d_status);
+    if (ctx->h_status) cudaFreeHost(ctx->h_status);
+    delete ctx;
+}
+
+int moara_get_hparams(const moara_ctx* ctx, moara_hparams* out) {
+    if (ctx == nullptr || out == nullptr) return MOARA_ERR_INVALID_ARG;
+    *out = ctx->hp;
+    return MOARA_OK;
+}
+
+int moara_state_bytes(int m, int n, int r, int block_size, int b_V, int b_M, int d_rule,
+                      int decompose, size_t* out) {
+    if (out == nullptr) return MOARA_ERR_INVALID_ARG;
+    if (m < 1 || n < 1 || block_size < 1 || b_V < 0 || b_M < 0) return MOARA_ERR_SHAPE;
+    if (r < 1 || r > std::min(m, n)) return MOARA_ERR_RANK;
+    if (d_rule != MOARA_DRULE_N && d_rule != MOARA_DRULE_MAX) return MOARA_ERR_INVALID_ARG;
+    const unsigned long long d = d_rule == MOARA_DRULE_N ? (unsigned long long)n
+                                                         : (unsigned long long)std::max(m, n);
+    const unsigned long long kb = (unsigned long long)blocks_of(n, block_size);
+    const long double dir = 2.0L * b_V * (long double)r * d;
+    const long double mag = decompose ? 2.0L * b_M * (long double)m * kb : 0.0L;
+    const long double tot = dir + mag;
+    if (tot > (long double)std::numeric_limits<size_t>::max()) return MOARA_ERR_SHAPE;
+    *out = static_cast<size_t>(2ull * b_V * r * d + (decompose ? 2ull * b_M * m * kb : 0ull));
+    return MOARA_OK;
+}
+
+int moara_rank_table(int r_base, uint32_t donor_mask, uint32_t receiver_mask, int delta_r,
+                     int out_ranks[7]) {
+    if (out_ranks == nullptr) return MOARA_ERR_INVALID_ARG;
+    if (r_base < 1) return MOARA_ERR_RANK;
+    if (((donor_mask | receiver_mask) >> 7) != 0) return MOARA_ERR_INVALID_ARG;
+    if (donor_mask & receiver_mask) return MOARA_ERR_INVALID_ARG;
+    if (delta_r < 0 || delta_r >= r_base) return MOARA_ERR_RANK;
+    int nd = 0, nr = 0;
+    for (int i = 0; i < 7; ++i) {
+        nd += (donor_mask >> i) & 1;
+        nr += (receiver_mask >> i) & 1;
+    }
+    if (nd > 0 && nr == 0) return MOARA_ERR_INVALID_ARG;
+    const long long moved = (long long)delta_r * nd;
+    const long long share = nr ? moved / nr : 0;
+    long long rem = nr ? moved - share * nr : 0;
+    for (int i = 0; i < 7; ++i) {
+        long long v = r_base;
+        if ((donor_mask >> i) & 1) v = r_base - delta_r;
+        if ((receiver_mask >> i) & 1) {
+            v = r_base + share + (rem > 0 ? 1 : 0);
+            if (rem > 0) --rem;
+        }
+        if (v > std::numeric_limits<int>::max()) return MOARA_ERR_RANK;
+        out_ranks[i] = static_cast<int>(v);
+    }
+    return MOARA_OK;
+}
+
+int moara_workspace_bytes(int m, int n, int r, int block_size, size_t* out) {
+    if (out == nullptr) return MOARA_ERR_INVALID_ARG;
+    if (m < 1 || n < 1 || block_size < 1) return MOARA_ERR_SHAPE;
+    if (r < 1 || r > std::min(m, n)) return MOARA_ERR_RANK;
+    *out = moara::workspace_layout(m, n, r, block_size).total;
+    return MOARA_OK;
+}
+
+int moara_init_module(moara_ctx* ctx, const moara_module_desc* d, int* module_id) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    if (d == nullptr || module_id == nullptr) return fail(ctx, MOARA_ERR_INVALID_ARG, "desc or module_id is NULL");
+    if (d->m < 1 || d->n < 1) return fail(ctx, MOARA_ERR_SHAPE, "m and n must be >= 1 (got %d x %d)", d->m, d->n);
+    if ((long long)d->m * d->n > (1LL << 40)) return fail(ctx, MOARA_ERR_SHAPE, "matrix too large");
+    if (d->r < 1 || d->r > std::min(d->m, d->n))
+        return fail(ctx, MOARA_ERR_RANK, "rank %d outside [1, min(m, n) = %d]", d->r, std::min(d->m, d->n));
+    if (d->grad_dtype != MOARA_DTYPE_F32 && d->grad_dtype != MOARA_DTYPE_BF16)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "unknown grad_dtype %d", d->grad_dtype);
+    const void* req[] = {d->W, d->P, d->exp_avg, d->exp_avg_sq, d->workspace};
+    const char* names[] = {"W", "P", "exp_avg", "exp_avg_sq", "workspace"};
+    for (int i = 0; i < 5; ++i) {
+        if (req[i] == nullptr) return fail(ctx, MOARA_ERR_INVALID_ARG, "%s is NULL", names[i]);
+        if (!aligned16(req[i])) return fail(ctx, MOARA_ERR_ALIGN, "%s is not 16-byte aligned", names[i]);
+    }
+    if (ctx->hp.decompose) {
+        if (d->mag_avg == nullptr || d->mag_avg_sq == nullptr)
+            return fail(ctx, MOARA_ERR_INVALID_ARG, "mag_avg / mag_avg_sq are NULL with decompose = 1");
+        if (!aligned16(d->mag_avg) || !aligned16(d->mag_avg_sq))
+            return fail(ctx, MOARA_ERR_ALIGN, "mag_avg / mag_avg_sq not 16-byte aligned");
+    }
+    if (d->P_bf16 != nullptr && !aligned16(d->P_bf16))
+        return fail(ctx, MOARA_ERR_ALIGN, "P_bf16 is not 16-byte aligned");
+    if (ctx->hp.precision == MOARA_PREC_BF16_TC && d->P_bf16 == nullptr)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "P_bf16 is required with precision BF16_TC");
+    const moara::WsLayout wl = moara::workspace_layout(d->m, d->n, d->r, ctx->hp.block_size);
+    if (d->workspace_bytes < wl.total)
+        return fail(ctx, MOARA_ERR_WORKSPACE, "workspace of %zu bytes, %zu needed", d->workspace_bytes, wl.total);
+    if (static_cast<int>(ctx->mods.size()) >= kMaxModules)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "too many modules");
+
+    DeviceGuard g(ctx->device);
+    if (static_cast<int>(ctx->mods.size()) >= ctx->cap) {
+        const int ncap = ctx->cap * 2;
+        moara::ModDev* nd = nullptr;
+        cudaError_t e = cudaMalloc(&nd, sizeof(moara::ModDev) * ncap);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMalloc module table");
+        if (!ctx->moddev.empty()) {
+            e = cudaMemcpy(nd, ctx->moddev.data(), sizeof(moara::ModDev) * ctx->moddev.size(),
+                           cudaMemcpyHostToDevice);
+            if (e != cudaSuccess) { cudaFree(nd); return cuda_fail(ctx, e, "module table copy"); }
+        }
+        cudaFree(ctx->d_mods);
+        ctx->d_mods = nd;
+        ctx->cap = ncap;
+    }
+    moara::ModDev md{};
+    md.m = d->m; md.n = d->n; md.r = d->r; md.kb = blocks_of(d->n, ctx->hp.block_size);
+    md.dtype = d->grad_dtype;
+    md.W = d->W; md.P = d->P; md.Pb = d->P_bf16;
+    md.exp_avg = d->exp_avg; md.exp_avg_sq = d->exp_avg_sq;
+    md.mag_avg = d->mag_avg; md.mag_avg_sq = d->mag_avg_sq;
+    char* ws = static_cast<char*>(d->workspace);
+    md.ws_N = reinterpret_cast<float*>(ws + wl.off_N);
+    md.ws_dM = reinterpret_cast<float*>(ws + wl.off_dM);
+    md.ws_inv = reinterpret_cast<float*>(ws + wl.off_inv);
+    const int id = static_cast<int>(ctx->mods.size());
+    cudaError_t e = cudaMemcpy(ctx->d_mods + id, &md, sizeof(md), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "module table copy");
+    if (ctx->tc) {
+        int rc = moara::tc_register(ctx->tc, id, md, ctx->hp);
+        if (rc != MOARA_OK) return fail(ctx, rc, "tensor-core registration of module %d failed", id);
+    }
+    ctx->mods.push_back(*d);
+    ctx->moddev.push_back(md);
+    ctx->refresh_count.push_back(0);
+    *module_id = id;
+    ctx->last_error.clear();
+    return MOARA_OK;
+}
+
+int moara_load_projector(moara_ctx* ctx, int module_id, const float* P_src, void* stream) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    if (module_id < 0 || module_id >= static_cast<int>(ctx->mods.size()))
+        return fail(ctx, MOARA_ERR_UNKNOWN_MODULE, "module id %d is not registered", module_id);
+    if (P_src == nullptr) return fail(ctx, MOARA_ERR_INVALID_ARG, "P_src is NULL");
+    if (!aligned16(P_src)) return fail(ctx, MOARA_ERR_ALIGN, "P_src is not 16-byte aligned");
+    DeviceGuard g(ctx->device);
+    const moara::ModDev& md = ctx->moddev[module_id];
+    cudaError_t e = moara::launch_f32_to_bf16(P_src, md.P, md.Pb, (long long)md.m * md.r,
+                                              static_cast<cudaStream_t>(stream), &ctx->launches);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "projector copy");
+    return MOARA_OK;
+}
+
+int moara_refresh_workspace_bytes(const moara_ctx* ctx, int m, int n, int r, size_t* out) {
+    if (ctx == nullptr || out == nullptr) return MOARA_ERR_INVALID_ARG;
+    if (m < 1 || n < 1) return MOARA_ERR_SHAPE;
+    if (r < 1 || r > std::min(m, n)) return MOARA_ERR_RANK;
+    const int src_v = (ctx->hp.refresh_src == MOARA_REFRESH_SRC_V && ctx->hp.decompose) ? 1 : 0;
+    *out = align_up(moara::refresh_ws_bytes(m, n, r, refresh_l(ctx, m, n, r), ctx->hp.block_size, src_v), 256);
+    return MOARA_OK;
+}
+
+int moara_set_refresh_workspace(moara_ctx* ctx, void* ptr, size_t bytes) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    if (ptr == nullptr && bytes != 0) return fail(ctx, MOARA_ERR_INVALID_ARG, "NULL workspace with nonzero size");
+    if (ptr != nullptr && (reinterpret_cast<uintptr_t>(ptr) & 255u) != 0)
+        return fail(ctx, MOARA_ERR_ALIGN, "refresh workspace must be 256-byte aligned");
+    ctx->refresh_ws = ptr;
+    ctx->refresh_ws_bytes = bytes;
+    return MOARA_OK;
+}
+
+int moara_refresh_projector(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, void* stream) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    int rc = check_ids(ctx, n_mod, ids, G);
+    if (rc != MOARA_OK) return rc;
+    if (n_mod == 0) return MOARA_OK;
+    if (ctx->refresh_ws == nullptr) return fail(ctx, MOARA_ERR_WORKSPACE, "no refresh workspace set");
+    DeviceGuard g(ctx->device);
+    ProfScope ps(ctx, MOARA_PHASE_REFRESH, static_cast<cudaStream_t>(stream));
+    return do_refresh(ctx, n_mod, ids, G, static_cast<cudaStream_t>(stream));
+}
+
+int moara_step_grouped(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, int64_t t,
+                       float lr, int auto_refresh, void* stream) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    int rc = check_ids(ctx, n_mod, ids, G);
+    if (rc != MOARA_OK) return rc;
+    if (t < 1) return fail(ctx, MOARA_ERR_INVALID_ARG, "step t must be >= 1 (got %lld)", (long long)t);
+    if (!std::isfinite(lr)) return fail(ctx, MOARA_ERR_INVALID_ARG, "lr must be finite");
+    if (n_mod == 0) return MOARA_OK;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DeviceGuard g(ctx->device);
+    if (auto_refresh && ((t - 1) % ctx->hp.refresh_interval) == 0) {
+        if (ctx->refresh_ws == nullptr) return fail(ctx, MOARA_ERR_WORKSPACE, "no refresh workspace set");
+        ProfScope ps(ctx, MOARA_PHASE_REFRESH, s);
+        rc = do_refresh(ctx, n_mod, ids, G, s);
+        if (rc != MOARA_OK) return rc;
+    }
+    std::vector<int> simt, tcm;
+    for (int i = 0; i < n_mod; ++i) (use_tc(ctx, ids[i]) ? tcm : simt).push_back(i);
+    if (!tcm.empty()) {
+        const double bc1 = 1.0 - std::pow((double)ctx->hp.beta1, (double)t);
+        const double bc2 = 1.0 - std::pow((double)ctx->hp.beta2, (double)t);
+        std::vector<int> mids(tcm.size());
+        std::vector<const void*> gp(tcm.size());
+        for (size_t q = 0; q < tcm.size(); ++q) { mids[q] = ids[tcm[q]]; gp[q] = G[tcm[q]]; }
+        moara::TcProfile tp{ctx->prof, [](void* c, int ph, cudaStream_t st, bool begin) {
+            moara_ctx* cx = static_cast<moara_ctx*>(c);
+            static thread_local cudaEvent_t open = nullptr;
+            if (begin) { open = take_event(cx); cudaEventRecord(open, st); }
+            else { cudaEvent_t b = take_event(cx); cudaEventRecord(b, st); cx->recs.push_back({ph, open, b}); }
+        }, ctx};
+        rc = moara::tc_step(ctx->tc, ctx->hp, static_cast<int>(mids.size()), mids.data(), gp.data(),
+                            static_cast<float>(bc1), static_cast<float>(bc2), lr, s, &ctx->launches, tp);
+        if (rc != MOARA_OK) return fail(ctx, rc, "tensor-core step launch failed: %s", moara::tc_last_error(ctx->tc));
+    }
+    if (!simt.empty()) {
+        rc = do_step_simt(ctx, simt, ids, G, t, lr, s);
+        if (rc != MOARA_OK) return rc;
+    }
+    return MOARA_OK;
+}
+
+int moara_get_device_status(moara_ctx* ctx, int* status, void* stream) {
+    if (ctx == nullptr || status == nullptr) return MOARA_ERR_INVALID_ARG;
+    DeviceGuard g(ctx->device);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(ctx->h_status, ctx->d_status, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(ctx->d_status, 0, sizeof(int), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "status read");
+    *status = ctx->h_status[0];
+    return MOARA_OK;
+}
+
+const char* moara_last_error(const moara_ctx* ctx) {
+    if (ctx == nullptr) return "context is NULL";
+    return ctx->last_error.c_str();
+}
+
+const char* moara_status_string(int code) {
+    switch (code) {
+        case MOARA_OK: return "ok";
+        case MOARA_ERR_INVALID_ARG: return "invalid argument";
+        case MOARA_ERR_SHAPE: return "invalid shape";
+        case MOARA_ERR_RANK: return "invalid rank";
+        case MOARA_ERR_ALIGN: return "misaligned pointer";
+        case MOARA_ERR_UNKNOWN_MODULE: return "unknown module";
+        case MOARA_ERR_CUDA: return "CUDA error";
+        case MOARA_ERR_DEVICE_TIMEOUT: return "device-side wait timed out";
+        case MOARA_ERR_WORKSPACE: return "workspace missing or too small";
+        case MOARA_ERR_UNSUPPORTED: return "unsupported";
+        default: return "unknown status";
+    }
+}
+
+int64_t moara_launch_count(const moara_ctx* ctx) { return ctx ? ctx->launches : -1; }
+
+int moara_profile_enable(moara_ctx* ctx, int enable) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    ctx->prof = enable != 0;
+    return MOARA_OK;
+}
+
+int moara_profile_read(moara_ctx* ctx, double ms[8], int64_t launches[8]) {
+    if (ctx == nullptr || ms == nullptr || launches == nullptr) return MOARA_ERR_INVALID_ARG;
+    DeviceGuard g(ctx->device);
+    for (auto& r : ctx->recs) {
+        cudaError_t e = cudaEventSynchronize(r.b);
+        float t = 0.0f;
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&t, r.a, r.b);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "profile event");
+        ctx->prof_ms[r.phase] += t;
+        ctx->prof_n[r.phase] += 1;
+        ctx->free_events.push_back(r.a);
+        ctx->free_events.push_back(r.b);
+    }
+    ctx->recs.clear();
+    for (int i = 0; i < MOARA_NUM_PHASES; ++i) {
+        ms[i] = ctx->prof_ms[i];
+        launches[i] = ctx->prof_n[i];
+        ctx->prof_ms[i] = 0.0;
+        ctx->prof_n[i] = 0;
+    }
+    return MOARA_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,155 @@
+// Internal declarations shared by the host API and the kernel translation
+// units of libmoara.  Plain C++ structs passed to kernels by value (grouped
+// launches) or stored in the context's device table.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+#include "../../include/moara.h"
+
+namespace moara {
+
+// Largest number of problems a grouped launch carries in its parameter block
+// (kernel parameters up to 32 KB are allowed on sm_70+ with CUDA >= 12.1).
+constexpr int kMaxGroup = 96;
+
+// Device-side image of one registered module.
+struct ModDev {
+    int m, n, r, kb;        // kb = ceil(n / B)
+    int dtype;              // MOARA_DTYPE_*
+    int pad_;
+    float* W;
+    float* P;
+    uint16_t* Pb;
+    float* exp_avg;
+    float* exp_avg_sq;
+    float* mag_avg;
+    float* mag_avg_sq;
+    float* ws_N;            // r x n update of the direction branch (fp32 or bf16)
+    float* ws_dM;           // m x kb update of the magnitude branch
+    float* ws_inv;          // m x kb inverse block scales 1 / (||g|| + eps)
+};
+
+// Workspace carve-up of one module (byte offsets, 256-byte aligned).
+struct WsLayout {
+    size_t off_N, off_dM, off_inv, total;
+};
+WsLayout workspace_layout(int m, int n, int r, int B);
+
+// ---------------------------------------------------------------- decompose
+struct DecompItem {
+    const void* G;
+    float* inv;       // m x kb, written
+    float* mag_avg;   // m x kb, updated when do_mag
+    float* mag_avg_sq;
+    float* dM;        // m x kb, written when do_mag
+    int m, n, kb, dtype;
+};
+
+struct DecompBatch {
+    int count;
+    int B;
+    int do_mag;
+    float decomp_eps, beta1, beta2, adam_eps, bc1, bc2;
+    long long item_start[kMaxGroup + 1];
+    DecompItem p[kMaxGroup];
+};
+
+// ------------------------------------------------------------- SIMT GEMM
+// C (M x N) = op(A) (M x K) * op(B) (K x N), fp32 accumulate.
+enum Epi { EPI_STORE = 0, EPI_ADAM = 1, EPI_UPDATE = 2 };
+
+struct GemmProb {
+    const void* A;
+    const void* Bm;
+    float* C;
+    const float* a_inv;   // block scales applied to A (V operand) or null
+    const float* b_inv;   // block scales applied to B or null
+    float* aux0;          // EPI_ADAM: exp_avg    EPI_UPDATE: W
+    float* aux1;          // EPI_ADAM: exp_avg_sq
+    const float* aux2;    // EPI_UPDATE: dM (m x kb) or null (no magnitude)
+    int M, N, K;
+    int lda, ldb, ldc;
+    int kb;               // blocks per row of the scaled operand / of dM
+    int a_bf16, b_bf16;
+};
+
+struct GemmBatch {
+    int count;
+    int B;                        // block size (scales, dM repetition)
+    float beta1, beta2, adam_eps, bc1, bc2;
+    float step_scale;             // lr * alpha (EPI_UPDATE)
+    int tiles_n[kMaxGroup];
+    int tile_start[kMaxGroup + 1];
+    GemmProb p[kMaxGroup];
+};
+
+// Operand layouts of the SIMT GEMM.
+//   A: KCONTIG  A[i][k] = A[i*lda + k];  MCONTIG  A[i][k] = A[k*lda + i]
+//   B: NCONTIG  B[k][j] = B[k*ldb + j];  KCONTIG  B[k][j] = B[j*ldb + k]
+enum ALayout { A_KCONTIG = 0, A_MCONTIG = 1 };
+enum BLayout { B_NCONTIG = 0, B_KCONTIG = 1 };
+
+struct GemmKind {
+    int a_layout, b_layout, a_scale, b_scale, a_bf16, b_bf16, epi;
+};
+
+// Host launchers (return cudaError_t of the launch).
+cudaError_t launch_decompose(const DecompBatch& b, cudaStream_t s, int64_t* launches);
+cudaError_t launch_gemm(const GemmKind& kind, GemmBatch& b, cudaStream_t s, int64_t* launches);
+int gemm_tile_m();
+int gemm_tile_n();
+
+cudaError_t launch_f32_to_bf16(const float* src, float* dst_f32, uint16_t* dst_bf16,
+                               long long count, cudaStream_t s, int64_t* launches);
+
+// ------------------------------------------------------------- refresh
+struct RefreshItem {
+    int m, n, r, l, kb, dtype;
+    const void* G;
+    float* inv;       // block scales (src V) or null (src G)
+    float* Omega;     // n x l
+    float* Qa; float* Qb;   // m x l
+    float* Za; float* Zb;   // n x l
+    float* Cg;        // l x l Gram / Cholesky factor
+    float* Linv;      // l x l
+    float* Cr;        // l x l Rayleigh-Ritz matrix
+    float* Xa; float* Xb;   // l x l
+    float* ritz;      // l
+    int* perm;        // l
+    int* fail;        // 1 int
+    float* P;         // m x r destination
+    uint16_t* Pb;     // m x r bf16 destination (may be null)
+    uint64_t key;     // RNG key (seed, module, refresh count)
+};
+
+size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v);
+void refresh_carve(RefreshItem& it, void* base, int m, int n, int r, int l, int B, int src_v);
+
+// Small dense kernels (one CTA per problem).
+struct SmallBatch {
+    int count;
+    int l[kMaxGroup];
+    int rows[kMaxGroup];
+    float* a[kMaxGroup];
+    float* b[kMaxGroup];
+    float* c[kMaxGroup];
+    int* fail[kMaxGroup];
+    int* iaux[kMaxGroup];
+    uint16_t* h[kMaxGroup];
+    float shift_rel;
+    uint64_t key[kMaxGroup];
+};
+
+cudaError_t launch_philox_gaussian(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+cudaError_t launch_cholesky(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+cudaError_t launch_tri_inverse(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+cudaError_t launch_set_identity(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+cudaError_t launch_ritz_sort(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+cudaError_t launch_sign_fix_store(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+
+}  // namespace moara

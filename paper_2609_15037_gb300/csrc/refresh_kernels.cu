@@ -1,0 +1,325 @@
+// Small dense kernels of the projector refresh (TruncatedSVD of Algorithm 1
+// computed by randomized subspace iteration): the Gaussian test matrix, the
+// Cholesky factorisation and triangular inverse of CholeskyQR, the ordering of
+// Ritz vectors, and the final sign convention.  One CTA per problem; the
+// problems of a group run side by side in one launch.
+#include <cuda_bf16.h>
+
+#include "internal.h"
+
+namespace moara {
+
+// ---------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as easy
+// as 1, 2, 3", SC'11): 10 rounds of the 4x32 S-box with the published
+// multipliers and Weyl key increments.  Box-Muller turns pairs of uniforms
+// into standard normals.
+// ---------------------------------------------------------------------------
+struct U4 { uint32_t x, y, z, w; };
+
+__device__ __forceinline__ U4 philox4x32_10(U4 c, uint32_t k0, uint32_t k1) {
+    const uint32_t M0 = 0xD2511F53u, M1 = 0xCD9E8D57u;
+    const uint32_t W0 = 0x9E3779B9u, W1 = 0xBB67AE85u;
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        const uint32_t hi0 = __umulhi(M0, c.x), lo0 = M0 * c.x;
+        const uint32_t hi1 = __umulhi(M1, c.z), lo1 = M1 * c.z;
+        U4 n;
+        n.x = hi1 ^ c.y ^ k0;
+        n.y = lo1;
+        n.z = hi0 ^ c.w ^ k1;
+        n.w = lo0;
+        c = n;
+        k0 += W0;
+        k1 += W1;
+    }
+    return c;
+}
+
+// uniform in (0, 1]: (x + 1) * 2^-32 with x the top 24 bits scaled
+__device__ __forceinline__ float u01(uint32_t x) {
+    return (static_cast<float>(x >> 8) + 1.0f) * (1.0f / 16777216.0f);
+}
+
+__global__ void k_philox_gaussian(const __grid_constant__ SmallBatch b) {
+    const int pi = blockIdx.y;
+    float* out = b.a[pi];
+    const long long count = (long long)b.rows[pi] * b.l[pi];
+    const uint32_t k0 = static_cast<uint32_t>(b.key[pi]);
+    const uint32_t k1 = static_cast<uint32_t>(b.key[pi] >> 32);
+    const long long groups = (count + 3) / 4;
+    for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < groups;
+         g += (long long)gridDim.x * blockDim.x) {
+        U4 c{static_cast<uint32_t>(g), static_cast<uint32_t>(g >> 32), 0x4D6F4152u, 0x52616E64u};
+        const U4 r = philox4x32_10(c, k0, k1);
+        const float u1 = u01(r.x), u2 = u01(r.y), u3 = u01(r.z), u4 = u01(r.w);
+        const float ra = sqrtf(-2.0f * logf(u1)), rb = sqrtf(-2.0f * logf(u3));
+        float s2, c2, s4, c4;
+        sincospif(2.0f * u2, &s2, &c2);
+        sincospif(2.0f * u4, &s4, &c4);
+        const float z[4] = {ra * c2, ra * s2, rb * c4, rb * s4};
+        const long long base = g * 4;
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            if (base + q < count) out[base + q] = z[q];
+    }
+}
+
+cudaError_t launch_philox_gaussian(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    dim3 grid(64, b.count);
+    k_philox_gaussian<<<grid, 256, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// In-place lower Cholesky of a symmetric l x l matrix a (row-major, lower
+// triangle read), with a diagonal shift shift_rel * sqrt(rows) * trace(a)
+// (shifted CholeskyQR: Fukaya, Kannan, Nakatsukasa, Yamamoto, Yanagisawa,
+// SIAM J. Sci. Comput. 2020).  A non-positive or non-finite pivot marks the
+// problem as failed (fail = 1) and is replaced by 1 so the sweep finishes
+// without NaNs.  The strict upper triangle is zeroed.
+// ---------------------------------------------------------------------------
+constexpr int kSmallThreads = 1024;
+
+__device__ float block_sum(float v, float* red) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) red[w] = v;
+    __syncthreads();
+    float t = 0.0f;
+    if (w == 0) {
+        t = (lane < static_cast<int>(blockDim.x >> 5)) ? red[lane] : 0.0f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0) red[32] = t;
+    }
+    __syncthreads();
+    return red[32];
+}
+
+__global__ void __launch_bounds__(kSmallThreads) k_cholesky(const __grid_constant__ SmallBatch b) {
+    extern __shared__ float rowj[];          // l floats: row j of L
+    __shared__ float red[33];
+    __shared__ float s_djj;
+    const int pi = blockIdx.x;
+    const int l = b.l[pi];
+    float* A = b.a[pi];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+
+    float tr = 0.0f;
+    for (int i = threadIdx.x; i < l; i += blockDim.x) tr += A[(long long)i * l + i];
+    tr = block_sum(tr, red);
+    const float shift = b.shift_rel * sqrtf(static_cast<float>(b.rows[pi])) * tr;
+    int failed = 0;
+
+    for (int j = 0; j < l; ++j) {
+        // row j of L (k < j) into shared memory, partial sum of squares
+        float ss = 0.0f;
+        for (int k = threadIdx.x; k < j; k += blockDim.x) {
+            const float v = A[(long long)j * l + k];
+            rowj[k] = v;
+            ss = fmaf(v, v, ss);
+        }
+        ss = block_sum(ss, red);
+        if (threadIdx.x == 0) {
+            float d = A[(long long)j * l + j] + shift - ss;
+            if (!(d > 0.0f) || !isfinite(d)) { d = 1.0f; failed = 1; }
+            d = sqrtf(d);
+            A[(long long)j * l + j] = d;
+            s_djj = d;
+        }
+        __syncthreads();
+        const float djj = s_djj;
+        for (int i = j + 1 + warp; i < l; i += nw) {
+            const float* Li = A + (long long)i * l;
+            float dot = 0.0f;
+            for (int k = lane; k < j; k += 32) dot = fmaf(Li[k], rowj[k], dot);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+            if (lane == 0) A[(long long)i * l + j] = (Li[j] - dot) / djj;
+        }
+        __syncthreads();
+    }
+    for (int i = 0; i < l; ++i)
+        for (int k = i + 1 + threadIdx.x; k < l; k += blockDim.x) A[(long long)i * l + k] = 0.0f;
+    if (threadIdx.x == 0 && failed && b.fail[pi] != nullptr) *b.fail[pi] = 1;
+}
+
+cudaError_t launch_cholesky(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    int lmax = 1;
+    for (int i = 0; i < b.count; ++i) lmax = b.l[i] > lmax ? b.l[i] : lmax;
+    const size_t smem = sizeof(float) * lmax;
+    if (smem > 48 * 1024) {
+        cudaFuncSetAttribute(k_cholesky, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    }
+    k_cholesky<<<b.count, kSmallThreads, smem, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Inverse of a lower-triangular l x l matrix (a -> c), row by row:
+// Linv[i][c] = (delta_ic - sum_{c <= k < i} L[i][k] Linv[k][c]) / L[i][i].
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kSmallThreads) k_tri_inverse(const __grid_constant__ SmallBatch b) {
+    extern __shared__ float rowi[];
+    const int pi = blockIdx.x;
+    const int l = b.l[pi];
+    const float* L = b.a[pi];
+    float* X = b.c[pi];
+    for (int i = 0; i < l; ++i) {
+        for (int k = threadIdx.x; k <= i; k += blockDim.x) rowi[k] = L[(long long)i * l + k];
+        __syncthreads();
+        const float dinv = 1.0f / rowi[i];
+        for (int c = threadIdx.x; c < l; c += blockDim.x) {
+            float v = 0.0f;
+            if (c <= i) {
+                float acc = (c == i) ? 1.0f : 0.0f;
+                for (int k = c; k < i; ++k) acc = fmaf(-rowi[k], X[(long long)k * l + c], acc);
+                v = acc * dinv;
+            }
+            X[(long long)i * l + c] = v;
+        }
+        __syncthreads();
+    }
+}
+
+cudaError_t launch_tri_inverse(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    int lmax = 1;
+    for (int i = 0; i < b.count; ++i) lmax = b.l[i] > lmax ? b.l[i] : lmax;
+    const size_t smem = sizeof(float) * lmax;
+    if (smem > 48 * 1024) {
+        cudaFuncSetAttribute(k_tri_inverse, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    }
+    k_tri_inverse<<<b.count, kSmallThreads, smem, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// a <- I (l x l)
+// ---------------------------------------------------------------------------
+__global__ void k_set_identity(const __grid_constant__ SmallBatch b) {
+    const int pi = blockIdx.y;
+    const int l = b.l[pi];
+    float* X = b.a[pi];
+    const long long n = (long long)l * l;
+    for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < n;
+         e += (long long)gridDim.x * blockDim.x) {
+        const long long i = e / l, c = e - i * l;
+        X[e] = (i == c) ? 1.0f : 0.0f;
+    }
+}
+
+cudaError_t launch_set_identity(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    k_set_identity<<<dim3(32, b.count), 256, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Ritz values d_j = x_j^T (C x_j) from X (a) and W = C X (b), then the
+// descending order: iaux[rank] = j, rank_j = #{i : d_i > d_j, or d_i == d_j
+// and i < j}.  Ritz values go to c.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kSmallThreads) k_ritz_sort(const __grid_constant__ SmallBatch b) {
+    const int pi = blockIdx.x;
+    const int l = b.l[pi];
+    const float* X = b.a[pi];
+    const float* W = b.b[pi];
+    float* d = b.c[pi];
+    int* perm = b.iaux[pi];
+    for (int j = threadIdx.x; j < l; j += blockDim.x) {
+        float acc = 0.0f;
+        for (int i = 0; i < l; ++i) acc = fmaf(X[(long long)i * l + j], W[(long long)i * l + j], acc);
+        d[j] = acc;
+    }
+    __syncthreads();
+    __threadfence_block();
+    for (int j = threadIdx.x; j < l; j += blockDim.x) {
+        const float dj = d[j];
+        int rank = 0;
+        for (int i = 0; i < l; ++i) {
+            const float di = d[i];
+            rank += (di > dj || (di == dj && i < j)) ? 1 : 0;
+        }
+        perm[rank] = j;
+    }
+}
+
+cudaError_t launch_ritz_sort(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    k_ritz_sort<<<b.count, kSmallThreads, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// c[:, q] = a[:, iaux[q]] for q < rows (a is l x l, c is l x rows).
+// ---------------------------------------------------------------------------
+__global__ void k_gather_cols(const __grid_constant__ SmallBatch b) {
+    const int pi = blockIdx.y;
+    const int l = b.l[pi], r = b.rows[pi];
+    const float* X = b.a[pi];
+    float* Xs = b.c[pi];
+    const int* perm = b.iaux[pi];
+    const long long n = (long long)l * r;
+    for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < n;
+         e += (long long)gridDim.x * blockDim.x) {
+        const long long i = e / r, q = e - i * r;
+        Xs[e] = X[i * l + perm[q]];
+    }
+}
+
+cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    k_gather_cols<<<dim3(64, b.count), 256, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Final projector: each column of a (rows x l, here l = r columns) is signed
+// so that its largest-magnitude entry is positive (lowest row wins ties), then
+// stored to c (fp32) and h (bf16).  Skipped when the problem's fail flag is
+// set, which leaves the previous projector in place.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kSmallThreads) k_sign_fix_store(const __grid_constant__ SmallBatch b) {
+    const int pi = blockIdx.y;
+    const int rows = b.rows[pi], r = b.l[pi];
+    if (b.fail[pi] != nullptr && *b.fail[pi] != 0) return;
+    const float* Pt = b.a[pi];
+    float* P = b.c[pi];
+    uint16_t* Pb = b.h[pi];
+    for (int q = blockIdx.x * blockDim.x + threadIdx.x; q < r; q += gridDim.x * blockDim.x) {
+        float best = -1.0f, sgnv = 1.0f;
+        for (int i = 0; i < rows; ++i) {
+            const float v = Pt[(long long)i * r + q];
+            if (fabsf(v) > best) { best = fabsf(v); sgnv = v < 0.0f ? -1.0f : 1.0f; }
+        }
+        for (int i = 0; i < rows; ++i) {
+            const float v = Pt[(long long)i * r + q] * sgnv;
+            P[(long long)i * r + q] = v;
+            if (Pb != nullptr) {
+                __nv_bfloat16 h = __float2bfloat16_rn(v);
+                Pb[(long long)i * r + q] = *reinterpret_cast<uint16_t*>(&h);
+            }
+        }
+    }
+}
+
+cudaError_t launch_sign_fix_store(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    k_sign_fix_store<<<dim3(4, b.count), 256, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+}  // namespace moara

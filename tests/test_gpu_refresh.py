@@ -1,0 +1,159 @@
+"""GPU projector refresh (TruncatedSVD of Algorithm 1 by randomized subspace
+iteration) against the oracle's exact fp64 SVD.
+
+Checks: P^T P = I within 1e-5; principal angles <= 1e-2 rad on the leading
+directions up to the spectral gap k_gap (largest k <= r with
+sigma_k / sigma_{k+1} >= 1.5); captured energy ||P^T X||_F^2 >= (1 - 1e-3)
+sum_{i<=r} sigma_i^2; and, on an input with a clear gap at r, all r angles.
+"""
+
+import numpy as np
+import pytest
+
+from oracle import moara_ref as o
+import synth
+
+from gpu_helpers import principal_angles, gap_index, make_inputs
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def M():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2609_15037_gb300 as pkg
+    return pkg
+
+
+def _dev(G, bf16=True):
+    t = torch.tensor(G, dtype=torch.float32)
+    return (t.to(torch.bfloat16) if bf16 else t).cuda()
+
+
+def _check_projector(P, X, r, tol_angle=1e-2):
+    U, S, _ = np.linalg.svd(X, full_matrices=False)
+    np.testing.assert_allclose(P.T @ P, np.eye(r), atol=1e-5)
+    k = gap_index(S, r)
+    if k > 0:
+        ang = principal_angles(P[:, :k], U[:, :k])
+        assert ang.max() <= tol_angle, (k, ang.max())
+    energy = np.sum((P.T @ X) ** 2)
+    assert energy >= (1 - 1e-3) * np.sum(S[:r] ** 2)
+    return k
+
+
+@pytest.mark.parametrize("src", ["V", "G"])
+def test_refresh_llama300m_attention_and_mlp(M, src):
+    shapes = [(1024, 1024, 128), (2816, 1024, 256), (1024, 2816, 256)]
+    B = 64
+    grads, W0 = make_inputs(shapes, B, 1, True, signal_rank=32)
+    g = M.MoaraGroup(block_size=B, refresh_src=(M.MOARA_REFRESH_SRC_V if src == "V"
+                                                 else M.MOARA_REFRESH_SRC_G))
+    for (m, n, r) in shapes:
+        g.add(m, n, r, "bf16")
+    g.refresh([_dev(grads[i][0]) for i in range(len(shapes))])
+    torch.cuda.synchronize()
+    assert g.status() == 0
+    for i, (m, n, r) in enumerate(shapes):
+        P = g.modules[i].P.double().cpu().numpy()
+        X = o.decompose(grads[i][0], B)[1] if src == "V" else grads[i][0]
+        _check_projector(P, X, r)
+        Pb = g.modules[i].P_bf16.view(torch.bfloat16).float().cpu().numpy()
+        np.testing.assert_allclose(Pb, P, rtol=2 ** -8, atol=1e-30)
+    g.close()
+
+
+def test_refresh_clear_gap_all_directions(M):
+    """Signal of rank r + 8 with a factor-3 drop after r: all r directions."""
+    m, n, r = 384, 512, 24
+    u, v = synth.lowrank_factors(m, n, r + 8, seed=5)
+    sig = np.concatenate([10.0 * 0.9 ** np.arange(r), 0.5 * 0.9 ** np.arange(8)])
+    G = (u * sig) @ v.T + 1e-4 * np.random.default_rng(1).standard_normal((m, n))
+    G = G.astype(np.float32).astype(np.float64)
+    g = M.MoaraGroup(block_size=64, refresh_src=M.MOARA_REFRESH_SRC_G)
+    g.add(m, n, r, "f32")
+    g.refresh([_dev(G, bf16=False)])
+    torch.cuda.synchronize()
+    P = g.modules[0].P.double().cpu().numpy()
+    U = np.linalg.svd(G, full_matrices=False)[0][:, :r]
+    assert principal_angles(P, U).max() <= 1e-2
+    Po = o.truncated_svd(G, r)[0]
+    # columns come in descending order with the oracle's sign convention
+    assert np.min(np.sum(P * Po, axis=0)) >= 0.999
+    g.close()
+
+
+def test_auto_refresh_step_equals_refresh_then_step(M):
+    """Refresh and step on the same step (t = 1, (t-1) mod T = 0) equals the
+    two calls made one after the other."""
+    shapes = [(512, 256, 64), (256, 512, 32)]
+    grads, W0 = make_inputs(shapes, 64, 2, True)
+    outs = []
+    for mode in ("auto", "manual"):
+        g = M.MoaraGroup(block_size=64)
+        for i, (m, n, r) in enumerate(shapes):
+            g.add(m, n, r, "bf16", W0=W0[i])
+        Gs = [_dev(grads[i][0]) for i in range(len(shapes))]
+        if mode == "auto":
+            g.step(Gs, 1, 1e-3, auto_refresh=True)
+        else:
+            g.refresh(Gs)
+            g.step(Gs, 1, 1e-3, auto_refresh=False)
+        torch.cuda.synchronize()
+        outs.append([(b.W.clone(), b.P.clone()) for b in g.modules])
+        g.close()
+    for (wa, pa), (wb, pb) in zip(*outs):
+        assert torch.equal(pa, pb) and torch.equal(wa, wb)
+
+
+def test_refresh_interval(M):
+    """auto_refresh runs the refresh exactly when (t - 1) mod T == 0."""
+    B = M.binding
+    g = M.MoaraGroup(block_size=32, refresh_interval=3)
+    g.add(128, 96, 8, "bf16")
+    G = _dev(make_inputs([(128, 96, 8)], 32, 1, True)[0][0][0])
+    counts = []
+    for t in range(1, 8):
+        before = B.moara_launch_count(g.ctx)
+        g.step([G], t, 1e-3, auto_refresh=True)
+        counts.append(B.moara_launch_count(g.ctx) - before)
+    torch.cuda.synchronize()
+    plain = min(counts)
+    assert [c > plain for c in counts] == [True, False, False, True, False, False, True]
+    g.close()
+
+
+def test_refresh_qwen2_7b_gqa_modules_with_step(M):
+    """Qwen2-7B shapes with heterogeneous ranks (k/v 512 x 3584 at r = 256,
+    q 3584 x 3584 at r = 896): refresh and step on the same step."""
+    shapes = [(3584, 3584, 896), (512, 3584, 256), (512, 3584, 256)]
+    B = 128
+    grads, W0 = make_inputs(shapes, B, 1, True, signal_rank=32)
+    g = M.MoaraGroup(block_size=B)
+    for i, (m, n, r) in enumerate(shapes):
+        g.add(m, n, r, "bf16", W0=W0[i])
+    g.step([_dev(grads[i][0]) for i in range(len(shapes))], 1, 1e-3, auto_refresh=True)
+    torch.cuda.synchronize()
+    assert g.status() == 0
+    for i, (m, n, r) in enumerate(shapes):
+        P = g.modules[i].P.double().cpu().numpy()
+        X = o.decompose(grads[i][0], B)[1]
+        _check_projector(P, X, r)
+        assert np.all(np.isfinite(g.modules[i].W.cpu().numpy()))
+    g.close()
+
+
+def test_refresh_workspace_too_small(M):
+    B = M.binding
+    g = M.MoaraGroup(block_size=32)
+    mid = g.add(128, 128, 16, "bf16")
+    tiny = torch.empty(1024, dtype=torch.uint8, device="cuda")
+    B.moara_set_refresh_workspace(g.ctx, tiny.data_ptr(), 1024)
+    G = torch.zeros(128, 128, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(B.MoaraError) as e:
+        B.moara_refresh_projector(g.ctx, [mid], [G.data_ptr()])
+    assert e.value.code == B.MOARA_ERR_WORKSPACE
+    g.close()
