@@ -153,7 +153,7 @@ def run_gpu(args):
     hp = M.moara_default_hparams()
     hp.block_size = B
     hp.adam_eps = wl["adam_eps"]
-    g = M.MoaraGroup(hp, device=local)
+    g = M.MoaraGroup(hp, device=local, refresh_workspace_bytes=int(args.refresh_ws_gb * (1 << 30)))
     stream = torch.cuda.current_stream(dev)
     grads = []
     for i, md in enumerate(mods):
@@ -410,6 +410,7 @@ def main():
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--refresh-ws-gb", type=float, default=12.0)
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

@@ -10,6 +10,7 @@ from __future__ import annotations
 import concurrent.futures as cf
 import glob
 import os
+import platform
 import shutil
 import subprocess
 import sys
@@ -17,7 +18,7 @@ import sys
 PKG = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
-OUT_DIR = os.path.join(PKG, "_build")
+OUT_DIR = os.path.join(PKG, "_build", platform.machine())
 LIB = os.path.join(PKG, "libmoara.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -70,13 +71,18 @@ def build(verbose_ptxas=False, jobs=None):
             if log:
                 sys.stderr.write(log)
     newest = max(os.path.getmtime(o) for o in objs)
-    if not os.path.exists(LIB) or os.path.getmtime(LIB) < newest:
+    stamp = os.path.join(OUT_DIR, "lib.stamp")
+    fresh = (os.path.exists(LIB) and os.path.exists(stamp) and
+             os.path.getmtime(LIB) >= newest and open(stamp).read() == LIB)
+    if not fresh:
         tmp = LIB + ".tmp"
-        cmd = [_nvcc()] + ARCH + ["-shared", "-o", tmp] + objs + ["-lcudart", "-lcuda"]
+        cmd = [_nvcc()] + ARCH + ["-shared", "-o", tmp] + objs + ["-lcudart"]
         p = subprocess.run(cmd, capture_output=True, text=True)
         if p.returncode != 0:
             raise RuntimeError(f"link failed:\n{p.stdout}\n{p.stderr}")
         os.replace(tmp, LIB)
+        with open(stamp, "w") as f:
+            f.write(LIB)
     return LIB
 
 

@@ -167,7 +167,7 @@ size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v) {
     add(sizeof(float) * (size_t)n * l);  // Zb
     add(sizeof(float) * (size_t)m * l);  // Qa
     add(sizeof(float) * (size_t)m * l);  // Qb
-    for (int i = 0; i < 5; ++i) add(sizeof(float) * (size_t)l * l);
+    for (int i = 0; i < 6; ++i) add(sizeof(float) * (size_t)l * l);
     add(sizeof(float) * (size_t)l);
     add(sizeof(int) * (size_t)l);
     add(sizeof(int) * 4);
@@ -188,6 +188,7 @@ void refresh_carve(RefreshItem& it, void* base, int m, int n, int r, int l, int 
     it.Qb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * l));
     it.Cg = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Linv = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
+    it.Tt = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Cr = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Xa = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Xb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
@@ -250,7 +251,7 @@ struct RefreshRunner {
             sb.fail[i] = it[i].fail;
         }
         chk(moara::launch_cholesky(sb, s, &ctx->launches));
-        chk(moara::launch_tri_inverse(sb, s, &ctx->launches));
+        tri_inverse();
         moara::GemmKind apply{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
         gemm(apply, [&](int i, moara::GemmProb& p) {
             const int l = it[i].l;
@@ -259,12 +260,65 @@ struct RefreshRunner {
         });
     }
 
-    // Shifted CholeskyQR followed by CholeskyQR2; result lands in `b`.
-    void cholqr3(std::vector<float*>& a, std::vector<float*>& b, const std::vector<int>& rows) {
+    // Linv <- Cg^-1 for the lower-triangular Cholesky factor in Cg: diagonal
+    // 64 x 64 blocks in shared memory, then the off-diagonal blocks level by
+    // level (block size s = 64, 128, ...) with two grouped GEMMs per level:
+    //   T = L[D, A] Linv[A, A];  Linv[D, A] = -Linv[D, D] T.
+    void tri_inverse() {
+        int lmax = 0;
+        for (auto& x : it) {
+            chk(cudaMemsetAsync(x.Linv, 0, sizeof(float) * (size_t)x.l * x.l, s));
+            lmax = std::max(lmax, x.l);
+        }
+        moara::SmallBatch sb = small();
+        for (size_t i = 0; i < it.size(); ++i) { sb.l[i] = it[i].l; sb.a[i] = it[i].Cg; sb.c[i] = it[i].Linv; }
+        chk(moara::launch_tri_inverse_diag(sb, s, &ctx->launches));
+        moara::GemmKind mul{moara::A_KCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
+        moara::GemmKind neg{moara::A_KCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE_NEG};
+        for (int sz = moara::kTriBase; sz < lmax; sz *= 2) {
+            struct Pair { int mod, a0, d0, dn; };
+            std::vector<Pair> pairs;
+            for (int i = 0; i < static_cast<int>(it.size()); ++i) {
+                const int l = it[i].l;
+                for (int a0 = 0; a0 + sz < l; a0 += 2 * sz)
+                    pairs.push_back({i, a0, a0 + sz, std::min(sz, l - a0 - sz)});
+            }
+            for (int pass = 0; pass < 2; ++pass) {
+                for (size_t c0 = 0; c0 < pairs.size(); c0 += moara::kMaxGroup) {
+                    moara::GemmBatch b{};
+                    b.count = static_cast<int>(std::min<size_t>(moara::kMaxGroup, pairs.size() - c0));
+                    b.B = 1;
+                    for (int q = 0; q < b.count; ++q) {
+                        const Pair& pr = pairs[c0 + q];
+                        const auto& x = it[pr.mod];
+                        const long long l = x.l;
+                        moara::GemmProb& p = b.p[q];
+                        p = moara::GemmProb{};
+                        p.lda = p.ldb = p.ldc = x.l;
+                        if (pass == 0) {          // T[D, A] = L[D, A] Linv[A, A]
+                            p.A = x.Cg + pr.d0 * l + pr.a0;
+                            p.Bm = x.Linv + pr.a0 * l + pr.a0;
+                            p.C = x.Tt + pr.d0 * l + pr.a0;
+                            p.M = pr.dn; p.N = sz; p.K = sz;
+                        } else {                  // Linv[D, A] = -Linv[D, D] T[D, A]
+                            p.A = x.Linv + pr.d0 * l + pr.d0;
+                            p.Bm = x.Tt + pr.d0 * l + pr.a0;
+                            p.C = x.Linv + pr.d0 * l + pr.a0;
+                            p.M = pr.dn; p.N = sz; p.K = pr.dn;
+                        }
+                    }
+                    chk(moara::launch_gemm(pass == 0 ? mul : neg, b, s, &ctx->launches));
+                }
+            }
+        }
+    }
+
+    // CholeskyQR2 with a shifted first pass; result lands in `b`.
+    void cholqr2s(std::vector<float*>& a, std::vector<float*>& b, const std::vector<int>& rows) {
         const float u = 5.9604645e-08f;   // fp32 unit roundoff
         cholqr_pass(a, b, rows, 2.0f * u);
         cholqr_pass(b, a, rows, 0.0f);
-        cholqr_pass(a, b, rows, 0.0f);
+        std::swap(a, b);
     }
 
     void run() {
@@ -345,12 +399,12 @@ struct RefreshRunner {
         };
         (void)bf;
         v_times(Za, Qa);
-        cholqr3(Qa, Qb, rows_m);          // Q in Qb
+        cholqr2s(Qa, Qb, rows_m);          // Q in Qb
         for (int q = 0; q < hp.power_iters; ++q) {
             vt_times(Qb, Za);
-            cholqr3(Za, Zb, rows_n);      // Z in Zb
+            cholqr2s(Za, Zb, rows_n);      // Z in Zb
             v_times(Zb, Qa);
-            cholqr3(Qa, Qb, rows_m);      // Q in Qb
+            cholqr2s(Qa, Qb, rows_m);      // Q in Qb
         }
         // Rayleigh-Ritz on span(Q): C = (V^T Q)^T (V^T Q), eigenvectors of C by
         // orthogonal iteration with CholeskyQR, ordered by Ritz value.
@@ -375,7 +429,7 @@ struct RefreshRunner {
                 p.A = it[i].Cr; p.Bm = Xa[i]; p.C = Xb[i];
                 p.M = l; p.N = l; p.K = l; p.lda = l; p.ldb = l; p.ldc = l;
             });
-            cholqr3(Xb, Xa, rows_l);      // X in Xa
+            cholqr2s(Xb, Xa, rows_l);      // X in Xa
         }
         // Ritz values and order: W = C X into Xb
         gemm(prod, [&](int i, moara::GemmProb& p) {
@@ -573,7 +627,7 @@ int moara_default_hparams(moara_hparams* out) {
     out->refresh_interval = 200;
     out->decompose = 1;
     out->refresh_src = MOARA_REFRESH_SRC_V;
-    out->oversample = 0;
+    out->oversample = 16;
     out->power_iters = 2;
     out->ritz_iters = 16;
     out->precision = MOARA_PREC_AUTO;

@@ -60,7 +60,7 @@ struct DecompBatch {
 
 // ------------------------------------------------------------- SIMT GEMM
 // C (M x N) = op(A) (M x K) * op(B) (K x N), fp32 accumulate.
-enum Epi { EPI_STORE = 0, EPI_ADAM = 1, EPI_UPDATE = 2 };
+enum Epi { EPI_STORE = 0, EPI_ADAM = 1, EPI_UPDATE = 2, EPI_STORE_NEG = 3 };
 
 struct GemmProb {
     const void* A;
@@ -115,6 +115,7 @@ struct RefreshItem {
     float* Qa; float* Qb;   // m x l
     float* Za; float* Zb;   // n x l
     float* Cg;        // l x l Gram / Cholesky factor
+    float* Tt;        // l x l temporary of the blocked triangular inverse
     float* Linv;      // l x l
     float* Cr;        // l x l Rayleigh-Ritz matrix
     float* Xa; float* Xb;   // l x l
@@ -147,6 +148,9 @@ struct SmallBatch {
 cudaError_t launch_philox_gaussian(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_cholesky(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_tri_inverse(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+// Inverts the diagonal blocks [64j, 64j+64) of each lower-triangular a into c.
+constexpr int kTriBase = 64;
+cudaError_t launch_tri_inverse_diag(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_set_identity(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_ritz_sort(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* launches);

@@ -203,6 +203,58 @@ cudaError_t launch_tri_inverse(const SmallBatch& b, cudaStream_t s, int64_t* lau
 }
 
 // ---------------------------------------------------------------------------
+// Diagonal blocks of a lower-triangular inverse: block j of problem y covers
+// rows/cols [64j, min(64j + 64, l)); the block of a is inverted in shared
+// memory by forward substitution and written to the same place in c.  The
+// off-diagonal blocks are filled afterwards level by level with GEMMs:
+//   inv([A 0; C D]) = [A^-1 0; -D^-1 C A^-1  D^-1].
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_tri_inverse_diag(const __grid_constant__ SmallBatch b) {
+    __shared__ float Ls[kTriBase][kTriBase + 1];
+    __shared__ float Xs[kTriBase][kTriBase + 1];
+    const int pi = blockIdx.y;
+    const int l = b.l[pi];
+    const int i0 = blockIdx.x * kTriBase;
+    if (i0 >= l) return;
+    const int sz = min(kTriBase, l - i0);
+    const float* L = b.a[pi];
+    float* X = b.c[pi];
+    for (int e = threadIdx.x; e < sz * sz; e += blockDim.x) {
+        const int i = e / sz, c = e - i * sz;
+        Ls[i][c] = L[(long long)(i0 + i) * l + i0 + c];
+    }
+    __syncthreads();
+    // row by row; thread c owns column c
+    for (int i = 0; i < sz; ++i) {
+        if (threadIdx.x < sz) {
+            const int c = threadIdx.x;
+            float v = 0.0f;
+            if (c <= i) {
+                float acc = (c == i) ? 1.0f : 0.0f;
+                for (int k = c; k < i; ++k) acc = fmaf(-Ls[i][k], Xs[k][c], acc);
+                v = acc / Ls[i][i];
+            }
+            Xs[i][c] = v;
+        }
+        __syncthreads();
+    }
+    for (int e = threadIdx.x; e < sz * sz; e += blockDim.x) {
+        const int i = e / sz, c = e - i * sz;
+        X[(long long)(i0 + i) * l + i0 + c] = Xs[i][c];
+    }
+}
+
+cudaError_t launch_tri_inverse_diag(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    int lmax = 1;
+    for (int i = 0; i < b.count; ++i) lmax = b.l[i] > lmax ? b.l[i] : lmax;
+    dim3 grid((lmax + kTriBase - 1) / kTriBase, b.count);
+    k_tri_inverse_diag<<<grid, 256, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // a <- I (l x l)
 // ---------------------------------------------------------------------------
 __global__ void k_set_identity(const __grid_constant__ SmallBatch b) {

@@ -193,6 +193,8 @@ __device__ __forceinline__ void epilogue(const GemmBatch& b, const GemmProb& p, 
     const long long o = (long long)i * p.ldc + j;
     if (EPI == EPI_STORE) {
         p.C[o] = acc;
+    } else if (EPI == EPI_STORE_NEG) {
+        p.C[o] = -acc;
     } else if (EPI == EPI_ADAM) {
         // Optimizer_V (Algorithm 1): Adam on the projected direction R = acc.
         float ea = b.beta1 * p.aux0[o] + (1.0f - b.beta1) * acc;
@@ -319,6 +321,7 @@ cudaError_t launch_gemm(const GemmKind& k, GemmBatch& b, cudaStream_t s, int64_t
     MOARA_GEMM_CASE(A_MCONTIG, false, false, B_NCONTIG, false, false, EPI_STORE)
     MOARA_GEMM_CASE(A_KCONTIG, false, false, B_NCONTIG, false, false, EPI_STORE)
     MOARA_GEMM_CASE(A_KCONTIG, false, false, B_KCONTIG, false, false, EPI_STORE)
+    MOARA_GEMM_CASE(A_KCONTIG, false, false, B_NCONTIG, false, false, EPI_STORE_NEG)
 #undef MOARA_GEMM_CASE
     return cudaErrorInvalidValue;
 }

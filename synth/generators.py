@@ -95,18 +95,18 @@ def signed_permutation(m, r, seed=0):
 
 def lowrank_grad_torch(m, n, s, sigma0, noise, step, seed=0, module=0,
                        noise_rel=False, device="cuda", dtype=None):
-    """The same recipe built with torch on ``device`` (for large workloads)."""
+    """The same recipe on a torch device (for workloads too large for the
+    host): the factors come from ``lowrank_factors`` (NumPy), the noise from
+    torch's generator on ``device`` seeded by (seed, module, step)."""
     import torch
     dtype = torch.bfloat16 if dtype is None else dtype
-    gen = torch.Generator(device=device)
-    gen.manual_seed((seed * 1_000_003 + module * 7919) & 0x7FFFFFFF)
-    u = torch.randn(m, s, generator=gen, device=device, dtype=torch.float32)
-    v = torch.randn(n, s, generator=gen, device=device, dtype=torch.float32)
-    u, _ = torch.linalg.qr(u)
-    v, _ = torch.linalg.qr(v)
-    sig = sigma0 * (0.7 ** torch.arange(s, device=device, dtype=torch.float32))
+    u, v = lowrank_factors(m, n, s, seed, module)
+    sig = sigma0 * 0.7 ** np.arange(s)
+    ut = torch.tensor(u * sig, dtype=torch.float32, device=device)
+    vt = torch.tensor(v, dtype=torch.float32, device=device)
     nu = noise * sigma0 / (n ** 0.5) if noise_rel else noise
+    gen = torch.Generator(device=device)
     gen.manual_seed((seed * 1_000_003 + module * 7919 + 104729 * (1 + step)) & 0x7FFFFFFF)
-    g = (u * sig) @ v.T
+    g = ut @ vt.T
     g.add_(torch.randn(m, n, generator=gen, device=device, dtype=torch.float32), alpha=nu)
     return g.to(dtype)

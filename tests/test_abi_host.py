@@ -16,8 +16,8 @@ GOLDEN = os.path.join(ROOT, "tests", "golden")
 
 @pytest.fixture(scope="module")
 def M():
-    from paper_2609_15037_gb300 import build as b
-    b.build()
+    import __graft_entry__
+    __graft_entry__.build()
     import paper_2609_15037_gb300 as pkg
     return pkg
 
