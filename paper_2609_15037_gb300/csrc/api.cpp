@@ -34,6 +34,7 @@ struct moara_ctx {
     struct Rec { int phase; cudaEvent_t a, b; };
     std::vector<Rec> recs;
     std::vector<cudaEvent_t> free_events;
+    cudaEvent_t open_event = nullptr;
     double prof_ms[MOARA_NUM_PHASES] = {0};
     int64_t prof_n[MOARA_NUM_PHASES] = {0};
 };
@@ -874,9 +875,14 @@ int moara_step_grouped(moara_ctx* ctx, int n_mod, const int* ids, const void* co
         for (size_t q = 0; q < tcm.size(); ++q) { mids[q] = ids[tcm[q]]; gp[q] = G[tcm[q]]; }
         moara::TcProfile tp{ctx->prof, [](void* c, int ph, cudaStream_t st, bool begin) {
             moara_ctx* cx = static_cast<moara_ctx*>(c);
-            static thread_local cudaEvent_t open = nullptr;
-            if (begin) { open = take_event(cx); cudaEventRecord(open, st); }
-            else { cudaEvent_t b = take_event(cx); cudaEventRecord(b, st); cx->recs.push_back({ph, open, b}); }
+            if (begin) {
+                cx->open_event = take_event(cx);
+                cudaEventRecord(cx->open_event, st);
+            } else {
+                cudaEvent_t b = take_event(cx);
+                cudaEventRecord(b, st);
+                cx->recs.push_back({ph, cx->open_event, b});
+            }
         }, ctx};
         rc = moara::tc_step(ctx->tc, ctx->hp, static_cast<int>(mids.size()), mids.data(), gp.data(),
                             static_cast<float>(bc1), static_cast<float>(bc2), lr, s, &ctx->launches, tp);

@@ -1,30 +1,848 @@
-// Tensor-core path of the step (placeholder until the tcgen05 kernels land).
+// Tensor-core path of the optimizer step for bf16 gradients (sm_103a):
+//
+//  K1  R = P^T V with V = Decompose(G, B) formed in shared memory as a pair
+//      of bf16 tiles V_hi + V_lo (two MMAs; P is exact in bf16), then
+//      Optimizer_V (Adam) on R in the epilogue; writes the Adam update N as
+//      bf16.  The block norms computed for V also drive Optimizer_M (Adam on
+//      the block magnitudes M), done once per (row, block) by the CTAs of the
+//      first rank tile.  (Algorithm 1; §3.1 / Appendix B.1.)
+//  K2  dV = P N, then W <- W - lr*alpha*(Rep_B(dM) (.) dV) in the epilogue,
+//      reading and writing W once.  (Algorithm 1.)
+//
+// Both kernels are persistent and warp specialised: one warp issues TMA tile
+// loads into a 4-stage shared-memory ring, one thread issues tcgen05.mma into
+// double-buffered TMEM accumulators, and epilogue warps drain TMEM while the
+// next tile's MMAs run.  Every mbarrier wait is bounded; on expiry the kernel
+// records MOARA_ERR_DEVICE_TIMEOUT in the context's status word, drains its
+// own TMA copies and MMAs, frees TMEM and returns.
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cstring>
+#include <map>
 #include <string>
+#include <vector>
 
 #include "tc.h"
+#include "tc_ptx.cuh"
 
 namespace moara {
 
-struct TcState {
-    int device;
-    int* d_status;
-    std::string err;
+namespace {
+
+constexpr int kTcGroup = 224;                 // modules per launch (G maps in params)
+constexpr long long kWaitLimit = 1LL << 32;   // ~2 s of SM clocks
+
+struct TcMod {
+    int m, n, r, kb;
+    float* W;
+    float* exp_avg;
+    float* exp_avg_sq;
+    float* mag_avg;
+    float* mag_avg_sq;
+    uint16_t* Nb;     // r x n bf16 Adam update of the direction branch
+    float* dM;        // m x kb Adam update of the magnitude branch
 };
 
-bool tc_supported(int, int, int, int, int, int) { return false; }
+struct TcTile {
+    int mod, slot, t0, t1;
+};
 
-TcState* tc_create(int device, int* d_status) { return new TcState{device, d_status, {}}; }
+// ------------------------------------------------------------------- K1
+constexpr int K1_BM = 256, K1_BN = 128, K1_BK = 64, K1_STAGES = 3;
+constexpr int K1_A_BYTES = K1_BM * K1_BK * 2;           // 32 KB: four 64-row chunks of P^T
+constexpr int K1_B_BYTES = K1_BK * K1_BN * 2;           // 16 KB: two 64-column chunks of G
+// stage: A | B (G, then V_hi after the transform) | V_lo (V - V_hi in bf16)
+constexpr int K1_STAGE_BYTES = K1_A_BYTES + 2 * K1_B_BYTES;
+constexpr int K1_TX_BYTES = K1_A_BYTES + K1_B_BYTES;    // bytes the TMA brings per stage
+constexpr int K1_WARPS = 14;                            // 0 TMA, 1 MMA, 2-5 transform, 6-13 epilogue
+constexpr int K1_THREADS = K1_WARPS * 32;
+constexpr int GUARD_BYTES = 16384;
+constexpr int K1_SMEM = 1024 + K1_STAGES * K1_STAGE_BYTES + GUARD_BYTES + 2048;
 
-void tc_destroy(TcState* st) { delete st; }
+struct K1Params {
+    CUtensorMap gmap[kTcGroup];        // G of each launch slot: dims {n, m}, box {64, 64}
+    const TcTile* tiles;
+    const TcMod* mods;
+    const CUtensorMap* maps;           // per module: [0] P for K1, [1] P for K2, [2] N for K2
+    int* status;
+    int n_tiles;
+    float beta1, beta2, adam_eps, bc1, bc2, decomp_eps;
+};
 
-int tc_register(TcState*, int, const ModDev&, const moara_hparams&) { return MOARA_OK; }
+// ------------------------------------------------------------------- K2
+constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64, K2_STAGES = 4;
+constexpr int K2_A_BYTES = K2_BM * K2_BK * 2;           // 16 KB: P rows, K-major
+constexpr int K2_B_BYTES = K2_BK * K2_BN * 2;           // 32 KB: four 64-column chunks of N
+constexpr int K2_STAGE_BYTES = K2_A_BYTES + K2_B_BYTES;
+constexpr int K2_WARPS = 10;                            // 0 TMA, 1 MMA, 2-9 epilogue
+constexpr int K2_THREADS = K2_WARPS * 32;
+constexpr int K2_SMEM = 1024 + K2_STAGES * K2_STAGE_BYTES + GUARD_BYTES + 2048;
 
-int tc_step(TcState* st, const moara_hparams&, int, const int*, const void* const*, float, float, float,
-            cudaStream_t, int64_t*, const TcProfile&) {
-    st->err = "tensor-core path not available";
-    return MOARA_ERR_UNSUPPORTED;
+struct K2Params {
+    const TcTile* tiles;
+    const TcMod* mods;
+    const CUtensorMap* maps;
+    int* status;
+    int n_tiles;
+    float step_scale;                  // lr * alpha
+    int decompose;
+};
+
+struct SmemCtl {
+    uint64_t full[4];
+    uint64_t xform[4];
+    uint64_t empty[4];   // sized for up to four stages
+    uint64_t accf[2];
+    uint64_t acce[2];
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort;
+};
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+    return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
-const char* tc_last_error(const TcState* st) { return st->err.c_str(); }
+__device__ __forceinline__ bool wait_drain(uint32_t bar, uint32_t parity) {
+    const long long t0 = clock64();
+    while (!ptx::mbar_try_wait(bar, parity)) {
+        if (clock64() - t0 > kWaitLimit) return false;
+    }
+    return true;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// ===========================================================================
+// K1: projection R = P^T V with the decomposition fused into the B operand,
+// direction-branch Adam in the epilogue, magnitude-branch Adam in the
+// transform warps.
+// ===========================================================================
+template <int BLK, bool DECOMP>
+__global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constant__ K1Params p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = align1024(smem_raw);
+    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + K1_STAGES * K1_STAGE_BYTES + GUARD_BYTES);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    volatile int* abort_flag = &ctl->abort;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < K1_STAGES; ++s) {
+            ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->xform[s]), 128);
+            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            ptx::mbar_init(ptx::smem_u32(&ctl->accf[b]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 8);
+        }
+        ptx::mbar_init(ptx::smem_u32(&ctl->drain), 1);
+        ctl->abort = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(ptx::smem_u32(&ctl->tmem_base), 512);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = ctl->tmem_base;
+
+    if (warp == 0) {
+        // ------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t issued = 0, last_par = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+                const TcTile tl = p.tiles[t];
+                const TcMod md = p.mods[tl.mod];
+                const CUtensorMap* pmap = &p.maps[tl.mod * 3 + 0];
+                const CUtensorMap* gmap = &p.gmap[tl.slot];
+                const int r0 = tl.t0 * K1_BM, n0 = tl.t1 * K1_BN;
+                const int nk = (md.m + K1_BK - 1) / K1_BK;
+                for (int kb = 0; kb < nk; ++kb) {
+                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
+                    ptx::mbar_arrive_expect_tx(fb, K1_TX_BYTES);
+                    const uint32_t a = ptx::smem_u32(smem + stage * K1_STAGE_BYTES);
+                    const uint32_t b = a + K1_A_BYTES;
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) ptx::tma_load_2d(a + c * 8192, pmap, fb, r0 + 64 * c, kb * K1_BK);
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) ptx::tma_load_2d(b + c * 8192, gmap, fb, n0 + 64 * c, kb * K1_BK);
+                    issued |= 1u << stage;
+                    last_par = (last_par & ~(1u << stage)) | (phase << stage);
+                    if (++stage == K1_STAGES) { stage = 0; phase ^= 1; }
+                }
+            }
+            if (!ok) {   // let the copies already in flight land before the CTA exits
+                for (int s = 0; s < K1_STAGES; ++s)
+                    if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = ptx::idesc_bf16(128, K1_BN, 1, 1);
+            int stage = 0;
+            uint32_t phase = 0;
+            int buf = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+                const TcTile tl = p.tiles[t];
+                const TcMod md = p.mods[tl.mod];
+                const int r0 = tl.t0 * K1_BM;
+                const int nh = (r0 + 128 < md.r) ? 2 : 1;
+                const int nk = (md.m + K1_BK - 1) / K1_BK;
+                if (!ptx::mbar_wait(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
+                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                ptx::tc_fence_after();
+                const uint32_t d0 = tmem + buf * 256;
+                for (int kb = 0; kb < nk; ++kb) {
+                    const uint32_t wb = DECOMP ? ptx::smem_u32(&ctl->xform[stage]) : ptx::smem_u32(&ctl->full[stage]);
+                    if (!ptx::mbar_wait(wb, phase, abort_flag, p.status, MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    const uint32_t a = ptx::smem_u32(smem + stage * K1_STAGE_BYTES);
+                    const uint32_t b = a + K1_A_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const uint64_t bdesc = ptx::smem_desc_sw128(b + kk * 2048, 8192, 1024);
+                        const uint64_t ldesc = ptx::smem_desc_sw128(b + K1_B_BYTES + kk * 2048, 8192, 1024);
+                        for (int h = 0; h < nh; ++h) {
+                            const uint64_t adesc = ptx::smem_desc_sw128(a + h * 16384 + kk * 2048, 8192, 1024);
+                            ptx::mma_f16(d0 + h * 128, adesc, bdesc, idesc, (kb | kk) != 0);
+                            // P^T V_lo: the bf16 rounding residual of V, so that R carries
+                            // about 16 significant bits (P is exact in bf16)
+                            if (DECOMP) ptx::mma_f16(d0 + h * 128, adesc, ldesc, idesc, 1);
+                        }
+                    }
+                    ptx::mma_commit(ptx::smem_u32(&ctl->empty[stage]));
+                    if (++stage == K1_STAGES) { stage = 0; phase ^= 1; }
+                }
+                if (!ok) break;
+                ptx::mma_commit(ptx::smem_u32(&ctl->accf[buf]));
+                if (++buf == 2) { buf = 0; acc_phase ^= 1; }
+            }
+            // wait for every MMA this thread issued before TMEM is released
+            ptx::mma_commit(ptx::smem_u32(&ctl->drain));
+            wait_drain(ptx::smem_u32(&ctl->drain), 0);
+        }
+    } else if (warp < 6) {
+        // ------------------------------------------------- transform warps
+        if (DECOMP) {
+            const int tid = threadIdx.x - 64;           // 0..127
+            const int k = tid >> 1;                     // row within the stage
+            const int hc = tid & 1;                     // 64-column chunk (partner: lane ^ 1)
+            const uint32_t x = static_cast<uint32_t>(k & 7);
+            constexpr int UB = BLK / 8;                 // 16-byte units per block
+            constexpr int NBT = UB <= 8 ? 8 / UB : 1;   // blocks held by this thread
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+                const TcTile tl = p.tiles[t];
+                const TcMod md = p.mods[tl.mod];
+                const int n0 = tl.t1 * K1_BN;
+                const bool do_mag = (tl.t0 == 0);
+                const int nk = (md.m + K1_BK - 1) / K1_BK;
+                for (int kb = 0; kb < nk; ++kb) {
+                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    uint8_t* row = smem + stage * K1_STAGE_BYTES + K1_A_BYTES + hc * 8192 + k * 128;
+                    uint4 d[8];
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) d[u] = *reinterpret_cast<const uint4*>(row + ((u ^ x) << 4));
+                    float ssu[8];
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const uint32_t w[4] = {d[u].x, d[u].y, d[u].z, d[u].w};
+                        float s = 0.0f;
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float lo = bf_lo(w[e]), hi = bf_hi(w[e]);
+                            s = fmaf(lo, lo, s);
+                            s = fmaf(hi, hi, s);
+                        }
+                        ssu[u] = s;
+                    }
+                    float ssb[NBT];
+#pragma unroll
+                    for (int bl = 0; bl < NBT; ++bl) {
+                        float s = 0.0f;
+#pragma unroll
+                        for (int u = 0; u < (UB <= 8 ? UB : 8); ++u) s += ssu[bl * (UB <= 8 ? UB : 8) + u];
+                        ssb[bl] = s;
+                    }
+                    if (UB > 8) {   // B = 128: the block spans both chunks; the partner is lane ^ 1
+                        ssb[0] += __shfl_xor_sync(0xffffffffu, ssb[0], 1);
+                    }
+                    float inv[NBT];
+                    float mag[NBT];
+#pragma unroll
+                    for (int bl = 0; bl < NBT; ++bl) {
+                        mag[bl] = sqrtf(ssb[bl]);
+                        inv[bl] = 1.0f / (mag[bl] + p.decomp_eps);
+                    }
+                    uint8_t* lrow = row + K1_B_BYTES;
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const float sc = inv[UB <= 8 ? u / UB : 0];
+                        const uint32_t w[4] = {d[u].x, d[u].y, d[u].z, d[u].w};
+                        uint32_t hi[4], lo[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float v0 = bf_lo(w[e]) * sc, v1 = bf_hi(w[e]) * sc;
+                            hi[e] = pack_bf16x2(v0, v1);
+                            lo[e] = pack_bf16x2(v0 - bf_lo(hi[e]), v1 - bf_hi(hi[e]));
+                        }
+                        const uint32_t off = (u ^ x) << 4;
+                        *reinterpret_cast<uint4*>(row + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                        *reinterpret_cast<uint4*>(lrow + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                    }
+                    ptx::fence_proxy_async_smem();
+                    ptx::mbar_arrive(ptx::smem_u32(&ctl->xform[stage]));
+                    // Optimizer_M on the block magnitudes, once per (row, block)
+                    const int grow = kb * K1_BK + k;
+                    if (do_mag && grow < md.m && (UB <= 8 || hc == 0)) {
+#pragma unroll
+                        for (int bl = 0; bl < NBT; ++bl) {
+                            const int gb = (n0 + hc * 64) / BLK + bl;
+                            if (gb < md.kb) {
+                                const long long o = (long long)grow * md.kb + gb;
+                                const float ma = p.beta1 * md.mag_avg[o] + (1.0f - p.beta1) * mag[bl];
+                                const float mas = p.beta2 * md.mag_avg_sq[o] + (1.0f - p.beta2) * mag[bl] * mag[bl];
+                                md.mag_avg[o] = ma;
+                                md.mag_avg_sq[o] = mas;
+                                md.dM[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
+                            }
+                        }
+                    }
+                    if (++stage == K1_STAGES) { stage = 0; phase ^= 1; }
+                }
+            }
+        }
+    } else {
+        // ------------------------------------------------- epilogue warps
+        const int ew = warp - 6;                       // 0..7
+        const int q = warp & 3;                        // TMEM lane quarter of this warp
+        const int h = ew >> 2;                         // accumulator half (rows 0-127 / 128-255)
+        int buf = 0;
+        uint32_t acc_phase = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+            const TcTile tl = p.tiles[t];
+            const TcMod md = p.mods[tl.mod];
+            const int r0 = tl.t0 * K1_BM, n0 = tl.t1 * K1_BN;
+            if (!ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
+                                MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+            ptx::tc_fence_after();
+            const bool half_valid = (r0 + h * 128) < md.r;
+            if (half_valid) {
+                const int a = r0 + h * 128 + q * 32 + lane;
+                const bool row_ok = a < md.r;
+#pragma unroll 1
+                for (int c = 0; c < K1_BN / 16; ++c) {
+                    float v[16];
+                    __syncwarp();
+                    ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + h * 128 + c * 16, v);
+                    const int j0 = n0 + c * 16;
+                    if (!row_ok || j0 >= md.n) continue;
+                    const long long o = (long long)a * md.n + j0;
+                    if (j0 + 16 <= md.n) {
+                        float4* ea4 = reinterpret_cast<float4*>(md.exp_avg + o);
+                        float4* es4 = reinterpret_cast<float4*>(md.exp_avg_sq + o);
+                        float ea[16], es[16];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float4 x = ea4[e], y = es4[e];
+                            ea[4 * e] = x.x; ea[4 * e + 1] = x.y; ea[4 * e + 2] = x.z; ea[4 * e + 3] = x.w;
+                            es[4 * e] = y.x; es[4 * e + 1] = y.y; es[4 * e + 2] = y.z; es[4 * e + 3] = y.w;
+                        }
+                        uint32_t nb[8];
+                        float nv[16];
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            ea[e] = p.beta1 * ea[e] + (1.0f - p.beta1) * v[e];
+                            es[e] = p.beta2 * es[e] + (1.0f - p.beta2) * v[e] * v[e];
+                            nv[e] = (ea[e] / p.bc1) / (sqrtf(es[e] / p.bc2) + p.adam_eps);
+                        }
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) nb[e] = pack_bf16x2(nv[2 * e], nv[2 * e + 1]);
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            ea4[e] = make_float4(ea[4 * e], ea[4 * e + 1], ea[4 * e + 2], ea[4 * e + 3]);
+                            es4[e] = make_float4(es[4 * e], es[4 * e + 1], es[4 * e + 2], es[4 * e + 3]);
+                        }
+                        uint4* n4 = reinterpret_cast<uint4*>(md.Nb + o);
+                        n4[0] = make_uint4(nb[0], nb[1], nb[2], nb[3]);
+                        n4[1] = make_uint4(nb[4], nb[5], nb[6], nb[7]);
+                    } else {
+                        for (int e = 0; e < 16 && j0 + e < md.n; ++e) {
+                            const float ea = p.beta1 * md.exp_avg[o + e] + (1.0f - p.beta1) * v[e];
+                            const float es = p.beta2 * md.exp_avg_sq[o + e] + (1.0f - p.beta2) * v[e] * v[e];
+                            md.exp_avg[o + e] = ea;
+                            md.exp_avg_sq[o + e] = es;
+                            const float nv = (ea / p.bc1) / (sqrtf(es / p.bc2) + p.adam_eps);
+                            __nv_bfloat16 hb = __float2bfloat16_rn(nv);
+                            md.Nb[o + e] = *reinterpret_cast<uint16_t*>(&hb);
+                        }
+                    }
+                }
+            }
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->acce[buf]));
+            if (++buf == 2) { buf = 0; acc_phase ^= 1; }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, 512);
+    }
+}
+
+// ===========================================================================
+// K2: back-projection dV = P N and the weight update in the epilogue.
+// ===========================================================================
+template <int BLK>
+__global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_constant__ K2Params p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = align1024(smem_raw);
+    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + K2_STAGES * K2_STAGE_BYTES + GUARD_BYTES);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    volatile int* abort_flag = &ctl->abort;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < K2_STAGES; ++s) {
+            ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            ptx::mbar_init(ptx::smem_u32(&ctl->accf[b]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 8);
+        }
+        ptx::mbar_init(ptx::smem_u32(&ctl->drain), 1);
+        ctl->abort = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(ptx::smem_u32(&ctl->tmem_base), 512);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = ctl->tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t issued = 0, last_par = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+                const TcTile tl = p.tiles[t];
+                const TcMod md = p.mods[tl.mod];
+                const CUtensorMap* amap = &p.maps[tl.mod * 3 + 1];
+                const CUtensorMap* bmap = &p.maps[tl.mod * 3 + 2];
+                const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
+                const int nk = (md.r + K2_BK - 1) / K2_BK;
+                for (int kb = 0; kb < nk; ++kb) {
+                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
+                    ptx::mbar_arrive_expect_tx(fb, K2_STAGE_BYTES);
+                    const uint32_t a = ptx::smem_u32(smem + stage * K2_STAGE_BYTES);
+                    const uint32_t b = a + K2_A_BYTES;
+                    ptx::tma_load_2d(a, amap, fb, kb * K2_BK, i0);
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) ptx::tma_load_2d(b + c * 8192, bmap, fb, n0 + 64 * c, kb * K2_BK);
+                    issued |= 1u << stage;
+                    last_par = (last_par & ~(1u << stage)) | (phase << stage);
+                    if (++stage == K2_STAGES) { stage = 0; phase ^= 1; }
+                }
+            }
+            if (!ok) {
+                for (int s = 0; s < K2_STAGES; ++s)
+                    if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = ptx::idesc_bf16(128, K2_BN, 0, 1);
+            int stage = 0;
+            uint32_t phase = 0;
+            int buf = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+                const TcTile tl = p.tiles[t];
+                const TcMod md = p.mods[tl.mod];
+                const int nk = (md.r + K2_BK - 1) / K2_BK;
+                if (!ptx::mbar_wait(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
+                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                ptx::tc_fence_after();
+                const uint32_t d0 = tmem + buf * 256;
+                for (int kb = 0; kb < nk; ++kb) {
+                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    ptx::tc_fence_after();
+                    const uint32_t a = ptx::smem_u32(smem + stage * K2_STAGE_BYTES);
+                    const uint32_t b = a + K2_A_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const uint64_t adesc = ptx::smem_desc_sw128(a + kk * 32, 16, 1024);
+                        const uint64_t bdesc = ptx::smem_desc_sw128(b + kk * 2048, 8192, 1024);
+                        ptx::mma_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
+                    }
+                    ptx::mma_commit(ptx::smem_u32(&ctl->empty[stage]));
+                    if (++stage == K2_STAGES) { stage = 0; phase ^= 1; }
+                }
+                if (!ok) break;
+                ptx::mma_commit(ptx::smem_u32(&ctl->accf[buf]));
+                if (++buf == 2) { buf = 0; acc_phase ^= 1; }
+            }
+            ptx::mma_commit(ptx::smem_u32(&ctl->drain));
+            wait_drain(ptx::smem_u32(&ctl->drain), 0);
+        }
+    } else {
+        const int ew = warp - 2;                        // 0..7
+        const int q = warp & 3;
+        const int ch = ew >> 2;                         // column half of the 256-wide tile
+        int buf = 0;
+        uint32_t acc_phase = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+            const TcTile tl = p.tiles[t];
+            const TcMod md = p.mods[tl.mod];
+            const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
+            if (!ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
+                                MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+            ptx::tc_fence_after();
+            const int i = i0 + q * 32 + lane;
+            const bool row_ok = i < md.m;
+#pragma unroll 1
+            for (int c = 0; c < 8; ++c) {
+                const int cc = ch * 128 + c * 16;
+                float v[16];
+                __syncwarp();
+                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + cc, v);
+                const int j0 = n0 + cc;
+                if (!row_ok || j0 >= md.n) continue;
+                const long long o = (long long)i * md.n + j0;
+                const float* dmr = md.dM + (long long)i * md.kb;
+                if (j0 + 16 <= md.n) {
+                    float4* w4 = reinterpret_cast<float4*>(md.W + o);
+                    float w[16];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float4 x = w4[e];
+                        w[4 * e] = x.x; w[4 * e + 1] = x.y; w[4 * e + 2] = x.z; w[4 * e + 3] = x.w;
+                    }
+                    if (p.decompose) {
+                        if (BLK >= 16) {
+                            const float dm = dmr[j0 / BLK];
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) w[e] -= p.step_scale * (dm * v[e]);
+                        } else {
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) w[e] -= p.step_scale * (dmr[(j0 + e) / BLK] * v[e]);
+                        }
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) w[e] -= p.step_scale * v[e];
+                    }
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) w4[e] = make_float4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
+                } else {
+                    for (int e = 0; e < 16 && j0 + e < md.n; ++e) {
+                        const float u = p.decompose ? dmr[(j0 + e) / BLK] * v[e] : v[e];
+                        md.W[o + e] -= p.step_scale * u;
+                    }
+                }
+            }
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->acce[buf]));
+            if (++buf == 2) { buf = 0; acc_phase ^= 1; }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, 512);
+    }
+}
+
+// ---------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+bool encode_bf16_2d(EncodeTiledFn enc, CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
+                    uint32_t box_inner, uint32_t box_outer) {
+    const cuuint64_t dims[2] = {inner, outer};
+    const cuuint64_t strides[1] = {inner * 2};
+    const cuuint32_t box[2] = {box_inner, box_outer};
+    const cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BLK>
+void set_smem_attrs() {
+    cudaFuncSetAttribute(k1_project<BLK, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
+    cudaFuncSetAttribute(k1_project<BLK, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
+    cudaFuncSetAttribute(k2_backproject<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize, K2_SMEM);
+}
+
+}  // namespace
+
+struct TcState {
+    int device = 0;
+    int* d_status = nullptr;
+    int sms = 148;
+    EncodeTiledFn encode = nullptr;
+    std::string err;
+    std::vector<TcMod> mods;               // indexed by module id (unsupported ones left zero)
+    std::vector<CUtensorMap> maps;         // 3 per module id
+    TcMod* d_mods = nullptr;
+    CUtensorMap* d_maps = nullptr;
+    int cap = 0;
+    bool dirty = false;
+    struct Tiles { TcTile* k1 = nullptr; int n1 = 0; TcTile* k2 = nullptr; int n2 = 0; };
+    std::map<std::vector<int>, Tiles> tiles;
+    bool attrs_set = false;
+    K1Params p1;                           // parameter block of the next K1 launch
+};
+
+bool tc_supported(int m, int n, int r, int B, int dtype, int decompose) {
+    if (dtype != MOARA_DTYPE_BF16) return false;
+    if (m < 1 || n < 8 || r < 8) return false;
+    if ((n % 8) != 0 || (r % 8) != 0) return false;
+    if (decompose && !(B == 8 || B == 16 || B == 32 || B == 64 || B == 128)) return false;
+    if (!decompose && !(B >= 1)) return false;
+    return true;
+}
+
+TcState* tc_create(int device, int* d_status) {
+    TcState* st = new TcState();
+    st->device = device;
+    st->d_status = d_status;
+    cudaDeviceProp prop{};
+    if (cudaGetDeviceProperties(&prop, device) == cudaSuccess) {
+        st->sms = prop.multiProcessorCount;
+        if (prop.major != 10 || prop.minor != 3) {   // these kernels are built for sm_103a only
+            delete st;
+            return nullptr;
+        }
+    }
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess || q != cudaDriverEntryPointSuccess || fn == nullptr) {
+        delete st;
+        return nullptr;
+    }
+    st->encode = reinterpret_cast<EncodeTiledFn>(fn);
+    return st;
+}
+
+void tc_destroy(TcState* st) {
+    if (st == nullptr) return;
+    if (st->d_mods) cudaFree(st->d_mods);
+    if (st->d_maps) cudaFree(st->d_maps);
+    for (auto& kv : st->tiles) {
+        if (kv.second.k1) cudaFree(kv.second.k1);
+        if (kv.second.k2) cudaFree(kv.second.k2);
+    }
+    delete st;
+}
+
+int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) {
+    if (st == nullptr) return MOARA_OK;
+    if (static_cast<int>(st->mods.size()) <= id) {
+        st->mods.resize(id + 1, TcMod{});
+        st->maps.resize(3 * (id + 1));
+    }
+    if (!tc_supported(md.m, md.n, md.r, hp.block_size, md.dtype, hp.decompose) || md.Pb == nullptr) return MOARA_OK;
+    TcMod t{};
+    t.m = md.m; t.n = md.n; t.r = md.r; t.kb = md.kb;
+    t.W = md.W; t.exp_avg = md.exp_avg; t.exp_avg_sq = md.exp_avg_sq;
+    t.mag_avg = md.mag_avg; t.mag_avg_sq = md.mag_avg_sq;
+    t.Nb = reinterpret_cast<uint16_t*>(md.ws_N);
+    t.dM = md.ws_dM;
+    CUtensorMap* mp = &st->maps[3 * id];
+    if (!encode_bf16_2d(st->encode, &mp[0], md.Pb, md.r, md.m, 64, 64) ||
+        !encode_bf16_2d(st->encode, &mp[1], md.Pb, md.r, md.m, 64, 128) ||
+        !encode_bf16_2d(st->encode, &mp[2], t.Nb, md.n, md.r, 64, 64)) {
+        st->err = "cuTensorMapEncodeTiled failed";
+        return MOARA_ERR_CUDA;
+    }
+    st->mods[id] = t;
+    st->dirty = true;
+    return MOARA_OK;
+}
+
+static int tc_upload(TcState* st) {
+    if (!st->dirty) return MOARA_OK;
+    const int n = static_cast<int>(st->mods.size());
+    if (n > st->cap) {
+        int ncap = std::max(64, st->cap);
+        while (ncap < n) ncap *= 2;
+        if (st->d_mods) cudaFree(st->d_mods);
+        if (st->d_maps) cudaFree(st->d_maps);
+        st->d_mods = nullptr;
+        st->d_maps = nullptr;
+        if (cudaMalloc(&st->d_mods, sizeof(TcMod) * ncap) != cudaSuccess ||
+            cudaMalloc(&st->d_maps, sizeof(CUtensorMap) * 3 * ncap) != cudaSuccess) {
+            st->err = "cudaMalloc of the tensor-core module table failed";
+            return MOARA_ERR_CUDA;
+        }
+        st->cap = ncap;
+    }
+    if (cudaMemcpy(st->d_mods, st->mods.data(), sizeof(TcMod) * n, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(st->d_maps, st->maps.data(), sizeof(CUtensorMap) * 3 * n, cudaMemcpyHostToDevice) !=
+            cudaSuccess) {
+        st->err = "upload of the tensor-core module table failed";
+        return MOARA_ERR_CUDA;
+    }
+    st->dirty = false;
+    return MOARA_OK;
+}
+
+// Work lists of one launch: K1 tiles (rank tile x 128-column strip) and K2
+// tiles (128-row tile x 256-column strip), longest reduction first; the rank
+// tiles of one column strip stay adjacent so they share the strip of G in L2.
+static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
+    auto it = st->tiles.find(ids);
+    if (it != st->tiles.end()) return &it->second;
+    std::vector<TcTile> k1, k2;
+    std::vector<int> order(ids.size());
+    for (size_t i = 0; i < ids.size(); ++i) order[i] = static_cast<int>(i);
+    std::stable_sort(order.begin(), order.end(),
+                     [&](int a, int b) { return st->mods[ids[a]].m > st->mods[ids[b]].m; });
+    for (int slot : order) {
+        const TcMod& md = st->mods[ids[slot]];
+        const int nt = (md.n + K1_BN - 1) / K1_BN, rt = (md.r + K1_BM - 1) / K1_BM;
+        for (int j = 0; j < nt; ++j)
+            for (int i = 0; i < rt; ++i) k1.push_back({ids[slot], slot, i, j});
+    }
+    std::stable_sort(order.begin(), order.end(),
+                     [&](int a, int b) { return st->mods[ids[a]].r > st->mods[ids[b]].r; });
+    for (int slot : order) {
+        const TcMod& md = st->mods[ids[slot]];
+        const int mt = (md.m + K2_BM - 1) / K2_BM, nt = (md.n + K2_BN - 1) / K2_BN;
+        for (int i = 0; i < mt; ++i)
+            for (int j = 0; j < nt; ++j) k2.push_back({ids[slot], slot, i, j});
+    }
+    TcState::Tiles t;
+    t.n1 = static_cast<int>(k1.size());
+    t.n2 = static_cast<int>(k2.size());
+    if (cudaMalloc(&t.k1, sizeof(TcTile) * std::max(1, t.n1)) != cudaSuccess ||
+        cudaMalloc(&t.k2, sizeof(TcTile) * std::max(1, t.n2)) != cudaSuccess ||
+        cudaMemcpy(t.k1, k1.data(), sizeof(TcTile) * t.n1, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(t.k2, k2.data(), sizeof(TcTile) * t.n2, cudaMemcpyHostToDevice) != cudaSuccess) {
+        if (t.k1) cudaFree(t.k1);
+        if (t.k2) cudaFree(t.k2);
+        return nullptr;
+    }
+    return &(st->tiles[ids] = t);
+}
+
+template <int BLK>
+static cudaError_t launch_pair(TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2,
+                               bool decomp, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, true);
+    if (decomp) k1_project<BLK, true><<<g1, K1_THREADS, K1_SMEM, s>>>(p1);
+    else k1_project<BLK, false><<<g1, K1_THREADS, K1_SMEM, s>>>(p1);
+    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, false);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    ++*launches;
+    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_BACKPROJECT, s, true);
+    k2_backproject<BLK><<<g2, K2_THREADS, K2_SMEM, s>>>(p2);
+    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_BACKPROJECT, s, false);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    ++*launches;
+    return cudaSuccess;
+}
+
+int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G, float bc1,
+            float bc2, float lr, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+    if (!st->attrs_set) {
+        set_smem_attrs<8>(); set_smem_attrs<16>(); set_smem_attrs<32>(); set_smem_attrs<64>();
+        set_smem_attrs<128>();
+        st->attrs_set = true;
+    }
+    int rc = tc_upload(st);
+    if (rc != MOARA_OK) return rc;
+    const int B = hp.decompose ? hp.block_size : 128;
+    for (int c0 = 0; c0 < n_mod; c0 += kTcGroup) {
+        const int cnt = std::min(kTcGroup, n_mod - c0);
+        std::vector<int> chunk(ids + c0, ids + c0 + cnt);
+        TcState::Tiles* tl = tc_tiles(st, chunk);
+        if (tl == nullptr) { st->err = "tile list allocation failed"; return MOARA_ERR_CUDA; }
+        K1Params& p1 = st->p1;
+        std::memset(&p1, 0, sizeof(p1));
+        for (int q = 0; q < cnt; ++q) {
+            const TcMod& md = st->mods[chunk[q]];
+            if (!encode_bf16_2d(st->encode, &p1.gmap[q], G[c0 + q], md.n, md.m, 64, 64)) {
+                st->err = "cuTensorMapEncodeTiled failed for a gradient";
+                return MOARA_ERR_CUDA;
+            }
+        }
+        p1.tiles = tl->k1; p1.mods = st->d_mods; p1.maps = st->d_maps; p1.status = st->d_status;
+        p1.n_tiles = tl->n1;
+        p1.beta1 = hp.beta1; p1.beta2 = hp.beta2; p1.adam_eps = hp.adam_eps;
+        p1.bc1 = bc1; p1.bc2 = bc2; p1.decomp_eps = hp.decomp_eps;
+        K2Params p2{};
+        p2.tiles = tl->k2; p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;
+        p2.n_tiles = tl->n2;
+        p2.step_scale = lr * hp.scale;
+        p2.decompose = hp.decompose;
+        const int g1 = std::max(1, std::min(tl->n1, st->sms));
+        const int g2 = std::max(1, std::min(tl->n2, st->sms));
+        const bool dec = hp.decompose != 0;
+        cudaError_t e;
+        switch (B) {
+            case 8: e = launch_pair<8>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
+            case 16: e = launch_pair<16>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
+            case 32: e = launch_pair<32>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
+            case 64: e = launch_pair<64>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
+            default: e = launch_pair<128>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
+        }
+        if (e != cudaSuccess) {
+            st->err = cudaGetErrorString(e);
+            return MOARA_ERR_CUDA;
+        }
+    }
+    return MOARA_OK;
+}
+
+const char* tc_last_error(const TcState* st) { return st ? st->err.c_str() : "no tensor-core state"; }
 
 }  // namespace moara
