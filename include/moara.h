@@ -242,6 +242,43 @@ int moara_profile_enable(moara_ctx* ctx, int enable);
  * counts per phase (arrays of MOARA_NUM_PHASES), and clears the record. */
 int moara_profile_read(moara_ctx* ctx, double ms[8], int64_t launches[8]);
 
+/* One optimizer step of a single weight that allocates no device memory.
+ *
+ * For callers that cannot allocate device memory when they run the step:
+ * code embedded in a host application that reserves the GPU's memory up
+ * front through its own pool (and forbids allocations outside it), or a step
+ * loop that must not pay the device-wide synchronisation that cudaMalloc and
+ * cudaFree can imply.  Such callers cannot create a context (moara_create
+ * allocates) or hand over a per-module workspace; this entry point takes the
+ * buffers directly and keeps its scratch -- the direction update N (r x n
+ * floats), the magnitude update and the block scales (m x ceil(n/B) floats
+ * each) -- in a 16 MiB array compiled into the library, which every GPU that
+ * loads the library holds until the process exits.  The paper has no
+ * counterpart; the computation is that of moara_step_grouped on the fp32
+ * path (MOARA_PREC_FP32), without the refresh.
+ *
+ *   hp          hyper-parameters (block size, betas, eps, scale, decompose)
+ *   m, n, r     shape and rank, 1 <= r <= min(m, n)
+ *   grad_dtype  MOARA_DTYPE_F32 or MOARA_DTYPE_BF16
+ *   G           m x n gradient (read);  W  m x n fp32 (updated)
+ *   P           m x r fp32 projector (read)
+ *   exp_avg, exp_avg_sq   r x n fp32 (updated)
+ *   mag_avg, mag_avg_sq   m x ceil(n/B) fp32 (updated; unused if decompose = 0)
+ *   t, lr       1-based Adam step and learning rate; stream as elsewhere
+ * All pointers are device pointers on the calling thread's current device,
+ * 16-byte aligned.  Returns MOARA_ERR_WORKSPACE when
+ * 4*(r*n + 2*m*ceil(n/B)) bytes (each part rounded up to 256 bytes) exceed
+ * the 16 MiB array; nothing is launched then.  The first call on a device
+ * looks up the array's device address (once per device) and should come
+ * before any stream capture.  All calls share the one array: calls whose
+ * kernels overlap on the GPU (different streams, or different host threads
+ * on the same device) race on it and must be serialised by the caller.  No
+ * scratch value is carried from one call to the next. */
+int moara_step_static_scratch(const moara_hparams* hp, int m, int n, int r, int grad_dtype,
+                              const void* G, float* W, const float* P, float* exp_avg,
+                              float* exp_avg_sq, float* mag_avg, float* mag_avg_sq, int64_t t,
+                              float lr, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -91,6 +91,8 @@ def _load():
         "moara_launch_count": (i64, [vp]),
         "moara_profile_enable": (i32, [vp, i32]),
         "moara_profile_read": (i32, [vp, P(ctypes.c_double), P(i64)]),
+        "moara_step_static_scratch": (i32, [P(moara_hparams), i32, i32, i32, i32, vp, vp, vp, vp,
+                                            vp, vp, vp, i64, f32, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -220,6 +222,15 @@ def moara_launch_count(ctx):
     return int(_lib.moara_launch_count(ctx))
 
 
+def moara_step_static_scratch(hp, m, n, r, grad_dtype, G, W, P, exp_avg, exp_avg_sq,
+                              mag_avg, mag_avg_sq, t, lr, stream=0):
+    """Single-module step with the library's built-in scratch (no device
+    allocation); returns the status code instead of raising."""
+    return _lib.moara_step_static_scratch(ctypes.byref(hp), m, n, r, grad_dtype, G, W, P,
+                                          exp_avg, exp_avg_sq, mag_avg, mag_avg_sq,
+                                          int(t), float(lr), stream)
+
+
 PHASES = ["decompose", "project", "backproject", "refresh", "tc_project",
           "tc_backproject", "phase6", "phase7"]
 
@@ -242,5 +253,5 @@ EXPORTED = [
     "moara_load_projector", "moara_refresh_workspace_bytes", "moara_set_refresh_workspace",
     "moara_refresh_projector", "moara_step_grouped", "moara_get_device_status",
     "moara_last_error", "moara_status_string", "moara_launch_count",
-    "moara_profile_enable", "moara_profile_read",
+    "moara_profile_enable", "moara_profile_read", "moara_step_static_scratch",
 ]
