@@ -169,6 +169,7 @@ size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v) {
     add(sizeof(float) * (size_t)m * l);  // Qa
     add(sizeof(float) * (size_t)m * l);  // Qb
     for (int i = 0; i < 6; ++i) add(sizeof(float) * (size_t)l * l);
+    add(sizeof(float) * 16);
     add(sizeof(float) * (size_t)l);
     add(sizeof(int) * (size_t)l);
     add(sizeof(int) * 4);
@@ -190,6 +191,7 @@ void refresh_carve(RefreshItem& it, void* base, int m, int n, int r, int l, int 
     it.Cg = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Linv = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Tt = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
+    it.scal = reinterpret_cast<float*>(take(sizeof(float) * 16));
     it.Cr = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Xa = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Xb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
@@ -245,14 +247,8 @@ struct RefreshRunner {
             p.A = Xin[i]; p.Bm = Xin[i]; p.C = it[i].Cg;
             p.M = l; p.N = l; p.K = rows[i]; p.lda = l; p.ldb = l; p.ldc = l;
         });
-        moara::SmallBatch sb = small();
-        sb.shift_rel = shift_rel;
-        for (size_t i = 0; i < it.size(); ++i) {
-            sb.l[i] = it[i].l; sb.rows[i] = rows[i]; sb.a[i] = it[i].Cg; sb.c[i] = it[i].Linv;
-            sb.fail[i] = it[i].fail;
-        }
-        chk(moara::launch_cholesky(sb, s, &ctx->launches));
-        tri_inverse();
+        cholesky_blocked(rows, shift_rel);
+        tri_inverse(/*have_diag=*/true);
         moara::GemmKind apply{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
         gemm(apply, [&](int i, moara::GemmProb& p) {
             const int l = it[i].l;
@@ -265,15 +261,69 @@ struct RefreshRunner {
     // 64 x 64 blocks in shared memory, then the off-diagonal blocks level by
     // level (block size s = 64, 128, ...) with two grouped GEMMs per level:
     //   T = L[D, A] Linv[A, A];  Linv[D, A] = -Linv[D, D] T.
-    void tri_inverse() {
+    // Lower Cholesky factor of Cg (+ shift on the diagonal) in place, by 64-wide
+    // panels: factor the diagonal block (its inverse goes to the diagonal block
+    // of Linv), solve the panel below it, update the trailing matrix.
+    void cholesky_blocked(const std::vector<int>& rows, float shift_rel) {
+        int lmax = 0;
+        moara::SmallBatch sb = small();
+        sb.shift_rel = shift_rel;
+        for (size_t i = 0; i < it.size(); ++i) {
+            chk(cudaMemsetAsync(it[i].Linv, 0, sizeof(float) * (size_t)it[i].l * it[i].l, s));
+            sb.l[i] = it[i].l; sb.rows[i] = rows[i]; sb.a[i] = it[i].Cg; sb.b[i] = it[i].scal;
+            sb.c[i] = it[i].Linv; sb.fail[i] = it[i].fail;
+            lmax = std::max(lmax, it[i].l);
+        }
+        chk(moara::launch_trace_shift(sb, s, &ctx->launches));
+        const int nb = moara::kTriBase;
+        moara::GemmKind solve{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
+        moara::GemmKind upd{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_SUB};
+        for (int j0 = 0; j0 < lmax; j0 += nb) {
+            chk(moara::launch_chol_diag(sb, j0, s, &ctx->launches));
+            std::vector<int> act;
+            for (int i = 0; i < static_cast<int>(it.size()); ++i)
+                if (j0 + nb < it[i].l) act.push_back(i);
+            if (act.empty()) continue;
+            for (int pass = 0; pass < 2; ++pass) {
+                moara::GemmBatch b{};
+                b.count = static_cast<int>(act.size());
+                b.B = 1;
+                for (int q = 0; q < b.count; ++q) {
+                    const auto& x = it[act[q]];
+                    const long long l = x.l;
+                    const int j1 = j0 + nb;
+                    moara::GemmProb& p = b.p[q];
+                    p = moara::GemmProb{};
+                    p.lda = p.ldb = p.ldc = x.l;
+                    if (pass == 0) {      // L[j1:, panel] = A[j1:, panel] * Ljj^-T (in place)
+                        p.A = x.Cg + j1 * l + j0;
+                        p.Bm = x.Linv + j0 * l + j0;
+                        p.C = x.Cg + j1 * l + j0;
+                        p.M = x.l - j1; p.N = nb; p.K = nb;
+                    } else {              // A[j1:, j1:] -= L[j1:, panel] L[j1:, panel]^T (lower tiles)
+                        p.A = x.Cg + j1 * l + j0;
+                        p.Bm = x.Cg + j1 * l + j0;
+                        p.C = x.Cg + j1 * l + j1;
+                        p.M = x.l - j1; p.N = x.l - j1; p.K = nb;
+                        p.lower_only = 1;
+                    }
+                }
+                chk(moara::launch_gemm(pass == 0 ? solve : upd, b, s, &ctx->launches));
+            }
+        }
+    }
+
+    void tri_inverse(bool have_diag) {
         int lmax = 0;
         for (auto& x : it) {
-            chk(cudaMemsetAsync(x.Linv, 0, sizeof(float) * (size_t)x.l * x.l, s));
+            if (!have_diag) chk(cudaMemsetAsync(x.Linv, 0, sizeof(float) * (size_t)x.l * x.l, s));
             lmax = std::max(lmax, x.l);
         }
-        moara::SmallBatch sb = small();
-        for (size_t i = 0; i < it.size(); ++i) { sb.l[i] = it[i].l; sb.a[i] = it[i].Cg; sb.c[i] = it[i].Linv; }
-        chk(moara::launch_tri_inverse_diag(sb, s, &ctx->launches));
+        if (!have_diag) {
+            moara::SmallBatch sb = small();
+            for (size_t i = 0; i < it.size(); ++i) { sb.l[i] = it[i].l; sb.a[i] = it[i].Cg; sb.c[i] = it[i].Linv; }
+            chk(moara::launch_tri_inverse_diag(sb, s, &ctx->launches));
+        }
         moara::GemmKind mul{moara::A_KCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
         moara::GemmKind neg{moara::A_KCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE_NEG};
         for (int sz = moara::kTriBase; sz < lmax; sz *= 2) {

@@ -60,7 +60,7 @@ struct DecompBatch {
 
 // ------------------------------------------------------------- SIMT GEMM
 // C (M x N) = op(A) (M x K) * op(B) (K x N), fp32 accumulate.
-enum Epi { EPI_STORE = 0, EPI_ADAM = 1, EPI_UPDATE = 2, EPI_STORE_NEG = 3 };
+enum Epi { EPI_STORE = 0, EPI_ADAM = 1, EPI_UPDATE = 2, EPI_STORE_NEG = 3, EPI_SUB = 4 };
 
 struct GemmProb {
     const void* A;
@@ -75,6 +75,7 @@ struct GemmProb {
     int lda, ldb, ldc;
     int kb;               // blocks per row of the scaled operand / of dM
     int a_bf16, b_bf16;
+    int lower_only;       // skip output tiles strictly above the diagonal
 };
 
 struct GemmBatch {
@@ -116,6 +117,7 @@ struct RefreshItem {
     float* Za; float* Zb;   // n x l
     float* Cg;        // l x l Gram / Cholesky factor
     float* Tt;        // l x l temporary of the blocked triangular inverse
+    float* scal;      // per-problem scalars (diagonal shift)
     float* Linv;      // l x l
     float* Cr;        // l x l Rayleigh-Ritz matrix
     float* Xa; float* Xb;   // l x l
@@ -146,11 +148,14 @@ struct SmallBatch {
 };
 
 cudaError_t launch_philox_gaussian(const SmallBatch& b, cudaStream_t s, int64_t* launches);
-cudaError_t launch_cholesky(const SmallBatch& b, cudaStream_t s, int64_t* launches);
-cudaError_t launch_tri_inverse(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 // Inverts the diagonal blocks [64j, 64j+64) of each lower-triangular a into c.
 constexpr int kTriBase = 64;
 cudaError_t launch_tri_inverse_diag(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+// Blocked Cholesky pieces: the diagonal shift shift_rel*sqrt(rows)*trace(a)
+// into b[0]; and the factorisation of the diagonal block starting at j0
+// (a: matrix, b: shift, c: inverse of the factor's block, written in place).
+cudaError_t launch_trace_shift(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+cudaError_t launch_chol_diag(const SmallBatch& b, int j0, cudaStream_t s, int64_t* launches);
 cudaError_t launch_set_identity(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_ritz_sort(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* launches);

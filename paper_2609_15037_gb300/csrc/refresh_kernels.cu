@@ -1,8 +1,9 @@
 // Small dense kernels of the projector refresh (TruncatedSVD of Algorithm 1
 // computed by randomized subspace iteration): the Gaussian test matrix, the
-// Cholesky factorisation and triangular inverse of CholeskyQR, the ordering of
-// Ritz vectors, and the final sign convention.  One CTA per problem; the
-// problems of a group run side by side in one launch.
+// diagonal blocks of the blocked Cholesky factorisation and of the triangular
+// inverse used by CholeskyQR, the ordering of Ritz vectors, and the final sign
+// convention.  One CTA per problem (or per diagonal block); the problems of a
+// group run side by side in one launch.
 #include <cuda_bf16.h>
 
 #include "internal.h"
@@ -73,14 +74,6 @@ cudaError_t launch_philox_gaussian(const SmallBatch& b, cudaStream_t s, int64_t*
     return cudaGetLastError();
 }
 
-// ---------------------------------------------------------------------------
-// In-place lower Cholesky of a symmetric l x l matrix a (row-major, lower
-// triangle read), with a diagonal shift shift_rel * sqrt(rows) * trace(a)
-// (shifted CholeskyQR: Fukaya, Kannan, Nakatsukasa, Yamamoto, Yanagisawa,
-// SIAM J. Sci. Comput. 2020).  A non-positive or non-finite pivot marks the
-// problem as failed (fail = 1) and is replaced by 1 so the sweep finishes
-// without NaNs.  The strict upper triangle is zeroed.
-// ---------------------------------------------------------------------------
 constexpr int kSmallThreads = 1024;
 
 __device__ float block_sum(float v, float* red) {
@@ -99,107 +92,6 @@ __device__ float block_sum(float v, float* red) {
     }
     __syncthreads();
     return red[32];
-}
-
-__global__ void __launch_bounds__(kSmallThreads) k_cholesky(const __grid_constant__ SmallBatch b) {
-    extern __shared__ float rowj[];          // l floats: row j of L
-    __shared__ float red[33];
-    __shared__ float s_djj;
-    const int pi = blockIdx.x;
-    const int l = b.l[pi];
-    float* A = b.a[pi];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-
-    float tr = 0.0f;
-    for (int i = threadIdx.x; i < l; i += blockDim.x) tr += A[(long long)i * l + i];
-    tr = block_sum(tr, red);
-    const float shift = b.shift_rel * sqrtf(static_cast<float>(b.rows[pi])) * tr;
-    int failed = 0;
-
-    for (int j = 0; j < l; ++j) {
-        // row j of L (k < j) into shared memory, partial sum of squares
-        float ss = 0.0f;
-        for (int k = threadIdx.x; k < j; k += blockDim.x) {
-            const float v = A[(long long)j * l + k];
-            rowj[k] = v;
-            ss = fmaf(v, v, ss);
-        }
-        ss = block_sum(ss, red);
-        if (threadIdx.x == 0) {
-            float d = A[(long long)j * l + j] + shift - ss;
-            if (!(d > 0.0f) || !isfinite(d)) { d = 1.0f; failed = 1; }
-            d = sqrtf(d);
-            A[(long long)j * l + j] = d;
-            s_djj = d;
-        }
-        __syncthreads();
-        const float djj = s_djj;
-        for (int i = j + 1 + warp; i < l; i += nw) {
-            const float* Li = A + (long long)i * l;
-            float dot = 0.0f;
-            for (int k = lane; k < j; k += 32) dot = fmaf(Li[k], rowj[k], dot);
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
-            if (lane == 0) A[(long long)i * l + j] = (Li[j] - dot) / djj;
-        }
-        __syncthreads();
-    }
-    for (int i = 0; i < l; ++i)
-        for (int k = i + 1 + threadIdx.x; k < l; k += blockDim.x) A[(long long)i * l + k] = 0.0f;
-    if (threadIdx.x == 0 && failed && b.fail[pi] != nullptr) *b.fail[pi] = 1;
-}
-
-cudaError_t launch_cholesky(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
-    if (b.count <= 0) return cudaSuccess;
-    int lmax = 1;
-    for (int i = 0; i < b.count; ++i) lmax = b.l[i] > lmax ? b.l[i] : lmax;
-    const size_t smem = sizeof(float) * lmax;
-    if (smem > 48 * 1024) {
-        cudaFuncSetAttribute(k_cholesky, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    }
-    k_cholesky<<<b.count, kSmallThreads, smem, s>>>(b);
-    ++*launches;
-    return cudaGetLastError();
-}
-
-// ---------------------------------------------------------------------------
-// Inverse of a lower-triangular l x l matrix (a -> c), row by row:
-// Linv[i][c] = (delta_ic - sum_{c <= k < i} L[i][k] Linv[k][c]) / L[i][i].
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kSmallThreads) k_tri_inverse(const __grid_constant__ SmallBatch b) {
-    extern __shared__ float rowi[];
-    const int pi = blockIdx.x;
-    const int l = b.l[pi];
-    const float* L = b.a[pi];
-    float* X = b.c[pi];
-    for (int i = 0; i < l; ++i) {
-        for (int k = threadIdx.x; k <= i; k += blockDim.x) rowi[k] = L[(long long)i * l + k];
-        __syncthreads();
-        const float dinv = 1.0f / rowi[i];
-        for (int c = threadIdx.x; c < l; c += blockDim.x) {
-            float v = 0.0f;
-            if (c <= i) {
-                float acc = (c == i) ? 1.0f : 0.0f;
-                for (int k = c; k < i; ++k) acc = fmaf(-rowi[k], X[(long long)k * l + c], acc);
-                v = acc * dinv;
-            }
-            X[(long long)i * l + c] = v;
-        }
-        __syncthreads();
-    }
-}
-
-cudaError_t launch_tri_inverse(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
-    if (b.count <= 0) return cudaSuccess;
-    int lmax = 1;
-    for (int i = 0; i < b.count; ++i) lmax = b.l[i] > lmax ? b.l[i] : lmax;
-    const size_t smem = sizeof(float) * lmax;
-    if (smem > 48 * 1024) {
-        cudaFuncSetAttribute(k_tri_inverse, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    }
-    k_tri_inverse<<<b.count, kSmallThreads, smem, s>>>(b);
-    ++*launches;
-    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------
@@ -250,6 +142,100 @@ cudaError_t launch_tri_inverse_diag(const SmallBatch& b, cudaStream_t s, int64_t
     for (int i = 0; i < b.count; ++i) lmax = b.l[i] > lmax ? b.l[i] : lmax;
     dim3 grid((lmax + kTriBase - 1) / kTriBase, b.count);
     k_tri_inverse_diag<<<grid, 256, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Blocked right-looking Cholesky.  k_trace_shift stores the diagonal shift of
+// the shifted CholeskyQR pass; k_chol_diag factors the (at most 64 x 64)
+// diagonal block at j0 in shared memory after the trailing updates of the
+// earlier panels, checks its pivots, writes the factor in place and its
+// inverse into the same block of c (the diagonal blocks of the triangular
+// inverse).  The panel below the block and the trailing matrix are updated by
+// grouped GEMMs on the host side.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_trace_shift(const __grid_constant__ SmallBatch b) {
+    __shared__ float red[33];
+    const int pi = blockIdx.x;
+    const int l = b.l[pi];
+    const float* A = b.a[pi];
+    float tr = 0.0f;
+    for (int i = threadIdx.x; i < l; i += blockDim.x) tr += A[(long long)i * l + i];
+    tr = block_sum(tr, red);
+    if (threadIdx.x == 0) b.b[pi][0] = b.shift_rel * sqrtf(static_cast<float>(b.rows[pi])) * tr;
+}
+
+cudaError_t launch_trace_shift(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    k_trace_shift<<<b.count, 256, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+__global__ void __launch_bounds__(256) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
+    __shared__ float Ls[kTriBase][kTriBase + 1];
+    __shared__ float Xs[kTriBase][kTriBase + 1];
+    __shared__ int s_fail;
+    const int pi = blockIdx.x;
+    const int l = b.l[pi];
+    if (j0 >= l) return;
+    const int sz = min(kTriBase, l - j0);
+    float* A = b.a[pi];
+    float* X = b.c[pi];
+    const float shift = b.b[pi][0];
+    if (threadIdx.x == 0) s_fail = 0;
+    for (int e = threadIdx.x; e < sz * sz; e += blockDim.x) {
+        const int i = e / sz, c = e - i * sz;
+        float v = A[(long long)(j0 + i) * l + j0 + c];
+        if (i == c) v += shift;
+        Ls[i][c] = v;
+    }
+    __syncthreads();
+    // column-by-column Cholesky of the block (lower triangle)
+    for (int j = 0; j < sz; ++j) {
+        if (threadIdx.x == 0) {
+            float d = Ls[j][j];
+            if (!(d > 0.0f) || !isfinite(d)) { d = 1.0f; s_fail = 1; }
+            Ls[j][j] = sqrtf(d);
+        }
+        __syncthreads();
+        const float djj = Ls[j][j];
+        for (int i = j + 1 + threadIdx.x; i < sz; i += blockDim.x) Ls[i][j] /= djj;
+        __syncthreads();
+        // trailing update of the block: rows/cols > j
+        const int rem = sz - j - 1;
+        for (int e = threadIdx.x; e < rem * rem; e += blockDim.x) {
+            const int i = j + 1 + e / rem, c = j + 1 + e % rem;
+            if (c <= i) Ls[i][c] = fmaf(-Ls[i][j], Ls[c][j], Ls[i][c]);
+        }
+        __syncthreads();
+    }
+    // inverse of the block factor, row by row (thread c owns column c)
+    for (int i = 0; i < sz; ++i) {
+        if (threadIdx.x < sz) {
+            const int c = threadIdx.x;
+            float v = 0.0f;
+            if (c <= i) {
+                float acc = (c == i) ? 1.0f : 0.0f;
+                for (int k = c; k < i; ++k) acc = fmaf(-Ls[i][k], Xs[k][c], acc);
+                v = acc / Ls[i][i];
+            }
+            Xs[i][c] = v;
+        }
+        __syncthreads();
+    }
+    for (int e = threadIdx.x; e < sz * sz; e += blockDim.x) {
+        const int i = e / sz, c = e - i * sz;
+        A[(long long)(j0 + i) * l + j0 + c] = (c <= i) ? Ls[i][c] : 0.0f;
+        X[(long long)(j0 + i) * l + j0 + c] = Xs[i][c];
+    }
+    if (threadIdx.x == 0 && s_fail && b.fail[pi] != nullptr) *b.fail[pi] = 1;
+}
+
+cudaError_t launch_chol_diag(const SmallBatch& b, int j0, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    k_chol_diag<<<b.count, 256, 0, s>>>(b, j0);
     ++*launches;
     return cudaGetLastError();
 }

@@ -195,6 +195,8 @@ __device__ __forceinline__ void epilogue(const GemmBatch& b, const GemmProb& p, 
         p.C[o] = acc;
     } else if (EPI == EPI_STORE_NEG) {
         p.C[o] = -acc;
+    } else if (EPI == EPI_SUB) {
+        p.C[o] = p.C[o] - acc;
     } else if (EPI == EPI_ADAM) {
         // Optimizer_V (Algorithm 1): Adam on the projected direction R = acc.
         float ea = b.beta1 * p.aux0[o] + (1.0f - b.beta1) * acc;
@@ -227,6 +229,7 @@ __global__ void __launch_bounds__(256) k_gemm(const __grid_constant__ GemmBatch 
     const int tn = b.tiles_n[lo];
     const int m0 = (local / tn) * TM;
     const int n0 = (local % tn) * TN;
+    if (p.lower_only && n0 >= m0 + TM) return;
 
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     float acc[8][8];
@@ -322,6 +325,7 @@ cudaError_t launch_gemm(const GemmKind& k, GemmBatch& b, cudaStream_t s, int64_t
     MOARA_GEMM_CASE(A_KCONTIG, false, false, B_NCONTIG, false, false, EPI_STORE)
     MOARA_GEMM_CASE(A_KCONTIG, false, false, B_KCONTIG, false, false, EPI_STORE)
     MOARA_GEMM_CASE(A_KCONTIG, false, false, B_NCONTIG, false, false, EPI_STORE_NEG)
+    MOARA_GEMM_CASE(A_KCONTIG, false, false, B_KCONTIG, false, false, EPI_SUB)
 #undef MOARA_GEMM_CASE
     return cudaErrorInvalidValue;
 }

@@ -56,18 +56,18 @@ constexpr int K1_B_BYTES = K1_BK * K1_BN * 2;           // 16 KB: two 64-column 
 // stage: A | B (G, then V_hi after the transform) | V_lo (V - V_hi in bf16)
 constexpr int K1_STAGE_BYTES = K1_A_BYTES + 2 * K1_B_BYTES;
 constexpr int K1_TX_BYTES = K1_A_BYTES + K1_B_BYTES;    // bytes the TMA brings per stage
-constexpr int K1_WARPS = 14;                            // 0 TMA, 1 MMA, 2-5 transform, 6-13 epilogue
+constexpr int K1_WARPS = 18;                            // 0 TMA, 1 MMA, 2-9 transform, 10-17 epilogue
 constexpr int K1_THREADS = K1_WARPS * 32;
 constexpr int GUARD_BYTES = 16384;
 constexpr int K1_SMEM = 1024 + K1_STAGES * K1_STAGE_BYTES + GUARD_BYTES + 2048;
 
 struct K1Params {
     CUtensorMap gmap[kTcGroup];        // G of each launch slot: dims {n, m}, box {64, 64}
+    const int* cta_start;              // tiles of CTA c: tiles[cta_start[c] .. cta_start[c+1])
     const TcTile* tiles;
     const TcMod* mods;
     const CUtensorMap* maps;           // per module: [0] P for K1, [1] P for K2, [2] N for K2
     int* status;
-    int n_tiles;
     float beta1, beta2, adam_eps, bc1, bc2, decomp_eps;
 };
 
@@ -76,16 +76,16 @@ constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64, K2_STAGES = 4;
 constexpr int K2_A_BYTES = K2_BM * K2_BK * 2;           // 16 KB: P rows, K-major
 constexpr int K2_B_BYTES = K2_BK * K2_BN * 2;           // 32 KB: four 64-column chunks of N
 constexpr int K2_STAGE_BYTES = K2_A_BYTES + K2_B_BYTES;
-constexpr int K2_WARPS = 10;                            // 0 TMA, 1 MMA, 2-9 epilogue
+constexpr int K2_WARPS = 18;                            // 0 TMA, 1 MMA, 2-17 epilogue
 constexpr int K2_THREADS = K2_WARPS * 32;
 constexpr int K2_SMEM = 1024 + K2_STAGES * K2_STAGE_BYTES + GUARD_BYTES + 2048;
 
 struct K2Params {
+    const int* cta_start;
     const TcTile* tiles;
     const TcMod* mods;
     const CUtensorMap* maps;
     int* status;
-    int n_tiles;
     float step_scale;                  // lr * alpha
     int decompose;
 };
@@ -137,7 +137,7 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
     if (threadIdx.x == 0) {
         for (int s = 0; s < K1_STAGES; ++s) {
             ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->xform[s]), 128);
+            ptx::mbar_init(ptx::smem_u32(&ctl->xform[s]), 256);
             ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -164,9 +164,9 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
             uint32_t phase = 0;
             uint32_t issued = 0, last_par = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
                 const TcTile tl = p.tiles[t];
-                const TcMod md = p.mods[tl.mod];
+                const TcMod& md = p.mods[tl.mod];
                 const CUtensorMap* pmap = &p.maps[tl.mod * 3 + 0];
                 const CUtensorMap* gmap = &p.gmap[tl.slot];
                 const int r0 = tl.t0 * K1_BM, n0 = tl.t1 * K1_BN;
@@ -201,9 +201,9 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
             int buf = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
                 const TcTile tl = p.tiles[t];
-                const TcMod md = p.mods[tl.mod];
+                const TcMod& md = p.mods[tl.mod];
                 const int r0 = tl.t0 * K1_BM;
                 const int nh = (r0 + 128 < md.r) ? 2 : 1;
                 const int nk = (md.m + K1_BK - 1) / K1_BK;
@@ -243,55 +243,67 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
             ptx::mma_commit(ptx::smem_u32(&ctl->drain));
             wait_drain(ptx::smem_u32(&ctl->drain), 0);
         }
-    } else if (warp < 6) {
+    } else if (warp < 10) {
         // ------------------------------------------------- transform warps
         if (DECOMP) {
-            const int tid = threadIdx.x - 64;           // 0..127
-            const int k = tid >> 1;                     // row within the stage
-            const int hc = tid & 1;                     // 64-column chunk (partner: lane ^ 1)
+            // 256 threads: lane bits 0-2 = row within an 8-row group, bit 3 = unit
+            // half (16-byte units 0-3 or 4-7 of the 128-byte row), bit 4 =
+            // 64-column chunk, warp = 8-row group.  Each quarter-warp then touches
+            // 8 distinct rows of one chunk (conflict-free under the 128-byte
+            // swizzle); the threads sharing a block are lanes ^ 8 and ^ 16.
+            const int tid = threadIdx.x - 64;           // 0..255
+            const int k = ((tid >> 5) << 3) | (tid & 7);  // row within the stage (0..63)
+            const int hu = (tid >> 3) & 1;              // unit half
+            const int hc = (tid >> 4) & 1;              // 64-column chunk
             const uint32_t x = static_cast<uint32_t>(k & 7);
             constexpr int UB = BLK / 8;                 // 16-byte units per block
-            constexpr int NBT = UB <= 8 ? 8 / UB : 1;   // blocks held by this thread
+            constexpr int UPB = UB < 4 ? UB : 4;        // units of a block held by this thread
+            constexpr int NBT = 4 / UPB;                // blocks (or block parts) per thread
             int stage = 0;
             uint32_t phase = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
                 const TcTile tl = p.tiles[t];
-                const TcMod md = p.mods[tl.mod];
+                const TcMod& md = p.mods[tl.mod];
                 const int n0 = tl.t1 * K1_BN;
                 const bool do_mag = (tl.t0 == 0);
-                const int nk = (md.m + K1_BK - 1) / K1_BK;
+                const int mm = md.m, mkb = md.kb;
+                float* const mag_avg = md.mag_avg;
+                float* const mag_avg_sq = md.mag_avg_sq;
+                float* const dMp = md.dM;
+                const int nk = (mm + K1_BK - 1) / K1_BK;
                 for (int kb = 0; kb < nk; ++kb) {
-                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
-                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
+                                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+                    if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
                     uint8_t* row = smem + stage * K1_STAGE_BYTES + K1_A_BYTES + hc * 8192 + k * 128;
-                    uint4 d[8];
+                    uint4 d[4];
 #pragma unroll
-                    for (int u = 0; u < 8; ++u) d[u] = *reinterpret_cast<const uint4*>(row + ((u ^ x) << 4));
-                    float ssu[8];
+                    for (int u = 0; u < 4; ++u)
+                        d[u] = *reinterpret_cast<const uint4*>(row + (((hu * 4 + u) ^ x) << 4));
+                    float ssu[4];
 #pragma unroll
-                    for (int u = 0; u < 8; ++u) {
+                    for (int u = 0; u < 4; ++u) {
                         const uint32_t w[4] = {d[u].x, d[u].y, d[u].z, d[u].w};
-                        float s = 0.0f;
+                        float s2 = 0.0f;
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
                             const float lo = bf_lo(w[e]), hi = bf_hi(w[e]);
-                            s = fmaf(lo, lo, s);
-                            s = fmaf(hi, hi, s);
+                            s2 = fmaf(lo, lo, s2);
+                            s2 = fmaf(hi, hi, s2);
                         }
-                        ssu[u] = s;
+                        ssu[u] = s2;
                     }
                     float ssb[NBT];
 #pragma unroll
                     for (int bl = 0; bl < NBT; ++bl) {
-                        float s = 0.0f;
+                        float s2 = 0.0f;
 #pragma unroll
-                        for (int u = 0; u < (UB <= 8 ? UB : 8); ++u) s += ssu[bl * (UB <= 8 ? UB : 8) + u];
-                        ssb[bl] = s;
+                        for (int u = 0; u < UPB; ++u) s2 += ssu[bl * UPB + u];
+                        ssb[bl] = s2;
                     }
-                    if (UB > 8) {   // B = 128: the block spans both chunks; the partner is lane ^ 1
-                        ssb[0] += __shfl_xor_sync(0xffffffffu, ssb[0], 1);
-                    }
+                    if (UB >= 8) ssb[0] += __shfl_xor_sync(0xffffffffu, ssb[0], 8);    // other unit half
+                    if (UB >= 16) ssb[0] += __shfl_xor_sync(0xffffffffu, ssb[0], 16);  // other chunk
                     float inv[NBT];
                     float mag[NBT];
 #pragma unroll
@@ -301,8 +313,8 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
                     }
                     uint8_t* lrow = row + K1_B_BYTES;
 #pragma unroll
-                    for (int u = 0; u < 8; ++u) {
-                        const float sc = inv[UB <= 8 ? u / UB : 0];
+                    for (int u = 0; u < 4; ++u) {
+                        const float sc = inv[u / UPB];
                         const uint32_t w[4] = {d[u].x, d[u].y, d[u].z, d[u].w};
                         uint32_t hi[4], lo[4];
 #pragma unroll
@@ -311,7 +323,7 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
                             hi[e] = pack_bf16x2(v0, v1);
                             lo[e] = pack_bf16x2(v0 - bf_lo(hi[e]), v1 - bf_hi(hi[e]));
                         }
-                        const uint32_t off = (u ^ x) << 4;
+                        const uint32_t off = ((hu * 4 + u) ^ x) << 4;
                         *reinterpret_cast<uint4*>(row + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
                         *reinterpret_cast<uint4*>(lrow + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
                     }
@@ -319,17 +331,18 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
                     ptx::mbar_arrive(ptx::smem_u32(&ctl->xform[stage]));
                     // Optimizer_M on the block magnitudes, once per (row, block)
                     const int grow = kb * K1_BK + k;
-                    if (do_mag && grow < md.m && (UB <= 8 || hc == 0)) {
+                    const bool owner = (UB < 8) || (hu == 0 && (UB < 16 || hc == 0));
+                    if (do_mag && owner && grow < mm) {
 #pragma unroll
                         for (int bl = 0; bl < NBT; ++bl) {
-                            const int gb = (n0 + hc * 64) / BLK + bl;
-                            if (gb < md.kb) {
-                                const long long o = (long long)grow * md.kb + gb;
-                                const float ma = p.beta1 * md.mag_avg[o] + (1.0f - p.beta1) * mag[bl];
-                                const float mas = p.beta2 * md.mag_avg_sq[o] + (1.0f - p.beta2) * mag[bl] * mag[bl];
-                                md.mag_avg[o] = ma;
-                                md.mag_avg_sq[o] = mas;
-                                md.dM[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
+                            const int gb = (n0 + hc * 64 + hu * 32) / BLK + (UB < 8 ? bl : 0);
+                            if (gb < mkb) {
+                                const long long o = (long long)grow * mkb + gb;
+                                const float ma = p.beta1 * mag_avg[o] + (1.0f - p.beta1) * mag[bl];
+                                const float mas = p.beta2 * mag_avg_sq[o] + (1.0f - p.beta2) * mag[bl] * mag[bl];
+                                mag_avg[o] = ma;
+                                mag_avg_sq[o] = mas;
+                                dMp[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
                             }
                         }
                     }
@@ -339,18 +352,19 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
         }
     } else {
         // ------------------------------------------------- epilogue warps
-        const int ew = warp - 6;                       // 0..7
+        const int ew = warp - 10;                      // 0..7
         const int q = warp & 3;                        // TMEM lane quarter of this warp
         const int h = ew >> 2;                         // accumulator half (rows 0-127 / 128-255)
         int buf = 0;
         uint32_t acc_phase = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+        for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
             const TcTile tl = p.tiles[t];
-            const TcMod md = p.mods[tl.mod];
+            const TcMod& md = p.mods[tl.mod];
             const int r0 = tl.t0 * K1_BM, n0 = tl.t1 * K1_BN;
-            if (!ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
-                                MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+            const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
+                                            MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+            if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
             ptx::tc_fence_after();
             const bool half_valid = (r0 + h * 128) < md.r;
             if (half_valid) {
@@ -393,7 +407,9 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
                         n4[0] = make_uint4(nb[0], nb[1], nb[2], nb[3]);
                         n4[1] = make_uint4(nb[4], nb[5], nb[6], nb[7]);
                     } else {
-                        for (int e = 0; e < 16 && j0 + e < md.n; ++e) {
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            if (j0 + e >= md.n) continue;
                             const float ea = p.beta1 * md.exp_avg[o + e] + (1.0f - p.beta1) * v[e];
                             const float es = p.beta2 * md.exp_avg_sq[o + e] + (1.0f - p.beta2) * v[e] * v[e];
                             md.exp_avg[o + e] = ea;
@@ -438,7 +454,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
         }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(ptx::smem_u32(&ctl->accf[b]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 8);
+            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 16);
         }
         ptx::mbar_init(ptx::smem_u32(&ctl->drain), 1);
         ctl->abort = 0;
@@ -459,9 +475,9 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             uint32_t phase = 0;
             uint32_t issued = 0, last_par = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
                 const TcTile tl = p.tiles[t];
-                const TcMod md = p.mods[tl.mod];
+                const TcMod& md = p.mods[tl.mod];
                 const CUtensorMap* amap = &p.maps[tl.mod * 3 + 1];
                 const CUtensorMap* bmap = &p.maps[tl.mod * 3 + 2];
                 const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
@@ -494,9 +510,9 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             int buf = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
                 const TcTile tl = p.tiles[t];
-                const TcMod md = p.mods[tl.mod];
+                const TcMod& md = p.mods[tl.mod];
                 const int nk = (md.r + K2_BK - 1) / K2_BK;
                 if (!ptx::mbar_wait(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
                                     MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
@@ -525,39 +541,51 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             wait_drain(ptx::smem_u32(&ctl->drain), 0);
         }
     } else {
-        const int ew = warp - 2;                        // 0..7
+        // 16 epilogue warps: lane quarter q = warp % 4, column quarter cq
+        // (64 of the 256 columns, 4 chunks of 16).  W of the next chunk is
+        // loaded while the current one is updated.
+        const int ew = warp - 2;                        // 0..15
         const int q = warp & 3;
-        const int ch = ew >> 2;                         // column half of the 256-wide tile
+        const int cq = ew >> 2;
         int buf = 0;
         uint32_t acc_phase = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+        for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
             const TcTile tl = p.tiles[t];
-            const TcMod md = p.mods[tl.mod];
+            const TcMod& md = p.mods[tl.mod];
+            const int mm = md.m, nn = md.n, mkb = md.kb;
+            float* const Wp = md.W;
+            const float* const dMp = md.dM;
             const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
-            if (!ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
-                                MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
-            ptx::tc_fence_after();
             const int i = i0 + q * 32 + lane;
-            const bool row_ok = i < md.m;
+            const bool row_ok = i < mm;
+            const int jbase = n0 + cq * 64;
+            // prefetch W of the first chunk before waiting for the accumulator
+            float4 wn0 = make_float4(0.f, 0.f, 0.f, 0.f), wn1 = wn0, wn2 = wn0, wn3 = wn0;
+            if (row_ok && jbase + 16 <= nn) {
+                const float4* w4 = reinterpret_cast<const float4*>(Wp + (long long)i * nn + jbase);
+                wn0 = w4[0]; wn1 = w4[1]; wn2 = w4[2]; wn3 = w4[3];
+            }
+            const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
+                                            MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+            if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
+            ptx::tc_fence_after();
 #pragma unroll 1
-            for (int c = 0; c < 8; ++c) {
-                const int cc = ch * 128 + c * 16;
+            for (int c = 0; c < 4; ++c) {
+                const int j0 = jbase + c * 16;
+                float w[16] = {wn0.x, wn0.y, wn0.z, wn0.w, wn1.x, wn1.y, wn1.z, wn1.w,
+                               wn2.x, wn2.y, wn2.z, wn2.w, wn3.x, wn3.y, wn3.z, wn3.w};
+                if (c + 1 < 4 && row_ok && j0 + 32 <= nn) {
+                    const float4* w4 = reinterpret_cast<const float4*>(Wp + (long long)i * nn + j0 + 16);
+                    wn0 = w4[0]; wn1 = w4[1]; wn2 = w4[2]; wn3 = w4[3];
+                }
                 float v[16];
                 __syncwarp();
-                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + cc, v);
-                const int j0 = n0 + cc;
-                if (!row_ok || j0 >= md.n) continue;
-                const long long o = (long long)i * md.n + j0;
-                const float* dmr = md.dM + (long long)i * md.kb;
-                if (j0 + 16 <= md.n) {
-                    float4* w4 = reinterpret_cast<float4*>(md.W + o);
-                    float w[16];
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float4 x = w4[e];
-                        w[4 * e] = x.x; w[4 * e + 1] = x.y; w[4 * e + 2] = x.z; w[4 * e + 3] = x.w;
-                    }
+                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + cq * 64 + c * 16, v);
+                if (!row_ok || j0 >= nn) continue;
+                const long long o = (long long)i * nn + j0;
+                const float* dmr = dMp + (long long)i * mkb;
+                if (j0 + 16 <= nn) {
                     if (p.decompose) {
                         if (BLK >= 16) {
                             const float dm = dmr[j0 / BLK];
@@ -571,12 +599,16 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
 #pragma unroll
                         for (int e = 0; e < 16; ++e) w[e] -= p.step_scale * v[e];
                     }
+                    float4* w4 = reinterpret_cast<float4*>(Wp + o);
 #pragma unroll
                     for (int e = 0; e < 4; ++e) w4[e] = make_float4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
                 } else {
-                    for (int e = 0; e < 16 && j0 + e < md.n; ++e) {
-                        const float u = p.decompose ? dmr[(j0 + e) / BLK] * v[e] : v[e];
-                        md.W[o + e] -= p.step_scale * u;
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        if (j0 + e < nn) {
+                            const float u = p.decompose ? dmr[(j0 + e) / BLK] * v[e] : v[e];
+                            Wp[o + e] -= p.step_scale * u;
+                        }
                     }
                 }
             }
@@ -632,7 +664,12 @@ struct TcState {
     CUtensorMap* d_maps = nullptr;
     int cap = 0;
     bool dirty = false;
-    struct Tiles { TcTile* k1 = nullptr; int n1 = 0; TcTile* k2 = nullptr; int n2 = 0; };
+    // Per-CTA work lists of one launch (CSR: start offsets, then tiles).
+    struct Tiles {
+        void* mem = nullptr;
+        const int* k1_start = nullptr; const TcTile* k1 = nullptr; int g1 = 0;
+        const int* k2_start = nullptr; const TcTile* k2 = nullptr; int g2 = 0;
+    };
     std::map<std::vector<int>, Tiles> tiles;
     bool attrs_set = false;
     K1Params p1;                           // parameter block of the next K1 launch
@@ -674,10 +711,8 @@ void tc_destroy(TcState* st) {
     if (st == nullptr) return;
     if (st->d_mods) cudaFree(st->d_mods);
     if (st->d_maps) cudaFree(st->d_maps);
-    for (auto& kv : st->tiles) {
-        if (kv.second.k1) cudaFree(kv.second.k1);
-        if (kv.second.k2) cudaFree(kv.second.k2);
-    }
+    for (auto& kv : st->tiles)
+        if (kv.second.mem) cudaFree(kv.second.mem);
     delete st;
 }
 
@@ -733,42 +768,90 @@ static int tc_upload(TcState* st) {
     return MOARA_OK;
 }
 
-// Work lists of one launch: K1 tiles (rank tile x 128-column strip) and K2
-// tiles (128-row tile x 256-column strip), longest reduction first; the rank
-// tiles of one column strip stay adjacent so they share the strip of G in L2.
+// Longest-processing-time assignment of weighted tiles to `grid` persistent
+// CTAs: tiles in descending cost, each to the CTA with the least work so far;
+// each CTA runs its tiles in that (descending) order.
+static void lpt_assign(const std::vector<TcTile>& tiles, const std::vector<double>& cost, int grid,
+                       std::vector<int>& start, std::vector<TcTile>& out) {
+    std::vector<int> order(tiles.size());
+    for (size_t i = 0; i < order.size(); ++i) order[i] = static_cast<int>(i);
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return cost[a] > cost[b]; });
+    std::vector<std::vector<int>> per(grid);
+    std::vector<std::pair<double, int>> heap;
+    for (int c = 0; c < grid; ++c) heap.push_back({0.0, c});
+    auto cmp = [](const std::pair<double, int>& a, const std::pair<double, int>& b) {
+        return a.first > b.first || (a.first == b.first && a.second > b.second);
+    };
+    std::make_heap(heap.begin(), heap.end(), cmp);
+    for (int i : order) {
+        std::pop_heap(heap.begin(), heap.end(), cmp);
+        auto& top = heap.back();
+        per[top.second].push_back(i);
+        top.first += cost[i];
+        std::push_heap(heap.begin(), heap.end(), cmp);
+    }
+    start.assign(grid + 1, 0);
+    out.clear();
+    for (int c = 0; c < grid; ++c) {
+        start[c] = static_cast<int>(out.size());
+        for (int i : per[c]) out.push_back(tiles[i]);
+    }
+    start[grid] = static_cast<int>(out.size());
+}
+
+// Work lists of one launch: K1 tiles (256-rank x 128-column) and K2 tiles
+// (128-row x 256-column), cost-weighted (MMA clocks vs. epilogue traffic).
 static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
     auto it = st->tiles.find(ids);
     if (it != st->tiles.end()) return &it->second;
     std::vector<TcTile> k1, k2;
-    std::vector<int> order(ids.size());
-    for (size_t i = 0; i < ids.size(); ++i) order[i] = static_cast<int>(i);
-    std::stable_sort(order.begin(), order.end(),
-                     [&](int a, int b) { return st->mods[ids[a]].m > st->mods[ids[b]].m; });
-    for (int slot : order) {
+    std::vector<double> c1, c2;
+    for (size_t slot = 0; slot < ids.size(); ++slot) {
         const TcMod& md = st->mods[ids[slot]];
         const int nt = (md.n + K1_BN - 1) / K1_BN, rt = (md.r + K1_BM - 1) / K1_BM;
         for (int j = 0; j < nt; ++j)
-            for (int i = 0; i < rt; ++i) k1.push_back({ids[slot], slot, i, j});
-    }
-    std::stable_sort(order.begin(), order.end(),
-                     [&](int a, int b) { return st->mods[ids[a]].r > st->mods[ids[b]].r; });
-    for (int slot : order) {
-        const TcMod& md = st->mods[ids[slot]];
-        const int mt = (md.m + K2_BM - 1) / K2_BM, nt = (md.n + K2_BN - 1) / K2_BN;
+            for (int i = 0; i < rt; ++i) {
+                const int rows = std::min(K1_BM, md.r - i * K1_BM);
+                const int nh = rows > 128 ? 2 : 1;
+                const double mma = 8.0 * nh * md.m;                       // clocks, with V_lo
+                const double epi = 0.8 * rows * std::min(K1_BN, md.n - j * K1_BN);
+                k1.push_back({ids[slot], static_cast<int>(slot), i, j});
+                c1.push_back(std::max(mma, epi));
+            }
+        const int mt = (md.m + K2_BM - 1) / K2_BM, nt2 = (md.n + K2_BN - 1) / K2_BN;
         for (int i = 0; i < mt; ++i)
-            for (int j = 0; j < nt; ++j) k2.push_back({ids[slot], slot, i, j});
+            for (int j = 0; j < nt2; ++j) {
+                const double mma = 8.0 * md.r;
+                const double epi = 0.36 * std::min(K2_BM, md.m - i * K2_BM) * std::min(K2_BN, md.n - j * K2_BN);
+                k2.push_back({ids[slot], static_cast<int>(slot), i, j});
+                c2.push_back(std::max(mma, epi));
+            }
     }
     TcState::Tiles t;
-    t.n1 = static_cast<int>(k1.size());
-    t.n2 = static_cast<int>(k2.size());
-    if (cudaMalloc(&t.k1, sizeof(TcTile) * std::max(1, t.n1)) != cudaSuccess ||
-        cudaMalloc(&t.k2, sizeof(TcTile) * std::max(1, t.n2)) != cudaSuccess ||
-        cudaMemcpy(t.k1, k1.data(), sizeof(TcTile) * t.n1, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(t.k2, k2.data(), sizeof(TcTile) * t.n2, cudaMemcpyHostToDevice) != cudaSuccess) {
-        if (t.k1) cudaFree(t.k1);
-        if (t.k2) cudaFree(t.k2);
+    t.g1 = std::max(1, std::min(static_cast<int>(k1.size()), st->sms));
+    t.g2 = std::max(1, std::min(static_cast<int>(k2.size()), st->sms));
+    std::vector<int> s1, s2;
+    std::vector<TcTile> o1, o2;
+    lpt_assign(k1, c1, t.g1, s1, o1);
+    lpt_assign(k2, c2, t.g2, s2, o2);
+    auto pad = [](size_t b) { return (b + 255) / 256 * 256; };
+    const size_t b_s1 = pad(sizeof(int) * s1.size()), b_o1 = pad(sizeof(TcTile) * std::max<size_t>(1, o1.size()));
+    const size_t b_s2 = pad(sizeof(int) * s2.size()), b_o2 = pad(sizeof(TcTile) * std::max<size_t>(1, o2.size()));
+    std::vector<char> host(b_s1 + b_o1 + b_s2 + b_o2, 0);
+    std::memcpy(host.data(), s1.data(), sizeof(int) * s1.size());
+    std::memcpy(host.data() + b_s1, o1.data(), sizeof(TcTile) * o1.size());
+    std::memcpy(host.data() + b_s1 + b_o1, s2.data(), sizeof(int) * s2.size());
+    std::memcpy(host.data() + b_s1 + b_o1 + b_s2, o2.data(), sizeof(TcTile) * o2.size());
+    if (cudaMalloc(&t.mem, host.size()) != cudaSuccess) return nullptr;
+    if (cudaMemcpy(t.mem, host.data(), host.size(), cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaFree(t.mem);
         return nullptr;
     }
+    char* base = static_cast<char*>(t.mem);
+    t.k1_start = reinterpret_cast<const int*>(base);
+    t.k1 = reinterpret_cast<const TcTile*>(base + b_s1);
+    t.k2_start = reinterpret_cast<const int*>(base + b_s1 + b_o1);
+    t.k2 = reinterpret_cast<const TcTile*>(base + b_s1 + b_o1 + b_s2);
     return &(st->tiles[ids] = t);
 }
 
@@ -815,17 +898,17 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
                 return MOARA_ERR_CUDA;
             }
         }
-        p1.tiles = tl->k1; p1.mods = st->d_mods; p1.maps = st->d_maps; p1.status = st->d_status;
-        p1.n_tiles = tl->n1;
+        p1.cta_start = tl->k1_start; p1.tiles = tl->k1;
+        p1.mods = st->d_mods; p1.maps = st->d_maps; p1.status = st->d_status;
         p1.beta1 = hp.beta1; p1.beta2 = hp.beta2; p1.adam_eps = hp.adam_eps;
         p1.bc1 = bc1; p1.bc2 = bc2; p1.decomp_eps = hp.decomp_eps;
         K2Params p2{};
-        p2.tiles = tl->k2; p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;
-        p2.n_tiles = tl->n2;
+        p2.cta_start = tl->k2_start; p2.tiles = tl->k2;
+        p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;
         p2.step_scale = lr * hp.scale;
         p2.decompose = hp.decompose;
-        const int g1 = std::max(1, std::min(tl->n1, st->sms));
-        const int g2 = std::max(1, std::min(tl->n2, st->sms));
+        const int g1 = tl->g1;
+        const int g2 = tl->g2;
         const bool dec = hp.decompose != 0;
         cudaError_t e;
         switch (B) {
