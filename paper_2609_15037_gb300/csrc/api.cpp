@@ -935,7 +935,8 @@ int moara_step_grouped(moara_ctx* ctx, int n_mod, const int* ids, const void* co
             }
         }, ctx};
         rc = moara::tc_step(ctx->tc, ctx->hp, static_cast<int>(mids.size()), mids.data(), gp.data(),
-                            static_cast<float>(bc1), static_cast<float>(bc2), lr, s, &ctx->launches, tp);
+                            static_cast<float>(bc1), static_cast<float>(bc2), lr, t == 1 ? 1 : 0, s,
+                            &ctx->launches, tp);
         if (rc != MOARA_OK) return fail(ctx, rc, "tensor-core step launch failed: %s", moara::tc_last_error(ctx->tc));
     }
     if (!simt.empty()) {

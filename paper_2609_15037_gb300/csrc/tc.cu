@@ -1,7 +1,8 @@
 // Tensor-core path of the optimizer step for bf16 gradients (sm_103a):
 //
-//  K1  R = P^T V with V = Decompose(G, B) formed in shared memory as a pair
-//      of bf16 tiles V_hi + V_lo (two MMAs; P is exact in bf16), then
+//  K1  R = P^T V with V = Decompose(G, B) formed in shared memory in bf16
+//      (at the first Adam step as the pair V_hi + V_lo, two MMAs; P is
+//      exact in bf16), then
 //      Optimizer_V (Adam) on R in the epilogue; writes the Adam update N as
 //      bf16.  The block norms computed for V also drive Optimizer_M (Adam on
 //      the block magnitudes M), done once per (row, block) by the CTAs of the
@@ -66,19 +67,24 @@ struct K1Params {
     const int* cta_start;              // tiles of CTA c: tiles[cta_start[c] .. cta_start[c+1])
     const TcTile* tiles;
     const TcMod* mods;
-    const CUtensorMap* maps;           // per module: [0] P for K1, [1] P for K2, [2] N for K2
+    const CUtensorMap* maps;           // per module: [0] P for K1, [1] P for K2, [2] N, [3] W
     int* status;
     float beta1, beta2, adam_eps, bc1, bc2, decomp_eps;
+    int hilo;                          // project V_hi + V_lo (first Adam step) or V_hi only
 };
 
 // ------------------------------------------------------------------- K2
-constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64, K2_STAGES = 4;
+constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64, K2_STAGES = 3;
 constexpr int K2_A_BYTES = K2_BM * K2_BK * 2;           // 16 KB: P rows, K-major
 constexpr int K2_B_BYTES = K2_BK * K2_BN * 2;           // 32 KB: four 64-column chunks of N
 constexpr int K2_STAGE_BYTES = K2_A_BYTES + K2_B_BYTES;
-constexpr int K2_WARPS = 18;                            // 0 TMA, 1 MMA, 2-17 epilogue
+// W streams through a ring of 128-row x 32-column fp32 chunks (TMA in and out)
+constexpr int K2_WCOLS = 32, K2_WBUF = 4;
+constexpr int K2_WBYTES = K2_BM * K2_WCOLS * 4;         // 16 KB
+constexpr int K2_WARPS = 12;                            // 0 TMA, 1 MMA, 2 W loader, 3 W storer, 4-11 epilogue
 constexpr int K2_THREADS = K2_WARPS * 32;
-constexpr int K2_SMEM = 1024 + K2_STAGES * K2_STAGE_BYTES + GUARD_BYTES + 2048;
+constexpr int K2_GUARD = 8192;
+constexpr int K2_SMEM = 1024 + K2_STAGES * K2_STAGE_BYTES + K2_WBUF * K2_WBYTES + K2_GUARD + 2048;
 
 struct K2Params {
     const int* cta_start;
@@ -97,6 +103,9 @@ struct SmemCtl {
     uint64_t accf[2];
     uint64_t acce[2];
     uint64_t drain;
+    uint64_t wfull[4];
+    uint64_t wdone[4];
+    uint64_t wempty[4];
     uint32_t tmem_base;
     int abort;
 };
@@ -167,7 +176,7 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
             for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
-                const CUtensorMap* pmap = &p.maps[tl.mod * 3 + 0];
+                const CUtensorMap* pmap = &p.maps[tl.mod * 4 + 0];
                 const CUtensorMap* gmap = &p.gmap[tl.slot];
                 const int r0 = tl.t0 * K1_BM, n0 = tl.t1 * K1_BN;
                 const int nk = (md.m + K1_BK - 1) / K1_BK;
@@ -229,7 +238,7 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
                             ptx::mma_f16(d0 + h * 128, adesc, bdesc, idesc, (kb | kk) != 0);
                             // P^T V_lo: the bf16 rounding residual of V, so that R carries
                             // about 16 significant bits (P is exact in bf16)
-                            if (DECOMP) ptx::mma_f16(d0 + h * 128, adesc, ldesc, idesc, 1);
+                            if (DECOMP && p.hilo) ptx::mma_f16(d0 + h * 128, adesc, ldesc, idesc, 1);
                         }
                     }
                     ptx::mma_commit(ptx::smem_u32(&ctl->empty[stage]));
@@ -272,7 +281,39 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
                 float* const mag_avg_sq = md.mag_avg_sq;
                 float* const dMp = md.dM;
                 const int nk = (mm + K1_BK - 1) / K1_BK;
+                const bool owner = (UB < 8) || (hu == 0 && (UB < 16 || hc == 0));
+                const bool mag_here = do_mag && owner;
+                const int gb0 = (n0 + hc * 64 + hu * 32) / BLK;
+                // the magnitude moments of the next stage are loaded one stage ahead,
+                // so their latency is not on the path to the MMA
+                float pma[NBT], pmas[NBT];
+#pragma unroll
+                for (int bl = 0; bl < NBT; ++bl) { pma[bl] = 0.0f; pmas[bl] = 0.0f; }
+                if (mag_here && k < mm) {
+#pragma unroll
+                    for (int bl = 0; bl < NBT; ++bl) {
+                        const int gb = gb0 + (UB < 8 ? bl : 0);
+                        if (gb < mkb) {
+                            pma[bl] = mag_avg[(long long)k * mkb + gb];
+                            pmas[bl] = mag_avg_sq[(long long)k * mkb + gb];
+                        }
+                    }
+                }
                 for (int kb = 0; kb < nk; ++kb) {
+                    float cma[NBT], cmas[NBT];
+#pragma unroll
+                    for (int bl = 0; bl < NBT; ++bl) { cma[bl] = pma[bl]; cmas[bl] = pmas[bl]; }
+                    const int nrow = (kb + 1) * K1_BK + k;
+                    if (mag_here && nrow < mm) {
+#pragma unroll
+                        for (int bl = 0; bl < NBT; ++bl) {
+                            const int gb = gb0 + (UB < 8 ? bl : 0);
+                            if (gb < mkb) {
+                                pma[bl] = mag_avg[(long long)nrow * mkb + gb];
+                                pmas[bl] = mag_avg_sq[(long long)nrow * mkb + gb];
+                            }
+                        }
+                    }
                     const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
                                                     MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
                     if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
@@ -325,21 +366,20 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
                         }
                         const uint32_t off = ((hu * 4 + u) ^ x) << 4;
                         *reinterpret_cast<uint4*>(row + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                        *reinterpret_cast<uint4*>(lrow + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                        if (p.hilo) *reinterpret_cast<uint4*>(lrow + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
                     }
                     ptx::fence_proxy_async_smem();
                     ptx::mbar_arrive(ptx::smem_u32(&ctl->xform[stage]));
                     // Optimizer_M on the block magnitudes, once per (row, block)
                     const int grow = kb * K1_BK + k;
-                    const bool owner = (UB < 8) || (hu == 0 && (UB < 16 || hc == 0));
-                    if (do_mag && owner && grow < mm) {
+                    if (mag_here && grow < mm) {
 #pragma unroll
                         for (int bl = 0; bl < NBT; ++bl) {
-                            const int gb = (n0 + hc * 64 + hu * 32) / BLK + (UB < 8 ? bl : 0);
+                            const int gb = gb0 + (UB < 8 ? bl : 0);
                             if (gb < mkb) {
                                 const long long o = (long long)grow * mkb + gb;
-                                const float ma = p.beta1 * mag_avg[o] + (1.0f - p.beta1) * mag[bl];
-                                const float mas = p.beta2 * mag_avg_sq[o] + (1.0f - p.beta2) * mag[bl] * mag[bl];
+                                const float ma = p.beta1 * cma[bl] + (1.0f - p.beta1) * mag[bl];
+                                const float mas = p.beta2 * cmas[bl] + (1.0f - p.beta2) * mag[bl] * mag[bl];
                                 mag_avg[o] = ma;
                                 mag_avg_sq[o] = mas;
                                 dMp[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
@@ -443,7 +483,8 @@ template <int BLK>
 __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_constant__ K2Params p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
-    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + K2_STAGES * K2_STAGE_BYTES + GUARD_BYTES);
+    uint8_t* wring = smem + K2_STAGES * K2_STAGE_BYTES;
+    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(wring + K2_WBUF * K2_WBYTES + K2_GUARD);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int* abort_flag = &ctl->abort;
 
@@ -454,7 +495,12 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
         }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(ptx::smem_u32(&ctl->accf[b]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 16);
+            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 8);
+        }
+        for (int b = 0; b < K2_WBUF; ++b) {
+            ptx::mbar_init(ptx::smem_u32(&ctl->wfull[b]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->wdone[b]), 8);
+            ptx::mbar_init(ptx::smem_u32(&ctl->wempty[b]), 1);
         }
         ptx::mbar_init(ptx::smem_u32(&ctl->drain), 1);
         ctl->abort = 0;
@@ -468,18 +514,20 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = ctl->tmem_base;
+    const int t_begin = p.cta_start[blockIdx.x], t_end = p.cta_start[blockIdx.x + 1];
 
     if (warp == 0) {
+        // ------------------------------------------------ operand TMA producer
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued = 0, last_par = 0;
             bool ok = true;
-            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
+            for (int t = t_begin; t < t_end && ok; ++t) {
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
-                const CUtensorMap* amap = &p.maps[tl.mod * 3 + 1];
-                const CUtensorMap* bmap = &p.maps[tl.mod * 3 + 2];
+                const CUtensorMap* amap = &p.maps[tl.mod * 4 + 1];
+                const CUtensorMap* bmap = &p.maps[tl.mod * 4 + 2];
                 const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
                 const int nk = (md.r + K2_BK - 1) / K2_BK;
                 for (int kb = 0; kb < nk; ++kb) {
@@ -503,6 +551,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             }
         }
     } else if (warp == 1) {
+        // ------------------------------------------------------ MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc = ptx::idesc_bf16(128, K2_BN, 0, 1);
             int stage = 0;
@@ -510,7 +559,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             int buf = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
-            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
+            for (int t = t_begin; t < t_end && ok; ++t) {
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
                 const int nk = (md.r + K2_BK - 1) / K2_BK;
@@ -540,78 +589,120 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             ptx::mma_commit(ptx::smem_u32(&ctl->drain));
             wait_drain(ptx::smem_u32(&ctl->drain), 0);
         }
+    } else if (warp == 2) {
+        // ------------------------------------------- W chunk loader (TMA in)
+        if (lane == 0) {
+            uint32_t g = 0;
+            uint32_t issued = 0, last_par = 0;
+            bool ok = true;
+            for (int t = t_begin; t < t_end && ok; ++t) {
+                const TcTile tl = p.tiles[t];
+                const TcMod& md = p.mods[tl.mod];
+                const CUtensorMap* wmap = &p.maps[tl.mod * 4 + 3];
+                const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
+                const int nc = min(K2_BN / K2_WCOLS, (md.n - n0 + K2_WCOLS - 1) / K2_WCOLS);
+                for (int c = 0; c < nc; ++c, ++g) {
+                    const int b = g % K2_WBUF;
+                    const uint32_t ph = (g / K2_WBUF) & 1;
+                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->wempty[b]), ph ^ 1, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    const uint32_t fb = ptx::smem_u32(&ctl->wfull[b]);
+                    ptx::mbar_arrive_expect_tx(fb, K2_WBYTES);
+                    ptx::tma_load_2d(ptx::smem_u32(wring + b * K2_WBYTES), wmap, fb, n0 + c * K2_WCOLS, i0);
+                    issued |= 1u << b;
+                    last_par = (last_par & ~(1u << b)) | (ph << b);
+                }
+            }
+            if (!ok) {
+                for (int b = 0; b < K2_WBUF; ++b)
+                    if (issued & (1u << b)) wait_drain(ptx::smem_u32(&ctl->wfull[b]), (last_par >> b) & 1);
+            }
+        }
+    } else if (warp == 3) {
+        // ------------------------------------------ W chunk storer (TMA out)
+        if (lane == 0) {
+            uint32_t g = 0;
+            bool ok = true;
+            for (int t = t_begin; t < t_end && ok; ++t) {
+                const TcTile tl = p.tiles[t];
+                const TcMod& md = p.mods[tl.mod];
+                const CUtensorMap* wmap = &p.maps[tl.mod * 4 + 3];
+                const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
+                const int nc = min(K2_BN / K2_WCOLS, (md.n - n0 + K2_WCOLS - 1) / K2_WCOLS);
+                for (int c = 0; c < nc; ++c, ++g) {
+                    const int b = g % K2_WBUF;
+                    const uint32_t ph = (g / K2_WBUF) & 1;
+                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->wdone[b]), ph, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    ptx::tma_store_2d(wmap, ptx::smem_u32(wring + b * K2_WBYTES), n0 + c * K2_WCOLS, i0);
+                    ptx::bulk_commit_group();
+                    ptx::bulk_wait_read_all();            // the chunk may be refilled once read
+                    ptx::mbar_arrive(ptx::smem_u32(&ctl->wempty[b]));
+                }
+            }
+            ptx::bulk_wait_all();
+        }
     } else {
-        // 16 epilogue warps: lane quarter q = warp % 4, column quarter cq
-        // (64 of the 256 columns, 4 chunks of 16).  W of the next chunk is
-        // loaded while the current one is updated.
-        const int ew = warp - 2;                        // 0..15
+        // ------------------------------------------------- epilogue warps
+        // 8 warps: TMEM lane quarter q = warp % 4, column half ch of each
+        // 32-column chunk; each thread updates 16 values of its W row in the
+        // swizzled shared-memory chunk: W -= lr * alpha * dM * (P N).
+        const int ew = warp - 4;                        // 0..7
         const int q = warp & 3;
-        const int cq = ew >> 2;
+        const int ch = ew >> 2;
+        const int il = q * 32 + lane;                   // row within the tile
+        constexpr int NDM = BLK >= 16 ? 1 : 16 / BLK;   // dM values per thread and chunk
         int buf = 0;
         uint32_t acc_phase = 0;
+        uint32_t g = 0;
         bool ok = true;
-        for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
+        for (int t = t_begin; t < t_end && ok; ++t) {
             const TcTile tl = p.tiles[t];
             const TcMod& md = p.mods[tl.mod];
             const int mm = md.m, nn = md.n, mkb = md.kb;
-            float* const Wp = md.W;
             const float* const dMp = md.dM;
             const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
-            const int i = i0 + q * 32 + lane;
+            const int i = i0 + il;
             const bool row_ok = i < mm;
-            const int jbase = n0 + cq * 64;
-            // prefetch W of the first chunk before waiting for the accumulator
-            float4 wn0 = make_float4(0.f, 0.f, 0.f, 0.f), wn1 = wn0, wn2 = wn0, wn3 = wn0;
-            if (row_ok && jbase + 16 <= nn) {
-                const float4* w4 = reinterpret_cast<const float4*>(Wp + (long long)i * nn + jbase);
-                wn0 = w4[0]; wn1 = w4[1]; wn2 = w4[2]; wn3 = w4[3];
-            }
+            const int nc = min(K2_BN / K2_WCOLS, (nn - n0 + K2_WCOLS - 1) / K2_WCOLS);
             const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
                                             MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
             if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
             ptx::tc_fence_after();
-#pragma unroll 1
-            for (int c = 0; c < 4; ++c) {
-                const int j0 = jbase + c * 16;
-                float w[16] = {wn0.x, wn0.y, wn0.z, wn0.w, wn1.x, wn1.y, wn1.z, wn1.w,
-                               wn2.x, wn2.y, wn2.z, wn2.w, wn3.x, wn3.y, wn3.z, wn3.w};
-                if (c + 1 < 4 && row_ok && j0 + 32 <= nn) {
-                    const float4* w4 = reinterpret_cast<const float4*>(Wp + (long long)i * nn + j0 + 16);
-                    wn0 = w4[0]; wn1 = w4[1]; wn2 = w4[2]; wn3 = w4[3];
+            for (int c = 0; c < nc; ++c, ++g) {
+                const int b = g % K2_WBUF;
+                const uint32_t ph = (g / K2_WBUF) & 1;
+                const int j0 = n0 + c * K2_WCOLS + ch * 16;
+                float dm[NDM];
+#pragma unroll
+                for (int d = 0; d < NDM; ++d) {
+                    const int jb = (j0 + 8 * d) / BLK;
+                    dm[d] = (p.decompose && row_ok && jb < mkb) ? dMp[(long long)i * mkb + jb] : 1.0f;
                 }
                 float v[16];
                 __syncwarp();
-                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + cq * 64 + c * 16, v);
-                if (!row_ok || j0 >= nn) continue;
-                const long long o = (long long)i * nn + j0;
-                const float* dmr = dMp + (long long)i * mkb;
-                if (j0 + 16 <= nn) {
-                    if (p.decompose) {
-                        if (BLK >= 16) {
-                            const float dm = dmr[j0 / BLK];
+                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + c * K2_WCOLS + ch * 16, v);
+                const bool gotw = ptx::mbar_wait(ptx::smem_u32(&ctl->wfull[b]), ph, abort_flag, p.status,
+                                                 MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+                if (!__all_sync(0xffffffffu, gotw)) { ok = false; break; }
+                uint8_t* wrow = wring + b * K2_WBYTES + il * 128;
+                const uint32_t x = static_cast<uint32_t>(il & 7);
 #pragma unroll
-                            for (int e = 0; e < 16; ++e) w[e] -= p.step_scale * (dm * v[e]);
-                        } else {
-#pragma unroll
-                            for (int e = 0; e < 16; ++e) w[e] -= p.step_scale * (dmr[(j0 + e) / BLK] * v[e]);
-                        }
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < 16; ++e) w[e] -= p.step_scale * v[e];
-                    }
-                    float4* w4 = reinterpret_cast<float4*>(Wp + o);
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) w4[e] = make_float4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        if (j0 + e < nn) {
-                            const float u = p.decompose ? dmr[(j0 + e) / BLK] * v[e] : v[e];
-                            Wp[o + e] -= p.step_scale * u;
-                        }
-                    }
+                for (int u = 0; u < 4; ++u) {
+                    float4* w4 = reinterpret_cast<float4*>(wrow + (((ch * 4 + u) ^ x) << 4));
+                    float4 w = *w4;
+                    const float d0 = dm[NDM == 1 ? 0 : (u * 4) / BLK];
+                    w.x -= p.step_scale * (d0 * v[4 * u + 0]);
+                    w.y -= p.step_scale * (d0 * v[4 * u + 1]);
+                    w.z -= p.step_scale * (d0 * v[4 * u + 2]);
+                    w.w -= p.step_scale * (d0 * v[4 * u + 3]);
+                    *w4 = w;
                 }
+                ptx::fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->wdone[b]));
             }
+            if (!ok) break;
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->acce[buf]));
@@ -632,15 +723,20 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-bool encode_bf16_2d(EncodeTiledFn enc, CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
-                    uint32_t box_inner, uint32_t box_outer) {
+bool encode_2d(EncodeTiledFn enc, CUtensorMap* map, CUtensorMapDataType dt, int esize, const void* ptr,
+               uint64_t inner, uint64_t outer, uint32_t box_inner, uint32_t box_outer) {
     const cuuint64_t dims[2] = {inner, outer};
-    const cuuint64_t strides[1] = {inner * 2};
+    const cuuint64_t strides[1] = {inner * esize};
     const cuuint32_t box[2] = {box_inner, box_outer};
     const cuuint32_t estr[2] = {1, 1};
-    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+    return enc(map, dt, 2, const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_bf16_2d(EncodeTiledFn enc, CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
+                    uint32_t box_inner, uint32_t box_outer) {
+    return encode_2d(enc, map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ptr, inner, outer, box_inner, box_outer);
 }
 
 template <int BLK>
@@ -659,7 +755,7 @@ struct TcState {
     EncodeTiledFn encode = nullptr;
     std::string err;
     std::vector<TcMod> mods;               // indexed by module id (unsupported ones left zero)
-    std::vector<CUtensorMap> maps;         // 3 per module id
+    std::vector<CUtensorMap> maps;         // 4 per module id
     TcMod* d_mods = nullptr;
     CUtensorMap* d_maps = nullptr;
     int cap = 0;
@@ -720,7 +816,7 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
     if (st == nullptr) return MOARA_OK;
     if (static_cast<int>(st->mods.size()) <= id) {
         st->mods.resize(id + 1, TcMod{});
-        st->maps.resize(3 * (id + 1));
+        st->maps.resize(4 * (id + 1));
     }
     if (!tc_supported(md.m, md.n, md.r, hp.block_size, md.dtype, hp.decompose) || md.Pb == nullptr) return MOARA_OK;
     TcMod t{};
@@ -729,10 +825,11 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
     t.mag_avg = md.mag_avg; t.mag_avg_sq = md.mag_avg_sq;
     t.Nb = reinterpret_cast<uint16_t*>(md.ws_N);
     t.dM = md.ws_dM;
-    CUtensorMap* mp = &st->maps[3 * id];
+    CUtensorMap* mp = &st->maps[4 * id];
     if (!encode_bf16_2d(st->encode, &mp[0], md.Pb, md.r, md.m, 64, 64) ||
         !encode_bf16_2d(st->encode, &mp[1], md.Pb, md.r, md.m, 64, 128) ||
-        !encode_bf16_2d(st->encode, &mp[2], t.Nb, md.n, md.r, 64, 64)) {
+        !encode_bf16_2d(st->encode, &mp[2], t.Nb, md.n, md.r, 64, 64) ||
+        !encode_2d(st->encode, &mp[3], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, md.W, md.n, md.m, K2_WCOLS, K2_BM)) {
         st->err = "cuTensorMapEncodeTiled failed";
         return MOARA_ERR_CUDA;
     }
@@ -752,14 +849,14 @@ static int tc_upload(TcState* st) {
         st->d_mods = nullptr;
         st->d_maps = nullptr;
         if (cudaMalloc(&st->d_mods, sizeof(TcMod) * ncap) != cudaSuccess ||
-            cudaMalloc(&st->d_maps, sizeof(CUtensorMap) * 3 * ncap) != cudaSuccess) {
+            cudaMalloc(&st->d_maps, sizeof(CUtensorMap) * 4 * ncap) != cudaSuccess) {
             st->err = "cudaMalloc of the tensor-core module table failed";
             return MOARA_ERR_CUDA;
         }
         st->cap = ncap;
     }
     if (cudaMemcpy(st->d_mods, st->mods.data(), sizeof(TcMod) * n, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(st->d_maps, st->maps.data(), sizeof(CUtensorMap) * 3 * n, cudaMemcpyHostToDevice) !=
+        cudaMemcpy(st->d_maps, st->maps.data(), sizeof(CUtensorMap) * 4 * n, cudaMemcpyHostToDevice) !=
             cudaSuccess) {
         st->err = "upload of the tensor-core module table failed";
         return MOARA_ERR_CUDA;
@@ -875,7 +972,7 @@ static cudaError_t launch_pair(TcState* st, const K1Params& p1, const K2Params& 
 }
 
 int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G, float bc1,
-            float bc2, float lr, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+            float bc2, float lr, int first_step, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
     if (!st->attrs_set) {
         set_smem_attrs<8>(); set_smem_attrs<16>(); set_smem_attrs<32>(); set_smem_attrs<64>();
         set_smem_attrs<128>();
@@ -902,6 +999,7 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
         p1.mods = st->d_mods; p1.maps = st->d_maps; p1.status = st->d_status;
         p1.beta1 = hp.beta1; p1.beta2 = hp.beta2; p1.adam_eps = hp.adam_eps;
         p1.bc1 = bc1; p1.bc2 = bc2; p1.decomp_eps = hp.decomp_eps;
+        p1.hilo = first_step ? 1 : 0;
         K2Params p2{};
         p2.cta_start = tl->k2_start; p2.tiles = tl->k2;
         p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;

@@ -21,7 +21,8 @@ TcState* tc_create(int device, int* d_status);
 void tc_destroy(TcState* st);
 int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp);
 int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G,
-            float bc1, float bc2, float lr, cudaStream_t s, int64_t* launches, const TcProfile& prof);
+            float bc1, float bc2, float lr, int first_step, cudaStream_t s, int64_t* launches,
+            const TcProfile& prof);
 const char* tc_last_error(const TcState* st);
 
 }  // namespace moara
