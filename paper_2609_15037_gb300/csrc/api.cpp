@@ -451,11 +451,14 @@ struct RefreshRunner {
         (void)bf;
         v_times(Za, Qa);
         cholqr2s(Qa, Qb, rows_m);          // Q in Qb
+        // power iterations Y = V (V^T Q): Z = V^T Q gets one shifted CholeskyQR
+        // pass (enough to keep V Z well conditioned), Y the full two passes
+        const float u_rnd = 5.9604645e-08f;
         for (int q = 0; q < hp.power_iters; ++q) {
             vt_times(Qb, Za);
-            cholqr2s(Za, Zb, rows_n);      // Z in Zb
+            cholqr_pass(Za, Zb, rows_n, 2.0f * u_rnd);   // Z in Zb
             v_times(Zb, Qa);
-            cholqr2s(Qa, Qb, rows_m);      // Q in Qb
+            cholqr2s(Qa, Qb, rows_m);                    // Q in Qb
         }
         // Rayleigh-Ritz on span(Q): C = (V^T Q)^T (V^T Q), eigenvectors of C by
         // orthogonal iteration with CholeskyQR, ordered by Ritz value.
@@ -680,7 +683,7 @@ int moara_default_hparams(moara_hparams* out) {
     out->refresh_src = MOARA_REFRESH_SRC_V;
     out->oversample = 16;
     out->power_iters = 2;
-    out->ritz_iters = 16;
+    out->ritz_iters = 12;
     out->precision = MOARA_PREC_AUTO;
     out->seed = 0;
     return MOARA_OK;

@@ -211,20 +211,23 @@ __global__ void __launch_bounds__(256) k_chol_diag(const __grid_constant__ Small
         }
         __syncthreads();
     }
-    // inverse of the block factor, row by row (thread c owns column c)
-    for (int i = 0; i < sz; ++i) {
-        if (threadIdx.x < sz) {
-            const int c = threadIdx.x;
-            float v = 0.0f;
-            if (c <= i) {
-                float acc = (c == i) ? 1.0f : 0.0f;
-                for (int k = c; k < i; ++k) acc = fmaf(-Ls[i][k], Xs[k][c], acc);
-                v = acc / Ls[i][i];
-            }
-            Xs[i][c] = v;
+    // inverse of the block factor by forward substitution; thread c keeps
+    // column c of the inverse in registers (loops fully unrolled) and reads
+    // the rows of the factor as shared-memory broadcasts
+    if (threadIdx.x < kTriBase) {
+        const int c = threadIdx.x;
+        float xcol[kTriBase];
+#pragma unroll
+        for (int i = 0; i < kTriBase; ++i) {
+            float acc = (i == c) ? 1.0f : 0.0f;
+#pragma unroll
+            for (int k = 0; k < i; ++k) acc = fmaf(-Ls[i][k], xcol[k], acc);
+            xcol[i] = (i < sz && c <= i) ? acc / Ls[i][i] : 0.0f;
         }
-        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < kTriBase; ++i) Xs[i][c] = xcol[i];
     }
+    __syncthreads();
     for (int e = threadIdx.x; e < sz * sz; e += blockDim.x) {
         const int i = e / sz, c = e - i * sz;
         A[(long long)(j0 + i) * l + j0 + c] = (c <= i) ? Ls[i][c] : 0.0f;
@@ -329,20 +332,31 @@ cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* lau
 // stored to c (fp32) and h (bf16).  Skipped when the problem's fail flag is
 // set, which leaves the previous projector in place.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kSmallThreads) k_sign_fix_store(const __grid_constant__ SmallBatch b) {
+__global__ void __launch_bounds__(256) k_sign_fix_store(const __grid_constant__ SmallBatch b) {
     const int pi = blockIdx.y;
     const int rows = b.rows[pi], r = b.l[pi];
     if (b.fail[pi] != nullptr && *b.fail[pi] != 0) return;
     const float* Pt = b.a[pi];
     float* P = b.c[pi];
     uint16_t* Pb = b.h[pi];
-    for (int q = blockIdx.x * blockDim.x + threadIdx.x; q < r; q += gridDim.x * blockDim.x) {
-        float best = -1.0f, sgnv = 1.0f;
-        for (int i = 0; i < rows; ++i) {
-            const float v = Pt[(long long)i * r + q];
-            if (fabsf(v) > best) { best = fabsf(v); sgnv = v < 0.0f ? -1.0f : 1.0f; }
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    for (int q = blockIdx.x * wpb + (threadIdx.x >> 5); q < r; q += gridDim.x * wpb) {
+        // one warp per column: largest |entry| (lowest row on ties)
+        float best = -1.0f;
+        int bi = 0x7fffffff;
+        for (int i = lane; i < rows; i += 32) {
+            const float a = fabsf(Pt[(long long)i * r + q]);
+            if (a > best) { best = a; bi = i; }
         }
-        for (int i = 0; i < rows; ++i) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+            if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
+        }
+        const float sgnv = (bi < rows && Pt[(long long)bi * r + q] < 0.0f) ? -1.0f : 1.0f;
+        for (int i = lane; i < rows; i += 32) {
             const float v = Pt[(long long)i * r + q] * sgnv;
             P[(long long)i * r + q] = v;
             if (Pb != nullptr) {
@@ -355,7 +369,7 @@ __global__ void __launch_bounds__(kSmallThreads) k_sign_fix_store(const __grid_c
 
 cudaError_t launch_sign_fix_store(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
     if (b.count <= 0) return cudaSuccess;
-    k_sign_fix_store<<<dim3(4, b.count), 256, 0, s>>>(b);
+    k_sign_fix_store<<<dim3(32, b.count), 256, 0, s>>>(b);
     ++*launches;
     return cudaGetLastError();
 }
