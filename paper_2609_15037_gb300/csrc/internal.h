@@ -81,6 +81,7 @@ struct GemmProb {
 struct GemmBatch {
     int count;
     int B;                        // block size (scales, dM repetition)
+    int log2B;                    // log2(B) when B is a power of two, else -1 (set at launch)
     float beta1, beta2, adam_eps, bc1, bc2;
     float step_scale;             // lr * alpha (EPI_UPDATE)
     int tiles_n[kMaxGroup];

@@ -122,21 +122,25 @@ cudaError_t launch_decompose(const DecompBatch& b, cudaStream_t s, int64_t* laun
 // register-staged double buffering.  blockIdx.x enumerates the tiles of all
 // problems of the batch (problems are ordered longest-K first by the host).
 // ---------------------------------------------------------------------------
-constexpr int TM = 128, TN = 128, TK = 8, TPAD = 4;
+constexpr int TM = 128, TN = 128, TK = 16, TPAD = 4;
+constexpr int NQ = TK * 128 / 256;   // elements of A (and of B) each thread stages per k-tile
 
 int gemm_tile_m() { return TM; }
 int gemm_tile_n() { return TN; }
 
+// Index of the block holding column c: a shift when B is a power of two.
+__device__ __forceinline__ int block_of(int c, int B, int log2B) { return log2B >= 0 ? (c >> log2B) : c / B; }
+
 template <int ALAY, bool ASC, bool ABF, int BLAY, bool BSC, bool BBF>
 struct TileLoader {
-    float ra[4], rb[4];
+    float ra[NQ], rb[NQ];
 
-    __device__ __forceinline__ void load(const GemmProb& p, int m0, int n0, int k0, int B) {
+    __device__ __forceinline__ void load(const GemmProb& p, int m0, int n0, int k0, int B, int log2B) {
         const int t = threadIdx.x;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < NQ; ++q) {
             int i, k;
-            if (ALAY == A_KCONTIG) { k = t & 7; i = (t >> 3) + 32 * q; }
+            if (ALAY == A_KCONTIG) { k = t & (TK - 1); i = (t / TK) + (256 / TK) * q; }
             else                   { i = t & 127; k = (t >> 7) + 2 * q; }
             const int gi = m0 + i, gk = k0 + k;
             float v = 0.0f;
@@ -146,15 +150,15 @@ struct TileLoader {
                 if (ALAY == A_KCONTIG) { idx = (long long)gi * p.lda + gk; vrow = gi; vcol = gk; }
                 else                   { idx = (long long)gk * p.lda + gi; vrow = gk; vcol = gi; }
                 v = load_elem<ABF>(p.A, idx);
-                if (ASC) v *= __ldg(p.a_inv + (long long)vrow * p.kb + vcol / B);
+                if (ASC) v *= __ldg(p.a_inv + (long long)vrow * p.kb + block_of(vcol, B, log2B));
             }
             ra[q] = v;
         }
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < NQ; ++q) {
             int j, k;
             if (BLAY == B_NCONTIG) { j = t & 127; k = (t >> 7) + 2 * q; }
-            else                   { k = t & 7; j = (t >> 3) + 32 * q; }
+            else                   { k = t & (TK - 1); j = (t / TK) + (256 / TK) * q; }
             const int gj = n0 + j, gk = k0 + k;
             float v = 0.0f;
             if (gj < p.N && gk < p.K) {
@@ -163,7 +167,7 @@ struct TileLoader {
                 if (BLAY == B_NCONTIG) { idx = (long long)gk * p.ldb + gj; vrow = gk; vcol = gj; }
                 else                   { idx = (long long)gj * p.ldb + gk; vrow = gj; vcol = gk; }
                 v = load_elem<BBF>(p.Bm, idx);
-                if (BSC) v *= __ldg(p.b_inv + (long long)vrow * p.kb + vcol / B);
+                if (BSC) v *= __ldg(p.b_inv + (long long)vrow * p.kb + block_of(vcol, B, log2B));
             }
             rb[q] = v;
         }
@@ -172,17 +176,17 @@ struct TileLoader {
     __device__ __forceinline__ void store(float (*As)[TM + TPAD], float (*Bs)[TN + TPAD]) {
         const int t = threadIdx.x;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < NQ; ++q) {
             int i, k;
-            if (ALAY == A_KCONTIG) { k = t & 7; i = (t >> 3) + 32 * q; }
+            if (ALAY == A_KCONTIG) { k = t & (TK - 1); i = (t / TK) + (256 / TK) * q; }
             else                   { i = t & 127; k = (t >> 7) + 2 * q; }
             As[k][i] = ra[q];
         }
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < NQ; ++q) {
             int j, k;
             if (BLAY == B_NCONTIG) { j = t & 127; k = (t >> 7) + 2 * q; }
-            else                   { k = t & 7; j = (t >> 3) + 32 * q; }
+            else                   { k = t & (TK - 1); j = (t / TK) + (256 / TK) * q; }
             Bs[k][j] = rb[q];
         }
     }
@@ -207,13 +211,13 @@ __device__ __forceinline__ void epilogue(const GemmBatch& b, const GemmProb& p, 
     } else {
         // W <- W - lr*alpha*(Rep_B(dM) (.) dV)  (Algorithm 1; Rep_B of §3.1).
         float u = acc;
-        if (p.aux2 != nullptr) u *= p.aux2[(long long)i * p.kb + j / b.B];
+        if (p.aux2 != nullptr) u *= p.aux2[(long long)i * p.kb + block_of(j, b.B, b.log2B)];
         p.aux0[o] = p.aux0[o] - b.step_scale * u;
     }
 }
 
 template <int ALAY, bool ASC, bool ABF, int BLAY, bool BSC, bool BBF, int EPI>
-__global__ void __launch_bounds__(256) k_gemm(const __grid_constant__ GemmBatch b) {
+__global__ void __launch_bounds__(256, 2) k_gemm(const __grid_constant__ GemmBatch b) {
     __shared__ __align__(16) float As[2][TK][TM + TPAD];
     __shared__ __align__(16) float Bs[2][TK][TN + TPAD];
 
@@ -240,12 +244,12 @@ __global__ void __launch_bounds__(256) k_gemm(const __grid_constant__ GemmBatch 
 
     TileLoader<ALAY, ASC, ABF, BLAY, BSC, BBF> ld;
     const int ktiles = (p.K + TK - 1) / TK;
-    ld.load(p, m0, n0, 0, b.B);
+    ld.load(p, m0, n0, 0, b.B, b.log2B);
     ld.store(As[0], Bs[0]);
     __syncthreads();
     for (int kt = 0; kt < ktiles; ++kt) {
         const int cur = kt & 1;
-        if (kt + 1 < ktiles) ld.load(p, m0, n0, (kt + 1) * TK, b.B);
+        if (kt + 1 < ktiles) ld.load(p, m0, n0, (kt + 1) * TK, b.B, b.log2B);
 #pragma unroll
         for (int k = 0; k < TK; ++k) {
             float av[8], bv[8];
@@ -282,6 +286,12 @@ __global__ void __launch_bounds__(256) k_gemm(const __grid_constant__ GemmBatch 
 
 template <int ALAY, bool ASC, bool ABF, int BLAY, bool BSC, bool BBF, int EPI>
 static cudaError_t launch_one(GemmBatch& b, cudaStream_t s, int64_t* launches) {
+    b.log2B = -1;
+    if (b.B > 0 && (b.B & (b.B - 1)) == 0) {
+        int lg = 0;
+        while ((1 << lg) < b.B) ++lg;
+        b.log2B = lg;
+    }
     int total = 0;
     for (int i = 0; i < b.count; ++i) {
         const GemmProb& p = b.p[i];
