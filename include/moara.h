@@ -158,7 +158,9 @@ int moara_rank_table(int r_base, uint32_t donor_mask, uint32_t receiver_mask,
                      int delta_r, int out_ranks[7]);
 
 /* Bytes of per-module scratch a module of this shape needs (Adam update of
- * the direction branch r x n, magnitude update m x k, block scales m x k). */
+ * the direction branch r x n, magnitude update m x k, block scales m x k,
+ * and the direction matrix V as two m x n bf16 planes for the tensor-core
+ * projection). */
 int moara_workspace_bytes(int m, int n, int r, int block_size, size_t* out);
 
 /* Registers a weight (see moara_module_desc).  Checks shapes (r <= min(m,n)),
@@ -235,6 +237,8 @@ int64_t moara_launch_count(const moara_ctx* ctx);
 #define MOARA_PHASE_REFRESH       3  /* one whole refresh call                       */
 #define MOARA_PHASE_TC_PROJECT    4  /* tensor-core projection kernel                */
 #define MOARA_PHASE_TC_BACKPROJECT 5 /* tensor-core back-projection kernel           */
+#define MOARA_PHASE_TC_DECOMPOSE  6  /* tensor-core path: block norms, magnitude Adam, V in bf16 */
+#define MOARA_PHASE_TC_REFRESH    7  /* refresh products V^T Q, V Z on tensor cores (inside REFRESH) */
 #define MOARA_NUM_PHASES          8
 int moara_profile_enable(moara_ctx* ctx, int enable);
 

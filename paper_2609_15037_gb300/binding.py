@@ -232,7 +232,7 @@ def moara_step_static_scratch(hp, m, n, r, grad_dtype, G, W, P, exp_avg, exp_avg
 
 
 PHASES = ["decompose", "project", "backproject", "refresh", "tc_project",
-          "tc_backproject", "phase6", "phase7"]
+          "tc_backproject", "tc_decompose", "tc_refresh"]
 
 
 def moara_profile_enable(ctx, enable=True):

@@ -154,6 +154,8 @@ WsLayout workspace_layout(int m, int n, int r, int B) {
     w.off_N = off;   off = align_up(off + sizeof(float) * (size_t)r * n, 256);
     w.off_dM = off;  off = align_up(off + sizeof(float) * (size_t)m * kb, 256);
     w.off_inv = off; off = align_up(off + sizeof(float) * (size_t)m * kb, 256);
+    w.off_Vhi = off; off = align_up(off + sizeof(uint16_t) * (size_t)m * n, 256);
+    w.off_Vlo = off; off = align_up(off + sizeof(uint16_t) * (size_t)m * n, 256);
     w.total = off;
     return w;
 }
@@ -168,6 +170,8 @@ size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v) {
     add(sizeof(float) * (size_t)n * l);  // Zb
     add(sizeof(float) * (size_t)m * l);  // Qa
     add(sizeof(float) * (size_t)m * l);  // Qb
+    add(sizeof(uint16_t) * (size_t)m * l);  // Qbf
+    add(sizeof(uint16_t) * (size_t)n * l);  // Zbf
     for (int i = 0; i < 6; ++i) add(sizeof(float) * (size_t)l * l);
     add(sizeof(float) * 16);
     add(sizeof(float) * (size_t)l);
@@ -188,6 +192,8 @@ void refresh_carve(RefreshItem& it, void* base, int m, int n, int r, int l, int 
     it.Zb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)n * l));
     it.Qa = reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * l));
     it.Qb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * l));
+    it.Qbf = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * (size_t)m * l));
+    it.Zbf = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * (size_t)n * l));
     it.Cg = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Linv = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Tt = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
@@ -239,13 +245,19 @@ struct RefreshRunner {
     }
 
     // X_out = X_in * chol(X_in^T X_in + shift)^-T for every item (rows(i) x l).
+    // Only the lower triangle of the Gram matrix is formed (the Cholesky
+    // factorisation reads no more), and the product with the lower-triangular
+    // inverse skips its zero upper part.  `bf` (per item, may hold nulls)
+    // receives a bf16 copy of X_out for the tensor-core products.
     void cholqr_pass(std::vector<float*>& Xin, std::vector<float*>& Xout,
-                     const std::vector<int>& rows, float shift_rel) {
+                     const std::vector<int>& rows, float shift_rel,
+                     const std::vector<uint16_t*>* bf = nullptr) {
         moara::GemmKind gram{moara::A_MCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
         gemm(gram, [&](int i, moara::GemmProb& p) {
             const int l = it[i].l;
             p.A = Xin[i]; p.Bm = Xin[i]; p.C = it[i].Cg;
             p.M = l; p.N = l; p.K = rows[i]; p.lda = l; p.ldb = l; p.ldc = l;
+            p.lower_only = 1;
         });
         cholesky_blocked(rows, shift_rel);
         tri_inverse(/*have_diag=*/true);
@@ -254,6 +266,8 @@ struct RefreshRunner {
             const int l = it[i].l;
             p.A = Xin[i]; p.Bm = it[i].Linv; p.C = Xout[i];
             p.M = rows[i]; p.N = l; p.K = l; p.lda = l; p.ldb = l; p.ldc = l;
+            p.k_tri = 1;
+            p.c_bf16 = bf != nullptr ? (*bf)[i] : nullptr;
         });
     }
 
@@ -364,11 +378,13 @@ struct RefreshRunner {
         }
     }
 
-    // CholeskyQR2 with a shifted first pass; result lands in `b`.
-    void cholqr2s(std::vector<float*>& a, std::vector<float*>& b, const std::vector<int>& rows) {
+    // CholeskyQR2 with a shifted first pass; result lands in `b` (and its bf16
+    // copy in `bf` when given).
+    void cholqr2s(std::vector<float*>& a, std::vector<float*>& b, const std::vector<int>& rows,
+                  const std::vector<uint16_t*>* bf = nullptr) {
         const float u = 5.9604645e-08f;   // fp32 unit roundoff
         cholqr_pass(a, b, rows, 2.0f * u);
-        cholqr_pass(b, a, rows, 0.0f);
+        cholqr_pass(b, a, rows, 0.0f, bf);
         std::swap(a, b);
     }
 
@@ -376,19 +392,30 @@ struct RefreshRunner {
         const int n_it = static_cast<int>(it.size());
         const moara_hparams& hp = ctx->hp;
         for (auto& x : it) chk(cudaMemsetAsync(x.fail, 0, sizeof(int), s));
-        // block scales of Decompose(G, B) when the source is V
-        if (src_v) {
+        std::vector<int> simt_ids, tc_ids;
+        for (int i = 0; i < n_it; ++i) (it[i].tc ? tc_ids : simt_ids).push_back(i);
+        // block scales of Decompose(G, B) when the source is V: fp32 scales for
+        // the SIMT products, bf16 planes V_hi + V_lo for the tensor-core ones
+        if (src_v && !simt_ids.empty()) {
             moara::DecompBatch db{};
-            db.count = n_it; db.B = hp.block_size; db.do_mag = 0; db.decomp_eps = hp.decomp_eps;
+            db.count = static_cast<int>(simt_ids.size()); db.B = hp.block_size; db.do_mag = 0;
+            db.decomp_eps = hp.decomp_eps;
             long long acc = 0;
-            for (int i = 0; i < n_it; ++i) {
-                db.item_start[i] = acc;
-                db.p[i] = moara::DecompItem{it[i].G, it[i].inv, nullptr, nullptr, nullptr,
-                                            it[i].m, it[i].n, it[i].kb, it[i].dtype};
-                acc += (long long)it[i].m * it[i].kb;
+            for (int q = 0; q < db.count; ++q) {
+                const auto& x = it[simt_ids[q]];
+                db.item_start[q] = acc;
+                db.p[q] = moara::DecompItem{x.G, x.inv, nullptr, nullptr, nullptr, x.m, x.n, x.kb, x.dtype};
+                acc += (long long)x.m * x.kb;
             }
-            db.item_start[n_it] = acc;
+            db.item_start[db.count] = acc;
             chk(moara::launch_decompose(db, s, &ctx->launches));
+        }
+        if (src_v && !tc_ids.empty()) {
+            std::vector<moara::TcSplitItem> sp;
+            for (int i : tc_ids) sp.push_back({it[i].G, it[i].Vhi_w, it[i].Vlo, it[i].m, it[i].n});
+            if (moara::tc_split_v(ctx->tc, sp.data(), static_cast<int>(sp.size()), hp.block_size, hp.decomp_eps, s,
+                                  &ctx->launches) != MOARA_OK)
+                chk(cudaErrorLaunchFailure);
         }
         // Gaussian test matrix Omega (n x l)
         {
@@ -398,19 +425,34 @@ struct RefreshRunner {
             }
             chk(moara::launch_philox_gaussian(sb, s, &ctx->launches));
         }
+        for (int i : tc_ids)
+            chk(moara::launch_f32_to_bf16(it[i].Omega, nullptr, it[i].Zbf, (long long)it[i].n * it[i].l, s,
+                                          &ctx->launches));
         std::vector<float*> Qa(n_it), Qb(n_it), Za(n_it), Zb(n_it), Xa(n_it), Xb(n_it);
         std::vector<int> rows_m(n_it), rows_n(n_it), rows_l(n_it);
+        std::vector<uint16_t*> qbf(n_it, nullptr), zbf(n_it, nullptr);
         for (int i = 0; i < n_it; ++i) {
             Qa[i] = it[i].Qa; Qb[i] = it[i].Qb; Za[i] = it[i].Za; Zb[i] = it[i].Zb;
             Xa[i] = it[i].Xa; Xb[i] = it[i].Xb;
             rows_m[i] = it[i].m; rows_n[i] = it[i].n; rows_l[i] = it[i].l;
+            if (it[i].tc) { qbf[i] = it[i].Qbf; zbf[i] = it[i].Zbf; }
         }
-        const int bf = it.empty() ? 0 : (it[0].dtype == MOARA_DTYPE_BF16);
-        // Y = V * Omega  (m x l)
+        // tensor-core products of the TC items: op 0 out = V^T Q_bf16, op 1 out = V Z_bf16
+        auto tc_products = [&](int op, std::vector<float*>& out) {
+            if (tc_ids.empty()) return;
+            ProfScope ps(ctx, MOARA_PHASE_TC_REFRESH, s);
+            std::vector<moara::TcProdItem> pi;
+            for (int i : tc_ids)
+                pi.push_back({it[i].Vhi, it[i].Vlo, it[i].Qbf, it[i].Zbf, out[i], it[i].m, it[i].n, it[i].l});
+            if (moara::tc_refresh_products(ctx->tc, op, pi.data(), static_cast<int>(pi.size()), s,
+                                           &ctx->launches) != MOARA_OK)
+                chk(cudaErrorLaunchFailure);
+        };
+        // Y = V * Z  (m x l); Z is Omega on the first call
         auto v_times = [&](std::vector<float*>& rhs, std::vector<float*>& out) {
             for (int d = 0; d < 2; ++d) {  // per-dtype sub-batches
                 std::vector<int> sel;
-                for (int i = 0; i < n_it; ++i) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
+                for (int i : simt_ids) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
                 if (sel.empty()) continue;
                 moara::GemmKind k{moara::A_KCONTIG, moara::B_NCONTIG, src_v, 0, d, 0, moara::EPI_STORE};
                 moara::GemmBatch b{};
@@ -426,12 +468,13 @@ struct RefreshRunner {
                 }
                 chk(moara::launch_gemm(k, b, s, &ctx->launches));
             }
+            tc_products(1, out);
         };
         // Z = V^T * Q  (n x l)
         auto vt_times = [&](std::vector<float*>& rhs, std::vector<float*>& out) {
             for (int d = 0; d < 2; ++d) {
                 std::vector<int> sel;
-                for (int i = 0; i < n_it; ++i) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
+                for (int i : simt_ids) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
                 if (sel.empty()) continue;
                 moara::GemmKind k{moara::A_MCONTIG, moara::B_NCONTIG, src_v, 0, d, 0, moara::EPI_STORE};
                 moara::GemmBatch b{};
@@ -447,18 +490,18 @@ struct RefreshRunner {
                 }
                 chk(moara::launch_gemm(k, b, s, &ctx->launches));
             }
+            tc_products(0, out);
         };
-        (void)bf;
         v_times(Za, Qa);
-        cholqr2s(Qa, Qb, rows_m);          // Q in Qb
+        cholqr2s(Qa, Qb, rows_m, &qbf);    // Q in Qb
         // power iterations Y = V (V^T Q): Z = V^T Q gets one shifted CholeskyQR
         // pass (enough to keep V Z well conditioned), Y the full two passes
         const float u_rnd = 5.9604645e-08f;
         for (int q = 0; q < hp.power_iters; ++q) {
             vt_times(Qb, Za);
-            cholqr_pass(Za, Zb, rows_n, 2.0f * u_rnd);   // Z in Zb
+            cholqr_pass(Za, Zb, rows_n, 2.0f * u_rnd, &zbf);   // Z in Zb
             v_times(Zb, Qa);
-            cholqr2s(Qa, Qb, rows_m);                    // Q in Qb
+            cholqr2s(Qa, Qb, rows_m, &qbf);                    // Q in Qb
         }
         // Rayleigh-Ritz on span(Q): C = (V^T Q)^T (V^T Q), eigenvectors of C by
         // orthogonal iteration with CholeskyQR, ordered by Ritz value.
@@ -550,6 +593,18 @@ int do_refresh(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, 
             moara::refresh_carve(x, static_cast<char*>(ctx->refresh_ws) + used, d.m, d.n, d.r, l,
                                  hp.block_size, src_v);
             x.P = d.P; x.Pb = d.P_bf16;
+            // products on tensor cores when the module's step runs there (bf16
+            // G, supported shape) and the bf16 planes of Q and Z have a TMA
+            // row pitch (l % 8 == 0)
+            if (use_tc(ctx, id) && (l % 8) == 0) {
+                const moara::ModDev& md = ctx->moddev[id];
+                x.tc = 1;
+                if (src_v) {
+                    x.Vhi = md.ws_Vhi; x.Vhi_w = md.ws_Vhi; x.Vlo = md.ws_Vlo;
+                } else {
+                    x.Vhi = static_cast<const uint16_t*>(G[end]); x.Vhi_w = nullptr; x.Vlo = nullptr;
+                }
+            }
             const uint64_t cnt = static_cast<uint64_t>(ctx->refresh_count[id]++);
             x.key = hp.seed ^ (0x9E3779B97F4A7C15ull * (static_cast<uint64_t>(id) + 1)) ^
                     (cnt * 0xD1B54A32D192ED03ull);
@@ -843,6 +898,8 @@ int moara_init_module(moara_ctx* ctx, const moara_module_desc* d, int* module_id
     md.ws_N = reinterpret_cast<float*>(ws + wl.off_N);
     md.ws_dM = reinterpret_cast<float*>(ws + wl.off_dM);
     md.ws_inv = reinterpret_cast<float*>(ws + wl.off_inv);
+    md.ws_Vhi = reinterpret_cast<uint16_t*>(ws + wl.off_Vhi);
+    md.ws_Vlo = reinterpret_cast<uint16_t*>(ws + wl.off_Vlo);
     const int id = static_cast<int>(ctx->mods.size());
     cudaError_t e = cudaMemcpy(ctx->d_mods + id, &md, sizeof(md), cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "module table copy");

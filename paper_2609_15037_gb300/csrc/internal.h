@@ -31,11 +31,13 @@ struct ModDev {
     float* ws_N;            // r x n update of the direction branch (fp32 or bf16)
     float* ws_dM;           // m x kb update of the magnitude branch
     float* ws_inv;          // m x kb inverse block scales 1 / (||g|| + eps)
+    uint16_t* ws_Vhi;       // m x n direction matrix V in bf16 (tensor-core path)
+    uint16_t* ws_Vlo;       // m x n bf16 residual V - V_hi (first Adam step)
 };
 
 // Workspace carve-up of one module (byte offsets, 256-byte aligned).
 struct WsLayout {
-    size_t off_N, off_dM, off_inv, total;
+    size_t off_N, off_dM, off_inv, off_Vhi, off_Vlo, total;
 };
 WsLayout workspace_layout(int m, int n, int r, int B);
 
@@ -76,6 +78,8 @@ struct GemmProb {
     int kb;               // blocks per row of the scaled operand / of dM
     int a_bf16, b_bf16;
     int lower_only;       // skip output tiles strictly above the diagonal
+    int k_tri;            // B is lower triangular in (j, k): column tile n0 needs k < n0 + tile width only
+    uint16_t* c_bf16;     // EPI_STORE: also write C rounded to bf16 here (same layout), or null
 };
 
 struct GemmBatch {
@@ -128,6 +132,12 @@ struct RefreshItem {
     float* P;         // m x r destination
     uint16_t* Pb;     // m x r bf16 destination (may be null)
     uint64_t key;     // RNG key (seed, module, refresh count)
+    int tc;           // products with V on tensor cores
+    const uint16_t* Vhi;    // m x n bf16 planes of V (or G) for the tensor-core products
+    uint16_t* Vhi_w;        // writable view of Vhi when V is formed here (null otherwise)
+    uint16_t* Vlo;          // residual plane, or null when Vhi is exact
+    uint16_t* Qbf;    // m x l bf16 copy of the latest orthonormal Q
+    uint16_t* Zbf;    // n x l bf16 copy of the latest Z (or of Omega)
 };
 
 size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v);

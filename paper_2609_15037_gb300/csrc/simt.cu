@@ -197,6 +197,10 @@ __device__ __forceinline__ void epilogue(const GemmBatch& b, const GemmProb& p, 
     const long long o = (long long)i * p.ldc + j;
     if (EPI == EPI_STORE) {
         p.C[o] = acc;
+        if (p.c_bf16 != nullptr) {
+            __nv_bfloat16 h = __float2bfloat16_rn(acc);
+            p.c_bf16[o] = *reinterpret_cast<uint16_t*>(&h);
+        }
     } else if (EPI == EPI_STORE_NEG) {
         p.C[o] = -acc;
     } else if (EPI == EPI_SUB) {
@@ -243,7 +247,8 @@ __global__ void __launch_bounds__(256, 2) k_gemm(const __grid_constant__ GemmBat
         for (int c = 0; c < 8; ++c) acc[a][c] = 0.0f;
 
     TileLoader<ALAY, ASC, ABF, BLAY, BSC, BBF> ld;
-    const int ktiles = (p.K + TK - 1) / TK;
+    const int kend = p.k_tri ? min(p.K, n0 + TN) : p.K;
+    const int ktiles = (kend + TK - 1) / TK;
     ld.load(p, m0, n0, 0, b.B, b.log2B);
     ld.store(As[0], Bs[0]);
     __syncthreads();

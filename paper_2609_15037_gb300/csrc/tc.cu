@@ -1,17 +1,17 @@
 // Tensor-core path of the optimizer step for bf16 gradients (sm_103a):
 //
-//  K1  R = P^T V with V = Decompose(G, B) formed in shared memory in bf16
-//      (at the first Adam step as the pair V_hi + V_lo, two MMAs; P is
-//      exact in bf16), then
+//  K0  Decompose(G, B) of §3.1 / Appendix B.1 as a memory-bound prepass: block
+//      norms in fp32, Optimizer_M (Adam on the block magnitudes), and the
+//      direction matrix V written in bf16 (at the first Adam step also the
+//      residual V - V_hi, so that the projection carries ~16 bits there).
+//  K1  R = P^T V on tcgen05 (128 x 256 tiles, P exact in bf16), then
 //      Optimizer_V (Adam) on R in the epilogue; writes the Adam update N as
-//      bf16.  The block norms computed for V also drive Optimizer_M (Adam on
-//      the block magnitudes M), done once per (row, block) by the CTAs of the
-//      first rank tile.  (Algorithm 1; §3.1 / Appendix B.1.)
+//      bf16.  (Algorithm 1.)
 //  K2  dV = P N, then W <- W - lr*alpha*(Rep_B(dM) (.) dV) in the epilogue,
-//      reading and writing W once.  (Algorithm 1.)
+//      reading and writing W once through TMA.  (Algorithm 1.)
 //
-// Both kernels are persistent and warp specialised: one warp issues TMA tile
-// loads into a 4-stage shared-memory ring, one thread issues tcgen05.mma into
+// K1 and K2 are persistent and warp specialised: one warp issues TMA tile
+// loads into a shared-memory ring, one thread issues tcgen05.mma into
 // double-buffered TMEM accumulators, and epilogue warps drain TMEM while the
 // next tile's MMAs run.  Every mbarrier wait is bounded; on expiry the kernel
 // records MOARA_ERR_DEVICE_TIMEOUT in the context's status word, drains its
@@ -34,9 +34,12 @@ namespace {
 
 constexpr int kTcGroup = 224;                 // modules per launch (G maps in params)
 constexpr long long kWaitLimit = 1LL << 32;   // ~2 s of SM clocks
+constexpr int kMaps = 6;                      // tensor maps per module
 
 struct TcMod {
     int m, n, r, kb;
+    uint16_t* Vhi;    // m x n bf16 direction matrix (written by K0)
+    uint16_t* Vlo;    // m x n bf16 residual (first Adam step)
     float* W;
     float* exp_avg;
     float* exp_avg_sq;
@@ -50,27 +53,48 @@ struct TcTile {
     int mod, slot, t0, t1;
 };
 
+// ------------------------------------------------------------------- K0
+struct K0Item {
+    const uint16_t* G;
+    uint16_t* Vhi;
+    uint16_t* Vlo;
+    float* mag_avg;
+    float* mag_avg_sq;
+    float* dM;
+    int m, n, kb, segs;                // segs = ceil(n / 1024) row segments
+};
+
+struct K0Params {
+    int count;
+    int hilo;                          // also write V_lo = V - V_hi
+    int do_mag;                        // run Optimizer_M (off when only V is wanted)
+    float decomp_eps, beta1, beta2, adam_eps, bc1, bc2;
+    long long start[kTcGroup + 1];     // warp items (row, 1024-column segment) per module
+    K0Item p[kTcGroup];
+};
+
 // ------------------------------------------------------------------- K1
-constexpr int K1_BM = 256, K1_BN = 128, K1_BK = 64, K1_STAGES = 3;
-constexpr int K1_A_BYTES = K1_BM * K1_BK * 2;           // 32 KB: four 64-row chunks of P^T
-constexpr int K1_B_BYTES = K1_BK * K1_BN * 2;           // 16 KB: two 64-column chunks of G
-// stage: A | B (G, then V_hi after the transform) | V_lo (V - V_hi in bf16)
-constexpr int K1_STAGE_BYTES = K1_A_BYTES + 2 * K1_B_BYTES;
-constexpr int K1_TX_BYTES = K1_A_BYTES + K1_B_BYTES;    // bytes the TMA brings per stage
-constexpr int K1_WARPS = 18;                            // 0 TMA, 1 MMA, 2-9 transform, 10-17 epilogue
+constexpr int K1_BM = 128, K1_BN = 256, K1_BK = 64;
+constexpr int K1_A_BYTES = K1_BM * K1_BK * 2;           // 16 KB: two 64-rank chunks of P^T (MN-major)
+constexpr int K1_B_BYTES = K1_BK * K1_BN * 2;           // 32 KB: four 64-column chunks of V (MN-major)
+template <bool HILO> struct K1Cfg {
+    static constexpr int STAGES = HILO ? 2 : 4;
+    static constexpr int STAGE_BYTES = K1_A_BYTES + (HILO ? 2 : 1) * K1_B_BYTES;
+};
+constexpr int K1_WARPS = 10;                            // 0 TMA, 1 MMA, 2-9 epilogue
 constexpr int K1_THREADS = K1_WARPS * 32;
 constexpr int GUARD_BYTES = 16384;
-constexpr int K1_SMEM = 1024 + K1_STAGES * K1_STAGE_BYTES + GUARD_BYTES + 2048;
+constexpr int K1_SMEM = 1024 + 4 * (K1_A_BYTES + K1_B_BYTES) + GUARD_BYTES + 2048;
 
 struct K1Params {
-    CUtensorMap gmap[kTcGroup];        // G of each launch slot: dims {n, m}, box {64, 64}
+    CUtensorMap gmap[kTcGroup];        // G of each launch slot (decomposition off): {n, m}, box {64, 64}
     const int* cta_start;              // tiles of CTA c: tiles[cta_start[c] .. cta_start[c+1])
     const TcTile* tiles;
     const TcMod* mods;
-    const CUtensorMap* maps;           // per module: [0] P for K1, [1] P for K2, [2] N, [3] W
+    const CUtensorMap* maps;           // per module: P (K1), P (K2), N, W, V_hi, V_lo
     int* status;
-    float beta1, beta2, adam_eps, bc1, bc2, decomp_eps;
-    int hilo;                          // project V_hi + V_lo (first Adam step) or V_hi only
+    float beta1, beta2, adam_eps, bc1, bc2;
+    int decompose;
 };
 
 // ------------------------------------------------------------------- K2
@@ -98,7 +122,6 @@ struct K2Params {
 
 struct SmemCtl {
     uint64_t full[4];
-    uint64_t xform[4];
     uint64_t empty[4];   // sized for up to four stages
     uint64_t accf[2];
     uint64_t acce[2];
@@ -131,22 +154,101 @@ __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w <<
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
 // ===========================================================================
-// K1: projection R = P^T V with the decomposition fused into the B operand,
-// direction-branch Adam in the epilogue, magnitude-branch Adam in the
-// transform warps.
+// K0: Decompose(G, B) (§3.1 / App. B.1) and Optimizer_M.  One warp per (row,
+// 1024-column segment), taken as four 256-column sub-segments whose loads are
+// all issued first; in a sub-segment lane l holds columns 8l..8l+7, so a block
+// of B columns spans B/8 lanes, reduced with xor shuffles.  Columns past n (the
+// right zero padding of the last block) contribute nothing; V is written for
+// c < n only.
 // ===========================================================================
-template <int BLK, bool DECOMP>
+constexpr int K0_SEG = 1024;
+
+template <int BLK>
+__global__ void __launch_bounds__(256) k0_decompose(const __grid_constant__ K0Params p) {
+    constexpr int LPB = BLK / 8;                       // lanes per block (1..16)
+    const int lane = threadIdx.x & 31;
+    const long long total = p.start[p.count];
+    const long long warp0 = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+    for (long long item = warp0; item < total; item += nwarps) {
+        int lo = 0, hi = p.count - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (p.start[mid] <= item) lo = mid; else hi = mid - 1;
+        }
+        const K0Item& it = p.p[lo];
+        const long long local = item - p.start[lo];
+        const int row = static_cast<int>(local / it.segs);
+        const int seg = static_cast<int>(local - (long long)row * it.segs);
+        const int n = it.n;
+        uint4 g[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int c0 = seg * K0_SEG + u * 256 + lane * 8;
+            g[u] = make_uint4(0u, 0u, 0u, 0u);
+            if (c0 < n) g[u] = __ldcs(reinterpret_cast<const uint4*>(it.G + (long long)row * n + c0));
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int cs = seg * K0_SEG + u * 256;      // first column of the sub-segment
+            if (cs >= n) break;                         // warp-uniform
+            const int c0 = cs + lane * 8;
+            const uint32_t w[4] = {g[u].x, g[u].y, g[u].z, g[u].w};
+            float ss = 0.0f;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float a = bf_lo(w[e]), b = bf_hi(w[e]);
+                ss = fmaf(a, a, ss);
+                ss = fmaf(b, b, ss);
+            }
+#pragma unroll
+            for (int o = 1; o < LPB; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+            const float mag = sqrtf(ss);
+            const float sc = 1.0f / (mag + p.decomp_eps);
+            if ((lane & (LPB - 1)) == 0 && c0 < n) {     // first lane of a block that starts before n
+                const long long o = (long long)row * it.kb + c0 / BLK;
+                if (p.do_mag) {
+                    const float ma = p.beta1 * it.mag_avg[o] + (1.0f - p.beta1) * mag;
+                    const float mas = p.beta2 * it.mag_avg_sq[o] + (1.0f - p.beta2) * mag * mag;
+                    it.mag_avg[o] = ma;
+                    it.mag_avg_sq[o] = mas;
+                    it.dM[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
+                }
+            }
+            if (c0 < n) {
+                const long long off = (long long)row * n + c0;
+                uint32_t vh[4], vl[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float v0 = bf_lo(w[e]) * sc, v1 = bf_hi(w[e]) * sc;
+                    vh[e] = pack_bf16x2(v0, v1);
+                    vl[e] = pack_bf16x2(v0 - bf_lo(vh[e]), v1 - bf_hi(vh[e]));
+                }
+                *reinterpret_cast<uint4*>(it.Vhi + off) = make_uint4(vh[0], vh[1], vh[2], vh[3]);
+                if (p.hilo) *reinterpret_cast<uint4*>(it.Vlo + off) = make_uint4(vl[0], vl[1], vl[2], vl[3]);
+            }
+        }
+    }
+}
+
+// ===========================================================================
+// K1: projection R = P^T V (tile 128 ranks x 256 columns x 64 rows, MN-major
+// operands), Optimizer_V (Adam) in the epilogue, N written in bf16.  HILO
+// adds the MMA with V_lo (first Adam step).
+// ===========================================================================
+template <bool HILO>
 __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constant__ K1Params p) {
+    constexpr int STAGES = K1Cfg<HILO>::STAGES;
+    constexpr int STAGE_BYTES = K1Cfg<HILO>::STAGE_BYTES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
-    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + K1_STAGES * K1_STAGE_BYTES + GUARD_BYTES);
+    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + 4 * (K1_A_BYTES + K1_B_BYTES) + GUARD_BYTES);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int* abort_flag = &ctl->abort;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < K1_STAGES; ++s) {
+        for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->xform[s]), 256);
             ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -165,6 +267,7 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = ctl->tmem_base;
+    const int t_begin = p.cta_start[blockIdx.x], t_end = p.cta_start[blockIdx.x + 1];
 
     if (warp == 0) {
         // ------------------------------------------------------ TMA producer
@@ -173,31 +276,37 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
             uint32_t phase = 0;
             uint32_t issued = 0, last_par = 0;
             bool ok = true;
-            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
+            for (int t = t_begin; t < t_end && ok; ++t) {
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
-                const CUtensorMap* pmap = &p.maps[tl.mod * 4 + 0];
-                const CUtensorMap* gmap = &p.gmap[tl.slot];
+                const CUtensorMap* pmap = &p.maps[tl.mod * kMaps + 0];
+                const CUtensorMap* vmap = p.decompose ? &p.maps[tl.mod * kMaps + 4] : &p.gmap[tl.slot];
+                const CUtensorMap* lmap = &p.maps[tl.mod * kMaps + 5];
                 const int r0 = tl.t0 * K1_BM, n0 = tl.t1 * K1_BN;
                 const int nk = (md.m + K1_BK - 1) / K1_BK;
                 for (int kb = 0; kb < nk; ++kb) {
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
                     const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
-                    ptx::mbar_arrive_expect_tx(fb, K1_TX_BYTES);
-                    const uint32_t a = ptx::smem_u32(smem + stage * K1_STAGE_BYTES);
+                    ptx::mbar_arrive_expect_tx(fb, STAGE_BYTES);
+                    const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
                     const uint32_t b = a + K1_A_BYTES;
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) ptx::tma_load_2d(a + c * 8192, pmap, fb, r0 + 64 * c, kb * K1_BK);
+                    for (int c = 0; c < 2; ++c) ptx::tma_load_2d(a + c * 8192, pmap, fb, r0 + 64 * c, kb * K1_BK);
 #pragma unroll
-                    for (int c = 0; c < 2; ++c) ptx::tma_load_2d(b + c * 8192, gmap, fb, n0 + 64 * c, kb * K1_BK);
+                    for (int c = 0; c < 4; ++c) ptx::tma_load_2d(b + c * 8192, vmap, fb, n0 + 64 * c, kb * K1_BK);
+                    if (HILO) {
+#pragma unroll
+                        for (int c = 0; c < 4; ++c)
+                            ptx::tma_load_2d(b + K1_B_BYTES + c * 8192, lmap, fb, n0 + 64 * c, kb * K1_BK);
+                    }
                     issued |= 1u << stage;
                     last_par = (last_par & ~(1u << stage)) | (phase << stage);
-                    if (++stage == K1_STAGES) { stage = 0; phase ^= 1; }
+                    if (++stage == STAGES) { stage = 0; phase ^= 1; }
                 }
             }
             if (!ok) {   // let the copies already in flight land before the CTA exits
-                for (int s = 0; s < K1_STAGES; ++s)
+                for (int s = 0; s < STAGES; ++s)
                     if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
             }
         }
@@ -210,39 +319,32 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
             int buf = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
-            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
+            for (int t = t_begin; t < t_end && ok; ++t) {
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
-                const int r0 = tl.t0 * K1_BM;
-                const int nh = (r0 + 128 < md.r) ? 2 : 1;
                 const int nk = (md.m + K1_BK - 1) / K1_BK;
                 if (!ptx::mbar_wait(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
                                     MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
                 ptx::tc_fence_after();
                 const uint32_t d0 = tmem + buf * 256;
                 for (int kb = 0; kb < nk; ++kb) {
-                    const uint32_t wb = DECOMP ? ptx::smem_u32(&ctl->xform[stage]) : ptx::smem_u32(&ctl->full[stage]);
-                    if (!ptx::mbar_wait(wb, phase, abort_flag, p.status, MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) {
-                        ok = false;
-                        break;
-                    }
+                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
                     ptx::tc_fence_after();
-                    const uint32_t a = ptx::smem_u32(smem + stage * K1_STAGE_BYTES);
+                    const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
                     const uint32_t b = a + K1_A_BYTES;
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk) {
+                        const uint64_t adesc = ptx::smem_desc_sw128(a + kk * 2048, 8192, 1024);
                         const uint64_t bdesc = ptx::smem_desc_sw128(b + kk * 2048, 8192, 1024);
-                        const uint64_t ldesc = ptx::smem_desc_sw128(b + K1_B_BYTES + kk * 2048, 8192, 1024);
-                        for (int h = 0; h < nh; ++h) {
-                            const uint64_t adesc = ptx::smem_desc_sw128(a + h * 16384 + kk * 2048, 8192, 1024);
-                            ptx::mma_f16(d0 + h * 128, adesc, bdesc, idesc, (kb | kk) != 0);
-                            // P^T V_lo: the bf16 rounding residual of V, so that R carries
-                            // about 16 significant bits (P is exact in bf16)
-                            if (DECOMP && p.hilo) ptx::mma_f16(d0 + h * 128, adesc, ldesc, idesc, 1);
+                        ptx::mma_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
+                        if (HILO) {   // P^T V_lo: the bf16 rounding residual of V
+                            const uint64_t ldesc = ptx::smem_desc_sw128(b + K1_B_BYTES + kk * 2048, 8192, 1024);
+                            ptx::mma_f16(d0, adesc, ldesc, idesc, 1);
                         }
                     }
                     ptx::mma_commit(ptx::smem_u32(&ctl->empty[stage]));
-                    if (++stage == K1_STAGES) { stage = 0; phase ^= 1; }
+                    if (++stage == STAGES) { stage = 0; phase ^= 1; }
                 }
                 if (!ok) break;
                 ptx::mma_commit(ptx::smem_u32(&ctl->accf[buf]));
@@ -252,212 +354,89 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
             ptx::mma_commit(ptx::smem_u32(&ctl->drain));
             wait_drain(ptx::smem_u32(&ctl->drain), 0);
         }
-    } else if (warp < 10) {
-        // ------------------------------------------------- transform warps
-        if (DECOMP) {
-            // 256 threads: lane bits 0-2 = row within an 8-row group, bit 3 = unit
-            // half (16-byte units 0-3 or 4-7 of the 128-byte row), bit 4 =
-            // 64-column chunk, warp = 8-row group.  Each quarter-warp then touches
-            // 8 distinct rows of one chunk (conflict-free under the 128-byte
-            // swizzle); the threads sharing a block are lanes ^ 8 and ^ 16.
-            const int tid = threadIdx.x - 64;           // 0..255
-            const int k = ((tid >> 5) << 3) | (tid & 7);  // row within the stage (0..63)
-            const int hu = (tid >> 3) & 1;              // unit half
-            const int hc = (tid >> 4) & 1;              // 64-column chunk
-            const uint32_t x = static_cast<uint32_t>(k & 7);
-            constexpr int UB = BLK / 8;                 // 16-byte units per block
-            constexpr int UPB = UB < 4 ? UB : 4;        // units of a block held by this thread
-            constexpr int NBT = 4 / UPB;                // blocks (or block parts) per thread
-            int stage = 0;
-            uint32_t phase = 0;
-            bool ok = true;
-            for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
-                const TcTile tl = p.tiles[t];
-                const TcMod& md = p.mods[tl.mod];
-                const int n0 = tl.t1 * K1_BN;
-                const bool do_mag = (tl.t0 == 0);
-                const int mm = md.m, mkb = md.kb;
-                float* const mag_avg = md.mag_avg;
-                float* const mag_avg_sq = md.mag_avg_sq;
-                float* const dMp = md.dM;
-                const int nk = (mm + K1_BK - 1) / K1_BK;
-                const bool owner = (UB < 8) || (hu == 0 && (UB < 16 || hc == 0));
-                const bool mag_here = do_mag && owner;
-                const int gb0 = (n0 + hc * 64 + hu * 32) / BLK;
-                // the magnitude moments of the next stage are loaded one stage ahead,
-                // so their latency is not on the path to the MMA
-                float pma[NBT], pmas[NBT];
-#pragma unroll
-                for (int bl = 0; bl < NBT; ++bl) { pma[bl] = 0.0f; pmas[bl] = 0.0f; }
-                if (mag_here && k < mm) {
-#pragma unroll
-                    for (int bl = 0; bl < NBT; ++bl) {
-                        const int gb = gb0 + (UB < 8 ? bl : 0);
-                        if (gb < mkb) {
-                            pma[bl] = mag_avg[(long long)k * mkb + gb];
-                            pmas[bl] = mag_avg_sq[(long long)k * mkb + gb];
-                        }
-                    }
-                }
-                for (int kb = 0; kb < nk; ++kb) {
-                    float cma[NBT], cmas[NBT];
-#pragma unroll
-                    for (int bl = 0; bl < NBT; ++bl) { cma[bl] = pma[bl]; cmas[bl] = pmas[bl]; }
-                    const int nrow = (kb + 1) * K1_BK + k;
-                    if (mag_here && nrow < mm) {
-#pragma unroll
-                        for (int bl = 0; bl < NBT; ++bl) {
-                            const int gb = gb0 + (UB < 8 ? bl : 0);
-                            if (gb < mkb) {
-                                pma[bl] = mag_avg[(long long)nrow * mkb + gb];
-                                pmas[bl] = mag_avg_sq[(long long)nrow * mkb + gb];
-                            }
-                        }
-                    }
-                    const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
-                                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
-                    if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
-                    uint8_t* row = smem + stage * K1_STAGE_BYTES + K1_A_BYTES + hc * 8192 + k * 128;
-                    uint4 d[4];
-#pragma unroll
-                    for (int u = 0; u < 4; ++u)
-                        d[u] = *reinterpret_cast<const uint4*>(row + (((hu * 4 + u) ^ x) << 4));
-                    float ssu[4];
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const uint32_t w[4] = {d[u].x, d[u].y, d[u].z, d[u].w};
-                        float s2 = 0.0f;
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float lo = bf_lo(w[e]), hi = bf_hi(w[e]);
-                            s2 = fmaf(lo, lo, s2);
-                            s2 = fmaf(hi, hi, s2);
-                        }
-                        ssu[u] = s2;
-                    }
-                    float ssb[NBT];
-#pragma unroll
-                    for (int bl = 0; bl < NBT; ++bl) {
-                        float s2 = 0.0f;
-#pragma unroll
-                        for (int u = 0; u < UPB; ++u) s2 += ssu[bl * UPB + u];
-                        ssb[bl] = s2;
-                    }
-                    if (UB >= 8) ssb[0] += __shfl_xor_sync(0xffffffffu, ssb[0], 8);    // other unit half
-                    if (UB >= 16) ssb[0] += __shfl_xor_sync(0xffffffffu, ssb[0], 16);  // other chunk
-                    float inv[NBT];
-                    float mag[NBT];
-#pragma unroll
-                    for (int bl = 0; bl < NBT; ++bl) {
-                        mag[bl] = sqrtf(ssb[bl]);
-                        inv[bl] = 1.0f / (mag[bl] + p.decomp_eps);
-                    }
-                    uint8_t* lrow = row + K1_B_BYTES;
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const float sc = inv[u / UPB];
-                        const uint32_t w[4] = {d[u].x, d[u].y, d[u].z, d[u].w};
-                        uint32_t hi[4], lo[4];
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float v0 = bf_lo(w[e]) * sc, v1 = bf_hi(w[e]) * sc;
-                            hi[e] = pack_bf16x2(v0, v1);
-                            lo[e] = pack_bf16x2(v0 - bf_lo(hi[e]), v1 - bf_hi(hi[e]));
-                        }
-                        const uint32_t off = ((hu * 4 + u) ^ x) << 4;
-                        *reinterpret_cast<uint4*>(row + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                        if (p.hilo) *reinterpret_cast<uint4*>(lrow + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-                    }
-                    ptx::fence_proxy_async_smem();
-                    ptx::mbar_arrive(ptx::smem_u32(&ctl->xform[stage]));
-                    // Optimizer_M on the block magnitudes, once per (row, block)
-                    const int grow = kb * K1_BK + k;
-                    if (mag_here && grow < mm) {
-#pragma unroll
-                        for (int bl = 0; bl < NBT; ++bl) {
-                            const int gb = gb0 + (UB < 8 ? bl : 0);
-                            if (gb < mkb) {
-                                const long long o = (long long)grow * mkb + gb;
-                                const float ma = p.beta1 * cma[bl] + (1.0f - p.beta1) * mag[bl];
-                                const float mas = p.beta2 * cmas[bl] + (1.0f - p.beta2) * mag[bl] * mag[bl];
-                                mag_avg[o] = ma;
-                                mag_avg_sq[o] = mas;
-                                dMp[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
-                            }
-                        }
-                    }
-                    if (++stage == K1_STAGES) { stage = 0; phase ^= 1; }
-                }
-            }
-        }
     } else {
         // ------------------------------------------------- epilogue warps
-        const int ew = warp - 10;                      // 0..7
-        const int q = warp & 3;                        // TMEM lane quarter of this warp
-        const int h = ew >> 2;                         // accumulator half (rows 0-127 / 128-255)
+        // 8 warps: TMEM lane quarter q = warp % 4 (rank row), column half ch
+        // (128 of the 256 columns, 8 chunks of 16).  The moments of the next
+        // chunk are loaded while the current one is updated.
+        const int ew = warp - 2;                       // 0..7
+        const int q = warp & 3;
+        const int ch = ew >> 2;
         int buf = 0;
         uint32_t acc_phase = 0;
         bool ok = true;
-        for (int t = p.cta_start[blockIdx.x]; t < p.cta_start[blockIdx.x + 1] && ok; ++t) {
+        for (int t = t_begin; t < t_end && ok; ++t) {
             const TcTile tl = p.tiles[t];
             const TcMod& md = p.mods[tl.mod];
+            const int rr = md.r, nn = md.n;
+            float* const ea_p = md.exp_avg;
+            float* const es_p = md.exp_avg_sq;
+            uint16_t* const nb_p = md.Nb;
             const int r0 = tl.t0 * K1_BM, n0 = tl.t1 * K1_BN;
+            const int a = r0 + q * 32 + lane;
+            const bool row_ok = a < rr;
+            const int jbase = n0 + ch * 128;
+            float4 pa0 = make_float4(0.f, 0.f, 0.f, 0.f), pa1 = pa0, pa2 = pa0, pa3 = pa0;
+            float4 ps0 = pa0, ps1 = pa0, ps2 = pa0, ps3 = pa0;
+            if (row_ok && jbase + 16 <= nn) {
+                const float4* x = reinterpret_cast<const float4*>(ea_p + (long long)a * nn + jbase);
+                const float4* y = reinterpret_cast<const float4*>(es_p + (long long)a * nn + jbase);
+                pa0 = x[0]; pa1 = x[1]; pa2 = x[2]; pa3 = x[3];
+                ps0 = y[0]; ps1 = y[1]; ps2 = y[2]; ps3 = y[3];
+            }
             const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
                                             MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
             if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
             ptx::tc_fence_after();
-            const bool half_valid = (r0 + h * 128) < md.r;
-            if (half_valid) {
-                const int a = r0 + h * 128 + q * 32 + lane;
-                const bool row_ok = a < md.r;
 #pragma unroll 1
-                for (int c = 0; c < K1_BN / 16; ++c) {
-                    float v[16];
-                    __syncwarp();
-                    ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + h * 128 + c * 16, v);
-                    const int j0 = n0 + c * 16;
-                    if (!row_ok || j0 >= md.n) continue;
-                    const long long o = (long long)a * md.n + j0;
-                    if (j0 + 16 <= md.n) {
-                        float4* ea4 = reinterpret_cast<float4*>(md.exp_avg + o);
-                        float4* es4 = reinterpret_cast<float4*>(md.exp_avg_sq + o);
-                        float ea[16], es[16];
+            for (int c = 0; c < 8; ++c) {
+                const int j0 = jbase + c * 16;
+                float ea[16] = {pa0.x, pa0.y, pa0.z, pa0.w, pa1.x, pa1.y, pa1.z, pa1.w,
+                                pa2.x, pa2.y, pa2.z, pa2.w, pa3.x, pa3.y, pa3.z, pa3.w};
+                float es[16] = {ps0.x, ps0.y, ps0.z, ps0.w, ps1.x, ps1.y, ps1.z, ps1.w,
+                                ps2.x, ps2.y, ps2.z, ps2.w, ps3.x, ps3.y, ps3.z, ps3.w};
+                if (c + 1 < 8 && row_ok && j0 + 32 <= nn) {
+                    const float4* x = reinterpret_cast<const float4*>(ea_p + (long long)a * nn + j0 + 16);
+                    const float4* y = reinterpret_cast<const float4*>(es_p + (long long)a * nn + j0 + 16);
+                    pa0 = x[0]; pa1 = x[1]; pa2 = x[2]; pa3 = x[3];
+                    ps0 = y[0]; ps1 = y[1]; ps2 = y[2]; ps3 = y[3];
+                }
+                float v[16];
+                __syncwarp();
+                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + ch * 128 + c * 16, v);
+                if (!row_ok || j0 >= nn) continue;
+                const long long o = (long long)a * nn + j0;
+                if (j0 + 16 <= nn) {
+                    float nv[16];
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float4 x = ea4[e], y = es4[e];
-                            ea[4 * e] = x.x; ea[4 * e + 1] = x.y; ea[4 * e + 2] = x.z; ea[4 * e + 3] = x.w;
-                            es[4 * e] = y.x; es[4 * e + 1] = y.y; es[4 * e + 2] = y.z; es[4 * e + 3] = y.w;
-                        }
-                        uint32_t nb[8];
-                        float nv[16];
+                    for (int e = 0; e < 16; ++e) {
+                        ea[e] = p.beta1 * ea[e] + (1.0f - p.beta1) * v[e];
+                        es[e] = p.beta2 * es[e] + (1.0f - p.beta2) * v[e] * v[e];
+                        nv[e] = (ea[e] / p.bc1) / (sqrtf(es[e] / p.bc2) + p.adam_eps);
+                    }
+                    float4* ea4 = reinterpret_cast<float4*>(ea_p + o);
+                    float4* es4 = reinterpret_cast<float4*>(es_p + o);
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            ea[e] = p.beta1 * ea[e] + (1.0f - p.beta1) * v[e];
-                            es[e] = p.beta2 * es[e] + (1.0f - p.beta2) * v[e] * v[e];
-                            nv[e] = (ea[e] / p.bc1) / (sqrtf(es[e] / p.bc2) + p.adam_eps);
-                        }
+                    for (int e = 0; e < 4; ++e) {
+                        ea4[e] = make_float4(ea[4 * e], ea[4 * e + 1], ea[4 * e + 2], ea[4 * e + 3]);
+                        es4[e] = make_float4(es[4 * e], es[4 * e + 1], es[4 * e + 2], es[4 * e + 3]);
+                    }
+                    uint4* n4 = reinterpret_cast<uint4*>(nb_p + o);
+                    n4[0] = make_uint4(pack_bf16x2(nv[0], nv[1]), pack_bf16x2(nv[2], nv[3]),
+                                       pack_bf16x2(nv[4], nv[5]), pack_bf16x2(nv[6], nv[7]));
+                    n4[1] = make_uint4(pack_bf16x2(nv[8], nv[9]), pack_bf16x2(nv[10], nv[11]),
+                                       pack_bf16x2(nv[12], nv[13]), pack_bf16x2(nv[14], nv[15]));
+                } else {
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) nb[e] = pack_bf16x2(nv[2 * e], nv[2 * e + 1]);
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            ea4[e] = make_float4(ea[4 * e], ea[4 * e + 1], ea[4 * e + 2], ea[4 * e + 3]);
-                            es4[e] = make_float4(es[4 * e], es[4 * e + 1], es[4 * e + 2], es[4 * e + 3]);
-                        }
-                        uint4* n4 = reinterpret_cast<uint4*>(md.Nb + o);
-                        n4[0] = make_uint4(nb[0], nb[1], nb[2], nb[3]);
-                        n4[1] = make_uint4(nb[4], nb[5], nb[6], nb[7]);
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            if (j0 + e >= md.n) continue;
-                            const float ea = p.beta1 * md.exp_avg[o + e] + (1.0f - p.beta1) * v[e];
-                            const float es = p.beta2 * md.exp_avg_sq[o + e] + (1.0f - p.beta2) * v[e] * v[e];
-                            md.exp_avg[o + e] = ea;
-                            md.exp_avg_sq[o + e] = es;
-                            const float nv = (ea / p.bc1) / (sqrtf(es / p.bc2) + p.adam_eps);
-                            __nv_bfloat16 hb = __float2bfloat16_rn(nv);
-                            md.Nb[o + e] = *reinterpret_cast<uint16_t*>(&hb);
-                        }
+                    for (int e = 0; e < 16; ++e) {
+                        if (j0 + e >= nn) continue;
+                        const float x = p.beta1 * ea_p[o + e] + (1.0f - p.beta1) * v[e];
+                        const float y = p.beta2 * es_p[o + e] + (1.0f - p.beta2) * v[e] * v[e];
+                        ea_p[o + e] = x;
+                        es_p[o + e] = y;
+                        const float nv = (x / p.bc1) / (sqrtf(y / p.bc2) + p.adam_eps);
+                        __nv_bfloat16 hb = __float2bfloat16_rn(nv);
+                        nb_p[o + e] = *reinterpret_cast<uint16_t*>(&hb);
                     }
                 }
             }
@@ -526,8 +505,8 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             for (int t = t_begin; t < t_end && ok; ++t) {
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
-                const CUtensorMap* amap = &p.maps[tl.mod * 4 + 1];
-                const CUtensorMap* bmap = &p.maps[tl.mod * 4 + 2];
+                const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 1];
+                const CUtensorMap* bmap = &p.maps[tl.mod * kMaps + 2];
                 const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
                 const int nk = (md.r + K2_BK - 1) / K2_BK;
                 for (int kb = 0; kb < nk; ++kb) {
@@ -598,7 +577,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             for (int t = t_begin; t < t_end && ok; ++t) {
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
-                const CUtensorMap* wmap = &p.maps[tl.mod * 4 + 3];
+                const CUtensorMap* wmap = &p.maps[tl.mod * kMaps + 3];
                 const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
                 const int nc = min(K2_BN / K2_WCOLS, (md.n - n0 + K2_WCOLS - 1) / K2_WCOLS);
                 for (int c = 0; c < nc; ++c, ++g) {
@@ -626,7 +605,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             for (int t = t_begin; t < t_end && ok; ++t) {
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
-                const CUtensorMap* wmap = &p.maps[tl.mod * 4 + 3];
+                const CUtensorMap* wmap = &p.maps[tl.mod * kMaps + 3];
                 const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
                 const int nc = min(K2_BN / K2_WCOLS, (md.n - n0 + K2_WCOLS - 1) / K2_WCOLS);
                 for (int c = 0; c < nc; ++c, ++g) {
@@ -719,6 +698,189 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
 }
 
 // ---------------------------------------------------------------- host side
+// ===========================================================================
+// KR: the products of the projector refresh (randomized subspace iteration,
+// §3.3 / App. B.2) on tensor cores:
+//   op ZT:  out (n x l) = V^T Q      (A = V read MN-major, M = n, K = m)
+//   op Y:   out (m x l) = V Z        (A = V read K-major,  M = m, K = n)
+// with V = V_hi + V_lo held as two bf16 planes (the two MMAs per k-step keep
+// ~16 significant bits of V) and the orthonormal factor Q or Z in bf16.
+// Tile 256 x 256 (two 128-row accumulators in TMEM), BK = 64, one tile per
+// CTA: the contraction (m or n >= 1024 in practice) is long enough that the
+// epilogue need not overlap the next tile.  The last column tile issues the
+// MMA with N = 64 * ceil(cols / 64), so a ragged l costs at most 48 columns.
+// ===========================================================================
+constexpr int KR_BM = 256, KR_BN = 256, KR_BK = 64;
+constexpr int KR_PLANE = KR_BM * KR_BK * 2;               // 32 KB: one A plane or the B tile
+template <bool LO> struct KrCfg {
+    static constexpr int STAGES = LO ? 2 : 3;
+    static constexpr int STAGE_BYTES = (LO ? 3 : 2) * KR_PLANE;
+};
+constexpr int KR_WARPS = 10;                              // 0 TMA, 1 MMA, 2-9 epilogue
+constexpr int KR_THREADS = KR_WARPS * 32;
+constexpr int KR_SMEM = 1024 + 6 * KR_PLANE + 2048;
+constexpr int kKrGroup = 48;
+
+struct KrParams {
+    CUtensorMap amap[kKrGroup];        // V_hi ({n, m}, box {64, 64})
+    CUtensorMap lmap[kKrGroup];        // V_lo (same geometry), unused without LO
+    CUtensorMap bmap[kKrGroup];        // Q ({l, m}) for ZT, Z ({l, n}) for Y; box {64, 64}
+    float* out[kKrGroup];
+    int M[kKrGroup], N[kKrGroup], K[kKrGroup];
+    int tiles_n[kKrGroup];
+    int tile_start[kKrGroup + 1];
+    int count;
+    int* status;
+};
+
+template <bool KMAJOR, bool LO>
+__global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constant__ KrParams p) {
+    constexpr int STAGES = KrCfg<LO>::STAGES;
+    constexpr int STAGE_BYTES = KrCfg<LO>::STAGE_BYTES;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = align1024(smem_raw);
+    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + 6 * KR_PLANE);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    volatile int* abort_flag = &ctl->abort;
+
+    // locate (problem, tile)
+    const int tile = blockIdx.x;
+    int lo = 0, hi = p.count - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.tile_start[mid] <= tile) lo = mid; else hi = mid - 1;
+    }
+    const int pi = lo;
+    const int local = tile - p.tile_start[pi];
+    const int M = p.M[pi], N = p.N[pi], K = p.K[pi];
+    const int i0 = (local / p.tiles_n[pi]) * KR_BM;
+    const int n0 = (local % p.tiles_n[pi]) * KR_BN;
+    const int nch = min(4, (N - n0 + 63) / 64);            // 64-column chunks of B in this tile
+    const int halves = (M - i0) > 128 ? 2 : 1;
+    const int nk = (K + KR_BK - 1) / KR_BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);
+        }
+        ptx::mbar_init(ptx::smem_u32(&ctl->accf[0]), 1);
+        ptx::mbar_init(ptx::smem_u32(&ctl->drain), 1);
+        ctl->abort = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(ptx::smem_u32(&ctl->tmem_base), 512);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = ctl->tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t issued = 0, last_par = 0;
+            const uint32_t bytes = (LO ? 2 : 1) * KR_PLANE + nch * 8192;
+            for (int kb = 0; kb < nk; ++kb) {
+                if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
+                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) {
+                    for (int s = 0; s < STAGES; ++s)
+                        if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
+                    break;
+                }
+                const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
+                ptx::mbar_arrive_expect_tx(fb, bytes);
+                const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
+                const uint32_t b = a + (LO ? 2 : 1) * KR_PLANE;
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    const int x = KMAJOR ? kb * KR_BK : i0 + 64 * c;
+                    const int y = KMAJOR ? i0 + 64 * c : kb * KR_BK;
+                    ptx::tma_load_2d(a + c * 8192, &p.amap[pi], fb, x, y);
+                    if (LO) ptx::tma_load_2d(a + KR_PLANE + c * 8192, &p.lmap[pi], fb, x, y);
+                }
+                for (int c = 0; c < nch; ++c) ptx::tma_load_2d(b + c * 8192, &p.bmap[pi], fb, n0 + 64 * c, kb * KR_BK);
+                issued |= 1u << stage;
+                last_par = (last_par & ~(1u << stage)) | (phase << stage);
+                if (++stage == STAGES) { stage = 0; phase ^= 1; }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t idesc = ptx::idesc_bf16(128, nch * 64, KMAJOR ? 0 : 1, 1);
+            int stage = 0;
+            uint32_t phase = 0;
+            for (int kb = 0; kb < nk; ++kb) {
+                if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
+                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) break;
+                ptx::tc_fence_after();
+                const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
+                const uint32_t b = a + (LO ? 2 : 1) * KR_PLANE;
+                for (int h = 0; h < halves; ++h) {
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const uint32_t ao = a + h * 16384 + (KMAJOR ? kk * 32 : kk * 2048);
+                        const uint64_t adesc = KMAJOR ? ptx::smem_desc_sw128(ao, 16, 1024)
+                                                      : ptx::smem_desc_sw128(ao, 8192, 1024);
+                        const uint64_t bdesc = ptx::smem_desc_sw128(b + kk * 2048, 8192, 1024);
+                        ptx::mma_f16(tmem + h * 256, adesc, bdesc, idesc, (kb | kk) != 0);
+                        if (LO) {
+                            const uint32_t lo_addr = ao + KR_PLANE;
+                            const uint64_t ldesc = KMAJOR ? ptx::smem_desc_sw128(lo_addr, 16, 1024)
+                                                          : ptx::smem_desc_sw128(lo_addr, 8192, 1024);
+                            ptx::mma_f16(tmem + h * 256, ldesc, bdesc, idesc, 1);
+                        }
+                    }
+                }
+                ptx::mma_commit(ptx::smem_u32(&ctl->empty[stage]));
+                if (++stage == STAGES) { stage = 0; phase ^= 1; }
+            }
+            ptx::mma_commit(ptx::smem_u32(&ctl->accf[0]));
+            ptx::mma_commit(ptx::smem_u32(&ctl->drain));
+            wait_drain(ptx::smem_u32(&ctl->drain), 0);
+        }
+    } else {
+        // 8 epilogue warps: lane quarter q = warp % 4, accumulator half h.
+        const int ew = warp - 2;
+        const int q = warp & 3;
+        const int h = ew >> 2;
+        const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[0]), 0, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+        if (__all_sync(0xffffffffu, got) && h < halves) {
+            ptx::tc_fence_after();
+            const int row = i0 + h * 128 + q * 32 + lane;
+            float* const orow = p.out[pi] + (long long)row * N;
+            for (int c = 0; c < nch * 4; ++c) {
+                const int j0 = n0 + c * 16;
+                if (j0 >= N) break;                       // warp-uniform
+                float v[16];
+                __syncwarp();
+                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + h * 256 + c * 16, v);
+                if (row >= M) continue;
+                if (j0 + 16 <= N && (N & 3) == 0) {
+                    float4* o4 = reinterpret_cast<float4*>(orow + j0);
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) o4[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e)
+                        if (j0 + e < N) orow[j0 + e] = v[e];
+                }
+            }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, 512);
+    }
+}
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -741,8 +903,6 @@ bool encode_bf16_2d(EncodeTiledFn enc, CUtensorMap* map, const void* ptr, uint64
 
 template <int BLK>
 void set_smem_attrs() {
-    cudaFuncSetAttribute(k1_project<BLK, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
-    cudaFuncSetAttribute(k1_project<BLK, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
     cudaFuncSetAttribute(k2_backproject<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize, K2_SMEM);
 }
 
@@ -755,7 +915,7 @@ struct TcState {
     EncodeTiledFn encode = nullptr;
     std::string err;
     std::vector<TcMod> mods;               // indexed by module id (unsupported ones left zero)
-    std::vector<CUtensorMap> maps;         // 4 per module id
+    std::vector<CUtensorMap> maps;         // kMaps per module id
     TcMod* d_mods = nullptr;
     CUtensorMap* d_maps = nullptr;
     int cap = 0;
@@ -769,6 +929,8 @@ struct TcState {
     std::map<std::vector<int>, Tiles> tiles;
     bool attrs_set = false;
     K1Params p1;                           // parameter block of the next K1 launch
+    K0Params p0;                           // parameter block of the next K0 launch
+    KrParams pr;                           // parameter block of the next refresh product launch
 };
 
 bool tc_supported(int m, int n, int r, int B, int dtype, int decompose) {
@@ -816,20 +978,23 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
     if (st == nullptr) return MOARA_OK;
     if (static_cast<int>(st->mods.size()) <= id) {
         st->mods.resize(id + 1, TcMod{});
-        st->maps.resize(4 * (id + 1));
+        st->maps.resize(kMaps * (id + 1));
     }
     if (!tc_supported(md.m, md.n, md.r, hp.block_size, md.dtype, hp.decompose) || md.Pb == nullptr) return MOARA_OK;
     TcMod t{};
     t.m = md.m; t.n = md.n; t.r = md.r; t.kb = md.kb;
+    t.Vhi = md.ws_Vhi; t.Vlo = md.ws_Vlo;
     t.W = md.W; t.exp_avg = md.exp_avg; t.exp_avg_sq = md.exp_avg_sq;
     t.mag_avg = md.mag_avg; t.mag_avg_sq = md.mag_avg_sq;
     t.Nb = reinterpret_cast<uint16_t*>(md.ws_N);
     t.dM = md.ws_dM;
-    CUtensorMap* mp = &st->maps[4 * id];
+    CUtensorMap* mp = &st->maps[kMaps * id];
     if (!encode_bf16_2d(st->encode, &mp[0], md.Pb, md.r, md.m, 64, 64) ||
         !encode_bf16_2d(st->encode, &mp[1], md.Pb, md.r, md.m, 64, 128) ||
         !encode_bf16_2d(st->encode, &mp[2], t.Nb, md.n, md.r, 64, 64) ||
-        !encode_2d(st->encode, &mp[3], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, md.W, md.n, md.m, K2_WCOLS, K2_BM)) {
+        !encode_2d(st->encode, &mp[3], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, md.W, md.n, md.m, K2_WCOLS, K2_BM) ||
+        !encode_bf16_2d(st->encode, &mp[4], t.Vhi, md.n, md.m, 64, 64) ||
+        !encode_bf16_2d(st->encode, &mp[5], t.Vlo, md.n, md.m, 64, 64)) {
         st->err = "cuTensorMapEncodeTiled failed";
         return MOARA_ERR_CUDA;
     }
@@ -849,14 +1014,14 @@ static int tc_upload(TcState* st) {
         st->d_mods = nullptr;
         st->d_maps = nullptr;
         if (cudaMalloc(&st->d_mods, sizeof(TcMod) * ncap) != cudaSuccess ||
-            cudaMalloc(&st->d_maps, sizeof(CUtensorMap) * 4 * ncap) != cudaSuccess) {
+            cudaMalloc(&st->d_maps, sizeof(CUtensorMap) * kMaps * ncap) != cudaSuccess) {
             st->err = "cudaMalloc of the tensor-core module table failed";
             return MOARA_ERR_CUDA;
         }
         st->cap = ncap;
     }
     if (cudaMemcpy(st->d_mods, st->mods.data(), sizeof(TcMod) * n, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(st->d_maps, st->maps.data(), sizeof(CUtensorMap) * 4 * n, cudaMemcpyHostToDevice) !=
+        cudaMemcpy(st->d_maps, st->maps.data(), sizeof(CUtensorMap) * kMaps * n, cudaMemcpyHostToDevice) !=
             cudaSuccess) {
         st->err = "upload of the tensor-core module table failed";
         return MOARA_ERR_CUDA;
@@ -896,8 +1061,11 @@ static void lpt_assign(const std::vector<TcTile>& tiles, const std::vector<doubl
     start[grid] = static_cast<int>(out.size());
 }
 
-// Work lists of one launch: K1 tiles (256-rank x 128-column) and K2 tiles
-// (128-row x 256-column), cost-weighted (MMA clocks vs. epilogue traffic).
+// Work lists of one launch: K1 tiles (128-rank x 256-column) and K2 tiles
+// (128-row x 256-column), cost-weighted in SM clocks: MMA time (8 clocks per
+// K row of a 128 x 256 tile) against the epilogue's HBM traffic (K1: the two
+// moments read and written and N stored, 18 bytes per entry; K2: W read and
+// written, 8 bytes per entry; about 27 bytes per clock per SM).
 static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
     auto it = st->tiles.find(ids);
     if (it != st->tiles.end()) return &it->second;
@@ -905,13 +1073,14 @@ static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
     std::vector<double> c1, c2;
     for (size_t slot = 0; slot < ids.size(); ++slot) {
         const TcMod& md = st->mods[ids[slot]];
+        // column tiles outer, rank tiles inner: CTAs that start together share
+        // the V panel of one column tile in L2
         const int nt = (md.n + K1_BN - 1) / K1_BN, rt = (md.r + K1_BM - 1) / K1_BM;
         for (int j = 0; j < nt; ++j)
             for (int i = 0; i < rt; ++i) {
                 const int rows = std::min(K1_BM, md.r - i * K1_BM);
-                const int nh = rows > 128 ? 2 : 1;
-                const double mma = 8.0 * nh * md.m;                       // clocks, with V_lo
-                const double epi = 0.8 * rows * std::min(K1_BN, md.n - j * K1_BN);
+                const double mma = 8.0 * md.m;
+                const double epi = 0.66 * rows * std::min(K1_BN, md.n - j * K1_BN);
                 k1.push_back({ids[slot], static_cast<int>(slot), i, j});
                 c1.push_back(std::max(mma, epi));
             }
@@ -919,7 +1088,7 @@ static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
         for (int i = 0; i < mt; ++i)
             for (int j = 0; j < nt2; ++j) {
                 const double mma = 8.0 * md.r;
-                const double epi = 0.36 * std::min(K2_BM, md.m - i * K2_BM) * std::min(K2_BN, md.n - j * K2_BN);
+                const double epi = 0.3 * std::min(K2_BM, md.m - i * K2_BM) * std::min(K2_BN, md.n - j * K2_BN);
                 k2.push_back({ids[slot], static_cast<int>(slot), i, j});
                 c2.push_back(std::max(mma, epi));
             }
@@ -953,13 +1122,22 @@ static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
 }
 
 template <int BLK>
-static cudaError_t launch_pair(TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2,
-                               bool decomp, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+static cudaError_t launch_blk(TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2, bool decomp,
+                              bool hilo, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+    cudaError_t e;
+    if (decomp) {
+        if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, true);
+        k0_decompose<BLK><<<st->sms * 4, 256, 0, s>>>(st->p0);
+        if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, false);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        ++*launches;
+    }
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, true);
-    if (decomp) k1_project<BLK, true><<<g1, K1_THREADS, K1_SMEM, s>>>(p1);
-    else k1_project<BLK, false><<<g1, K1_THREADS, K1_SMEM, s>>>(p1);
+    if (hilo) k1_project<true><<<g1, K1_THREADS, K1_SMEM, s>>>(p1);
+    else k1_project<false><<<g1, K1_THREADS, K1_SMEM, s>>>(p1);
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, false);
-    cudaError_t e = cudaGetLastError();
+    e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     ++*launches;
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_BACKPROJECT, s, true);
@@ -974,13 +1152,17 @@ static cudaError_t launch_pair(TcState* st, const K1Params& p1, const K2Params& 
 int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G, float bc1,
             float bc2, float lr, int first_step, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
     if (!st->attrs_set) {
+        cudaFuncSetAttribute(k1_project<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
+        cudaFuncSetAttribute(k1_project<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
         set_smem_attrs<8>(); set_smem_attrs<16>(); set_smem_attrs<32>(); set_smem_attrs<64>();
         set_smem_attrs<128>();
         st->attrs_set = true;
     }
     int rc = tc_upload(st);
     if (rc != MOARA_OK) return rc;
-    const int B = hp.decompose ? hp.block_size : 128;
+    const bool dec = hp.decompose != 0;
+    const bool hilo = dec && first_step;
+    const int B = dec ? hp.block_size : 128;
     for (int c0 = 0; c0 < n_mod; c0 += kTcGroup) {
         const int cnt = std::min(kTcGroup, n_mod - c0);
         std::vector<int> chunk(ids + c0, ids + c0 + cnt);
@@ -988,18 +1170,39 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
         if (tl == nullptr) { st->err = "tile list allocation failed"; return MOARA_ERR_CUDA; }
         K1Params& p1 = st->p1;
         std::memset(&p1, 0, sizeof(p1));
-        for (int q = 0; q < cnt; ++q) {
-            const TcMod& md = st->mods[chunk[q]];
-            if (!encode_bf16_2d(st->encode, &p1.gmap[q], G[c0 + q], md.n, md.m, 64, 64)) {
-                st->err = "cuTensorMapEncodeTiled failed for a gradient";
-                return MOARA_ERR_CUDA;
+        if (dec) {
+            K0Params& p0 = st->p0;
+            std::memset(&p0, 0, sizeof(p0));
+            p0.count = cnt;
+            p0.hilo = hilo ? 1 : 0;
+            p0.do_mag = 1;
+            p0.decomp_eps = hp.decomp_eps;
+            p0.beta1 = hp.beta1; p0.beta2 = hp.beta2; p0.adam_eps = hp.adam_eps;
+            p0.bc1 = bc1; p0.bc2 = bc2;
+            long long acc = 0;
+            for (int q = 0; q < cnt; ++q) {
+                const TcMod& md = st->mods[chunk[q]];
+                const int segs = (md.n + K0_SEG - 1) / K0_SEG;
+                p0.start[q] = acc;
+                p0.p[q] = K0Item{static_cast<const uint16_t*>(G[c0 + q]), md.Vhi, md.Vlo, md.mag_avg,
+                                 md.mag_avg_sq, md.dM, md.m, md.n, md.kb, segs};
+                acc += static_cast<long long>(md.m) * segs;
+            }
+            p0.start[cnt] = acc;
+        } else {
+            for (int q = 0; q < cnt; ++q) {
+                const TcMod& md = st->mods[chunk[q]];
+                if (!encode_bf16_2d(st->encode, &p1.gmap[q], G[c0 + q], md.n, md.m, 64, 64)) {
+                    st->err = "cuTensorMapEncodeTiled failed for a gradient";
+                    return MOARA_ERR_CUDA;
+                }
             }
         }
         p1.cta_start = tl->k1_start; p1.tiles = tl->k1;
         p1.mods = st->d_mods; p1.maps = st->d_maps; p1.status = st->d_status;
         p1.beta1 = hp.beta1; p1.beta2 = hp.beta2; p1.adam_eps = hp.adam_eps;
-        p1.bc1 = bc1; p1.bc2 = bc2; p1.decomp_eps = hp.decomp_eps;
-        p1.hilo = first_step ? 1 : 0;
+        p1.bc1 = bc1; p1.bc2 = bc2;
+        p1.decompose = dec ? 1 : 0;
         K2Params p2{};
         p2.cta_start = tl->k2_start; p2.tiles = tl->k2;
         p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;
@@ -1007,14 +1210,13 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
         p2.decompose = hp.decompose;
         const int g1 = tl->g1;
         const int g2 = tl->g2;
-        const bool dec = hp.decompose != 0;
         cudaError_t e;
         switch (B) {
-            case 8: e = launch_pair<8>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
-            case 16: e = launch_pair<16>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
-            case 32: e = launch_pair<32>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
-            case 64: e = launch_pair<64>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
-            default: e = launch_pair<128>(st, p1, p2, g1, g2, dec, s, launches, prof); break;
+            case 8: e = launch_blk<8>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
+            case 16: e = launch_blk<16>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
+            case 32: e = launch_blk<32>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
+            case 64: e = launch_blk<64>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
+            default: e = launch_blk<128>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
         }
         if (e != cudaSuccess) {
             st->err = cudaGetErrorString(e);
@@ -1025,5 +1227,103 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
 }
 
 const char* tc_last_error(const TcState* st) { return st ? st->err.c_str() : "no tensor-core state"; }
+
+int tc_refresh_products(TcState* st, int op, const TcProdItem* items, int count, cudaStream_t s,
+                        int64_t* launches) {
+    static bool attrs = false;
+    if (!attrs) {
+        cudaFuncSetAttribute(kr_product<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
+        cudaFuncSetAttribute(kr_product<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
+        cudaFuncSetAttribute(kr_product<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
+        cudaFuncSetAttribute(kr_product<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
+        attrs = true;
+    }
+    // two sub-launches: items with and without the V_lo plane
+    for (int with_lo = 0; with_lo < 2; ++with_lo) {
+        std::vector<int> sel;
+        for (int i = 0; i < count; ++i)
+            if ((items[i].Vlo != nullptr) == (with_lo == 1)) sel.push_back(i);
+        for (size_t c0 = 0; c0 < sel.size(); c0 += kKrGroup) {
+            const int cnt = static_cast<int>(std::min<size_t>(kKrGroup, sel.size() - c0));
+            KrParams& kp = st->pr;
+            std::memset(&kp, 0, sizeof(kp));
+            int total = 0;
+            for (int q = 0; q < cnt; ++q) {
+                const TcProdItem& x = items[sel[c0 + q]];
+                const int M = op == 0 ? x.n : x.m;
+                const int K = op == 0 ? x.m : x.n;
+                bool ok = encode_bf16_2d(st->encode, &kp.amap[q], x.Vhi, x.n, x.m, 64, 64);
+                if (with_lo) ok = ok && encode_bf16_2d(st->encode, &kp.lmap[q], x.Vlo, x.n, x.m, 64, 64);
+                ok = ok && encode_bf16_2d(st->encode, &kp.bmap[q], op == 0 ? x.Qbf : x.Zbf, x.l,
+                                          op == 0 ? x.m : x.n, 64, 64);
+                if (!ok) {
+                    st->err = "cuTensorMapEncodeTiled failed for a refresh operand";
+                    return MOARA_ERR_CUDA;
+                }
+                kp.out[q] = x.out;
+                kp.M[q] = M; kp.N[q] = x.l; kp.K[q] = K;
+                kp.tiles_n[q] = (x.l + KR_BN - 1) / KR_BN;
+                kp.tile_start[q] = total;
+                total += ((M + KR_BM - 1) / KR_BM) * kp.tiles_n[q];
+            }
+            kp.tile_start[cnt] = total;
+            kp.count = cnt;
+            kp.status = st->d_status;
+            if (total == 0) continue;
+            if (op == 0) {
+                if (with_lo) kr_product<false, true><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
+                else kr_product<false, false><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
+            } else {
+                if (with_lo) kr_product<true, true><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
+                else kr_product<true, false><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
+            }
+            const cudaError_t e = cudaGetLastError();
+            if (e != cudaSuccess) {
+                st->err = cudaGetErrorString(e);
+                return MOARA_ERR_CUDA;
+            }
+            ++*launches;
+        }
+    }
+    return MOARA_OK;
+}
+
+int tc_split_v(TcState* st, const TcSplitItem* items, int count, int B, float decomp_eps, cudaStream_t s,
+               int64_t* launches) {
+    for (int c0 = 0; c0 < count; c0 += kTcGroup) {
+        const int cnt = std::min(kTcGroup, count - c0);
+        K0Params& p0 = st->p0;
+        std::memset(&p0, 0, sizeof(p0));
+        p0.count = cnt;
+        p0.hilo = 1;
+        p0.do_mag = 0;
+        p0.decomp_eps = decomp_eps;
+        long long acc = 0;
+        for (int q = 0; q < cnt; ++q) {
+            const TcSplitItem& x = items[c0 + q];
+            const int segs = (x.n + K0_SEG - 1) / K0_SEG;
+            p0.start[q] = acc;
+            p0.p[q] = K0Item{static_cast<const uint16_t*>(x.G), x.Vhi, x.Vlo, nullptr, nullptr, nullptr,
+                             x.m, x.n, (x.n + B - 1) / B, segs};
+            acc += static_cast<long long>(x.m) * segs;
+        }
+        p0.start[cnt] = acc;
+        switch (B) {
+            case 8: k0_decompose<8><<<st->sms * 4, 256, 0, s>>>(p0); break;
+            case 16: k0_decompose<16><<<st->sms * 4, 256, 0, s>>>(p0); break;
+            case 32: k0_decompose<32><<<st->sms * 4, 256, 0, s>>>(p0); break;
+            case 64: k0_decompose<64><<<st->sms * 4, 256, 0, s>>>(p0); break;
+            case 128: k0_decompose<128><<<st->sms * 4, 256, 0, s>>>(p0); break;
+            default: st->err = "block size not supported on the tensor-core path"; return MOARA_ERR_UNSUPPORTED;
+        }
+        const cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) {
+            st->err = cudaGetErrorString(e);
+            return MOARA_ERR_CUDA;
+        }
+        ++*launches;
+    }
+    return MOARA_OK;
+}
 
 }  // namespace moara
