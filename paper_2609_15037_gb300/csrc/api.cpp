@@ -388,33 +388,93 @@ struct RefreshRunner {
         std::swap(a, b);
     }
 
+    // ---------------------------------------------- tensor-core helpers
+    void tc_gemm(int a_kmajor, const std::vector<moara::TcGemmItem>& items) {
+        if (items.empty()) return;
+        ProfScope ps(ctx, MOARA_PHASE_TC_REFRESH, s);
+        if (moara::tc_gemm_bf16(ctx->tc, a_kmajor, items.data(), static_cast<int>(items.size()), s,
+                                &ctx->launches) != MOARA_OK)
+            chk(cudaErrorLaunchFailure);
+    }
+
+    // out (n x l) = V^T X with X (m x l) in bf16; fp32 and/or bf16 output
+    void tc_vt_times(const std::vector<uint16_t*>& X, const std::vector<float*>& out,
+                     const std::vector<uint16_t*>& out_bf) {
+        std::vector<moara::TcGemmItem> g;
+        for (size_t i = 0; i < it.size(); ++i) {
+            const auto& x = it[i];
+            g.push_back({x.Vhi, x.Vlo, X[i], out[i], out_bf[i], x.n, x.l, x.m, 0});
+        }
+        tc_gemm(0, g);
+    }
+
+    // out (m x l) = V Z with Z (n x l) in bf16
+    void tc_v_times(const std::vector<uint16_t*>& Z, const std::vector<float*>& out,
+                    const std::vector<uint16_t*>& out_bf) {
+        std::vector<moara::TcGemmItem> g;
+        for (size_t i = 0; i < it.size(); ++i) {
+            const auto& x = it[i];
+            g.push_back({x.Vhi, x.Vlo, Z[i], out[i], out_bf[i], x.m, x.l, x.n, 0});
+        }
+        tc_gemm(1, g);
+    }
+
+    // One shifted CholeskyQR pass on tensor cores: X_out = X_in R^-1 with
+    // R^T R = X_in^T X_in + shift, X_in and X_out bf16 (rows x l).  The Gram
+    // matrix of the bf16 X_in is exact up to fp32 accumulation; R^-1 is
+    // applied in bf16.  Upper-triangular R keeps the nested column spans of
+    // X_in, which is all the subspace iteration needs from this step.
+    void tc_cholqr_pass(const std::vector<uint16_t*>& Xin, const std::vector<uint16_t*>& Xout,
+                        const std::vector<int>& rows, float shift_rel) {
+        std::vector<moara::TcGemmItem> gram;
+        for (size_t i = 0; i < it.size(); ++i) {
+            const int l = it[i].l;
+            gram.push_back({Xin[i], nullptr, Xin[i], it[i].Cg, nullptr, l, l, rows[i], 0});
+        }
+        tc_gemm(0, gram);
+        cholesky_blocked(rows, shift_rel);
+        tri_inverse(/*have_diag=*/true);
+        {   // (R^-1) in bf16: the transpose of the lower-triangular Linv, into Tt
+            moara::SmallBatch sb = small();
+            for (size_t i = 0; i < it.size(); ++i) {
+                sb.a[i] = it[i].Linv; sb.h[i] = reinterpret_cast<uint16_t*>(it[i].Tt); sb.l[i] = it[i].l;
+            }
+            chk(moara::launch_transpose_bf16(sb, s, &ctx->launches));
+        }
+        std::vector<moara::TcGemmItem> apply;
+        for (size_t i = 0; i < it.size(); ++i) {
+            const int l = it[i].l;
+            apply.push_back({Xin[i], nullptr, reinterpret_cast<const uint16_t*>(it[i].Tt), nullptr, Xout[i],
+                             rows[i], l, l, 1});
+        }
+        tc_gemm(1, apply);
+    }
+
     void run() {
         const int n_it = static_cast<int>(it.size());
         const moara_hparams& hp = ctx->hp;
+        const bool tc = n_it > 0 && it[0].tc;   // groups are all tensor-core or all fp32
         for (auto& x : it) chk(cudaMemsetAsync(x.fail, 0, sizeof(int), s));
-        std::vector<int> simt_ids, tc_ids;
-        for (int i = 0; i < n_it; ++i) (it[i].tc ? tc_ids : simt_ids).push_back(i);
-        // block scales of Decompose(G, B) when the source is V: fp32 scales for
-        // the SIMT products, bf16 planes V_hi + V_lo for the tensor-core ones
-        if (src_v && !simt_ids.empty()) {
+        // Decompose(G, B) when the source is V: fp32 block scales for the fp32
+        // products, bf16 planes V_hi + V_lo for the tensor-core ones
+        if (src_v && !tc) {
             moara::DecompBatch db{};
-            db.count = static_cast<int>(simt_ids.size()); db.B = hp.block_size; db.do_mag = 0;
-            db.decomp_eps = hp.decomp_eps;
+            db.count = n_it; db.B = hp.block_size; db.do_mag = 0; db.decomp_eps = hp.decomp_eps;
             long long acc = 0;
-            for (int q = 0; q < db.count; ++q) {
-                const auto& x = it[simt_ids[q]];
-                db.item_start[q] = acc;
-                db.p[q] = moara::DecompItem{x.G, x.inv, nullptr, nullptr, nullptr, x.m, x.n, x.kb, x.dtype};
-                acc += (long long)x.m * x.kb;
+            for (int i = 0; i < n_it; ++i) {
+                db.item_start[i] = acc;
+                db.p[i] = moara::DecompItem{it[i].G, it[i].inv, nullptr, nullptr, nullptr,
+                                            it[i].m, it[i].n, it[i].kb, it[i].dtype};
+                acc += (long long)it[i].m * it[i].kb;
             }
-            db.item_start[db.count] = acc;
+            db.item_start[n_it] = acc;
             chk(moara::launch_decompose(db, s, &ctx->launches));
         }
-        if (src_v && !tc_ids.empty()) {
+        if (src_v && tc) {
             std::vector<moara::TcSplitItem> sp;
-            for (int i : tc_ids) sp.push_back({it[i].G, it[i].Vhi_w, it[i].Vlo, it[i].m, it[i].n});
-            if (moara::tc_split_v(ctx->tc, sp.data(), static_cast<int>(sp.size()), hp.block_size, hp.decomp_eps, s,
-                                  &ctx->launches) != MOARA_OK)
+            for (auto& x : it) sp.push_back({x.G, x.Vhi_w, x.Vlo, x.m, x.n});
+            if (moara::tc_split_v(ctx->tc, sp.data(), n_it, hp.block_size, hp.decomp_eps, s, &ctx->launches) !=
+                MOARA_OK)
                 chk(cudaErrorLaunchFailure);
         }
         // Gaussian test matrix Omega (n x l)
@@ -425,88 +485,108 @@ struct RefreshRunner {
             }
             chk(moara::launch_philox_gaussian(sb, s, &ctx->launches));
         }
-        for (int i : tc_ids)
-            chk(moara::launch_f32_to_bf16(it[i].Omega, nullptr, it[i].Zbf, (long long)it[i].n * it[i].l, s,
-                                          &ctx->launches));
         std::vector<float*> Qa(n_it), Qb(n_it), Za(n_it), Zb(n_it), Xa(n_it), Xb(n_it);
         std::vector<int> rows_m(n_it), rows_n(n_it), rows_l(n_it);
-        std::vector<uint16_t*> qbf(n_it, nullptr), zbf(n_it, nullptr);
+        std::vector<uint16_t*> qbf(n_it), zbf(n_it), ybf(n_it), zraw(n_it);
+        std::vector<float*> nof(n_it, nullptr);
+        std::vector<uint16_t*> nob(n_it, nullptr);
         for (int i = 0; i < n_it; ++i) {
             Qa[i] = it[i].Qa; Qb[i] = it[i].Qb; Za[i] = it[i].Za; Zb[i] = it[i].Zb;
             Xa[i] = it[i].Xa; Xb[i] = it[i].Xb;
             rows_m[i] = it[i].m; rows_n[i] = it[i].n; rows_l[i] = it[i].l;
-            if (it[i].tc) { qbf[i] = it[i].Qbf; zbf[i] = it[i].Zbf; }
+            qbf[i] = it[i].Qbf; zbf[i] = it[i].Zbf;
+            // bf16 iterates of the tensor-core power iterations live in the
+            // fp32 buffers (4 bytes per entry hold the 2-byte plane)
+            ybf[i] = reinterpret_cast<uint16_t*>(it[i].Qa);
+            zraw[i] = reinterpret_cast<uint16_t*>(it[i].Za);
         }
-        // tensor-core products of the TC items: op 0 out = V^T Q_bf16, op 1 out = V Z_bf16
-        auto tc_products = [&](int op, std::vector<float*>& out) {
-            if (tc_ids.empty()) return;
-            ProfScope ps(ctx, MOARA_PHASE_TC_REFRESH, s);
-            std::vector<moara::TcProdItem> pi;
-            for (int i : tc_ids)
-                pi.push_back({it[i].Vhi, it[i].Vlo, it[i].Qbf, it[i].Zbf, out[i], it[i].m, it[i].n, it[i].l});
-            if (moara::tc_refresh_products(ctx->tc, op, pi.data(), static_cast<int>(pi.size()), s,
-                                           &ctx->launches) != MOARA_OK)
-                chk(cudaErrorLaunchFailure);
-        };
-        // Y = V * Z  (m x l); Z is Omega on the first call
-        auto v_times = [&](std::vector<float*>& rhs, std::vector<float*>& out) {
-            for (int d = 0; d < 2; ++d) {  // per-dtype sub-batches
-                std::vector<int> sel;
-                for (int i : simt_ids) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
-                if (sel.empty()) continue;
-                moara::GemmKind k{moara::A_KCONTIG, moara::B_NCONTIG, src_v, 0, d, 0, moara::EPI_STORE};
-                moara::GemmBatch b{};
-                b.count = static_cast<int>(sel.size());
-                b.B = hp.block_size;
-                for (int q = 0; q < b.count; ++q) {
-                    const auto& x = it[sel[q]];
-                    moara::GemmProb& p = b.p[q];
-                    p = moara::GemmProb{};
-                    p.A = x.G; p.a_inv = x.inv; p.Bm = rhs[sel[q]]; p.C = out[sel[q]];
-                    p.M = x.m; p.N = x.l; p.K = x.n; p.lda = x.n; p.ldb = x.l; p.ldc = x.l; p.kb = x.kb;
-                    p.a_bf16 = d;
+        const float u_rnd = 5.9604645e-08f;   // fp32 unit roundoff
+        if (tc) {
+            // Subspace iteration with every product and every intermediate
+            // orthonormalisation on tensor cores; only the last Y gets the
+            // fp32 CholeskyQR2 that makes Q orthonormal for the Rayleigh-Ritz step.
+            for (int i = 0; i < n_it; ++i)
+                chk(moara::launch_f32_to_bf16(it[i].Omega, nullptr, it[i].Zbf, (long long)it[i].n * it[i].l, s,
+                                              &ctx->launches));
+            const int q_it = hp.power_iters;
+            if (q_it == 0) {
+                tc_v_times(zbf, Qa, nob);
+            } else {
+                tc_v_times(zbf, nof, ybf);
+                tc_cholqr_pass(ybf, qbf, rows_m, 2.0f * u_rnd);
+                for (int q = 0; q < q_it; ++q) {
+                    tc_vt_times(qbf, nof, zraw);
+                    tc_cholqr_pass(zraw, zbf, rows_n, 2.0f * u_rnd);
+                    if (q + 1 < q_it) {
+                        tc_v_times(zbf, nof, ybf);
+                        tc_cholqr_pass(ybf, qbf, rows_m, 2.0f * u_rnd);
+                    } else {
+                        tc_v_times(zbf, Qa, nob);
+                    }
                 }
-                chk(moara::launch_gemm(k, b, s, &ctx->launches));
             }
-            tc_products(1, out);
-        };
-        // Z = V^T * Q  (n x l)
-        auto vt_times = [&](std::vector<float*>& rhs, std::vector<float*>& out) {
-            for (int d = 0; d < 2; ++d) {
-                std::vector<int> sel;
-                for (int i : simt_ids) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
-                if (sel.empty()) continue;
-                moara::GemmKind k{moara::A_MCONTIG, moara::B_NCONTIG, src_v, 0, d, 0, moara::EPI_STORE};
-                moara::GemmBatch b{};
-                b.count = static_cast<int>(sel.size());
-                b.B = hp.block_size;
-                for (int q = 0; q < b.count; ++q) {
-                    const auto& x = it[sel[q]];
-                    moara::GemmProb& p = b.p[q];
-                    p = moara::GemmProb{};
-                    p.A = x.G; p.a_inv = x.inv; p.Bm = rhs[sel[q]]; p.C = out[sel[q]];
-                    p.M = x.n; p.N = x.l; p.K = x.m; p.lda = x.n; p.ldb = x.l; p.ldc = x.l; p.kb = x.kb;
-                    p.a_bf16 = d;
+            cholqr2s(Qa, Qb, rows_m, &qbf);     // Q in Qb (fp32) and qbf
+            // Rayleigh-Ritz matrix C = Z^T Z with Z = V^T Q (bf16 operands)
+            tc_vt_times(qbf, nof, zraw);
+            std::vector<moara::TcGemmItem> gram;
+            for (int i = 0; i < n_it; ++i)
+                gram.push_back({zraw[i], nullptr, zraw[i], it[i].Cr, nullptr, it[i].l, it[i].l, it[i].n, 0});
+            tc_gemm(0, gram);
+        } else {
+            // Y = V * Z  (m x l), fp32 SIMT products (V scaled on the fly)
+            auto v_times = [&](std::vector<float*>& rhs, std::vector<float*>& out) {
+                for (int d = 0; d < 2; ++d) {  // per-dtype sub-batches
+                    std::vector<int> sel;
+                    for (int i = 0; i < n_it; ++i) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
+                    if (sel.empty()) continue;
+                    moara::GemmKind k{moara::A_KCONTIG, moara::B_NCONTIG, src_v, 0, d, 0, moara::EPI_STORE};
+                    moara::GemmBatch b{};
+                    b.count = static_cast<int>(sel.size());
+                    b.B = hp.block_size;
+                    for (int q = 0; q < b.count; ++q) {
+                        const auto& x = it[sel[q]];
+                        moara::GemmProb& p = b.p[q];
+                        p = moara::GemmProb{};
+                        p.A = x.G; p.a_inv = x.inv; p.Bm = rhs[sel[q]]; p.C = out[sel[q]];
+                        p.M = x.m; p.N = x.l; p.K = x.n; p.lda = x.n; p.ldb = x.l; p.ldc = x.l; p.kb = x.kb;
+                        p.a_bf16 = d;
+                    }
+                    chk(moara::launch_gemm(k, b, s, &ctx->launches));
                 }
-                chk(moara::launch_gemm(k, b, s, &ctx->launches));
+            };
+            // Z = V^T * Q  (n x l)
+            auto vt_times = [&](std::vector<float*>& rhs, std::vector<float*>& out) {
+                for (int d = 0; d < 2; ++d) {
+                    std::vector<int> sel;
+                    for (int i = 0; i < n_it; ++i) if ((it[i].dtype == MOARA_DTYPE_BF16) == (d == 1)) sel.push_back(i);
+                    if (sel.empty()) continue;
+                    moara::GemmKind k{moara::A_MCONTIG, moara::B_NCONTIG, src_v, 0, d, 0, moara::EPI_STORE};
+                    moara::GemmBatch b{};
+                    b.count = static_cast<int>(sel.size());
+                    b.B = hp.block_size;
+                    for (int q = 0; q < b.count; ++q) {
+                        const auto& x = it[sel[q]];
+                        moara::GemmProb& p = b.p[q];
+                        p = moara::GemmProb{};
+                        p.A = x.G; p.a_inv = x.inv; p.Bm = rhs[sel[q]]; p.C = out[sel[q]];
+                        p.M = x.n; p.N = x.l; p.K = x.m; p.lda = x.n; p.ldb = x.l; p.ldc = x.l; p.kb = x.kb;
+                        p.a_bf16 = d;
+                    }
+                    chk(moara::launch_gemm(k, b, s, &ctx->launches));
+                }
+            };
+            v_times(Za, Qa);
+            cholqr2s(Qa, Qb, rows_m);          // Q in Qb
+            // power iterations Y = V (V^T Q): Z = V^T Q gets one shifted CholeskyQR
+            // pass (enough to keep V Z well conditioned), Y the full two passes
+            for (int q = 0; q < hp.power_iters; ++q) {
+                vt_times(Qb, Za);
+                cholqr_pass(Za, Zb, rows_n, 2.0f * u_rnd);   // Z in Zb
+                v_times(Zb, Qa);
+                cholqr2s(Qa, Qb, rows_m);                    // Q in Qb
             }
-            tc_products(0, out);
-        };
-        v_times(Za, Qa);
-        cholqr2s(Qa, Qb, rows_m, &qbf);    // Q in Qb
-        // power iterations Y = V (V^T Q): Z = V^T Q gets one shifted CholeskyQR
-        // pass (enough to keep V Z well conditioned), Y the full two passes
-        const float u_rnd = 5.9604645e-08f;
-        for (int q = 0; q < hp.power_iters; ++q) {
+            // Rayleigh-Ritz matrix C = (V^T Q)^T (V^T Q)
             vt_times(Qb, Za);
-            cholqr_pass(Za, Zb, rows_n, 2.0f * u_rnd, &zbf);   // Z in Zb
-            v_times(Zb, Qa);
-            cholqr2s(Qa, Qb, rows_m, &qbf);                    // Q in Qb
-        }
-        // Rayleigh-Ritz on span(Q): C = (V^T Q)^T (V^T Q), eigenvectors of C by
-        // orthogonal iteration with CholeskyQR, ordered by Ritz value.
-        vt_times(Qb, Za);
-        {
             moara::GemmKind gram{moara::A_MCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
             gemm(gram, [&](int i, moara::GemmProb& p) {
                 const int l = it[i].l;
@@ -514,6 +594,10 @@ struct RefreshRunner {
                 p.M = l; p.N = l; p.K = it[i].n; p.lda = l; p.ldb = l; p.ldc = l;
             });
         }
+        // Eigenvectors of C by orthogonal iteration X <- C X with CholeskyQR2
+        // (shifted, then plain) every iteration: each X is orthonormal, so
+        // directions of C below its rounding level only ever fill an
+        // orthonormal completion.  Then the Ritz order.
         {
             moara::SmallBatch sb = small();
             for (int i = 0; i < n_it; ++i) { sb.a[i] = Xa[i]; sb.l[i] = it[i].l; }
@@ -528,7 +612,8 @@ struct RefreshRunner {
             });
             cholqr2s(Xb, Xa, rows_l);      // X in Xa
         }
-        // Ritz values and order: W = C X into Xb
+        // Ritz values (Rayleigh quotients of the columns of X) and order:
+        // W = C X into Xb
         gemm(prod, [&](int i, moara::GemmProb& p) {
             const int l = it[i].l;
             p.A = it[i].Cr; p.Bm = Xa[i]; p.C = Xb[i];
@@ -542,17 +627,17 @@ struct RefreshRunner {
             }
             chk(moara::launch_ritz_sort(sb, s, &ctx->launches));
         }
-        {   // Xs (l x r) = X[:, perm[:r]] into Linv
+        {   // Xs (l x r) = X[:, perm[:r]] into Xb
             moara::SmallBatch sb = small();
             for (int i = 0; i < n_it; ++i) {
-                sb.a[i] = Xa[i]; sb.c[i] = it[i].Linv; sb.iaux[i] = it[i].perm;
+                sb.a[i] = Xa[i]; sb.c[i] = Xb[i]; sb.iaux[i] = it[i].perm;
                 sb.l[i] = it[i].l; sb.rows[i] = it[i].r;
             }
             chk(moara::launch_gather_cols(sb, s, &ctx->launches));
         }
         // P_tmp (m x r) = Q * Xs into Qa
         gemm(prod, [&](int i, moara::GemmProb& p) {
-            p.A = Qb[i]; p.Bm = it[i].Linv; p.C = Qa[i];
+            p.A = Qb[i]; p.Bm = Xb[i]; p.C = Qa[i];
             p.M = it[i].m; p.N = it[i].r; p.K = it[i].l; p.lda = it[i].l; p.ldb = it[i].r; p.ldc = it[i].r;
         });
         {
@@ -569,52 +654,65 @@ struct RefreshRunner {
 int do_refresh(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, cudaStream_t s) {
     const moara_hparams& hp = ctx->hp;
     const int src_v = (hp.refresh_src == MOARA_REFRESH_SRC_V && hp.decompose) ? 1 : 0;
-    // group modules so that each group fits the refresh workspace
-    int start = 0;
-    while (start < n_mod) {
-        RefreshRunner rr{ctx, s, {}, src_v};
-        size_t used = 0;
-        int end = start;
-        while (end < n_mod && static_cast<int>(rr.it.size()) < moara::kMaxGroup) {
-            const int id = ids[end];
-            const moara_module_desc& d = ctx->mods[id];
-            const int l = refresh_l(ctx, d.m, d.n, d.r);
-            const size_t need = align_up(moara::refresh_ws_bytes(d.m, d.n, d.r, l, hp.block_size, src_v), 256);
-            if (used + need > ctx->refresh_ws_bytes) {
-                if (rr.it.empty())
-                    return fail(ctx, MOARA_ERR_WORKSPACE,
-                                "refresh workspace of %zu bytes is smaller than the %zu bytes module %d needs",
-                                ctx->refresh_ws_bytes, need, id);
-                break;
-            }
-            moara::RefreshItem x{};
-            x.m = d.m; x.n = d.n; x.r = d.r; x.l = l; x.kb = blocks_of(d.n, hp.block_size);
-            x.dtype = d.grad_dtype; x.G = G[end];
-            moara::refresh_carve(x, static_cast<char*>(ctx->refresh_ws) + used, d.m, d.n, d.r, l,
-                                 hp.block_size, src_v);
-            x.P = d.P; x.Pb = d.P_bf16;
-            // products on tensor cores when the module's step runs there (bf16
-            // G, supported shape) and the bf16 planes of Q and Z have a TMA
-            // row pitch (l % 8 == 0)
-            if (use_tc(ctx, id) && (l % 8) == 0) {
-                const moara::ModDev& md = ctx->moddev[id];
-                x.tc = 1;
-                if (src_v) {
-                    x.Vhi = md.ws_Vhi; x.Vhi_w = md.ws_Vhi; x.Vlo = md.ws_Vlo;
-                } else {
-                    x.Vhi = static_cast<const uint16_t*>(G[end]); x.Vhi_w = nullptr; x.Vlo = nullptr;
+    // Modules whose step runs on tensor cores refresh there too (their bf16
+    // planes of Q and Z need l % 8 == 0 for the TMA row pitch); the others use
+    // the fp32 path.  Each kind is grouped so that a group fits the workspace.
+    std::vector<int> kinds[2];
+    for (int i = 0; i < n_mod; ++i) {
+        const moara_module_desc& d = ctx->mods[ids[i]];
+        const int l = refresh_l(ctx, d.m, d.n, d.r);
+        kinds[(use_tc(ctx, ids[i]) && (l % 8) == 0) ? 1 : 0].push_back(i);
+    }
+    for (int kind = 0; kind < 2; ++kind) {
+        const std::vector<int>& sel = kinds[kind];
+        size_t start = 0;
+        while (start < sel.size()) {
+            RefreshRunner rr{ctx, s, {}, src_v};
+            size_t used = 0;
+            size_t end = start;
+            while (end < sel.size() && static_cast<int>(rr.it.size()) < moara::kMaxGroup) {
+                const int gi = sel[end];
+                const int id = ids[gi];
+                const moara_module_desc& d = ctx->mods[id];
+                const int l = refresh_l(ctx, d.m, d.n, d.r);
+                const size_t need = align_up(moara::refresh_ws_bytes(d.m, d.n, d.r, l, hp.block_size, src_v), 256);
+                if (used + need > ctx->refresh_ws_bytes) {
+                    if (rr.it.empty())
+                        return fail(ctx, MOARA_ERR_WORKSPACE,
+                                    "refresh workspace of %zu bytes is smaller than the %zu bytes module %d needs",
+                                    ctx->refresh_ws_bytes, need, id);
+                    break;
                 }
+                moara::RefreshItem x{};
+                x.m = d.m; x.n = d.n; x.r = d.r; x.l = l; x.kb = blocks_of(d.n, hp.block_size);
+                x.dtype = d.grad_dtype; x.G = G[gi];
+                moara::refresh_carve(x, static_cast<char*>(ctx->refresh_ws) + used, d.m, d.n, d.r, l,
+                                     hp.block_size, src_v);
+                x.P = d.P; x.Pb = d.P_bf16;
+                const uint64_t cnt = static_cast<uint64_t>(ctx->refresh_count[id]++);
+                x.key = hp.seed ^ (0x9E3779B97F4A7C15ull * (static_cast<uint64_t>(id) + 1)) ^
+                        (cnt * 0xD1B54A32D192ED03ull);
+                if (kind == 1) {
+                    const moara::ModDev& md = ctx->moddev[id];
+                    x.tc = 1;
+                    if (src_v) {
+                        x.Vhi = md.ws_Vhi; x.Vhi_w = md.ws_Vhi; x.Vlo = md.ws_Vlo;
+                    } else {
+                        x.Vhi = static_cast<const uint16_t*>(G[gi]); x.Vhi_w = nullptr; x.Vlo = nullptr;
+                    }
+                }
+                rr.it.push_back(x);
+                used += need;
+                ++end;
             }
-            const uint64_t cnt = static_cast<uint64_t>(ctx->refresh_count[id]++);
-            x.key = hp.seed ^ (0x9E3779B97F4A7C15ull * (static_cast<uint64_t>(id) + 1)) ^
-                    (cnt * 0xD1B54A32D192ED03ull);
-            rr.it.push_back(x);
-            used += need;
-            ++end;
+            rr.run();
+            if (rr.err != cudaSuccess) {
+                if (kind == 1 && ctx->tc != nullptr)
+                    return fail(ctx, MOARA_ERR_CUDA, "tensor-core refresh: %s", moara::tc_last_error(ctx->tc));
+                return cuda_fail(ctx, rr.err, "refresh launch");
+            }
+            start = end;
         }
-        rr.run();
-        if (rr.err != cudaSuccess) return cuda_fail(ctx, rr.err, "refresh launch");
-        start = end;
     }
     return MOARA_OK;
 }

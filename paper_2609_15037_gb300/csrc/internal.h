@@ -154,7 +154,7 @@ struct SmallBatch {
     int* fail[kMaxGroup];
     int* iaux[kMaxGroup];
     uint16_t* h[kMaxGroup];
-    float shift_rel;
+    float shift_rel;      // diagonal shift: shift_rel * sqrt(rows) * trace
     uint64_t key[kMaxGroup];
 };
 
@@ -171,5 +171,6 @@ cudaError_t launch_set_identity(const SmallBatch& b, cudaStream_t s, int64_t* la
 cudaError_t launch_ritz_sort(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_sign_fix_store(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+cudaError_t launch_transpose_bf16(const SmallBatch& b, cudaStream_t s, int64_t* launches);  // h = bf16(a^T)
 
 }  // namespace moara

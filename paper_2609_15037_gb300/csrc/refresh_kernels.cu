@@ -173,9 +173,8 @@ cudaError_t launch_trace_shift(const SmallBatch& b, cudaStream_t s, int64_t* lau
     return cudaGetLastError();
 }
 
-__global__ void __launch_bounds__(256) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
+__global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
     __shared__ float Ls[kTriBase][kTriBase + 1];
-    __shared__ float Xs[kTriBase][kTriBase + 1];
     __shared__ int s_fail;
     const int pi = blockIdx.x;
     const int l = b.l[pi];
@@ -184,37 +183,56 @@ __global__ void __launch_bounds__(256) k_chol_diag(const __grid_constant__ Small
     float* A = b.a[pi];
     float* X = b.c[pi];
     const float shift = b.b[pi][0];
-    if (threadIdx.x == 0) s_fail = 0;
-    for (int e = threadIdx.x; e < sz * sz; e += blockDim.x) {
-        const int i = e / sz, c = e - i * sz;
-        float v = A[(long long)(j0 + i) * l + j0 + c];
-        if (i == c) v += shift;
-        Ls[i][c] = v;
+    if (threadIdx.x < 32) {
+        // Warp 0 factors the block in registers: lane holds rows lane and
+        // lane + 32 (rows and columns past sz padded with the identity).  The
+        // loops are fully unrolled, so every register index is a constant;
+        // column j of the factor is broadcast with shuffles.
+        const int lane = threadIdx.x;
+        float r0[kTriBase], r1[kTriBase];
+#pragma unroll
+        for (int c = 0; c < kTriBase; ++c) {
+            float v0 = (c == lane) ? 1.0f : 0.0f, v1 = (c == lane + 32) ? 1.0f : 0.0f;
+            if (lane < sz && c < sz) v0 = A[(long long)(j0 + lane) * l + j0 + c] + (c == lane ? shift : 0.0f);
+            if (lane + 32 < sz && c < sz)
+                v1 = A[(long long)(j0 + lane + 32) * l + j0 + c] + (c == lane + 32 ? shift : 0.0f);
+            r0[c] = v0;
+            r1[c] = v1;
+        }
+        int bad = 0;
+#pragma unroll
+        for (int j = 0; j < kTriBase; ++j) {
+            float d = __shfl_sync(0xffffffffu, j < 32 ? r0[j] : r1[j], j & 31);
+            if (!(d > 0.0f) || !isfinite(d)) { d = 1.0f; bad = 1; }
+            const float dj = sqrtf(d);
+            const float inv = 1.0f / dj;
+            // column j below the diagonal (entries above it are never read)
+            if (j < 32) {
+                r0[j] = (lane == j) ? dj : r0[j] * inv;
+                r1[j] *= inv;
+            } else {
+                r1[j] = (lane + 32 == j) ? dj : r1[j] * inv;
+            }
+#pragma unroll
+            for (int c = j + 1; c < kTriBase; ++c) {
+                const float lcj = __shfl_sync(0xffffffffu, c < 32 ? r0[j] : r1[j], c & 31);
+                if (c < 32) r0[c] = fmaf(-r0[j], lcj, r0[c]);
+                r1[c] = fmaf(-r1[j], lcj, r1[c]);
+            }
+        }
+#pragma unroll
+        for (int c = 0; c < kTriBase; ++c) {
+            Ls[lane][c] = (c <= lane) ? r0[c] : 0.0f;
+            Ls[lane + 32][c] = (c <= lane + 32) ? r1[c] : 0.0f;
+        }
+        if (lane == 0) s_fail = bad;
     }
     __syncthreads();
-    // column-by-column Cholesky of the block (lower triangle)
-    for (int j = 0; j < sz; ++j) {
-        if (threadIdx.x == 0) {
-            float d = Ls[j][j];
-            if (!(d > 0.0f) || !isfinite(d)) { d = 1.0f; s_fail = 1; }
-            Ls[j][j] = sqrtf(d);
-        }
-        __syncthreads();
-        const float djj = Ls[j][j];
-        for (int i = j + 1 + threadIdx.x; i < sz; i += blockDim.x) Ls[i][j] /= djj;
-        __syncthreads();
-        // trailing update of the block: rows/cols > j
-        const int rem = sz - j - 1;
-        for (int e = threadIdx.x; e < rem * rem; e += blockDim.x) {
-            const int i = j + 1 + e / rem, c = j + 1 + e % rem;
-            if (c <= i) Ls[i][c] = fmaf(-Ls[i][j], Ls[c][j], Ls[i][c]);
-        }
-        __syncthreads();
-    }
     // inverse of the block factor by forward substitution; thread c keeps
     // column c of the inverse in registers (loops fully unrolled) and reads
-    // the rows of the factor as shared-memory broadcasts
-    if (threadIdx.x < kTriBase) {
+    // the rows of the factor as shared-memory broadcasts; then both the
+    // factor and the inverse go back to global memory
+    {
         const int c = threadIdx.x;
         float xcol[kTriBase];
 #pragma unroll
@@ -222,23 +240,60 @@ __global__ void __launch_bounds__(256) k_chol_diag(const __grid_constant__ Small
             float acc = (i == c) ? 1.0f : 0.0f;
 #pragma unroll
             for (int k = 0; k < i; ++k) acc = fmaf(-Ls[i][k], xcol[k], acc);
-            xcol[i] = (i < sz && c <= i) ? acc / Ls[i][i] : 0.0f;
+            xcol[i] = (c <= i) ? acc / Ls[i][i] : 0.0f;
         }
+        if (c < sz) {
 #pragma unroll
-        for (int i = 0; i < kTriBase; ++i) Xs[i][c] = xcol[i];
-    }
-    __syncthreads();
-    for (int e = threadIdx.x; e < sz * sz; e += blockDim.x) {
-        const int i = e / sz, c = e - i * sz;
-        A[(long long)(j0 + i) * l + j0 + c] = (c <= i) ? Ls[i][c] : 0.0f;
-        X[(long long)(j0 + i) * l + j0 + c] = Xs[i][c];
+            for (int i = 0; i < kTriBase; ++i) {
+                if (i < sz) {
+                    A[(long long)(j0 + i) * l + j0 + c] = Ls[i][c];
+                    X[(long long)(j0 + i) * l + j0 + c] = xcol[i];
+                }
+            }
+        }
     }
     if (threadIdx.x == 0 && s_fail && b.fail[pi] != nullptr) *b.fail[pi] = 1;
 }
 
 cudaError_t launch_chol_diag(const SmallBatch& b, int j0, cudaStream_t s, int64_t* launches) {
     if (b.count <= 0) return cudaSuccess;
-    k_chol_diag<<<b.count, 256, 0, s>>>(b, j0);
+    k_chol_diag<<<b.count, kTriBase, 0, s>>>(b, j0);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// h <- a^T rounded to bf16 (l x l): 32 x 32 tiles through shared memory.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_transpose_bf16(const __grid_constant__ SmallBatch b) {
+    __shared__ float t[32][33];
+    const int pi = blockIdx.z;
+    const int l = b.l[pi];
+    const float* src = b.a[pi];
+    uint16_t* dst = b.h[pi];
+    const int tiles = (l + 31) / 32;
+    for (int tile = blockIdx.x; tile < tiles * tiles; tile += gridDim.x) {
+        const int ti = tile / tiles, tj = tile - ti * tiles;
+        const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+        for (int r = ty; r < 32; r += 8) {
+            const int i = ti * 32 + r, j = tj * 32 + tx;
+            t[r][tx] = (i < l && j < l) ? src[(long long)i * l + j] : 0.0f;
+        }
+        __syncthreads();
+        for (int r = ty; r < 32; r += 8) {
+            const int i = tj * 32 + r, j = ti * 32 + tx;   // dst row i = src column
+            if (i < l && j < l) {
+                __nv_bfloat16 h = __float2bfloat16_rn(t[tx][r]);
+                dst[(long long)i * l + j] = *reinterpret_cast<uint16_t*>(&h);
+            }
+        }
+        __syncthreads();
+    }
+}
+
+cudaError_t launch_transpose_bf16(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    k_transpose_bf16<<<dim3(128, 1, b.count), 256, 0, s>>>(b);
     ++*launches;
     return cudaGetLastError();
 }
@@ -266,7 +321,7 @@ cudaError_t launch_set_identity(const SmallBatch& b, cudaStream_t s, int64_t* la
 }
 
 // ---------------------------------------------------------------------------
-// Ritz values d_j = x_j^T (C x_j) from X (a) and W = C X (b), then the
+// Ritz values d_j = x_j^T (C x_j) / x_j^T x_j from X (a) and W = C X (b), then the
 // descending order: iaux[rank] = j, rank_j = #{i : d_i > d_j, or d_i == d_j
 // and i < j}.  Ritz values go to c.
 // ---------------------------------------------------------------------------
@@ -278,9 +333,13 @@ __global__ void __launch_bounds__(kSmallThreads) k_ritz_sort(const __grid_consta
     float* d = b.c[pi];
     int* perm = b.iaux[pi];
     for (int j = threadIdx.x; j < l; j += blockDim.x) {
-        float acc = 0.0f;
-        for (int i = 0; i < l; ++i) acc = fmaf(X[(long long)i * l + j], W[(long long)i * l + j], acc);
-        d[j] = acc;
+        float acc = 0.0f, nrm = 0.0f;
+        for (int i = 0; i < l; ++i) {
+            const float x = X[(long long)i * l + j];
+            acc = fmaf(x, W[(long long)i * l + j], acc);
+            nrm = fmaf(x, x, nrm);
+        }
+        d[j] = nrm > 0.0f ? acc / nrm : 0.0f;
     }
     __syncthreads();
     __threadfence_block();

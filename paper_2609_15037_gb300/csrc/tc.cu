@@ -699,16 +699,17 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
 
 // ---------------------------------------------------------------- host side
 // ===========================================================================
-// KR: the products of the projector refresh (randomized subspace iteration,
-// §3.3 / App. B.2) on tensor cores:
-//   op ZT:  out (n x l) = V^T Q      (A = V read MN-major, M = n, K = m)
-//   op Y:   out (m x l) = V Z        (A = V read K-major,  M = m, K = n)
-// with V = V_hi + V_lo held as two bf16 planes (the two MMAs per k-step keep
-// ~16 significant bits of V) and the orthonormal factor Q or Z in bf16.
-// Tile 256 x 256 (two 128-row accumulators in TMEM), BK = 64, one tile per
-// CTA: the contraction (m or n >= 1024 in practice) is long enough that the
-// epilogue need not overlap the next tile.  The last column tile issues the
-// MMA with N = 64 * ceil(cols / 64), so a ragged l costs at most 48 columns.
+// KR: bf16 tensor-core GEMM of the projector refresh (randomized subspace
+// iteration, §3.3 / App. B.2): out (M x N) = op(A) B with fp32 accumulation,
+// written in fp32 and/or bf16.  A is read K-major (stored M x K) or MN-major
+// (stored K x M), optionally as two planes A_hi + A_lo (two MMAs per k-step
+// keep ~16 significant bits of A, used for V); B is stored K x N (MN-major).
+// Used for V^T Q, V Z, the Gram matrices X^T X and the triangular factor
+// products X R^-1.  Tile 256 x 256 (two 128-row accumulators in TMEM), BK =
+// 64, one tile per CTA: the contractions are long enough that the epilogue
+// need not overlap the next tile.  The last column tile issues the MMA with
+// N = 64 * ceil(cols / 64), so a ragged N costs at most 48 columns; with
+// `ktri` the K loop of column tile n0 stops at n0 + 256 (B upper triangular).
 // ===========================================================================
 constexpr int KR_BM = 256, KR_BN = 256, KR_BK = 64;
 constexpr int KR_PLANE = KR_BM * KR_BK * 2;               // 32 KB: one A plane or the B tile
@@ -722,11 +723,13 @@ constexpr int KR_SMEM = 1024 + 6 * KR_PLANE + 2048;
 constexpr int kKrGroup = 48;
 
 struct KrParams {
-    CUtensorMap amap[kKrGroup];        // V_hi ({n, m}, box {64, 64})
-    CUtensorMap lmap[kKrGroup];        // V_lo (same geometry), unused without LO
-    CUtensorMap bmap[kKrGroup];        // Q ({l, m}) for ZT, Z ({l, n}) for Y; box {64, 64}
-    float* out[kKrGroup];
+    CUtensorMap amap[kKrGroup];        // A_hi, box {64, 64}
+    CUtensorMap lmap[kKrGroup];        // A_lo (same geometry), unused without LO
+    CUtensorMap bmap[kKrGroup];        // B ({N, K}), box {64, 64}
+    float* out[kKrGroup];              // M x N fp32 or null
+    uint16_t* out_bf[kKrGroup];        // M x N bf16 or null
     int M[kKrGroup], N[kKrGroup], K[kKrGroup];
+    int ktri[kKrGroup];
     int tiles_n[kKrGroup];
     int tile_start[kKrGroup + 1];
     int count;
@@ -757,7 +760,8 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
     const int n0 = (local % p.tiles_n[pi]) * KR_BN;
     const int nch = min(4, (N - n0 + 63) / 64);            // 64-column chunks of B in this tile
     const int halves = (M - i0) > 128 ? 2 : 1;
-    const int nk = (K + KR_BK - 1) / KR_BK;
+    const int kend = p.ktri[pi] ? min(K, n0 + KR_BN) : K;
+    const int nk = (kend + KR_BK - 1) / KR_BK;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -852,7 +856,9 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
         if (__all_sync(0xffffffffu, got) && h < halves) {
             ptx::tc_fence_after();
             const int row = i0 + h * 128 + q * 32 + lane;
-            float* const orow = p.out[pi] + (long long)row * N;
+            float* const of = p.out[pi];
+            uint16_t* const ob = p.out_bf[pi];
+            const long long ro = (long long)row * N;
             for (int c = 0; c < nch * 4; ++c) {
                 const int j0 = n0 + c * 16;
                 if (j0 >= N) break;                       // warp-uniform
@@ -860,14 +866,30 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
                 __syncwarp();
                 ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + h * 256 + c * 16, v);
                 if (row >= M) continue;
-                if (j0 + 16 <= N && (N & 3) == 0) {
-                    float4* o4 = reinterpret_cast<float4*>(orow + j0);
+                if (j0 + 16 <= N) {                       // N % 8 == 0: 16-byte aligned rows
+                    if (of != nullptr) {
+                        float4* o4 = reinterpret_cast<float4*>(of + ro + j0);
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) o4[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+                        for (int e = 0; e < 4; ++e)
+                            o4[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+                    }
+                    if (ob != nullptr) {
+                        uint4* b4 = reinterpret_cast<uint4*>(ob + ro + j0);
+                        b4[0] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                                           pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+                        b4[1] = make_uint4(pack_bf16x2(v[8], v[9]), pack_bf16x2(v[10], v[11]),
+                                           pack_bf16x2(v[12], v[13]), pack_bf16x2(v[14], v[15]));
+                    }
                 } else {
 #pragma unroll
-                    for (int e = 0; e < 16; ++e)
-                        if (j0 + e < N) orow[j0 + e] = v[e];
+                    for (int e = 0; e < 16; ++e) {
+                        if (j0 + e >= N) continue;
+                        if (of != nullptr) of[ro + j0 + e] = v[e];
+                        if (ob != nullptr) {
+                            __nv_bfloat16 hb = __float2bfloat16_rn(v[e]);
+                            ob[ro + j0 + e] = *reinterpret_cast<uint16_t*>(&hb);
+                        }
+                    }
                 }
             }
         }
@@ -930,7 +952,8 @@ struct TcState {
     bool attrs_set = false;
     K1Params p1;                           // parameter block of the next K1 launch
     K0Params p0;                           // parameter block of the next K0 launch
-    KrParams pr;                           // parameter block of the next refresh product launch
+    KrParams pr;                           // parameter block of the next refresh GEMM launch
+    bool kr_attrs = false;
 };
 
 bool tc_supported(int m, int n, int r, int B, int dtype, int decompose) {
@@ -1228,49 +1251,56 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
 
 const char* tc_last_error(const TcState* st) { return st ? st->err.c_str() : "no tensor-core state"; }
 
-int tc_refresh_products(TcState* st, int op, const TcProdItem* items, int count, cudaStream_t s,
-                        int64_t* launches) {
-    static bool attrs = false;
-    if (!attrs) {
+int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, cudaStream_t s,
+                 int64_t* launches) {
+    if (!st->kr_attrs) {
         cudaFuncSetAttribute(kr_product<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
         cudaFuncSetAttribute(kr_product<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
         cudaFuncSetAttribute(kr_product<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
         cudaFuncSetAttribute(kr_product<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
-        attrs = true;
+        st->kr_attrs = true;
     }
-    // two sub-launches: items with and without the V_lo plane
+    for (int i = 0; i < count; ++i) {
+        const TcGemmItem& x = items[i];
+        const int a_inner = a_kmajor ? x.K : x.M;
+        if (x.M < 1 || x.N < 1 || x.K < 1 || (a_inner % 8) != 0 || (x.N % 8) != 0) {
+            st->err = "tensor-core refresh GEMM: row pitches must be multiples of 16 bytes";
+            return MOARA_ERR_UNSUPPORTED;
+        }
+    }
+    // two sub-launches: items with and without the A_lo plane
     for (int with_lo = 0; with_lo < 2; ++with_lo) {
         std::vector<int> sel;
         for (int i = 0; i < count; ++i)
-            if ((items[i].Vlo != nullptr) == (with_lo == 1)) sel.push_back(i);
+            if ((items[i].A_lo != nullptr) == (with_lo == 1)) sel.push_back(i);
         for (size_t c0 = 0; c0 < sel.size(); c0 += kKrGroup) {
             const int cnt = static_cast<int>(std::min<size_t>(kKrGroup, sel.size() - c0));
             KrParams& kp = st->pr;
             std::memset(&kp, 0, sizeof(kp));
             int total = 0;
             for (int q = 0; q < cnt; ++q) {
-                const TcProdItem& x = items[sel[c0 + q]];
-                const int M = op == 0 ? x.n : x.m;
-                const int K = op == 0 ? x.m : x.n;
-                bool ok = encode_bf16_2d(st->encode, &kp.amap[q], x.Vhi, x.n, x.m, 64, 64);
-                if (with_lo) ok = ok && encode_bf16_2d(st->encode, &kp.lmap[q], x.Vlo, x.n, x.m, 64, 64);
-                ok = ok && encode_bf16_2d(st->encode, &kp.bmap[q], op == 0 ? x.Qbf : x.Zbf, x.l,
-                                          op == 0 ? x.m : x.n, 64, 64);
+                const TcGemmItem& x = items[sel[c0 + q]];
+                const uint64_t a_cols = a_kmajor ? x.K : x.M, a_rows = a_kmajor ? x.M : x.K;
+                bool ok = encode_bf16_2d(st->encode, &kp.amap[q], x.A, a_cols, a_rows, 64, 64);
+                if (with_lo) ok = ok && encode_bf16_2d(st->encode, &kp.lmap[q], x.A_lo, a_cols, a_rows, 64, 64);
+                ok = ok && encode_bf16_2d(st->encode, &kp.bmap[q], x.B, x.N, x.K, 64, 64);
                 if (!ok) {
                     st->err = "cuTensorMapEncodeTiled failed for a refresh operand";
                     return MOARA_ERR_CUDA;
                 }
                 kp.out[q] = x.out;
-                kp.M[q] = M; kp.N[q] = x.l; kp.K[q] = K;
-                kp.tiles_n[q] = (x.l + KR_BN - 1) / KR_BN;
+                kp.out_bf[q] = x.out_bf16;
+                kp.M[q] = x.M; kp.N[q] = x.N; kp.K[q] = x.K;
+                kp.ktri[q] = x.ktri;
+                kp.tiles_n[q] = (x.N + KR_BN - 1) / KR_BN;
                 kp.tile_start[q] = total;
-                total += ((M + KR_BM - 1) / KR_BM) * kp.tiles_n[q];
+                total += ((x.M + KR_BM - 1) / KR_BM) * kp.tiles_n[q];
             }
             kp.tile_start[cnt] = total;
             kp.count = cnt;
             kp.status = st->d_status;
             if (total == 0) continue;
-            if (op == 0) {
+            if (!a_kmajor) {
                 if (with_lo) kr_product<false, true><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
                 else kr_product<false, false><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
             } else {

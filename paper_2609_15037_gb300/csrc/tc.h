@@ -23,20 +23,23 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp);
 int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G,
             float bc1, float bc2, float lr, int first_step, cudaStream_t s, int64_t* launches,
             const TcProfile& prof);
-// One module's operands of the refresh products on tensor cores.
-struct TcProdItem {
-    const uint16_t* Vhi;   // m x n bf16 (V, or G when the refresh source is G)
-    const uint16_t* Vlo;   // m x n bf16 residual, or null when Vhi is exact
-    const uint16_t* Qbf;   // m x l bf16 (op 0)
-    const uint16_t* Zbf;   // n x l bf16 (op 1)
-    float* out;            // n x l (op 0) or m x l (op 1), fp32
-    int m, n, l;
+// One problem of the refresh GEMM on tensor cores: out = op(A) B, bf16
+// operands, fp32 accumulation.
+struct TcGemmItem {
+    const uint16_t* A;     // K-major: M x K row-major;  MN-major: K x M row-major
+    const uint16_t* A_lo;  // residual plane of A in the same layout, or null
+    const uint16_t* B;     // K x N row-major
+    float* out;            // M x N row-major fp32, or null
+    uint16_t* out_bf16;    // M x N row-major bf16, or null
+    int M, N, K;
+    int ktri;              // B upper triangular: column j needs k <= j only
 };
 
-// op 0: out = V^T Qbf;  op 1: out = V Zbf.  Requires n % 8 == 0 and l % 8 == 0
-// (TMA row pitch) and 16-byte aligned planes.
-int tc_refresh_products(TcState* st, int op, const TcProdItem* items, int count, cudaStream_t s,
-                        int64_t* launches);
+// Grouped launch of TcGemmItems (A read K-major when a_kmajor, else
+// MN-major).  A's row pitch (K or M) and N must be multiples of 8 and every
+// plane 16-byte aligned; returns MOARA_ERR_UNSUPPORTED otherwise.
+int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, cudaStream_t s,
+                 int64_t* launches);
 
 // V = Decompose(G, B) direction as two bf16 planes (V_hi, V_lo) for the
 // refresh products; G bf16 m x n, B in {8, ..., 128}.
