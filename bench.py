@@ -69,7 +69,7 @@ class Clocks:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
@@ -120,20 +120,30 @@ def _algorithmic(mods, B):
 
 
 def _kernel_bytes(mods, B, tc):
-    """Algorithmic bytes per launch of the projection and back-projection
-    kernels as built (tc: bf16 N hand-off; otherwise fp32 N, fp32 P)."""
-    pb = bb = 0
+    """Algorithmic bytes per step of each step kernel as built.
+
+    tensor-core path: tc_decompose reads G (bf16), writes V (bf16) and updates
+    the magnitude moments (read+write) and dM; tc_project reads V, P (bf16) and
+    the direction moments (read+write) and writes N (bf16); tc_backproject
+    reads and writes W and reads N, P (bf16) and dM.  fp32 path: decompose
+    reads G and writes the block scales, project reads G, the scales, P (fp32)
+    and the moments and writes N (fp32), backproject as above with fp32 N, P.
+    """
+    kb = {}
     for md in mods:
         m, n, r = md.m, md.n, md.r
         k = -(-n // B)
-        nb = 2 if tc else 4
-        pbytes = 2 if tc else 4
-        # projection: G read, moments read+write, N write, P read, magnitude
-        # moments read+write and dM write
-        pb += 2 * m * n + 16 * r * n + nb * r * n + pbytes * m * r + 20 * m * k
-        # back-projection: W read+write, N read, P read, dM read
-        bb += 8 * m * n + nb * r * n + pbytes * m * r + 4 * m * k
-    return pb, bb
+        if tc:
+            add = {"tc_decompose": 2 * m * n + 2 * m * n + 20 * m * k,
+                   "tc_project": 2 * m * n + 2 * m * r + 16 * r * n + 2 * r * n,
+                   "tc_backproject": 8 * m * n + 2 * r * n + 2 * m * r + 4 * m * k}
+        else:
+            add = {"decompose": 2 * m * n + 20 * m * k + 4 * m * k,
+                   "project": 2 * m * n + 4 * m * k + 4 * m * r + 16 * r * n + 4 * r * n,
+                   "backproject": 8 * m * n + 4 * r * n + 4 * m * r + 4 * m * k}
+        for key, v in add.items():
+            kb[key] = kb.get(key, 0) + v
+    return kb
 
 
 def run_gpu(args):
@@ -216,23 +226,27 @@ def run_gpu(args):
     step_ms = elapsed / args.steps
     status = M.moara_get_device_status(g.ctx, cs)
 
-    # end to end through the C ABI with host buffers
+    # end to end through the C ABI with host buffers: every step uploads its
+    # gradients from page-locked host memory (moara_step_grouped_host overlaps
+    # the chunked upload with the step kernels) and reads the device status
+    # word back
     host = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for x in grads]
     for h, x in zip(host, grads):
         h.copy_(x)
-    st_host = torch.empty(1, dtype=torch.int32, pin_memory=True)
-    st_dev = torch.zeros(1, dtype=torch.int32, device=dev)
-    e2e_steps = max(1, min(args.steps, 5))
+    hptr = [h.data_ptr() for h in host]
+    e2e_steps = max(1, min(args.steps, 10))
+    chunk = int(args.chunk_mb) << 20
+    M.moara_step_grouped_host(g.ctx, ids, hptr, step, LR, False, chunk, cs)   # staging allocation
+    step += 1
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
+    e2e_status = 0
     for _ in range(e2e_steps):
-        for h, x in zip(host, grads):
-            x.copy_(h, non_blocking=True)
-        M.moara_step_grouped(g.ctx, ids, gptr, step, LR, False, cs)
+        M.moara_step_grouped_host(g.ctx, ids, hptr, step, LR, False, chunk, cs)
         step += 1
-        st_host.copy_(st_dev, non_blocking=True)
+        e2e_status |= M.moara_get_device_status(g.ctx, cs)
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
@@ -245,8 +259,8 @@ def run_gpu(args):
 
     # dominant kernel
     used_tc = prof["tc_project"][1] > 0
-    pbytes, bbytes = _kernel_bytes(mods, B, used_tc)
-    names = ["decompose", "project", "backproject", "tc_project", "tc_backproject"]
+    kbytes = _kernel_bytes(mods, B, used_tc)
+    names = ["decompose", "project", "backproject", "tc_decompose", "tc_project", "tc_backproject"]
     dom = max(names, key=lambda k: prof[k][0])
     dom_ms = prof[dom][0] / max(prof[dom][1], 1)
     n_launch_per_step = max(prof[dom][1] // args.steps, 1)
@@ -264,16 +278,20 @@ def run_gpu(args):
                 "unit": "TFLOP/s", "frac": round(achieved / bf16_sus, 4), "traffic": None,
                 "kernel": dom, "peak_source": f"bf16_tflops_sustained ({peak_src})"}
     else:
-        by = (bbytes if dom in ("backproject", "tc_backproject") else pbytes) / n_launch_per_step
+        by = kbytes[dom] / n_launch_per_step
         achieved = by / (dom_ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
                 "frac": round(achieved / hbm, 4), "traffic": None, "kernel": dom,
                 "peak_source": f"hbm_gbs ({peak_src})"}
 
-    kernels = {k: {"ms_per_step": round(prof[k][0] / args.steps, 4),
-                   "launches_per_step": prof[k][1] / args.steps,
-                   "share": round(prof[k][0] / max(sum(prof[x][0] for x in names), 1e-9), 4)}
-               for k in names if prof[k][1] > 0}
+    kernels = {}
+    for k in names:
+        if prof[k][1] == 0:
+            continue
+        ms = prof[k][0] / args.steps
+        kernels[k] = {"ms_per_step": round(ms, 4), "launches_per_step": prof[k][1] / args.steps,
+                      "share": round(prof[k][0] / max(sum(prof[x][0] for x in names), 1e-9), 4),
+                      "alg_gbs": round(kbytes.get(k, 0) / (ms * 1e-3) / 1e9, 1)}
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args, budget_s=args.cpu_seconds)
@@ -299,7 +317,7 @@ def run_gpu(args):
         "e2e": {"value": round(e2e_ms + refresh_ms / 200.0, 4), "unit": "ms",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4},
         "gpu_launches": int(launches),
-        "device_status": status,
+        "device_status": status | e2e_status,
         "clocks": clk,
     }
     if cpu is not None:
@@ -404,13 +422,15 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=25)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--refresh-ws-gb", type=float, default=12.0)
+    ap.add_argument("--chunk-mb", type=int, default=256,
+                    help="gradient chunk of the host-gradient step (e2e)")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

@@ -212,6 +212,20 @@ int moara_step_grouped(moara_ctx* ctx, int n_mod, const int* ids,
                        const void* const* G, int64_t t, float lr,
                        int auto_refresh, void* stream);
 
+/* The same step with the gradients in host memory: G_host[i] is module
+ * ids[i]'s gradient in page-locked host memory (m x n, the module's dtype).
+ * The modules are taken in order, in chunks of at most chunk_bytes of
+ * gradient (a larger module is a chunk of its own).  Each chunk is copied on
+ * an internal stream into one of two device staging buffers while the step
+ * kernels of the previous chunk run on `stream`, so the transfer overlaps the
+ * computation.  The staging buffers (2 x the largest chunk) are allocated on
+ * first use and kept until moara_destroy.  Asynchronous like
+ * cudaMemcpyAsync: G_host must stay valid and unchanged until the work
+ * enqueued on `stream` by this call has finished. */
+int moara_step_grouped_host(moara_ctx* ctx, int n_mod, const int* ids,
+                            const void* const* G_host, int64_t t, float lr,
+                            int auto_refresh, size_t chunk_bytes, void* stream);
+
 /* Reads and clears the device status word (0, or a MOARA_ERR_* code a kernel
  * recorded, e.g. MOARA_ERR_DEVICE_TIMEOUT from a bounded wait).  Synchronizes
  * `stream`.  *status receives the code. */

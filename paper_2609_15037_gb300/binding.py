@@ -85,6 +85,7 @@ def _load():
         "moara_set_refresh_workspace": (i32, [vp, vp, sz]),
         "moara_refresh_projector": (i32, [vp, i32, P(i32), P(vp), vp]),
         "moara_step_grouped": (i32, [vp, i32, P(i32), P(vp), i64, f32, i32, vp]),
+        "moara_step_grouped_host": (i32, [vp, i32, P(i32), P(vp), i64, f32, i32, sz, vp]),
         "moara_get_device_status": (i32, [vp, P(i32), vp]),
         "moara_last_error": (ctypes.c_char_p, [vp]),
         "moara_status_string": (ctypes.c_char_p, [i32]),
@@ -211,6 +212,14 @@ def moara_step_grouped(ctx, ids, grads, t, lr, auto_refresh=False, stream=0):
                                    stream), ctx, "moara_step_grouped")
 
 
+def moara_step_grouped_host(ctx, ids, host_grads, t, lr, auto_refresh=False,
+                            chunk_bytes=256 << 20, stream=0):
+    """host_grads: addresses of page-locked host gradients (one per id)."""
+    n, ia, ga = _arrays(ids, host_grads)
+    _check(_lib.moara_step_grouped_host(ctx, n, ia, ga, int(t), float(lr), int(bool(auto_refresh)),
+                                        int(chunk_bytes), stream), ctx, "moara_step_grouped_host")
+
+
 def moara_get_device_status(ctx, stream=0):
     st = ctypes.c_int()
     _check(_lib.moara_get_device_status(ctx, ctypes.byref(st), stream), ctx,
@@ -251,7 +260,8 @@ EXPORTED = [
     "moara_default_hparams", "moara_create", "moara_destroy", "moara_get_hparams",
     "moara_state_bytes", "moara_rank_table", "moara_workspace_bytes", "moara_init_module",
     "moara_load_projector", "moara_refresh_workspace_bytes", "moara_set_refresh_workspace",
-    "moara_refresh_projector", "moara_step_grouped", "moara_get_device_status",
+    "moara_refresh_projector", "moara_step_grouped", "moara_step_grouped_host",
+    "moara_get_device_status",
     "moara_last_error", "moara_status_string", "moara_launch_count",
     "moara_profile_enable", "moara_profile_read", "moara_step_static_scratch",
 ]

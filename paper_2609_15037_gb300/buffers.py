@@ -118,6 +118,16 @@ class MoaraGroup:
         B.moara_step_grouped(self.ctx, ids, [g.data_ptr() for g in grads], t, lr,
                              auto_refresh, stream)
 
+    def step_host(self, host_grads, t, lr, auto_refresh=False, ids=None, chunk_bytes=256 << 20,
+                  stream=0):
+        """Step with gradients in page-locked host tensors (see
+        moara_step_grouped_host)."""
+        ids = self.ids if ids is None else ids
+        if auto_refresh:
+            self.ensure_refresh_workspace()
+        B.moara_step_grouped_host(self.ctx, ids, [g.data_ptr() for g in host_grads], t, lr,
+                                  auto_refresh, chunk_bytes, stream)
+
     def status(self, stream=0):
         return B.moara_get_device_status(self.ctx, stream)
 

@@ -29,6 +29,12 @@ struct moara_ctx {
     std::string last_error;
     int64_t launches = 0;
     moara::TcState* tc = nullptr;
+    // host-gradient step: two device staging buffers, a copy stream, events
+    void* stage[2] = {nullptr, nullptr};
+    size_t stage_bytes = 0;
+    cudaStream_t copy_stream = nullptr;
+    cudaEvent_t copy_done[2] = {nullptr, nullptr};
+    cudaEvent_t compute_done[2] = {nullptr, nullptr};
     // per-kernel CUDA-event timing (moara_profile_enable)
     bool prof = false;
     struct Rec { int phase; cudaEvent_t a, b; };
@@ -872,6 +878,13 @@ void moara_destroy(moara_ctx* ctx) {
     if (ctx == nullptr) return;
     DeviceGuard g(ctx->device);
     if (ctx->tc) moara::tc_destroy(ctx->tc);
+    if (ctx->copy_stream) cudaStreamSynchronize(ctx->copy_stream);
+    for (int b = 0; b < 2; ++b) {
+        if (ctx->stage[b]) cudaFree(ctx->stage[b]);
+        if (ctx->copy_done[b]) cudaEventDestroy(ctx->copy_done[b]);
+        if (ctx->compute_done[b]) cudaEventDestroy(ctx->compute_done[b]);
+    }
+    if (ctx->copy_stream) cudaStreamDestroy(ctx->copy_stream);
     for (auto& r : ctx->recs) { cudaEventDestroy(r.a); cudaEventDestroy(r.b); }
     for (auto e : ctx->free_events) cudaEventDestroy(e);
     if (ctx->d_mods) cudaFree(ctx->d_mods);
@@ -1057,16 +1070,14 @@ int moara_refresh_projector(moara_ctx* ctx, int n_mod, const int* ids, const voi
     return do_refresh(ctx, n_mod, ids, G, static_cast<cudaStream_t>(stream));
 }
 
-int moara_step_grouped(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, int64_t t,
-                       float lr, int auto_refresh, void* stream) {
-    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
-    int rc = check_ids(ctx, n_mod, ids, G);
-    if (rc != MOARA_OK) return rc;
-    if (t < 1) return fail(ctx, MOARA_ERR_INVALID_ARG, "step t must be >= 1 (got %lld)", (long long)t);
-    if (!std::isfinite(lr)) return fail(ctx, MOARA_ERR_INVALID_ARG, "lr must be finite");
-    if (n_mod == 0) return MOARA_OK;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    DeviceGuard g(ctx->device);
+}  // extern "C"
+
+namespace {
+
+// The step on validated arguments (device gradients), enqueued on s.
+int step_impl(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, int64_t t, float lr,
+              int auto_refresh, cudaStream_t s) {
+    int rc = MOARA_OK;
     if (auto_refresh && ((t - 1) % ctx->hp.refresh_interval) == 0) {
         if (ctx->refresh_ws == nullptr) return fail(ctx, MOARA_ERR_WORKSPACE, "no refresh workspace set");
         ProfScope ps(ctx, MOARA_PHASE_REFRESH, s);
@@ -1100,6 +1111,111 @@ int moara_step_grouped(moara_ctx* ctx, int n_mod, const int* ids, const void* co
     if (!simt.empty()) {
         rc = do_step_simt(ctx, simt, ids, G, t, lr, s);
         if (rc != MOARA_OK) return rc;
+    }
+    return MOARA_OK;
+}
+
+
+// Two staging buffers of at least `bytes` each, the copy stream and events.
+int ensure_staging(moara_ctx* ctx, size_t bytes) {
+    if (ctx->copy_stream == nullptr) {
+        cudaError_t e = cudaStreamCreateWithFlags(&ctx->copy_stream, cudaStreamNonBlocking);
+        for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+            e = cudaEventCreateWithFlags(&ctx->copy_done[b], cudaEventDisableTiming);
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->compute_done[b], cudaEventDisableTiming);
+        }
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "copy stream / events");
+    }
+    if (ctx->stage_bytes >= bytes) return MOARA_OK;
+    // earlier steps may still read the old buffers
+    for (int b = 0; b < 2; ++b) {
+        if (ctx->stage[b] != nullptr) {
+            cudaError_t e = cudaEventSynchronize(ctx->compute_done[b]);
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "staging buffer release");
+            cudaFree(ctx->stage[b]);
+            ctx->stage[b] = nullptr;
+        }
+    }
+    ctx->stage_bytes = 0;
+    for (int b = 0; b < 2; ++b) {
+        cudaError_t e = cudaMalloc(&ctx->stage[b], bytes);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMalloc of a gradient staging buffer");
+    }
+    ctx->stage_bytes = bytes;
+    return MOARA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int moara_step_grouped(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, int64_t t,
+                       float lr, int auto_refresh, void* stream) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    int rc = check_ids(ctx, n_mod, ids, G);
+    if (rc != MOARA_OK) return rc;
+    if (t < 1) return fail(ctx, MOARA_ERR_INVALID_ARG, "step t must be >= 1 (got %lld)", (long long)t);
+    if (!std::isfinite(lr)) return fail(ctx, MOARA_ERR_INVALID_ARG, "lr must be finite");
+    if (n_mod == 0) return MOARA_OK;
+    DeviceGuard g(ctx->device);
+    return step_impl(ctx, n_mod, ids, G, t, lr, auto_refresh, static_cast<cudaStream_t>(stream));
+}
+
+int moara_step_grouped_host(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G_host, int64_t t,
+                            float lr, int auto_refresh, size_t chunk_bytes, void* stream) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    int rc = check_ids(ctx, n_mod, ids, G_host);
+    if (rc != MOARA_OK) return rc;
+    if (t < 1) return fail(ctx, MOARA_ERR_INVALID_ARG, "step t must be >= 1 (got %lld)", (long long)t);
+    if (!std::isfinite(lr)) return fail(ctx, MOARA_ERR_INVALID_ARG, "lr must be finite");
+    if (chunk_bytes == 0) return fail(ctx, MOARA_ERR_INVALID_ARG, "chunk_bytes must be > 0");
+    if (n_mod == 0) return MOARA_OK;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DeviceGuard g(ctx->device);
+    // chunks of consecutive modules, at most chunk_bytes of gradient each
+    // (a larger module forms its own chunk); 256-byte aligned offsets
+    auto gbytes = [&](int i) {
+        const moara_module_desc& d = ctx->mods[ids[i]];
+        const size_t es = d.grad_dtype == MOARA_DTYPE_BF16 ? 2 : 4;
+        return align_up(es * (size_t)d.m * d.n, 256);
+    };
+    std::vector<int> cstart{0};
+    size_t cur = 0, maxc = 0;
+    for (int i = 0; i < n_mod; ++i) {
+        const size_t b = gbytes(i);
+        if (cur > 0 && cur + b > chunk_bytes) {
+            maxc = std::max(maxc, cur);
+            cstart.push_back(i);
+            cur = 0;
+        }
+        cur += b;
+    }
+    maxc = std::max(maxc, cur);
+    cstart.push_back(n_mod);
+    rc = ensure_staging(ctx, maxc);
+    if (rc != MOARA_OK) return rc;
+    std::vector<const void*> gdev(n_mod);
+    for (size_t c = 0; c + 1 < cstart.size(); ++c) {
+        const int b = static_cast<int>(c & 1);
+        // the copy into buffer b waits for the step that last read it
+        cudaError_t e = cudaStreamWaitEvent(ctx->copy_stream, ctx->compute_done[b], 0);
+        size_t off = 0;
+        for (int i = cstart[c]; i < cstart[c + 1] && e == cudaSuccess; ++i) {
+            const moara_module_desc& d = ctx->mods[ids[i]];
+            const size_t es = d.grad_dtype == MOARA_DTYPE_BF16 ? 2 : 4;
+            void* dst = static_cast<char*>(ctx->stage[b]) + off;
+            e = cudaMemcpyAsync(dst, G_host[i], es * (size_t)d.m * d.n, cudaMemcpyHostToDevice, ctx->copy_stream);
+            gdev[i] = dst;
+            off += gbytes(i);
+        }
+        if (e == cudaSuccess) e = cudaEventRecord(ctx->copy_done[b], ctx->copy_stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ctx->copy_done[b], 0);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "gradient upload");
+        rc = step_impl(ctx, cstart[c + 1] - cstart[c], ids + cstart[c], gdev.data() + cstart[c], t, lr,
+                       auto_refresh, s);
+        if (rc != MOARA_OK) return rc;
+        e = cudaEventRecord(ctx->compute_done[b], s);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "step event");
     }
     return MOARA_OK;
 }

@@ -34,7 +34,7 @@ namespace {
 
 constexpr int kTcGroup = 224;                 // modules per launch (G maps in params)
 constexpr long long kWaitLimit = 1LL << 32;   // ~2 s of SM clocks
-constexpr int kMaps = 6;                      // tensor maps per module
+constexpr int kMaps = 8;                      // tensor maps per module
 
 struct TcMod {
     int m, n, r, kb;
@@ -77,21 +77,28 @@ struct K0Params {
 constexpr int K1_BM = 128, K1_BN = 256, K1_BK = 64;
 constexpr int K1_A_BYTES = K1_BM * K1_BK * 2;           // 16 KB: two 64-rank chunks of P^T (MN-major)
 constexpr int K1_B_BYTES = K1_BK * K1_BN * 2;           // 32 KB: four 64-column chunks of V (MN-major)
+// The Adam moments stream through a ring of slots, each one 32-column chunk
+// of exp_avg and of exp_avg_sq (128 rank rows x 32 fp32, 16 KB each), loaded
+// and stored by TMA.
+constexpr int K1_MCOLS = 32;
+constexpr int K1_MCHUNK = K1_BM * K1_MCOLS * 4;          // 16 KB
 template <bool HILO> struct K1Cfg {
-    static constexpr int STAGES = HILO ? 2 : 4;
+    static constexpr int STAGES = HILO ? 2 : 3;
     static constexpr int STAGE_BYTES = K1_A_BYTES + (HILO ? 2 : 1) * K1_B_BYTES;
+    static constexpr int MSLOTS = HILO ? 1 : 2;
+    static constexpr int RING = STAGES * STAGE_BYTES;     // offset of the moment slots
+    static constexpr int CTL = RING + MSLOTS * 2 * K1_MCHUNK;
 };
-constexpr int K1_WARPS = 10;                            // 0 TMA, 1 MMA, 2-9 epilogue
+constexpr int K1_WARPS = 12;                            // 0 TMA, 1 MMA, 2 moment loader, 3 moment storer, 4-11 epilogue
 constexpr int K1_THREADS = K1_WARPS * 32;
-constexpr int GUARD_BYTES = 16384;
-constexpr int K1_SMEM = 1024 + 4 * (K1_A_BYTES + K1_B_BYTES) + GUARD_BYTES + 2048;
+constexpr int K1_SMEM = 1024 + (K1Cfg<false>::CTL > K1Cfg<true>::CTL ? K1Cfg<false>::CTL : K1Cfg<true>::CTL) + 2048;
 
 struct K1Params {
     CUtensorMap gmap[kTcGroup];        // G of each launch slot (decomposition off): {n, m}, box {64, 64}
     const int* cta_start;              // tiles of CTA c: tiles[cta_start[c] .. cta_start[c+1])
     const TcTile* tiles;
     const TcMod* mods;
-    const CUtensorMap* maps;           // per module: P (K1), P (K2), N, W, V_hi, V_lo
+    const CUtensorMap* maps;           // per module: P (K1), P (K2), N, W, V_hi, V_lo, exp_avg, exp_avg_sq
     int* status;
     float beta1, beta2, adam_eps, bc1, bc2;
     int decompose;
@@ -164,36 +171,52 @@ __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 
 constexpr int K0_SEG = 1024;
 
 template <int BLK>
-__global__ void __launch_bounds__(256) k0_decompose(const __grid_constant__ K0Params p) {
+__global__ void __launch_bounds__(256, 3) k0_decompose(const __grid_constant__ K0Params p) {
     constexpr int LPB = BLK / 8;                       // lanes per block (1..16)
     const int lane = threadIdx.x & 31;
     const long long total = p.start[p.count];
-    const long long warp0 = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
     const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
-    for (long long item = warp0; item < total; item += nwarps) {
-        int lo = 0, hi = p.count - 1;
-        while (lo < hi) {
-            const int mid = (lo + hi + 1) >> 1;
-            if (p.start[mid] <= item) lo = mid; else hi = mid - 1;
-        }
-        const K0Item& it = p.p[lo];
-        const long long local = item - p.start[lo];
-        const int row = static_cast<int>(local / it.segs);
-        const int seg = static_cast<int>(local - (long long)row * it.segs);
-        const int n = it.n;
-        uint4 g[4];
+    long long item = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+    int mod = 0;                                       // module of `item` (items only increase)
+    // G of the next item is loaded before the current one is processed, so
+    // each warp keeps a 1024-column row segment in flight
+    auto locate = [&](long long x, int& row, int& seg) {
+        while (mod + 1 < p.count && p.start[mod + 1] <= x) ++mod;
+        const int local = static_cast<int>(x - p.start[mod]);
+        row = local / p.p[mod].segs;
+        seg = local - row * p.p[mod].segs;
+    };
+    auto load = [&](int md, int row, int seg, uint4 (&g)[4]) {
+        const K0Item& it = p.p[md];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             const int c0 = seg * K0_SEG + u * 256 + lane * 8;
             g[u] = make_uint4(0u, 0u, 0u, 0u);
-            if (c0 < n) g[u] = __ldcs(reinterpret_cast<const uint4*>(it.G + (long long)row * n + c0));
+            if (c0 < it.n) g[u] = __ldcs(reinterpret_cast<const uint4*>(it.G + (long long)row * it.n + c0));
         }
+    };
+    if (item >= total) return;
+    int row, seg;
+    locate(item, row, seg);
+    uint4 g[4];
+    load(mod, row, seg, g);
+    while (true) {
+        const int cmod = mod, crow = row, cseg = seg;
+        uint4 cg[4] = {g[0], g[1], g[2], g[3]};
+        item += nwarps;
+        const bool more = item < total;
+        if (more) {
+            locate(item, row, seg);
+            load(mod, row, seg, g);
+        }
+        const K0Item& it = p.p[cmod];
+        const int n = it.n;
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-            const int cs = seg * K0_SEG + u * 256;      // first column of the sub-segment
+            const int cs = cseg * K0_SEG + u * 256;     // first column of the sub-segment
             if (cs >= n) break;                         // warp-uniform
             const int c0 = cs + lane * 8;
-            const uint32_t w[4] = {g[u].x, g[u].y, g[u].z, g[u].w};
+            const uint32_t w[4] = {cg[u].x, cg[u].y, cg[u].z, cg[u].w};
             float ss = 0.0f;
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
@@ -205,18 +228,16 @@ __global__ void __launch_bounds__(256) k0_decompose(const __grid_constant__ K0Pa
             for (int o = 1; o < LPB; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
             const float mag = sqrtf(ss);
             const float sc = 1.0f / (mag + p.decomp_eps);
-            if ((lane & (LPB - 1)) == 0 && c0 < n) {     // first lane of a block that starts before n
-                const long long o = (long long)row * it.kb + c0 / BLK;
-                if (p.do_mag) {
-                    const float ma = p.beta1 * it.mag_avg[o] + (1.0f - p.beta1) * mag;
-                    const float mas = p.beta2 * it.mag_avg_sq[o] + (1.0f - p.beta2) * mag * mag;
-                    it.mag_avg[o] = ma;
-                    it.mag_avg_sq[o] = mas;
-                    it.dM[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
-                }
+            if (p.do_mag && (lane & (LPB - 1)) == 0 && c0 < n) {   // first lane of a block that starts before n
+                const long long o = (long long)crow * it.kb + c0 / BLK;
+                const float ma = p.beta1 * it.mag_avg[o] + (1.0f - p.beta1) * mag;
+                const float mas = p.beta2 * it.mag_avg_sq[o] + (1.0f - p.beta2) * mag * mag;
+                it.mag_avg[o] = ma;
+                it.mag_avg_sq[o] = mas;
+                it.dM[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
             }
             if (c0 < n) {
-                const long long off = (long long)row * n + c0;
+                const long long off = (long long)crow * n + c0;
                 uint32_t vh[4], vl[4];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
@@ -228,6 +249,7 @@ __global__ void __launch_bounds__(256) k0_decompose(const __grid_constant__ K0Pa
                 if (p.hilo) *reinterpret_cast<uint4*>(it.Vlo + off) = make_uint4(vl[0], vl[1], vl[2], vl[3]);
             }
         }
+        if (!more) break;
     }
 }
 
@@ -237,23 +259,33 @@ __global__ void __launch_bounds__(256) k0_decompose(const __grid_constant__ K0Pa
 // adds the MMA with V_lo (first Adam step).
 // ===========================================================================
 template <bool HILO>
-__global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constant__ K1Params p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(K1_THREADS, 1)
+k1_project(const __grid_constant__ K1Params p) {
     constexpr int STAGES = K1Cfg<HILO>::STAGES;
     constexpr int STAGE_BYTES = K1Cfg<HILO>::STAGE_BYTES;
+    constexpr int MSLOTS = K1Cfg<HILO>::MSLOTS;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
-    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + 4 * (K1_A_BYTES + K1_B_BYTES) + GUARD_BYTES);
+    uint8_t* mring = smem + K1Cfg<HILO>::RING;
+    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + K1Cfg<HILO>::CTL);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int crank = static_cast<int>(ptx::cluster_ctarank());   // rank tile 2 t0 + crank of each pair tile
+    const int cluster = blockIdx.x >> 1;
     volatile int* abort_flag = &ctl->abort;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 2);    // both CTAs' MMAs consumed the stage
         }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(ptx::smem_u32(&ctl->accf[b]), 1);
             ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 8);
+        }
+        for (int b = 0; b < MSLOTS; ++b) {
+            ptx::mbar_init(ptx::smem_u32(&ctl->wfull[b]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->wdone[b]), 8);
+            ptx::mbar_init(ptx::smem_u32(&ctl->wempty[b]), 1);
         }
         ptx::mbar_init(ptx::smem_u32(&ctl->drain), 1);
         ctl->abort = 0;
@@ -264,13 +296,16 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
         ptx::tmem_relinquish();
     }
     ptx::tc_fence_before();
-    __syncthreads();
+    __syncwarp();
+    ptx::cluster_sync();            // barriers of both CTAs initialised before any remote signal
     ptx::tc_fence_after();
     const uint32_t tmem = ctl->tmem_base;
-    const int t_begin = p.cta_start[blockIdx.x], t_end = p.cta_start[blockIdx.x + 1];
+    const int t_begin = p.cta_start[cluster], t_end = p.cta_start[cluster + 1];
 
     if (warp == 0) {
         // ------------------------------------------------------ TMA producer
+        // P^T rows of this CTA's rank tile; the V tile (shared by the pair) is
+        // loaded half by each CTA and multicast to both.
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
@@ -282,7 +317,7 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
                 const CUtensorMap* pmap = &p.maps[tl.mod * kMaps + 0];
                 const CUtensorMap* vmap = p.decompose ? &p.maps[tl.mod * kMaps + 4] : &p.gmap[tl.slot];
                 const CUtensorMap* lmap = &p.maps[tl.mod * kMaps + 5];
-                const int r0 = tl.t0 * K1_BM, n0 = tl.t1 * K1_BN;
+                const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
                 const int nk = (md.m + K1_BK - 1) / K1_BK;
                 for (int kb = 0; kb < nk; ++kb) {
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
@@ -294,11 +329,11 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
 #pragma unroll
                     for (int c = 0; c < 2; ++c) ptx::tma_load_2d(a + c * 8192, pmap, fb, r0 + 64 * c, kb * K1_BK);
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) ptx::tma_load_2d(b + c * 8192, vmap, fb, n0 + 64 * c, kb * K1_BK);
-                    if (HILO) {
-#pragma unroll
-                        for (int c = 0; c < 4; ++c)
-                            ptx::tma_load_2d(b + K1_B_BYTES + c * 8192, lmap, fb, n0 + 64 * c, kb * K1_BK);
+                    for (int h = 0; h < 2; ++h) {
+                        const int c = 2 * crank + h;
+                        ptx::tma_load_2d_mc(b + c * 8192, vmap, fb, n0 + 64 * c, kb * K1_BK, 0x3);
+                        if (HILO)
+                            ptx::tma_load_2d_mc(b + K1_B_BYTES + c * 8192, lmap, fb, n0 + 64 * c, kb * K1_BK, 0x3);
                     }
                     issued |= 1u << stage;
                     last_par = (last_par & ~(1u << stage)) | (phase << stage);
@@ -343,7 +378,7 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
                             ptx::mma_f16(d0, adesc, ldesc, idesc, 1);
                         }
                     }
-                    ptx::mma_commit(ptx::smem_u32(&ctl->empty[stage]));
+                    ptx::mma_commit_mc(ptx::smem_u32(&ctl->empty[stage]), 0x3);
                     if (++stage == STAGES) { stage = 0; phase ^= 1; }
                 }
                 if (!ok) break;
@@ -354,92 +389,146 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
             ptx::mma_commit(ptx::smem_u32(&ctl->drain));
             wait_drain(ptx::smem_u32(&ctl->drain), 0);
         }
+    } else if (warp == 2) {
+        // ------------------------------------- moment chunk loader (TMA in)
+        if (lane == 0) {
+            uint32_t g = 0;
+            uint32_t issued = 0, last_par = 0;
+            bool ok = true;
+            for (int t = t_begin; t < t_end && ok; ++t) {
+                const TcTile tl = p.tiles[t];
+                const TcMod& md = p.mods[tl.mod];
+                const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 6];
+                const CUtensorMap* smap = &p.maps[tl.mod * kMaps + 7];
+                const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
+                const int nc = min(K1_BN / K1_MCOLS, (md.n - n0 + K1_MCOLS - 1) / K1_MCOLS);
+                for (int c = 0; c < nc; ++c, ++g) {
+                    const int b = g % MSLOTS;
+                    const uint32_t ph = (g / MSLOTS) & 1;
+                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->wempty[b]), ph ^ 1, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    const uint32_t fb = ptx::smem_u32(&ctl->wfull[b]);
+                    ptx::mbar_arrive_expect_tx(fb, 2 * K1_MCHUNK);
+                    const uint32_t dst = ptx::smem_u32(mring + b * 2 * K1_MCHUNK);
+                    ptx::tma_load_2d(dst, amap, fb, n0 + c * K1_MCOLS, r0);
+                    ptx::tma_load_2d(dst + K1_MCHUNK, smap, fb, n0 + c * K1_MCOLS, r0);
+                    issued |= 1u << b;
+                    last_par = (last_par & ~(1u << b)) | (ph << b);
+                }
+            }
+            if (!ok) {
+                for (int b = 0; b < MSLOTS; ++b)
+                    if (issued & (1u << b)) wait_drain(ptx::smem_u32(&ctl->wfull[b]), (last_par >> b) & 1);
+            }
+        }
+    } else if (warp == 3) {
+        // ------------------------------------ moment chunk storer (TMA out)
+        if (lane == 0) {
+            uint32_t g = 0;
+            bool ok = true;
+            for (int t = t_begin; t < t_end && ok; ++t) {
+                const TcTile tl = p.tiles[t];
+                const TcMod& md = p.mods[tl.mod];
+                const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 6];
+                const CUtensorMap* smap = &p.maps[tl.mod * kMaps + 7];
+                const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
+                const int nc = min(K1_BN / K1_MCOLS, (md.n - n0 + K1_MCOLS - 1) / K1_MCOLS);
+                for (int c = 0; c < nc; ++c, ++g) {
+                    const int b = g % MSLOTS;
+                    const uint32_t ph = (g / MSLOTS) & 1;
+                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->wdone[b]), ph, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    const uint32_t src = ptx::smem_u32(mring + b * 2 * K1_MCHUNK);
+                    ptx::tma_store_2d(amap, src, n0 + c * K1_MCOLS, r0);
+                    ptx::tma_store_2d(smap, src + K1_MCHUNK, n0 + c * K1_MCOLS, r0);
+                    ptx::bulk_commit_group();
+                    ptx::bulk_wait_read_all();            // the slot may be refilled once read
+                    ptx::mbar_arrive(ptx::smem_u32(&ctl->wempty[b]));
+                }
+            }
+            ptx::bulk_wait_all();
+        }
     } else {
         // ------------------------------------------------- epilogue warps
         // 8 warps: TMEM lane quarter q = warp % 4 (rank row), column half ch
-        // (128 of the 256 columns, 8 chunks of 16).  The moments of the next
-        // chunk are loaded while the current one is updated.
-        const int ew = warp - 2;                       // 0..7
+        // of each 32-column chunk.  Optimizer_V (Adam) on R: each thread
+        // updates 16 entries of both moments of its rank row in the swizzled
+        // ring slot and writes the update N in bf16 to global memory.
+        const int ew = warp - 4;                       // 0..7
         const int q = warp & 3;
         const int ch = ew >> 2;
+        const int il = q * 32 + lane;                  // rank row within the tile
         int buf = 0;
         uint32_t acc_phase = 0;
+        uint32_t g = 0;
         bool ok = true;
         for (int t = t_begin; t < t_end && ok; ++t) {
             const TcTile tl = p.tiles[t];
             const TcMod& md = p.mods[tl.mod];
             const int rr = md.r, nn = md.n;
-            float* const ea_p = md.exp_avg;
-            float* const es_p = md.exp_avg_sq;
             uint16_t* const nb_p = md.Nb;
-            const int r0 = tl.t0 * K1_BM, n0 = tl.t1 * K1_BN;
-            const int a = r0 + q * 32 + lane;
+            const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
+            const int a = r0 + il;
             const bool row_ok = a < rr;
-            const int jbase = n0 + ch * 128;
-            float4 pa0 = make_float4(0.f, 0.f, 0.f, 0.f), pa1 = pa0, pa2 = pa0, pa3 = pa0;
-            float4 ps0 = pa0, ps1 = pa0, ps2 = pa0, ps3 = pa0;
-            if (row_ok && jbase + 16 <= nn) {
-                const float4* x = reinterpret_cast<const float4*>(ea_p + (long long)a * nn + jbase);
-                const float4* y = reinterpret_cast<const float4*>(es_p + (long long)a * nn + jbase);
-                pa0 = x[0]; pa1 = x[1]; pa2 = x[2]; pa3 = x[3];
-                ps0 = y[0]; ps1 = y[1]; ps2 = y[2]; ps3 = y[3];
-            }
+            const int nc = min(K1_BN / K1_MCOLS, (nn - n0 + K1_MCOLS - 1) / K1_MCOLS);
             const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
                                             MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
             if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
             ptx::tc_fence_after();
-#pragma unroll 1
-            for (int c = 0; c < 8; ++c) {
-                const int j0 = jbase + c * 16;
-                float ea[16] = {pa0.x, pa0.y, pa0.z, pa0.w, pa1.x, pa1.y, pa1.z, pa1.w,
-                                pa2.x, pa2.y, pa2.z, pa2.w, pa3.x, pa3.y, pa3.z, pa3.w};
-                float es[16] = {ps0.x, ps0.y, ps0.z, ps0.w, ps1.x, ps1.y, ps1.z, ps1.w,
-                                ps2.x, ps2.y, ps2.z, ps2.w, ps3.x, ps3.y, ps3.z, ps3.w};
-                if (c + 1 < 8 && row_ok && j0 + 32 <= nn) {
-                    const float4* x = reinterpret_cast<const float4*>(ea_p + (long long)a * nn + j0 + 16);
-                    const float4* y = reinterpret_cast<const float4*>(es_p + (long long)a * nn + j0 + 16);
-                    pa0 = x[0]; pa1 = x[1]; pa2 = x[2]; pa3 = x[3];
-                    ps0 = y[0]; ps1 = y[1]; ps2 = y[2]; ps3 = y[3];
-                }
+            for (int c = 0; c < nc; ++c, ++g) {
+                const int b = g % MSLOTS;
+                const uint32_t ph = (g / MSLOTS) & 1;
+                const int j0 = n0 + c * K1_MCOLS + ch * 16;
                 float v[16];
                 __syncwarp();
-                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + ch * 128 + c * 16, v);
-                if (!row_ok || j0 >= nn) continue;
-                const long long o = (long long)a * nn + j0;
-                if (j0 + 16 <= nn) {
-                    float nv[16];
+                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + c * K1_MCOLS + ch * 16, v);
+                const bool gotm = ptx::mbar_wait(ptx::smem_u32(&ctl->wfull[b]), ph, abort_flag, p.status,
+                                                 MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+                if (!__all_sync(0xffffffffu, gotm)) { ok = false; break; }
+                uint8_t* arow = mring + b * 2 * K1_MCHUNK + il * 128;
+                uint8_t* srow = arow + K1_MCHUNK;
+                const uint32_t x = static_cast<uint32_t>(il & 7);
+                float nv[16];
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        ea[e] = p.beta1 * ea[e] + (1.0f - p.beta1) * v[e];
-                        es[e] = p.beta2 * es[e] + (1.0f - p.beta2) * v[e] * v[e];
-                        nv[e] = (ea[e] / p.bc1) / (sqrtf(es[e] / p.bc2) + p.adam_eps);
-                    }
-                    float4* ea4 = reinterpret_cast<float4*>(ea_p + o);
-                    float4* es4 = reinterpret_cast<float4*>(es_p + o);
+                for (int u = 0; u < 4; ++u) {
+                    const uint32_t off = ((ch * 4 + u) ^ x) << 4;
+                    float4* a4 = reinterpret_cast<float4*>(arow + off);
+                    float4* s4 = reinterpret_cast<float4*>(srow + off);
+                    const float4 av = *a4, sv = *s4;
+                    float ea[4] = {av.x, av.y, av.z, av.w};
+                    float es[4] = {sv.x, sv.y, sv.z, sv.w};
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        ea4[e] = make_float4(ea[4 * e], ea[4 * e + 1], ea[4 * e + 2], ea[4 * e + 3]);
-                        es4[e] = make_float4(es[4 * e], es[4 * e + 1], es[4 * e + 2], es[4 * e + 3]);
+                        const float rv = v[4 * u + e];
+                        ea[e] = p.beta1 * ea[e] + (1.0f - p.beta1) * rv;
+                        es[e] = p.beta2 * es[e] + (1.0f - p.beta2) * rv * rv;
+                        nv[4 * u + e] = (ea[e] / p.bc1) / (sqrtf(es[e] / p.bc2) + p.adam_eps);
                     }
-                    uint4* n4 = reinterpret_cast<uint4*>(nb_p + o);
-                    n4[0] = make_uint4(pack_bf16x2(nv[0], nv[1]), pack_bf16x2(nv[2], nv[3]),
-                                       pack_bf16x2(nv[4], nv[5]), pack_bf16x2(nv[6], nv[7]));
-                    n4[1] = make_uint4(pack_bf16x2(nv[8], nv[9]), pack_bf16x2(nv[10], nv[11]),
-                                       pack_bf16x2(nv[12], nv[13]), pack_bf16x2(nv[14], nv[15]));
-                } else {
+                    *a4 = make_float4(ea[0], ea[1], ea[2], ea[3]);
+                    *s4 = make_float4(es[0], es[1], es[2], es[3]);
+                }
+                ptx::fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->wdone[b]));
+                if (row_ok && j0 < nn) {
+                    const long long o = (long long)a * nn + j0;
+                    if (j0 + 16 <= nn) {
+                        uint4* n4 = reinterpret_cast<uint4*>(nb_p + o);
+                        n4[0] = make_uint4(pack_bf16x2(nv[0], nv[1]), pack_bf16x2(nv[2], nv[3]),
+                                           pack_bf16x2(nv[4], nv[5]), pack_bf16x2(nv[6], nv[7]));
+                        n4[1] = make_uint4(pack_bf16x2(nv[8], nv[9]), pack_bf16x2(nv[10], nv[11]),
+                                           pack_bf16x2(nv[12], nv[13]), pack_bf16x2(nv[14], nv[15]));
+                    } else {
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        if (j0 + e >= nn) continue;
-                        const float x = p.beta1 * ea_p[o + e] + (1.0f - p.beta1) * v[e];
-                        const float y = p.beta2 * es_p[o + e] + (1.0f - p.beta2) * v[e] * v[e];
-                        ea_p[o + e] = x;
-                        es_p[o + e] = y;
-                        const float nv = (x / p.bc1) / (sqrtf(y / p.bc2) + p.adam_eps);
-                        __nv_bfloat16 hb = __float2bfloat16_rn(nv);
-                        nb_p[o + e] = *reinterpret_cast<uint16_t*>(&hb);
+                        for (int e = 0; e < 16; ++e) {
+                            if (j0 + e >= nn) continue;
+                            __nv_bfloat16 hb = __float2bfloat16_rn(nv[e]);
+                            nb_p[o + e] = *reinterpret_cast<uint16_t*>(&hb);
+                        }
                     }
                 }
             }
+            if (!ok) break;
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->acce[buf]));
@@ -448,7 +537,8 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
     }
 
     ptx::tc_fence_before();
-    __syncthreads();
+    __syncwarp();
+    ptx::cluster_sync();            // no CTA leaves while its peer may still signal or fill it
     if (warp == 1) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, 512);
@@ -459,18 +549,21 @@ __global__ void __launch_bounds__(K1_THREADS, 1) k1_project(const __grid_constan
 // K2: back-projection dV = P N and the weight update in the epilogue.
 // ===========================================================================
 template <int BLK>
-__global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_constant__ K2Params p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(K2_THREADS, 1)
+k2_backproject(const __grid_constant__ K2Params p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
     uint8_t* wring = smem + K2_STAGES * K2_STAGE_BYTES;
     SmemCtl* ctl = reinterpret_cast<SmemCtl*>(wring + K2_WBUF * K2_WBYTES + K2_GUARD);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int crank = static_cast<int>(ptx::cluster_ctarank());   // row tile 2 t0 + crank of each pair tile
+    const int cluster = blockIdx.x >> 1;
     volatile int* abort_flag = &ctl->abort;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < K2_STAGES; ++s) {
             ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 2);    // both CTAs' MMAs consumed the stage
         }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(ptx::smem_u32(&ctl->accf[b]), 1);
@@ -490,10 +583,11 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
         ptx::tmem_relinquish();
     }
     ptx::tc_fence_before();
-    __syncthreads();
+    __syncwarp();
+    ptx::cluster_sync();            // barriers of both CTAs initialised before any remote signal
     ptx::tc_fence_after();
     const uint32_t tmem = ctl->tmem_base;
-    const int t_begin = p.cta_start[blockIdx.x], t_end = p.cta_start[blockIdx.x + 1];
+    const int t_begin = p.cta_start[cluster], t_end = p.cta_start[cluster + 1];
 
     if (warp == 0) {
         // ------------------------------------------------ operand TMA producer
@@ -507,7 +601,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
                 const TcMod& md = p.mods[tl.mod];
                 const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 1];
                 const CUtensorMap* bmap = &p.maps[tl.mod * kMaps + 2];
-                const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
+                const int i0 = (2 * tl.t0 + crank) * K2_BM, n0 = tl.t1 * K2_BN;
                 const int nk = (md.r + K2_BK - 1) / K2_BK;
                 for (int kb = 0; kb < nk; ++kb) {
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
@@ -518,7 +612,10 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
                     const uint32_t b = a + K2_A_BYTES;
                     ptx::tma_load_2d(a, amap, fb, kb * K2_BK, i0);
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) ptx::tma_load_2d(b + c * 8192, bmap, fb, n0 + 64 * c, kb * K2_BK);
+                    for (int h = 0; h < 2; ++h) {   // the N tile is shared by the pair: half each, multicast
+                        const int c = 2 * crank + h;
+                        ptx::tma_load_2d_mc(b + c * 8192, bmap, fb, n0 + 64 * c, kb * K2_BK, 0x3);
+                    }
                     issued |= 1u << stage;
                     last_par = (last_par & ~(1u << stage)) | (phase << stage);
                     if (++stage == K2_STAGES) { stage = 0; phase ^= 1; }
@@ -558,7 +655,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
                         const uint64_t bdesc = ptx::smem_desc_sw128(b + kk * 2048, 8192, 1024);
                         ptx::mma_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
                     }
-                    ptx::mma_commit(ptx::smem_u32(&ctl->empty[stage]));
+                    ptx::mma_commit_mc(ptx::smem_u32(&ctl->empty[stage]), 0x3);
                     if (++stage == K2_STAGES) { stage = 0; phase ^= 1; }
                 }
                 if (!ok) break;
@@ -578,7 +675,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
                 const CUtensorMap* wmap = &p.maps[tl.mod * kMaps + 3];
-                const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
+                const int i0 = (2 * tl.t0 + crank) * K2_BM, n0 = tl.t1 * K2_BN;
                 const int nc = min(K2_BN / K2_WCOLS, (md.n - n0 + K2_WCOLS - 1) / K2_WCOLS);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % K2_WBUF;
@@ -606,7 +703,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
                 const CUtensorMap* wmap = &p.maps[tl.mod * kMaps + 3];
-                const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
+                const int i0 = (2 * tl.t0 + crank) * K2_BM, n0 = tl.t1 * K2_BN;
                 const int nc = min(K2_BN / K2_WCOLS, (md.n - n0 + K2_WCOLS - 1) / K2_WCOLS);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % K2_WBUF;
@@ -640,7 +737,7 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
             const TcMod& md = p.mods[tl.mod];
             const int mm = md.m, nn = md.n, mkb = md.kb;
             const float* const dMp = md.dM;
-            const int i0 = tl.t0 * K2_BM, n0 = tl.t1 * K2_BN;
+            const int i0 = (2 * tl.t0 + crank) * K2_BM, n0 = tl.t1 * K2_BN;
             const int i = i0 + il;
             const bool row_ok = i < mm;
             const int nc = min(K2_BN / K2_WCOLS, (nn - n0 + K2_WCOLS - 1) / K2_WCOLS);
@@ -690,7 +787,8 @@ __global__ void __launch_bounds__(K2_THREADS, 1) k2_backproject(const __grid_con
     }
 
     ptx::tc_fence_before();
-    __syncthreads();
+    __syncwarp();
+    ptx::cluster_sync();            // no CTA leaves while its peer may still signal or fill it
     if (warp == 1) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, 512);
@@ -923,6 +1021,20 @@ bool encode_bf16_2d(EncodeTiledFn enc, CUtensorMap* map, const void* ptr, uint64
     return encode_2d(enc, map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ptr, inner, outer, box_inner, box_outer);
 }
 
+// Largest number of 2-CTA clusters of `fn` resident at once (at most `cap`).
+int max_clusters(const void* fn, int threads, int smem, int cap) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * cap, 1, 1);
+    cfg.blockDim = dim3(threads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess || n < 1) {
+        cudaGetLastError();
+        return cap;
+    }
+    return std::min(n, cap);
+}
+
 template <int BLK>
 void set_smem_attrs() {
     cudaFuncSetAttribute(k2_backproject<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize, K2_SMEM);
@@ -950,6 +1062,7 @@ struct TcState {
     };
     std::map<std::vector<int>, Tiles> tiles;
     bool attrs_set = false;
+    int k1_clusters = 1, k2_clusters = 1;  // co-resident 2-CTA clusters of K1 / K2
     K1Params p1;                           // parameter block of the next K1 launch
     K0Params p0;                           // parameter block of the next K0 launch
     KrParams pr;                           // parameter block of the next refresh GEMM launch
@@ -1017,7 +1130,10 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
         !encode_bf16_2d(st->encode, &mp[2], t.Nb, md.n, md.r, 64, 64) ||
         !encode_2d(st->encode, &mp[3], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, md.W, md.n, md.m, K2_WCOLS, K2_BM) ||
         !encode_bf16_2d(st->encode, &mp[4], t.Vhi, md.n, md.m, 64, 64) ||
-        !encode_bf16_2d(st->encode, &mp[5], t.Vlo, md.n, md.m, 64, 64)) {
+        !encode_bf16_2d(st->encode, &mp[5], t.Vlo, md.n, md.m, 64, 64) ||
+        !encode_2d(st->encode, &mp[6], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, md.exp_avg, md.n, md.r, K1_MCOLS, K1_BM) ||
+        !encode_2d(st->encode, &mp[7], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, md.exp_avg_sq, md.n, md.r, K1_MCOLS,
+                   K1_BM)) {
         st->err = "cuTensorMapEncodeTiled failed";
         return MOARA_ERR_CUDA;
     }
@@ -1092,33 +1208,35 @@ static void lpt_assign(const std::vector<TcTile>& tiles, const std::vector<doubl
 static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
     auto it = st->tiles.find(ids);
     if (it != st->tiles.end()) return &it->second;
+    // Work units are pair tiles: the two CTAs of a cluster take rank (K1) or
+    // row (K2) tiles 2 t0 and 2 t0 + 1 of the same column tile t1.
     std::vector<TcTile> k1, k2;
     std::vector<double> c1, c2;
     for (size_t slot = 0; slot < ids.size(); ++slot) {
         const TcMod& md = st->mods[ids[slot]];
-        // column tiles outer, rank tiles inner: CTAs that start together share
-        // the V panel of one column tile in L2
+        // column tiles outer, rank pairs inner: clusters that start together
+        // share the V panel of one column tile in L2
         const int nt = (md.n + K1_BN - 1) / K1_BN, rt = (md.r + K1_BM - 1) / K1_BM;
         for (int j = 0; j < nt; ++j)
-            for (int i = 0; i < rt; ++i) {
-                const int rows = std::min(K1_BM, md.r - i * K1_BM);
+            for (int i = 0; i < (rt + 1) / 2; ++i) {
+                const int rows = std::min(K1_BM, md.r - 2 * i * K1_BM);
                 const double mma = 8.0 * md.m;
                 const double epi = 0.66 * rows * std::min(K1_BN, md.n - j * K1_BN);
                 k1.push_back({ids[slot], static_cast<int>(slot), i, j});
                 c1.push_back(std::max(mma, epi));
             }
         const int mt = (md.m + K2_BM - 1) / K2_BM, nt2 = (md.n + K2_BN - 1) / K2_BN;
-        for (int i = 0; i < mt; ++i)
+        for (int i = 0; i < (mt + 1) / 2; ++i)
             for (int j = 0; j < nt2; ++j) {
                 const double mma = 8.0 * md.r;
-                const double epi = 0.3 * std::min(K2_BM, md.m - i * K2_BM) * std::min(K2_BN, md.n - j * K2_BN);
+                const double epi = 0.3 * std::min(K2_BM, md.m - 2 * i * K2_BM) * std::min(K2_BN, md.n - j * K2_BN);
                 k2.push_back({ids[slot], static_cast<int>(slot), i, j});
                 c2.push_back(std::max(mma, epi));
             }
     }
     TcState::Tiles t;
-    t.g1 = std::max(1, std::min(static_cast<int>(k1.size()), st->sms));
-    t.g2 = std::max(1, std::min(static_cast<int>(k2.size()), st->sms));
+    t.g1 = std::max(1, std::min(static_cast<int>(k1.size()), st->k1_clusters));   // clusters
+    t.g2 = std::max(1, std::min(static_cast<int>(k2.size()), st->k2_clusters));
     std::vector<int> s1, s2;
     std::vector<TcTile> o1, o2;
     lpt_assign(k1, c1, t.g1, s1, o1);
@@ -1150,21 +1268,21 @@ static cudaError_t launch_blk(TcState* st, const K1Params& p1, const K2Params& p
     cudaError_t e;
     if (decomp) {
         if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, true);
-        k0_decompose<BLK><<<st->sms * 4, 256, 0, s>>>(st->p0);
+        k0_decompose<BLK><<<st->sms * 3, 256, 0, s>>>(st->p0);
         if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, false);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         ++*launches;
     }
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, true);
-    if (hilo) k1_project<true><<<g1, K1_THREADS, K1_SMEM, s>>>(p1);
-    else k1_project<false><<<g1, K1_THREADS, K1_SMEM, s>>>(p1);
+    if (hilo) k1_project<true><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+    else k1_project<false><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, false);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     ++*launches;
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_BACKPROJECT, s, true);
-    k2_backproject<BLK><<<g2, K2_THREADS, K2_SMEM, s>>>(p2);
+    k2_backproject<BLK><<<2 * g2, K2_THREADS, K2_SMEM, s>>>(p2);
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_BACKPROJECT, s, false);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -1179,6 +1297,11 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
         cudaFuncSetAttribute(k1_project<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
         set_smem_attrs<8>(); set_smem_attrs<16>(); set_smem_attrs<32>(); set_smem_attrs<64>();
         set_smem_attrs<128>();
+        // clusters of two that fit on the GPU at once (persistent grids)
+        st->k1_clusters = max_clusters(reinterpret_cast<const void*>(k1_project<false>), K1_THREADS, K1_SMEM,
+                                       st->sms / 2);
+        st->k2_clusters = max_clusters(reinterpret_cast<const void*>(k2_backproject<128>), K2_THREADS, K2_SMEM,
+                                       st->sms / 2);
         st->attrs_set = true;
     }
     int rc = tc_upload(st);
@@ -1339,11 +1462,11 @@ int tc_split_v(TcState* st, const TcSplitItem* items, int count, int B, float de
         }
         p0.start[cnt] = acc;
         switch (B) {
-            case 8: k0_decompose<8><<<st->sms * 4, 256, 0, s>>>(p0); break;
-            case 16: k0_decompose<16><<<st->sms * 4, 256, 0, s>>>(p0); break;
-            case 32: k0_decompose<32><<<st->sms * 4, 256, 0, s>>>(p0); break;
-            case 64: k0_decompose<64><<<st->sms * 4, 256, 0, s>>>(p0); break;
-            case 128: k0_decompose<128><<<st->sms * 4, 256, 0, s>>>(p0); break;
+            case 8: k0_decompose<8><<<st->sms * 3, 256, 0, s>>>(p0); break;
+            case 16: k0_decompose<16><<<st->sms * 3, 256, 0, s>>>(p0); break;
+            case 32: k0_decompose<32><<<st->sms * 3, 256, 0, s>>>(p0); break;
+            case 64: k0_decompose<64><<<st->sms * 3, 256, 0, s>>>(p0); break;
+            case 128: k0_decompose<128><<<st->sms * 3, 256, 0, s>>>(p0); break;
             default: st->err = "block size not supported on the tensor-core path"; return MOARA_ERR_UNSUPPORTED;
         }
         const cudaError_t e = cudaGetLastError();
