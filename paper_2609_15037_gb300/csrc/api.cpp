@@ -178,6 +178,7 @@ size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v) {
     add(sizeof(float) * (size_t)m * l);  // Qb
     add(sizeof(uint16_t) * (size_t)m * l);  // Qbf
     add(sizeof(uint16_t) * (size_t)n * l);  // Zbf
+    for (int i = 0; i < 3; ++i) add(3 * sizeof(uint16_t) * (size_t)l * l);   // Cp, P1, P2
     for (int i = 0; i < 6; ++i) add(sizeof(float) * (size_t)l * l);
     add(sizeof(float) * 16);
     add(sizeof(float) * (size_t)l);
@@ -200,6 +201,9 @@ void refresh_carve(RefreshItem& it, void* base, int m, int n, int r, int l, int 
     it.Qb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * l));
     it.Qbf = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * (size_t)m * l));
     it.Zbf = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * (size_t)n * l));
+    it.Cp = reinterpret_cast<uint16_t*>(take(3 * sizeof(uint16_t) * (size_t)l * l));
+    it.P1 = reinterpret_cast<uint16_t*>(take(3 * sizeof(uint16_t) * (size_t)l * l));
+    it.P2 = reinterpret_cast<uint16_t*>(take(3 * sizeof(uint16_t) * (size_t)l * l));
     it.Cg = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Linv = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
     it.Tt = reinterpret_cast<float*>(take(sizeof(float) * (size_t)l * l));
@@ -456,6 +460,49 @@ struct RefreshRunner {
         tc_gemm(1, apply);
     }
 
+    // ------------------------------------- split-precision l x l products
+    void split3(const std::vector<float*>& src, const std::vector<uint16_t*>& dst, int transpose) {
+        moara::SmallBatch sb = small();
+        for (size_t i = 0; i < it.size(); ++i) {
+            sb.a[i] = src[i]; sb.h[i] = dst[i]; sb.rows[i] = it[i].l; sb.l[i] = it[i].l;
+        }
+        chk(moara::launch_split3(sb, transpose, s, &ctx->launches));
+    }
+
+    // out = A B (l x l) from three-plane operands (A stored K x M, B K x N)
+    void ks_gemm(const std::vector<uint16_t*>& A, const std::vector<uint16_t*>& B, const std::vector<float*>& out,
+                 int ktri) {
+        std::vector<moara::TcSplitGemmItem> g;
+        for (size_t i = 0; i < it.size(); ++i) {
+            const int l = it[i].l;
+            const size_t pl = (size_t)l * l;
+            g.push_back({A[i], B[i], pl, pl, out[i], l, l, l, ktri});
+        }
+        ProfScope ps(ctx, MOARA_PHASE_TC_REFRESH, s);
+        if (moara::tc_gemm_split3(ctx->tc, g.data(), static_cast<int>(g.size()), s, &ctx->launches) != MOARA_OK)
+            chk(cudaErrorLaunchFailure);
+    }
+
+    // One CholeskyQR pass on an l x l matrix with the Gram matrix and the
+    // triangular apply as split-precision tensor-core products (fp32-accurate):
+    // Xout = Win R^-1, R^T R = Win^T Win + shift.
+    void ks_cholqr_pass(std::vector<float*>& Win, std::vector<float*>& Xout, const std::vector<int>& rows_l,
+                        float shift_rel) {
+        std::vector<uint16_t*> p1(it.size()), p2(it.size());
+        for (size_t i = 0; i < it.size(); ++i) { p1[i] = it[i].P1; p2[i] = it[i].P2; }
+        std::vector<float*> cg(it.size());
+        for (size_t i = 0; i < it.size(); ++i) cg[i] = it[i].Cg;
+        split3(Win, p1, 0);                 // W (as A = W^T, MN-major, and as B)
+        ks_gemm(p1, p1, cg, 0);             // Gram W^T W
+        cholesky_blocked(rows_l, shift_rel);
+        tri_inverse(/*have_diag=*/true);
+        std::vector<float*> linv(it.size());
+        for (size_t i = 0; i < it.size(); ++i) linv[i] = it[i].Linv;
+        split3(linv, p2, 1);                // B = Linv^T (upper triangular)
+        split3(Win, p1, 1);                 // A = W read MN-major: its transpose
+        ks_gemm(p1, p2, Xout, 1);
+    }
+
     void run() {
         const int n_it = static_cast<int>(it.size());
         const moara_hparams& hp = ctx->hp;
@@ -603,28 +650,51 @@ struct RefreshRunner {
         // Eigenvectors of C by orthogonal iteration X <- C X with CholeskyQR2
         // (shifted, then plain) every iteration: each X is orthonormal, so
         // directions of C below its rounding level only ever fill an
-        // orthonormal completion.  Then the Ritz order.
+        // orthonormal completion.  Then the Ritz order.  On the tensor-core
+        // path the l x l products run as split-precision (3 x bf16) MMAs.
         {
             moara::SmallBatch sb = small();
             for (int i = 0; i < n_it; ++i) { sb.a[i] = Xa[i]; sb.l[i] = it[i].l; }
             chk(moara::launch_set_identity(sb, s, &ctx->launches));
         }
         moara::GemmKind prod{moara::A_KCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
+        std::vector<uint16_t*> cp(n_it), p1(n_it);
+        for (int i = 0; i < n_it; ++i) { cp[i] = it[i].Cp; p1[i] = it[i].P1; }
+        std::vector<float*> cr(n_it);
+        for (int i = 0; i < n_it; ++i) cr[i] = it[i].Cr;
+        if (tc) split3(cr, cp, 0);          // C is symmetric: read MN-major as A
         for (int q = 0; q < hp.ritz_iters; ++q) {
+            if (tc) {
+                split3(Xa, p1, 0);
+                ks_gemm(cp, p1, Xb, 0);                  // W = C X
+                ks_cholqr_pass(Xb, Xa, rows_l, 2.0f * u_rnd);
+                // the tensor cores accumulate long sums less tightly than
+                // fp32 FMAs: the pass that fixes the final orthonormality of
+                // X runs on the fp32 units
+                if (q + 1 < hp.ritz_iters) ks_cholqr_pass(Xa, Xb, rows_l, 0.0f);
+                else cholqr_pass(Xa, Xb, rows_l, 0.0f);
+                std::swap(Xa, Xb);                       // X in Xa
+            } else {
+                gemm(prod, [&](int i, moara::GemmProb& p) {
+                    const int l = it[i].l;
+                    p.A = it[i].Cr; p.Bm = Xa[i]; p.C = Xb[i];
+                    p.M = l; p.N = l; p.K = l; p.lda = l; p.ldb = l; p.ldc = l;
+                });
+                cholqr2s(Xb, Xa, rows_l);      // X in Xa
+            }
+        }
+        // Ritz values (Rayleigh quotients of the columns of X) and order:
+        // W = C X into Xb
+        if (tc) {
+            split3(Xa, p1, 0);
+            ks_gemm(cp, p1, Xb, 0);
+        } else {
             gemm(prod, [&](int i, moara::GemmProb& p) {
                 const int l = it[i].l;
                 p.A = it[i].Cr; p.Bm = Xa[i]; p.C = Xb[i];
                 p.M = l; p.N = l; p.K = l; p.lda = l; p.ldb = l; p.ldc = l;
             });
-            cholqr2s(Xb, Xa, rows_l);      // X in Xa
         }
-        // Ritz values (Rayleigh quotients of the columns of X) and order:
-        // W = C X into Xb
-        gemm(prod, [&](int i, moara::GemmProb& p) {
-            const int l = it[i].l;
-            p.A = it[i].Cr; p.Bm = Xa[i]; p.C = Xb[i];
-            p.M = l; p.N = l; p.K = l; p.lda = l; p.ldb = l; p.ldc = l;
-        });
         {
             moara::SmallBatch sb = small();
             for (int i = 0; i < n_it; ++i) {

@@ -138,6 +138,9 @@ struct RefreshItem {
     uint16_t* Vlo;          // residual plane, or null when Vhi is exact
     uint16_t* Qbf;    // m x l bf16 copy of the latest orthonormal Q
     uint16_t* Zbf;    // n x l bf16 copy of the latest Z (or of Omega)
+    uint16_t* Cp;     // 3 x l x l bf16 planes of the Rayleigh-Ritz matrix
+    uint16_t* P1;     // 3 x l x l planes of X / W / W^T
+    uint16_t* P2;     // 3 x l x l planes of Linv^T
 };
 
 size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v);
@@ -172,5 +175,7 @@ cudaError_t launch_ritz_sort(const SmallBatch& b, cudaStream_t s, int64_t* launc
 cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_sign_fix_store(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_transpose_bf16(const SmallBatch& b, cudaStream_t s, int64_t* launches);  // h = bf16(a^T)
+// three bf16 planes (hi, mid, lo) of a (rows x l) at h, or of its transpose
+cudaError_t launch_split3(const SmallBatch& b, int transpose, cudaStream_t s, int64_t* launches);
 
 }  // namespace moara

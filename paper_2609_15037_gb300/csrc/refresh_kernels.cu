@@ -299,6 +299,57 @@ cudaError_t launch_transpose_bf16(const SmallBatch& b, cudaStream_t s, int64_t* 
 }
 
 // ---------------------------------------------------------------------------
+// Three bf16 planes of an fp32 matrix (rows x l, row-major): hi = bf16(x),
+// mid = bf16(x - hi), lo = bf16(x - hi - mid), so hi + mid + lo carries 24
+// significant bits.  With `transpose` the planes hold the l x rows transpose.
+// Planes are consecutive at h, each rows * l elements.  32 x 32 tiles through
+// shared memory keep both sides coalesced.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_split3(const __grid_constant__ SmallBatch b, int transpose) {
+    __shared__ float t[32][33];
+    const int pi = blockIdx.z;
+    const int rows = b.rows[pi], cols = b.l[pi];
+    const float* src = b.a[pi];
+    uint16_t* dst = b.h[pi];
+    const long long plane = (long long)rows * cols;
+    const int tr = (rows + 31) / 32, tc = (cols + 31) / 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    for (int tile = blockIdx.x; tile < tr * tc; tile += gridDim.x) {
+        const int ti = tile / tc, tj = tile - ti * tc;
+        for (int r = ty; r < 32; r += 8) {
+            const int i = ti * 32 + r, j = tj * 32 + tx;
+            t[r][tx] = (i < rows && j < cols) ? src[(long long)i * cols + j] : 0.0f;
+        }
+        __syncthreads();
+        for (int r = ty; r < 32; r += 8) {
+            int i, j, oc;
+            float x;
+            if (transpose) { i = tj * 32 + r; j = ti * 32 + tx; oc = rows; x = t[tx][r]; }   // out row i = src column
+            else           { i = ti * 32 + r; j = tj * 32 + tx; oc = cols; x = t[r][tx]; }
+            const bool in = transpose ? (i < cols && j < rows) : (i < rows && j < cols);
+            if (in) {
+                const __nv_bfloat16 h0 = __float2bfloat16_rn(x);
+                const float r1 = x - __bfloat162float(h0);
+                const __nv_bfloat16 h1 = __float2bfloat16_rn(r1);
+                const __nv_bfloat16 h2 = __float2bfloat16_rn(r1 - __bfloat162float(h1));
+                const long long o = (long long)i * oc + j;
+                dst[o] = *reinterpret_cast<const uint16_t*>(&h0);
+                dst[plane + o] = *reinterpret_cast<const uint16_t*>(&h1);
+                dst[2 * plane + o] = *reinterpret_cast<const uint16_t*>(&h2);
+            }
+        }
+        __syncthreads();
+    }
+}
+
+cudaError_t launch_split3(const SmallBatch& b, int transpose, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    k_split3<<<dim3(256, 1, b.count), 256, 0, s>>>(b, transpose);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // a <- I (l x l)
 // ---------------------------------------------------------------------------
 __global__ void k_set_identity(const __grid_constant__ SmallBatch b) {

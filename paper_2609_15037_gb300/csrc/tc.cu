@@ -1001,6 +1001,178 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
     }
 }
 
+// ===========================================================================
+// KS: fp32-accurate GEMM of the Rayleigh-Ritz step on tensor cores.  Both
+// operands arrive as three bf16 planes (x = hi + mid + lo, 24 significant
+// bits); six MMAs per k-step (hi.hi, hi.mid, mid.hi, hi.lo, mid.mid, lo.hi)
+// leave out terms of relative size 2^-24 and below.  out (M x N, fp32) =
+// A B with A stored K x M and B stored K x N (both MN-major), tile 256 x 256
+// (two 128-row accumulators in TMEM), BK = 32, two stages of 96 KB; `ktri`
+// stops the K loop of column tile n0 at n0 + 256 (B upper triangular).
+// ===========================================================================
+constexpr int KS_BM = 256, KS_BN = 256, KS_BK = 32;
+constexpr int KS_PLANE = KS_BM * KS_BK * 2;               // 16 KB: one plane of A (or B)
+constexpr int KS_STAGE = 6 * KS_PLANE;                    // 96 KB
+constexpr int KS_STAGES = 2;
+constexpr int KS_SMEM = 1024 + KS_STAGES * KS_STAGE + 2048;
+constexpr int kKsGroup = 36;                              // problems per launch (six maps each in the parameters)
+
+struct KsParams {
+    CUtensorMap amap[kKsGroup][3];     // A planes ({M, K}, box {64, 32})
+    CUtensorMap bmap[kKsGroup][3];     // B planes ({N, K}, box {64, 32})
+    float* out[kKsGroup];
+    int M[kKsGroup], N[kKsGroup], K[kKsGroup];
+    int ktri[kKsGroup];
+    int tiles_n[kKsGroup];
+    int tile_start[kKsGroup + 1];
+    int count;
+    int* status;
+};
+
+__global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constant__ KsParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = align1024(smem_raw);
+    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + KS_STAGES * KS_STAGE);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    volatile int* abort_flag = &ctl->abort;
+
+    const int tile = blockIdx.x;
+    int lo = 0, hi = p.count - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.tile_start[mid] <= tile) lo = mid; else hi = mid - 1;
+    }
+    const int pi = lo;
+    const int local = tile - p.tile_start[pi];
+    const int M = p.M[pi], N = p.N[pi], K = p.K[pi];
+    const int i0 = (local / p.tiles_n[pi]) * KS_BM;
+    const int n0 = (local % p.tiles_n[pi]) * KS_BN;
+    const int nch = min(4, (N - n0 + 63) / 64);
+    const int halves = (M - i0) > 128 ? 2 : 1;
+    const int kend = p.ktri[pi] ? min(K, n0 + KS_BN) : K;
+    const int nk = (kend + KS_BK - 1) / KS_BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < KS_STAGES; ++s) {
+            ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
+            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);
+        }
+        ptx::mbar_init(ptx::smem_u32(&ctl->accf[0]), 1);
+        ptx::mbar_init(ptx::smem_u32(&ctl->drain), 1);
+        ctl->abort = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(ptx::smem_u32(&ctl->tmem_base), 512);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = ctl->tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t issued = 0, last_par = 0;
+            const uint32_t bytes = 3 * KS_PLANE + 3 * nch * 4096;
+            for (int kb = 0; kb < nk; ++kb) {
+                if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
+                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) {
+                    for (int s = 0; s < KS_STAGES; ++s)
+                        if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
+                    break;
+                }
+                const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
+                ptx::mbar_arrive_expect_tx(fb, bytes);
+                const uint32_t a = ptx::smem_u32(smem + stage * KS_STAGE);
+                const uint32_t b = a + 3 * KS_PLANE;
+#pragma unroll
+                for (int q = 0; q < 3; ++q) {
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        ptx::tma_load_2d(a + q * KS_PLANE + c * 4096, &p.amap[pi][q], fb, i0 + 64 * c, kb * KS_BK);
+                    for (int c = 0; c < nch; ++c)
+                        ptx::tma_load_2d(b + q * KS_PLANE + c * 4096, &p.bmap[pi][q], fb, n0 + 64 * c, kb * KS_BK);
+                }
+                issued |= 1u << stage;
+                last_par = (last_par & ~(1u << stage)) | (phase << stage);
+                if (++stage == KS_STAGES) { stage = 0; phase ^= 1; }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t idesc = ptx::idesc_bf16(128, nch * 64, 1, 1);
+            // plane pairs (A, B) of the six products
+            constexpr int PA[6] = {0, 0, 1, 0, 1, 2};
+            constexpr int PB[6] = {0, 1, 0, 2, 1, 0};
+            int stage = 0;
+            uint32_t phase = 0;
+            for (int kb = 0; kb < nk; ++kb) {
+                if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
+                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) break;
+                ptx::tc_fence_after();
+                const uint32_t a = ptx::smem_u32(smem + stage * KS_STAGE);
+                const uint32_t b = a + 3 * KS_PLANE;
+#pragma unroll
+                for (int kk = 0; kk < 2; ++kk) {
+#pragma unroll
+                    for (int e = 0; e < 6; ++e) {
+                        const uint64_t bdesc = ptx::smem_desc_sw128(b + PB[e] * KS_PLANE + kk * 2048, 4096, 1024);
+                        for (int h = 0; h < halves; ++h) {
+                            const uint64_t adesc =
+                                ptx::smem_desc_sw128(a + PA[e] * KS_PLANE + h * 8192 + kk * 2048, 4096, 1024);
+                            ptx::mma_f16(tmem + h * 256, adesc, bdesc, idesc, (kb | kk | e) != 0);
+                        }
+                    }
+                }
+                ptx::mma_commit(ptx::smem_u32(&ctl->empty[stage]));
+                if (++stage == KS_STAGES) { stage = 0; phase ^= 1; }
+            }
+            ptx::mma_commit(ptx::smem_u32(&ctl->accf[0]));
+            ptx::mma_commit(ptx::smem_u32(&ctl->drain));
+            wait_drain(ptx::smem_u32(&ctl->drain), 0);
+        }
+    } else {
+        const int ew = warp - 2;
+        const int q = warp & 3;
+        const int h = ew >> 2;
+        const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[0]), 0, abort_flag, p.status,
+                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+        if (__all_sync(0xffffffffu, got) && h < halves) {
+            ptx::tc_fence_after();
+            const int row = i0 + h * 128 + q * 32 + lane;
+            float* const of = p.out[pi];
+            const long long ro = (long long)row * N;
+            for (int c = 0; c < nch * 4; ++c) {
+                const int j0 = n0 + c * 16;
+                if (j0 >= N) break;                       // warp-uniform
+                float v[16];
+                __syncwarp();
+                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + h * 256 + c * 16, v);
+                if (row >= M) continue;
+                if (j0 + 16 <= N) {
+                    float4* o4 = reinterpret_cast<float4*>(of + ro + j0);
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) o4[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e)
+                        if (j0 + e < N) of[ro + j0 + e] = v[e];
+                }
+            }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, 512);
+    }
+}
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -1067,6 +1239,8 @@ struct TcState {
     K0Params p0;                           // parameter block of the next K0 launch
     KrParams pr;                           // parameter block of the next refresh GEMM launch
     bool kr_attrs = false;
+    KsParams ps;                           // parameter block of the next split-precision GEMM launch
+    bool ks_attrs = false;
 };
 
 bool tc_supported(int m, int n, int r, int B, int dtype, int decompose) {
@@ -1469,6 +1643,56 @@ int tc_split_v(TcState* st, const TcSplitItem* items, int count, int B, float de
             case 128: k0_decompose<128><<<st->sms * 3, 256, 0, s>>>(p0); break;
             default: st->err = "block size not supported on the tensor-core path"; return MOARA_ERR_UNSUPPORTED;
         }
+        const cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) {
+            st->err = cudaGetErrorString(e);
+            return MOARA_ERR_CUDA;
+        }
+        ++*launches;
+    }
+    return MOARA_OK;
+}
+
+int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, cudaStream_t s, int64_t* launches) {
+    if (!st->ks_attrs) {
+        cudaFuncSetAttribute(ks_product, cudaFuncAttributeMaxDynamicSharedMemorySize, KS_SMEM);
+        st->ks_attrs = true;
+    }
+    for (int i = 0; i < count; ++i) {
+        const TcSplitGemmItem& x = items[i];
+        if (x.M < 1 || x.N < 1 || x.K < 1 || (x.M % 8) != 0 || (x.N % 8) != 0) {
+            st->err = "split-precision GEMM: M and N must be multiples of 8";
+            return MOARA_ERR_UNSUPPORTED;
+        }
+    }
+    for (int c0 = 0; c0 < count; c0 += kKsGroup) {
+        const int cnt = std::min(kKsGroup, count - c0);
+        KsParams& kp = st->ps;
+        std::memset(&kp, 0, sizeof(kp));
+        int total = 0;
+        for (int q = 0; q < cnt; ++q) {
+            const TcSplitGemmItem& x = items[c0 + q];
+            bool ok = true;
+            for (int pl = 0; pl < 3; ++pl) {
+                ok = ok && encode_bf16_2d(st->encode, &kp.amap[q][pl], x.A + (size_t)pl * x.a_plane, x.M, x.K, 64, 32);
+                ok = ok && encode_bf16_2d(st->encode, &kp.bmap[q][pl], x.B + (size_t)pl * x.b_plane, x.N, x.K, 64, 32);
+            }
+            if (!ok) {
+                st->err = "cuTensorMapEncodeTiled failed for a split-precision operand";
+                return MOARA_ERR_CUDA;
+            }
+            kp.out[q] = x.out;
+            kp.M[q] = x.M; kp.N[q] = x.N; kp.K[q] = x.K;
+            kp.ktri[q] = x.ktri;
+            kp.tiles_n[q] = (x.N + KS_BN - 1) / KS_BN;
+            kp.tile_start[q] = total;
+            total += ((x.M + KS_BM - 1) / KS_BM) * kp.tiles_n[q];
+        }
+        kp.tile_start[cnt] = total;
+        kp.count = cnt;
+        kp.status = st->d_status;
+        if (total == 0) continue;
+        ks_product<<<total, KR_THREADS, KS_SMEM, s>>>(kp);
         const cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) {
             st->err = cudaGetErrorString(e);

@@ -41,6 +41,22 @@ struct TcGemmItem {
 int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, cudaStream_t s,
                  int64_t* launches);
 
+// One problem of the split-precision GEMM: out (M x N fp32) = A B with A
+// stored K x M and B stored K x N, each as three consecutive bf16 planes
+// (hi, mid, lo; plane strides a_plane / b_plane elements) whose sum is the
+// fp32 operand.
+struct TcSplitGemmItem {
+    const uint16_t* A;
+    const uint16_t* B;
+    size_t a_plane, b_plane;
+    float* out;
+    int M, N, K;
+    int ktri;              // B upper triangular: column j needs k <= j only
+};
+
+// Grouped launch; M and N multiples of 8, planes 16-byte aligned.
+int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, cudaStream_t s, int64_t* launches);
+
 // V = Decompose(G, B) direction as two bf16 planes (V_hi, V_lo) for the
 // refresh products; G bf16 m x n, B in {8, ..., 128}.
 struct TcSplitItem {
