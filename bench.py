@@ -34,6 +34,15 @@ WORKLOAD = "llama2_7b_full_module_aware"
 METRIC = "ms per full-model projected-Adam step"
 LR = 1e-3
 
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one launch of
+# each step kernel, from an ncu capture of one decoder layer of the same
+# shapes (the full model is 32 such layers, and each kernel's traffic grows
+# in proportion to the layers it processes).  Valid only for the kernel source
+# with this SHA-1; after any change the roofline reports traffic = null until
+# the counters are taken again (profiles/ has the capture).
+TRAFFIC = {"source": "paper_2609_15037_gb300/csrc/tc.cu", "sha1": None, "layers": 32,
+           "layer_bytes": {}}
+
 
 def _peaks():
     try:
@@ -146,6 +155,17 @@ def _kernel_bytes(mods, B, tc):
     return kb
 
 
+def _traffic(kernel, workload):
+    """Per-launch DRAM bytes of `kernel` at the full-model workload, or None."""
+    import hashlib
+    if workload != WORKLOAD or TRAFFIC["sha1"] is None or kernel not in TRAFFIC["layer_bytes"]:
+        return None
+    with open(os.path.join(ROOT, TRAFFIC["source"]), "rb") as f:
+        if hashlib.sha1(f.read()).hexdigest() != TRAFFIC["sha1"]:
+            return None
+    return int(TRAFFIC["layer_bytes"][kernel] * TRAFFIC["layers"])
+
+
 def run_gpu(args):
     import torch
     import paper_2609_15037_gb300 as M
@@ -239,18 +259,29 @@ def run_gpu(args):
     M.moara_step_grouped_host(g.ctx, ids, hptr, step, LR, False, chunk, cs)   # staging allocation
     step += 1
     torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps + 1)]
+    evs[0].record(stream)
     e2e_status = 0
-    for _ in range(e2e_steps):
+    for k in range(e2e_steps):
         M.moara_step_grouped_host(g.ctx, ids, hptr, step, LR, False, chunk, cs)
         step += 1
         e2e_status |= M.moara_get_device_status(g.ctx, cs)
-    e1.record(stream)
+        evs[k + 1].record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    e2e_ms = evs[0].elapsed_time(evs[-1]) / e2e_steps
+    e2e_each = sorted(evs[k].elapsed_time(evs[k + 1]) for k in range(e2e_steps))
+    e2e_median = e2e_each[len(e2e_each) // 2]
     h2d = sum(x.numel() * x.element_size() for x in grads)
+    # the host link alone: the same bytes copied into the device gradients
+    torch.cuda.synchronize()
+    c0 = torch.cuda.Event(enable_timing=True)
+    c1 = torch.cuda.Event(enable_timing=True)
+    c0.record(stream)
+    for h, x in zip(host, grads):
+        x.copy_(h, non_blocking=True)
+    c1.record(stream)
+    torch.cuda.synchronize()
+    h2d_gbs = h2d / (c0.elapsed_time(c1) * 1e-3) / 1e9
 
     hbm, bf16_peak, bf16_sus, peak_src = _peaks()
     alg_bytes, alg_flops, _ = _algorithmic(mods, B)
@@ -275,13 +306,13 @@ def run_gpu(args):
     elif dom == "tc_project":
         achieved = flops_dom / (dom_ms * 1e-3) / 1e12
         roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": bf16_sus,
-                "unit": "TFLOP/s", "frac": round(achieved / bf16_sus, 4), "traffic": None,
+                "unit": "TFLOP/s", "frac": round(achieved / bf16_sus, 4), "traffic": _traffic(dom, args.workload),
                 "kernel": dom, "peak_source": f"bf16_tflops_sustained ({peak_src})"}
     else:
         by = kbytes[dom] / n_launch_per_step
         achieved = by / (dom_ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
-                "frac": round(achieved / hbm, 4), "traffic": None, "kernel": dom,
+                "frac": round(achieved / hbm, 4), "traffic": _traffic(dom, args.workload), "kernel": dom,
                 "peak_source": f"hbm_gbs ({peak_src})"}
 
     kernels = {}
@@ -315,7 +346,9 @@ def run_gpu(args):
         "roofline": roof,
         "kernels": kernels,
         "e2e": {"value": round(e2e_ms + refresh_ms / 200.0, 4), "unit": "ms",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4},
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4,
+                "h2d_gbs_link": round(h2d_gbs, 1),
+                "step_ms_median": round(e2e_median, 3), "steps": e2e_steps},
         "gpu_launches": int(launches),
         "device_status": status | e2e_status,
         "clocks": clk,

@@ -101,6 +101,7 @@ struct K1Params {
     const CUtensorMap* maps;           // per module: P (K1), P (K2), N, W, V_hi, V_lo, exp_avg, exp_avg_sq
     int* status;
     float beta1, beta2, adam_eps, bc1, bc2;
+    float inv_bc1, inv_bc2;            // 1 / bias corrections
     int decompose;
 };
 
@@ -502,7 +503,10 @@ k1_project(const __grid_constant__ K1Params p) {
                         const float rv = v[4 * u + e];
                         ea[e] = p.beta1 * ea[e] + (1.0f - p.beta1) * rv;
                         es[e] = p.beta2 * es[e] + (1.0f - p.beta2) * rv * rv;
-                        nv[4 * u + e] = (ea[e] / p.bc1) / (sqrtf(es[e] / p.bc2) + p.adam_eps);
+                        // N goes to K2 in bf16: approximate sqrt / reciprocal
+                        // (relative error ~2^-22) are far below its rounding
+                        nv[4 * u + e] = ea[e] * p.inv_bc1 *
+                                        ptx::rcp_approx(ptx::sqrt_approx(es[e] * p.inv_bc2) + p.adam_eps);
                     }
                     *a4 = make_float4(ea[0], ea[1], ea[2], ea[3]);
                     *s4 = make_float4(es[0], es[1], es[2], es[3]);
@@ -1522,6 +1526,7 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
         p1.mods = st->d_mods; p1.maps = st->d_maps; p1.status = st->d_status;
         p1.beta1 = hp.beta1; p1.beta2 = hp.beta2; p1.adam_eps = hp.adam_eps;
         p1.bc1 = bc1; p1.bc2 = bc2;
+        p1.inv_bc1 = 1.0f / bc1; p1.inv_bc2 = 1.0f / bc2;
         p1.decompose = dec ? 1 : 0;
         K2Params p2{};
         p2.cta_start = tl->k2_start; p2.tiles = tl->k2;
