@@ -76,14 +76,14 @@ struct K0Params {
 // ------------------------------------------------------------------- K1
 constexpr int K1_BM = 128, K1_BN = 256, K1_BK = 64;
 constexpr int K1_A_BYTES = K1_BM * K1_BK * 2;           // 16 KB: two 64-rank chunks of P^T (MN-major)
-constexpr int K1_B_BYTES = K1_BK * K1_BN * 2;           // 32 KB: four 64-column chunks of V (MN-major)
+constexpr int K1_B_BYTES = K1_BK * (K1_BN / 2) * 2;     // 16 KB: this CTA's two 64-column chunks of V
 // The Adam moments stream through a ring of slots, each one 32-column chunk
 // of exp_avg and of exp_avg_sq (128 rank rows x 32 fp32, 16 KB each), loaded
 // and stored by TMA.
 constexpr int K1_MCOLS = 32;
 constexpr int K1_MCHUNK = K1_BM * K1_MCOLS * 4;          // 16 KB
 template <bool HILO> struct K1Cfg {
-    static constexpr int STAGES = HILO ? 2 : 3;
+    static constexpr int STAGES = HILO ? 3 : 4;
     static constexpr int STAGE_BYTES = K1_A_BYTES + (HILO ? 2 : 1) * K1_B_BYTES;
     static constexpr int MSLOTS = HILO ? 1 : 2;
     static constexpr int RING = STAGES * STAGE_BYTES;     // offset of the moment slots
@@ -277,11 +277,11 @@ k1_project(const __grid_constant__ K1Params p) {
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 2);    // both CTAs' MMAs consumed the stage
+            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);    // the pair MMA consumed the stage
         }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(ptx::smem_u32(&ctl->accf[b]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 8);
+            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 16);    // both CTAs' epilogue warps
         }
         for (int b = 0; b < MSLOTS; ++b) {
             ptx::mbar_init(ptx::smem_u32(&ctl->wfull[b]), 1);
@@ -292,9 +292,9 @@ k1_project(const __grid_constant__ K1Params p) {
         ctl->abort = 0;
         ptx::fence_barrier_init();
     }
-    if (warp == 1) {
-        ptx::tmem_alloc(ptx::smem_u32(&ctl->tmem_base), 512);
-        ptx::tmem_relinquish();
+    if (warp == 1) {                // collective: one warp of each CTA of the pair
+        ptx::tmem_alloc2(ptx::smem_u32(&ctl->tmem_base), 512);
+        ptx::tmem_relinquish2();
     }
     ptx::tc_fence_before();
     __syncwarp();
@@ -305,8 +305,10 @@ k1_project(const __grid_constant__ K1Params p) {
 
     if (warp == 0) {
         // ------------------------------------------------------ TMA producer
-        // P^T rows of this CTA's rank tile; the V tile (shared by the pair) is
-        // loaded half by each CTA and multicast to both.
+        // P^T rows of this CTA's rank tile and this CTA's half (128 columns)
+        // of the V tile: the pair MMA reads A rows and B columns from both.
+        // Both CTAs' copies complete on the even CTA's full barrier, which
+        // the even CTA arms with the bytes of both.
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
@@ -323,72 +325,76 @@ k1_project(const __grid_constant__ K1Params p) {
                 for (int kb = 0; kb < nk; ++kb) {
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
-                    const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
-                    ptx::mbar_arrive_expect_tx(fb, STAGE_BYTES);
+                    const uint32_t own = ptx::smem_u32(&ctl->full[stage]);
+                    const uint32_t fb = ptx::mapa(own, 0);
+                    if (crank == 0) ptx::mbar_arrive_expect_tx(own, 2 * STAGE_BYTES);
                     const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
                     const uint32_t b = a + K1_A_BYTES;
 #pragma unroll
-                    for (int c = 0; c < 2; ++c) ptx::tma_load_2d(a + c * 8192, pmap, fb, r0 + 64 * c, kb * K1_BK);
+                    for (int c = 0; c < 2; ++c) ptx::tma_load_2d_pair(a + c * 8192, pmap, fb, r0 + 64 * c, kb * K1_BK);
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
                         const int c = 2 * crank + h;
-                        ptx::tma_load_2d_mc(b + c * 8192, vmap, fb, n0 + 64 * c, kb * K1_BK, 0x3);
-                        if (HILO)
-                            ptx::tma_load_2d_mc(b + K1_B_BYTES + c * 8192, lmap, fb, n0 + 64 * c, kb * K1_BK, 0x3);
+                        ptx::tma_load_2d_pair(b + h * 8192, vmap, fb, n0 + 64 * c, kb * K1_BK);
+                        if (HILO) ptx::tma_load_2d_pair(b + K1_B_BYTES + h * 8192, lmap, fb, n0 + 64 * c, kb * K1_BK);
                     }
                     issued |= 1u << stage;
                     last_par = (last_par & ~(1u << stage)) | (phase << stage);
                     if (++stage == STAGES) { stage = 0; phase ^= 1; }
                 }
             }
-            if (!ok) {   // let the copies already in flight land before the CTA exits
+            if (!ok && crank == 0) {   // let the copies already in flight land before the CTA exits
                 for (int s = 0; s < STAGES; ++s)
                     if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idesc = ptx::idesc_bf16(128, K1_BN, 1, 1);
-            int stage = 0;
-            uint32_t phase = 0;
-            int buf = 0;
-            uint32_t acc_phase = 0;
-            bool ok = true;
-            for (int t = t_begin; t < t_end && ok; ++t) {
-                const TcTile tl = p.tiles[t];
-                const TcMod& md = p.mods[tl.mod];
-                const int nk = (md.m + K1_BK - 1) / K1_BK;
-                if (!ptx::mbar_wait(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
-                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
-                ptx::tc_fence_after();
-                const uint32_t d0 = tmem + buf * 256;
-                for (int kb = 0; kb < nk; ++kb) {
-                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
-                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+        if (crank == 0) {
+            // -------------------------------------------- MMA issuer (even CTA)
+            // M = 256 (both CTAs' rank tiles), N = 256, K = 16 per MMA; the
+            // full barrier of a stage counts both CTAs' copies
+            if (lane == 0) {
+                constexpr uint32_t idesc = ptx::idesc_bf16(256, K1_BN, 1, 1);
+                int stage = 0;
+                uint32_t phase = 0;
+                int buf = 0;
+                uint32_t acc_phase = 0;
+                bool ok = true;
+                for (int t = t_begin; t < t_end && ok; ++t) {
+                    const TcTile tl = p.tiles[t];
+                    const TcMod& md = p.mods[tl.mod];
+                    const int nk = (md.m + K1_BK - 1) / K1_BK;
+                    if (!ptx::mbar_wait_cluster(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
+                                                MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
                     ptx::tc_fence_after();
-                    const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
-                    const uint32_t b = a + K1_A_BYTES;
+                    const uint32_t d0 = tmem + buf * 256;
+                    for (int kb = 0; kb < nk; ++kb) {
+                        if (!ptx::mbar_wait_cluster(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
+                                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                        ptx::tc_fence_after();
+                        const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
+                        const uint32_t b = a + K1_A_BYTES;
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk) {
-                        const uint64_t adesc = ptx::smem_desc_sw128(a + kk * 2048, 8192, 1024);
-                        const uint64_t bdesc = ptx::smem_desc_sw128(b + kk * 2048, 8192, 1024);
-                        ptx::mma_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
-                        if (HILO) {   // P^T V_lo: the bf16 rounding residual of V
-                            const uint64_t ldesc = ptx::smem_desc_sw128(b + K1_B_BYTES + kk * 2048, 8192, 1024);
-                            ptx::mma_f16(d0, adesc, ldesc, idesc, 1);
+                        for (int kk = 0; kk < 4; ++kk) {
+                            const uint64_t adesc = ptx::smem_desc_sw128(a + kk * 2048, 8192, 1024);
+                            const uint64_t bdesc = ptx::smem_desc_sw128(b + kk * 2048, 8192, 1024);
+                            ptx::mma2_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
+                            if (HILO) {   // P^T V_lo: the bf16 rounding residual of V
+                                const uint64_t ldesc = ptx::smem_desc_sw128(b + K1_B_BYTES + kk * 2048, 8192, 1024);
+                                ptx::mma2_f16(d0, adesc, ldesc, idesc, 1);
+                            }
                         }
+                        ptx::mma2_commit_mc(ptx::smem_u32(&ctl->empty[stage]), 0x3);
+                        if (++stage == STAGES) { stage = 0; phase ^= 1; }
                     }
-                    ptx::mma_commit_mc(ptx::smem_u32(&ctl->empty[stage]), 0x3);
-                    if (++stage == STAGES) { stage = 0; phase ^= 1; }
+                    if (!ok) break;
+                    ptx::mma2_commit_mc(ptx::smem_u32(&ctl->accf[buf]), 0x3);
+                    if (++buf == 2) { buf = 0; acc_phase ^= 1; }
                 }
-                if (!ok) break;
-                ptx::mma_commit(ptx::smem_u32(&ctl->accf[buf]));
-                if (++buf == 2) { buf = 0; acc_phase ^= 1; }
+                // wait for every MMA this thread issued before TMEM is released
+                ptx::mma2_commit_mc(ptx::smem_u32(&ctl->drain), 0x1);
+                wait_drain(ptx::smem_u32(&ctl->drain), 0);
             }
-            // wait for every MMA this thread issued before TMEM is released
-            ptx::mma_commit(ptx::smem_u32(&ctl->drain));
-            wait_drain(ptx::smem_u32(&ctl->drain), 0);
         }
     } else if (warp == 2) {
         // ------------------------------------- moment chunk loader (TMA in)
@@ -535,7 +541,10 @@ k1_project(const __grid_constant__ K1Params p) {
             if (!ok) break;
             ptx::tc_fence_before();
             __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->acce[buf]));
+            if (lane == 0) {   // the even CTA's issuer waits for both CTAs' epilogues
+                if (crank == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->acce[buf]));
+                else ptx::mbar_arrive_remote(ptx::mapa(ptx::smem_u32(&ctl->acce[buf]), 0));
+            }
             if (++buf == 2) { buf = 0; acc_phase ^= 1; }
         }
     }
@@ -545,7 +554,7 @@ k1_project(const __grid_constant__ K1Params p) {
     ptx::cluster_sync();            // no CTA leaves while its peer may still signal or fill it
     if (warp == 1) {
         ptx::tc_fence_after();
-        ptx::tmem_dealloc(tmem, 512);
+        ptx::tmem_dealloc2(tmem, 512);
     }
 }
 
