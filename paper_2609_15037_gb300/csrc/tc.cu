@@ -106,9 +106,9 @@ struct K1Params {
 };
 
 // ------------------------------------------------------------------- K2
-constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64, K2_STAGES = 3;
+constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64, K2_STAGES = 4;
 constexpr int K2_A_BYTES = K2_BM * K2_BK * 2;           // 16 KB: P rows, K-major
-constexpr int K2_B_BYTES = K2_BK * K2_BN * 2;           // 32 KB: four 64-column chunks of N
+constexpr int K2_B_BYTES = K2_BK * (K2_BN / 2) * 2;     // 16 KB: this CTA's two 64-column chunks of N
 constexpr int K2_STAGE_BYTES = K2_A_BYTES + K2_B_BYTES;
 // W streams through a ring of 128-row x 32-column fp32 chunks (TMA in and out)
 constexpr int K2_WCOLS = 32, K2_WBUF = 4;
@@ -576,11 +576,11 @@ k2_backproject(const __grid_constant__ K2Params p) {
     if (threadIdx.x == 0) {
         for (int s = 0; s < K2_STAGES; ++s) {
             ptx::mbar_init(ptx::smem_u32(&ctl->full[s]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 2);    // both CTAs' MMAs consumed the stage
+            ptx::mbar_init(ptx::smem_u32(&ctl->empty[s]), 1);    // the pair MMA consumed the stage
         }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(ptx::smem_u32(&ctl->accf[b]), 1);
-            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 8);
+            ptx::mbar_init(ptx::smem_u32(&ctl->acce[b]), 16);    // both CTAs' epilogue warps
         }
         for (int b = 0; b < K2_WBUF; ++b) {
             ptx::mbar_init(ptx::smem_u32(&ctl->wfull[b]), 1);
@@ -591,9 +591,9 @@ k2_backproject(const __grid_constant__ K2Params p) {
         ctl->abort = 0;
         ptx::fence_barrier_init();
     }
-    if (warp == 1) {
-        ptx::tmem_alloc(ptx::smem_u32(&ctl->tmem_base), 512);
-        ptx::tmem_relinquish();
+    if (warp == 1) {                // collective: one warp of each CTA of the pair
+        ptx::tmem_alloc2(ptx::smem_u32(&ctl->tmem_base), 512);
+        ptx::tmem_relinquish2();
     }
     ptx::tc_fence_before();
     __syncwarp();
@@ -604,6 +604,8 @@ k2_backproject(const __grid_constant__ K2Params p) {
 
     if (warp == 0) {
         // ------------------------------------------------ operand TMA producer
+        // P rows of this CTA's row tile and this CTA's half (128 columns) of
+        // the N tile; both CTAs' copies complete on the even CTA's barrier.
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
@@ -619,30 +621,32 @@ k2_backproject(const __grid_constant__ K2Params p) {
                 for (int kb = 0; kb < nk; ++kb) {
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
-                    const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
-                    ptx::mbar_arrive_expect_tx(fb, K2_STAGE_BYTES);
+                    const uint32_t own = ptx::smem_u32(&ctl->full[stage]);
+                    const uint32_t fb = ptx::mapa(own, 0);
+                    if (crank == 0) ptx::mbar_arrive_expect_tx(own, 2 * K2_STAGE_BYTES);
                     const uint32_t a = ptx::smem_u32(smem + stage * K2_STAGE_BYTES);
                     const uint32_t b = a + K2_A_BYTES;
-                    ptx::tma_load_2d(a, amap, fb, kb * K2_BK, i0);
+                    ptx::tma_load_2d_pair(a, amap, fb, kb * K2_BK, i0);
 #pragma unroll
-                    for (int h = 0; h < 2; ++h) {   // the N tile is shared by the pair: half each, multicast
+                    for (int h = 0; h < 2; ++h) {
                         const int c = 2 * crank + h;
-                        ptx::tma_load_2d_mc(b + c * 8192, bmap, fb, n0 + 64 * c, kb * K2_BK, 0x3);
+                        ptx::tma_load_2d_pair(b + h * 8192, bmap, fb, n0 + 64 * c, kb * K2_BK);
                     }
                     issued |= 1u << stage;
                     last_par = (last_par & ~(1u << stage)) | (phase << stage);
                     if (++stage == K2_STAGES) { stage = 0; phase ^= 1; }
                 }
             }
-            if (!ok) {
+            if (!ok && crank == 0) {
                 for (int s = 0; s < K2_STAGES; ++s)
                     if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idesc = ptx::idesc_bf16(128, K2_BN, 0, 1);
+        // ------------------------------------------ MMA issuer (even CTA)
+        // M = 256 (both CTAs' row tiles), N = 256, K = 16 per MMA
+        if (crank == 0 && lane == 0) {
+            constexpr uint32_t idesc = ptx::idesc_bf16(256, K2_BN, 0, 1);
             int stage = 0;
             uint32_t phase = 0;
             int buf = 0;
@@ -652,13 +656,13 @@ k2_backproject(const __grid_constant__ K2Params p) {
                 const TcTile tl = p.tiles[t];
                 const TcMod& md = p.mods[tl.mod];
                 const int nk = (md.r + K2_BK - 1) / K2_BK;
-                if (!ptx::mbar_wait(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
-                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                if (!ptx::mbar_wait_cluster(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
+                                            MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
                 ptx::tc_fence_after();
                 const uint32_t d0 = tmem + buf * 256;
                 for (int kb = 0; kb < nk; ++kb) {
-                    if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
-                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
+                    if (!ptx::mbar_wait_cluster(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
+                                                MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
                     ptx::tc_fence_after();
                     const uint32_t a = ptx::smem_u32(smem + stage * K2_STAGE_BYTES);
                     const uint32_t b = a + K2_A_BYTES;
@@ -666,16 +670,16 @@ k2_backproject(const __grid_constant__ K2Params p) {
                     for (int kk = 0; kk < 4; ++kk) {
                         const uint64_t adesc = ptx::smem_desc_sw128(a + kk * 32, 16, 1024);
                         const uint64_t bdesc = ptx::smem_desc_sw128(b + kk * 2048, 8192, 1024);
-                        ptx::mma_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
+                        ptx::mma2_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
                     }
-                    ptx::mma_commit_mc(ptx::smem_u32(&ctl->empty[stage]), 0x3);
+                    ptx::mma2_commit_mc(ptx::smem_u32(&ctl->empty[stage]), 0x3);
                     if (++stage == K2_STAGES) { stage = 0; phase ^= 1; }
                 }
                 if (!ok) break;
-                ptx::mma_commit(ptx::smem_u32(&ctl->accf[buf]));
+                ptx::mma2_commit_mc(ptx::smem_u32(&ctl->accf[buf]), 0x3);
                 if (++buf == 2) { buf = 0; acc_phase ^= 1; }
             }
-            ptx::mma_commit(ptx::smem_u32(&ctl->drain));
+            ptx::mma2_commit_mc(ptx::smem_u32(&ctl->drain), 0x1);
             wait_drain(ptx::smem_u32(&ctl->drain), 0);
         }
     } else if (warp == 2) {
@@ -794,7 +798,10 @@ k2_backproject(const __grid_constant__ K2Params p) {
             if (!ok) break;
             ptx::tc_fence_before();
             __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->acce[buf]));
+            if (lane == 0) {   // the even CTA's issuer waits for both CTAs' epilogues
+                if (crank == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->acce[buf]));
+                else ptx::mbar_arrive_remote(ptx::mapa(ptx::smem_u32(&ctl->acce[buf]), 0));
+            }
             if (++buf == 2) { buf = 0; acc_phase ^= 1; }
         }
     }
@@ -804,7 +811,7 @@ k2_backproject(const __grid_constant__ K2Params p) {
     ptx::cluster_sync();            // no CTA leaves while its peer may still signal or fill it
     if (warp == 1) {
         ptx::tc_fence_after();
-        ptx::tmem_dealloc(tmem, 512);
+        ptx::tmem_dealloc2(tmem, 512);
     }
 }
 
