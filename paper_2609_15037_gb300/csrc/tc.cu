@@ -83,7 +83,7 @@ constexpr int K1_B_BYTES = K1_BK * (K1_BN / 2) * 2;     // 16 KB: this CTA's two
 constexpr int K1_MCOLS = 32;
 constexpr int K1_MCHUNK = K1_BM * K1_MCOLS * 4;          // 16 KB
 template <bool HILO> struct K1Cfg {
-    static constexpr int STAGES = HILO ? 3 : 4;
+    static constexpr int STAGES = HILO ? 3 : 5;
     static constexpr int STAGE_BYTES = K1_A_BYTES + (HILO ? 2 : 1) * K1_B_BYTES;
     static constexpr int MSLOTS = HILO ? 1 : 2;
     static constexpr int RING = STAGES * STAGE_BYTES;     // offset of the moment slots
@@ -106,7 +106,7 @@ struct K1Params {
 };
 
 // ------------------------------------------------------------------- K2
-constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64, K2_STAGES = 4;
+constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64, K2_STAGES = 5;
 constexpr int K2_A_BYTES = K2_BM * K2_BK * 2;           // 16 KB: P rows, K-major
 constexpr int K2_B_BYTES = K2_BK * (K2_BN / 2) * 2;     // 16 KB: this CTA's two 64-column chunks of N
 constexpr int K2_STAGE_BYTES = K2_A_BYTES + K2_B_BYTES;
@@ -115,7 +115,7 @@ constexpr int K2_WCOLS = 32, K2_WBUF = 4;
 constexpr int K2_WBYTES = K2_BM * K2_WCOLS * 4;         // 16 KB
 constexpr int K2_WARPS = 12;                            // 0 TMA, 1 MMA, 2 W loader, 3 W storer, 4-11 epilogue
 constexpr int K2_THREADS = K2_WARPS * 32;
-constexpr int K2_GUARD = 8192;
+constexpr int K2_GUARD = 0;
 constexpr int K2_SMEM = 1024 + K2_STAGES * K2_STAGE_BYTES + K2_WBUF * K2_WBYTES + K2_GUARD + 2048;
 
 struct K2Params {
@@ -129,17 +129,18 @@ struct K2Params {
 };
 
 struct SmemCtl {
-    uint64_t full[4];
-    uint64_t empty[4];   // sized for up to four stages
+    uint64_t full[8];
+    uint64_t empty[8];   // sized for up to eight stages
     uint64_t accf[2];
     uint64_t acce[2];
     uint64_t drain;
-    uint64_t wfull[4];
-    uint64_t wdone[4];
-    uint64_t wempty[4];
+    uint64_t wfull[8];
+    uint64_t wdone[8];
+    uint64_t wempty[8];
     uint32_t tmem_base;
     int abort;
 };
+static_assert(sizeof(SmemCtl) <= 2048, "the barrier block fits the 2 KB each kernel reserves for it");
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
     return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
