@@ -43,6 +43,7 @@ struct TcMod {
     float* W;
     float* exp_avg;
     float* exp_avg_sq;
+    float* mag;       // m x kb block norms (K0 -> magnitude Adam)
     float* mag_avg;
     float* mag_avg_sq;
     uint16_t* Nb;     // r x n bf16 Adam update of the direction branch
@@ -58,6 +59,7 @@ struct K0Item {
     const uint16_t* G;
     uint16_t* Vhi;
     uint16_t* Vlo;
+    float* mag;                        // m x kb block norms M (written when do_mag)
     float* mag_avg;
     float* mag_avg_sq;
     float* dM;
@@ -70,6 +72,7 @@ struct K0Params {
     int do_mag;                        // run Optimizer_M (off when only V is wanted)
     float decomp_eps, beta1, beta2, adam_eps, bc1, bc2;
     long long start[kTcGroup + 1];     // warp items (row, 1024-column segment) per module
+    long long mstart[kTcGroup + 1];    // magnitude entries (m x kb) per module, prefix sums
     K0Item p[kTcGroup];
 };
 
@@ -230,14 +233,8 @@ __global__ void __launch_bounds__(256, 3) k0_decompose(const __grid_constant__ K
             for (int o = 1; o < LPB; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
             const float mag = sqrtf(ss);
             const float sc = 1.0f / (mag + p.decomp_eps);
-            if (p.do_mag && (lane & (LPB - 1)) == 0 && c0 < n) {   // first lane of a block that starts before n
-                const long long o = (long long)crow * it.kb + c0 / BLK;
-                const float ma = p.beta1 * it.mag_avg[o] + (1.0f - p.beta1) * mag;
-                const float mas = p.beta2 * it.mag_avg_sq[o] + (1.0f - p.beta2) * mag * mag;
-                it.mag_avg[o] = ma;
-                it.mag_avg_sq[o] = mas;
-                it.dM[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
-            }
+            if (p.do_mag && (lane & (LPB - 1)) == 0 && c0 < n)   // first lane of a block that starts before n
+                it.mag[(long long)crow * it.kb + c0 / BLK] = mag;
             if (c0 < n) {
                 const long long off = (long long)crow * n + c0;
                 uint32_t vh[4], vl[4];
@@ -252,6 +249,26 @@ __global__ void __launch_bounds__(256, 3) k0_decompose(const __grid_constant__ K
             }
         }
         if (!more) break;
+    }
+}
+
+// Optimizer_M (Algorithm 1) on the block norms K0 wrote: Adam on M, dM out.
+// A separate pass over the m x kb entries keeps these dependent loads out of
+// K0's streaming loop.
+__global__ void __launch_bounds__(256) k0_mag_adam(const __grid_constant__ K0Params p) {
+    const long long total = p.mstart[p.count];
+    int mod = 0;
+    for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+         e += (long long)gridDim.x * blockDim.x) {
+        while (mod + 1 < p.count && p.mstart[mod + 1] <= e) ++mod;
+        const K0Item& it = p.p[mod];
+        const long long o = e - p.mstart[mod];
+        const float mag = it.mag[o];
+        const float ma = p.beta1 * it.mag_avg[o] + (1.0f - p.beta1) * mag;
+        const float mas = p.beta2 * it.mag_avg_sq[o] + (1.0f - p.beta2) * mag * mag;
+        it.mag_avg[o] = ma;
+        it.mag_avg_sq[o] = mas;
+        it.dM[o] = (ma / p.bc1) / (sqrtf(mas / p.bc2) + p.adam_eps);
     }
 }
 
@@ -1316,6 +1333,7 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
     t.m = md.m; t.n = md.n; t.r = md.r; t.kb = md.kb;
     t.Vhi = md.ws_Vhi; t.Vlo = md.ws_Vlo;
     t.W = md.W; t.exp_avg = md.exp_avg; t.exp_avg_sq = md.exp_avg_sq;
+    t.mag = md.ws_inv;     // the block-scale buffer of the fp32 path holds the norms here
     t.mag_avg = md.mag_avg; t.mag_avg_sq = md.mag_avg_sq;
     t.Nb = reinterpret_cast<uint16_t*>(md.ws_N);
     t.dM = md.ws_dM;
@@ -1464,10 +1482,11 @@ static cudaError_t launch_blk(TcState* st, const K1Params& p1, const K2Params& p
     if (decomp) {
         if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, true);
         k0_decompose<BLK><<<st->sms * 3, 256, 0, s>>>(st->p0);
+        k0_mag_adam<<<st->sms * 4, 256, 0, s>>>(st->p0);
         if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, false);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
-        ++*launches;
+        *launches += 2;
     }
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, true);
     if (hilo) k1_project<true><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
@@ -1520,16 +1539,19 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             p0.decomp_eps = hp.decomp_eps;
             p0.beta1 = hp.beta1; p0.beta2 = hp.beta2; p0.adam_eps = hp.adam_eps;
             p0.bc1 = bc1; p0.bc2 = bc2;
-            long long acc = 0;
+            long long acc = 0, macc = 0;
             for (int q = 0; q < cnt; ++q) {
                 const TcMod& md = st->mods[chunk[q]];
                 const int segs = (md.n + K0_SEG - 1) / K0_SEG;
                 p0.start[q] = acc;
-                p0.p[q] = K0Item{static_cast<const uint16_t*>(G[c0 + q]), md.Vhi, md.Vlo, md.mag_avg,
+                p0.mstart[q] = macc;
+                p0.p[q] = K0Item{static_cast<const uint16_t*>(G[c0 + q]), md.Vhi, md.Vlo, md.mag, md.mag_avg,
                                  md.mag_avg_sq, md.dM, md.m, md.n, md.kb, segs};
                 acc += static_cast<long long>(md.m) * segs;
+                macc += static_cast<long long>(md.m) * md.kb;
             }
             p0.start[cnt] = acc;
+            p0.mstart[cnt] = macc;
         } else {
             for (int q = 0; q < cnt; ++q) {
                 const TcMod& md = st->mods[chunk[q]];
@@ -1652,7 +1674,7 @@ int tc_split_v(TcState* st, const TcSplitItem* items, int count, int B, float de
             const TcSplitItem& x = items[c0 + q];
             const int segs = (x.n + K0_SEG - 1) / K0_SEG;
             p0.start[q] = acc;
-            p0.p[q] = K0Item{static_cast<const uint16_t*>(x.G), x.Vhi, x.Vlo, nullptr, nullptr, nullptr,
+            p0.p[q] = K0Item{static_cast<const uint16_t*>(x.G), x.Vhi, x.Vlo, nullptr, nullptr, nullptr, nullptr,
                              x.m, x.n, (x.n + B - 1) / B, segs};
             acc += static_cast<long long>(x.m) * segs;
         }
