@@ -35,15 +35,15 @@ METRIC = "ms per full-model projected-Adam step"
 LR = 1e-3
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one launch of
-# each step kernel, from an ncu capture of one decoder layer of the same
-# shapes (the full model is 32 such layers, and each kernel's traffic grows
-# in proportion to the layers it processes).  Valid only for the kernel source
-# with this SHA-1; after any change the roofline reports traffic = null until
-# the counters are taken again (profiles/ has the capture).
+# each step kernel, from an ncu capture on the one-layer workload named here
+# (profiles/step_kernels_llama7b_layer.md).  A full-model launch processes the
+# same kinds of tiles, so its traffic is scaled by the ratio of the kernel's
+# algorithmic bytes (full model / captured workload).  Valid only for the
+# kernel source with this SHA-1; after any change the roofline reports
+# traffic = null until the counters are taken again.
 TRAFFIC = {"source": "paper_2609_15037_gb300/csrc/tc.cu", "sha1": "77767beb9e49718a8c2ca20a68a7cdc27da47523",
-           "layers": 32,
-           "layer_bytes": {"tc_decompose": 757169152, "tc_project": 1055578624,
-                           "tc_backproject": 1736584960}}
+           "workload": "llama7b_layer",
+           "bytes": {"tc_decompose": 757169152, "tc_project": 1055578624, "tc_backproject": 1736584960}}
 
 
 def _peaks():
@@ -158,14 +158,20 @@ def _kernel_bytes(mods, B, tc):
 
 
 def _traffic(kernel, workload):
-    """Per-launch DRAM bytes of `kernel` at the full-model workload, or None."""
+    """Per-launch DRAM bytes of `kernel` at `workload` (from the captured
+    counters, scaled by algorithmic bytes), or None."""
     import hashlib
-    if workload != WORKLOAD or TRAFFIC["sha1"] is None or kernel not in TRAFFIC["layer_bytes"]:
+    import synth
+    if TRAFFIC["sha1"] is None or kernel not in TRAFFIC["bytes"]:
         return None
     with open(os.path.join(ROOT, TRAFFIC["source"]), "rb") as f:
         if hashlib.sha1(f.read()).hexdigest() != TRAFFIC["sha1"]:
             return None
-    return int(TRAFFIC["layer_bytes"][kernel] * TRAFFIC["layers"])
+    cap = synth.workload(TRAFFIC["workload"])
+    cur = synth.workload(workload)
+    scale = (_kernel_bytes(cur["modules"], cur["block_size"], True)[kernel] /
+             _kernel_bytes(cap["modules"], cap["block_size"], True)[kernel])
+    return int(TRAFFIC["bytes"][kernel] * scale)
 
 
 def run_gpu(args):
