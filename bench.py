@@ -469,7 +469,7 @@ def main():
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--refresh-ws-gb", type=float, default=12.0)
+    ap.add_argument("--refresh-ws-gb", type=float, default=44.0)
     ap.add_argument("--chunk-mb", type=int, default=256,
                     help="gradient chunk of the host-gradient step (e2e)")
     args = ap.parse_args()

@@ -14,7 +14,7 @@ namespace moara {
 
 // Largest number of problems a grouped launch carries in its parameter block
 // (kernel parameters up to 32 KB are allowed on sm_70+ with CUDA >= 12.1).
-constexpr int kMaxGroup = 96;
+constexpr int kMaxGroup = 224;
 
 // Device-side image of one registered module.
 struct ModDev {
