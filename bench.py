@@ -39,9 +39,10 @@ LR = 1e-3
 # (profiles/step_kernels_llama7b_layer.md).  A full-model launch processes the
 # same kinds of tiles, so its traffic is scaled by the ratio of the kernel's
 # algorithmic bytes (full model / captured workload).  Valid only for the
-# kernel source with this SHA-1; after any change the roofline reports
-# traffic = null until the counters are taken again.
-TRAFFIC = {"source": "paper_2609_15037_gb300/csrc/tc.cu", "sha1": "77767beb9e49718a8c2ca20a68a7cdc27da47523",
+# kernel source with this code fingerprint (SHA-1 of the source with `//`
+# comments and blank lines removed); after any code change the roofline
+# reports traffic = null until the counters are taken again.
+TRAFFIC = {"source": "paper_2609_15037_gb300/csrc/tc.cu", "sha1": "7c0ce9207a53ea1e52cb2dd96a1536ce1904d0c8",
            "workload": "llama7b_layer",
            "bytes": {"tc_decompose": 757169152, "tc_project": 1055578624, "tc_backproject": 1736584960}}
 
@@ -157,6 +158,18 @@ def _kernel_bytes(mods, B, tc):
     return kb
 
 
+def _code_sha1(path):
+    """SHA-1 of a C++/CUDA source with `//` comments and blank lines removed."""
+    import hashlib
+    lines = []
+    with open(path, encoding="utf-8") as f:
+        for ln in f:
+            ln = ln.split("//", 1)[0].strip()
+            if ln:
+                lines.append(ln)
+    return hashlib.sha1("\n".join(lines).encode()).hexdigest()
+
+
 def _traffic(kernel, workload):
     """Per-launch DRAM bytes of `kernel` at `workload` (from the captured
     counters, scaled by algorithmic bytes), or None."""
@@ -164,9 +177,8 @@ def _traffic(kernel, workload):
     import synth
     if TRAFFIC["sha1"] is None or kernel not in TRAFFIC["bytes"]:
         return None
-    with open(os.path.join(ROOT, TRAFFIC["source"]), "rb") as f:
-        if hashlib.sha1(f.read()).hexdigest() != TRAFFIC["sha1"]:
-            return None
+    if _code_sha1(os.path.join(ROOT, TRAFFIC["source"])) != TRAFFIC["sha1"]:
+        return None
     cap = synth.workload(TRAFFIC["workload"])
     cur = synth.workload(workload)
     scale = (_kernel_bytes(cur["modules"], cur["block_size"], True)[kernel] /

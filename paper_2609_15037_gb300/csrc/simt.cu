@@ -277,6 +277,50 @@ __global__ void __launch_bounds__(256, 2) k_gemm(const __grid_constant__ GemmBat
         __syncthreads();
     }
 
+    // Plain stores and read-modify-writes move four consecutive columns per
+    // thread as one 16-byte access when the layout allows it.
+    if (EPI == EPI_STORE || EPI == EPI_STORE_NEG || EPI == EPI_SUB) {
+        const bool vec = (p.ldc & 3) == 0 && (reinterpret_cast<uintptr_t>(p.C) & 15) == 0 &&
+                         (EPI != EPI_STORE || p.c_bf16 == nullptr ||
+                          (reinterpret_cast<uintptr_t>(p.c_bf16) & 7) == 0);
+        if (vec) {
+#pragma unroll
+            for (int a = 0; a < 8; ++a) {
+                const int i = m0 + (a < 4 ? ty * 4 + a : 64 + ty * 4 + (a - 4));
+                if (i >= p.M) continue;
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int j = n0 + h * 64 + tx * 4;
+                    if (j + 3 < p.N) {
+                        const long long o = (long long)i * p.ldc + j;
+                        float4 v = make_float4(acc[a][4 * h], acc[a][4 * h + 1], acc[a][4 * h + 2],
+                                               acc[a][4 * h + 3]);
+                        float4* dst = reinterpret_cast<float4*>(p.C + o);
+                        if (EPI == EPI_SUB) {
+                            const float4 c = *dst;
+                            v = make_float4(c.x - v.x, c.y - v.y, c.z - v.z, c.w - v.w);
+                        } else if (EPI == EPI_STORE_NEG) {
+                            v = make_float4(-v.x, -v.y, -v.z, -v.w);
+                        }
+                        *dst = v;
+                        if (EPI == EPI_STORE && p.c_bf16 != nullptr) {
+                            const __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y);
+                            const __nv_bfloat162 hi = __floats2bfloat162_rn(v.z, v.w);
+                            uint2 pk;
+                            pk.x = *reinterpret_cast<const uint32_t*>(&lo);
+                            pk.y = *reinterpret_cast<const uint32_t*>(&hi);
+                            *reinterpret_cast<uint2*>(p.c_bf16 + o) = pk;
+                        }
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 4; ++c)
+                            if (j + c < p.N) epilogue<EPI>(b, p, i, j + c, acc[a][4 * h + c]);
+                    }
+                }
+            }
+            return;
+        }
+    }
 #pragma unroll
     for (int a = 0; a < 8; ++a) {
         const int i = m0 + (a < 4 ? ty * 4 + a : 64 + ty * 4 + (a - 4));

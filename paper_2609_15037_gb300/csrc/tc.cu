@@ -1,21 +1,24 @@
 // Tensor-core path of the optimizer step for bf16 gradients (sm_103a):
 //
 //  K0  Decompose(G, B) of §3.1 / Appendix B.1 as a memory-bound prepass: block
-//      norms in fp32, Optimizer_M (Adam on the block magnitudes), and the
-//      direction matrix V written in bf16 (at the first Adam step also the
-//      residual V - V_hi, so that the projection carries ~16 bits there).
-//  K1  R = P^T V on tcgen05 (128 x 256 tiles, P exact in bf16), then
-//      Optimizer_V (Adam) on R in the epilogue; writes the Adam update N as
-//      bf16.  (Algorithm 1.)
-//  K2  dV = P N, then W <- W - lr*alpha*(Rep_B(dM) (.) dV) in the epilogue,
-//      reading and writing W once through TMA.  (Algorithm 1.)
+//      norms in fp32 and the direction matrix V written in bf16 (at the first
+//      Adam step also the residual V - V_hi, so that the projection carries
+//      ~16 bits there); a second, small pass runs Optimizer_M (Adam on the
+//      block magnitudes).
+//  K1  R = P^T V on tcgen05 (2-SM pairs: 256 ranks x 256 columns per CTA pair,
+//      P exact in bf16), then Optimizer_V (Adam) on R in the epilogue; writes
+//      the Adam update N as bf16.  (Algorithm 1.)
+//  K2  dV = P N (2-SM pairs: 256 rows x 256 columns per CTA pair), then
+//      W <- W - lr*alpha*(Rep_B(dM) (.) dV) in the epilogue, reading and
+//      writing W once through TMA.  (Algorithm 1.)
 //
 // K1 and K2 are persistent and warp specialised: one warp issues TMA tile
-// loads into a shared-memory ring, one thread issues tcgen05.mma into
-// double-buffered TMEM accumulators, and epilogue warps drain TMEM while the
-// next tile's MMAs run.  Every mbarrier wait is bounded; on expiry the kernel
-// records MOARA_ERR_DEVICE_TIMEOUT in the context's status word, drains its
-// own TMA copies and MMAs, frees TMEM and returns.
+// loads into a shared-memory ring, one thread of the even CTA of each pair
+// issues tcgen05.mma (cta_group::2) into double-buffered TMEM accumulators,
+// and epilogue warps drain TMEM while the next tile's MMAs run.  Every
+// mbarrier wait is bounded; on expiry the kernel records
+// MOARA_ERR_DEVICE_TIMEOUT in the context's status word, drains its own TMA
+// copies and MMAs, frees TMEM and returns.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
