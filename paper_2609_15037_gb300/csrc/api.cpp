@@ -276,7 +276,7 @@ struct RefreshRunner {
             const int l = it[i].l;
             p.A = Xin[i]; p.Bm = it[i].Linv; p.C = Xout[i];
             p.M = rows[i]; p.N = l; p.K = l; p.lda = l; p.ldb = l; p.ldc = l;
-            p.k_tri = 1;
+            p.k_tri = moara::KTRI_B_UPPER;
             p.c_bf16 = bf != nullptr ? (*bf)[i] : nullptr;
         });
     }
@@ -370,16 +370,18 @@ struct RefreshRunner {
                         moara::GemmProb& p = b.p[q];
                         p = moara::GemmProb{};
                         p.lda = p.ldb = p.ldc = x.l;
-                        if (pass == 0) {          // T[D, A] = L[D, A] Linv[A, A]
+                        if (pass == 0) {          // T[D, A] = L[D, A] Linv[A, A]  (Linv[A, A] lower)
                             p.A = x.Cg + pr.d0 * l + pr.a0;
                             p.Bm = x.Linv + pr.a0 * l + pr.a0;
                             p.C = x.Tt + pr.d0 * l + pr.a0;
                             p.M = pr.dn; p.N = sz; p.K = sz;
-                        } else {                  // Linv[D, A] = -Linv[D, D] T[D, A]
+                            p.k_tri = moara::KTRI_B_LOWER;
+                        } else {                  // Linv[D, A] = -Linv[D, D] T[D, A]  (Linv[D, D] lower)
                             p.A = x.Linv + pr.d0 * l + pr.d0;
                             p.Bm = x.Tt + pr.d0 * l + pr.a0;
                             p.C = x.Linv + pr.d0 * l + pr.a0;
                             p.M = pr.dn; p.N = sz; p.K = pr.dn;
+                            p.k_tri = moara::KTRI_A_LOWER;
                         }
                     }
                     chk(moara::launch_gemm(pass == 0 ? mul : neg, b, s, &ctx->launches));

@@ -64,6 +64,15 @@ struct DecompBatch {
 // C (M x N) = op(A) (M x K) * op(B) (K x N), fp32 accumulate.
 enum Epi { EPI_STORE = 0, EPI_ADAM = 1, EPI_UPDATE = 2, EPI_STORE_NEG = 3, EPI_SUB = 4 };
 
+// Triangular operands of the SIMT GEMM (zeros stored explicitly): the K loop
+// of an output tile at (m0, n0) covers only the range that can be nonzero.
+enum KTri {
+    KTRI_NONE = 0,
+    KTRI_B_UPPER = 1,     // B[k][j] = 0 for k > j:  k < n0 + tile width
+    KTRI_B_LOWER = 2,     // B[k][j] = 0 for k < j:  k >= n0
+    KTRI_A_LOWER = 3,     // A[i][k] = 0 for k > i:  k < m0 + tile height
+};
+
 struct GemmProb {
     const void* A;
     const void* Bm;
@@ -78,7 +87,7 @@ struct GemmProb {
     int kb;               // blocks per row of the scaled operand / of dM
     int a_bf16, b_bf16;
     int lower_only;       // skip output tiles strictly above the diagonal
-    int k_tri;            // B is lower triangular in (j, k): column tile n0 needs k < n0 + tile width only
+    int k_tri;            // triangular operand: the K range of an output tile shrinks (KTRI_*)
     uint16_t* c_bf16;     // EPI_STORE: also write C rounded to bf16 here (same layout), or null
 };
 

@@ -173,91 +173,123 @@ cudaError_t launch_trace_shift(const SmallBatch& b, cudaStream_t s, int64_t* lau
     return cudaGetLastError();
 }
 
-__global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
-    __shared__ float Ls[kTriBase][kTriBase + 1];
+__global__ void __launch_bounds__(256) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
+    constexpr int NB = kTriBase, NT = 256, RPT = NB * NB / NT;   // 16 rows per thread
+    __shared__ float Lf[NB][NB + 1];   // the factor, one finished column per step
+    __shared__ float Xs[NB][NB + 1];   // the inverse, one finished row per step
+    __shared__ float dg[NB];           // current diagonal of the trailing matrix
     __shared__ int s_fail;
     const int pi = blockIdx.x;
     const int l = b.l[pi];
     if (j0 >= l) return;
-    const int sz = min(kTriBase, l - j0);
+    const int sz = min(NB, l - j0);
     float* A = b.a[pi];
     float* X = b.c[pi];
     const float shift = b.b[pi][0];
-    if (threadIdx.x < 32) {
-        // Warp 0 factors the block in registers: lane holds rows lane and
-        // lane + 32 (rows and columns past sz padded with the identity).  The
-        // loops are fully unrolled, so every register index is a constant;
-        // column j of the factor is broadcast with shuffles.
-        const int lane = threadIdx.x;
-        float r0[kTriBase], r1[kTriBase];
+    const int t = threadIdx.x;
+    // thread t keeps column c, rows i = g + 4s (s < 16), of the block in
+    // registers; rows and columns past sz are padded with the identity
+    const int c = t % NB, g = t / NB;
+    float a[RPT];
 #pragma unroll
-        for (int c = 0; c < kTriBase; ++c) {
-            float v0 = (c == lane) ? 1.0f : 0.0f, v1 = (c == lane + 32) ? 1.0f : 0.0f;
-            if (lane < sz && c < sz) v0 = A[(long long)(j0 + lane) * l + j0 + c] + (c == lane ? shift : 0.0f);
-            if (lane + 32 < sz && c < sz)
-                v1 = A[(long long)(j0 + lane + 32) * l + j0 + c] + (c == lane + 32 ? shift : 0.0f);
-            r0[c] = v0;
-            r1[c] = v1;
+    for (int s = 0; s < RPT; ++s) {
+        const int i = g + 4 * s;
+        float v = (i == c) ? 1.0f : 0.0f;
+        if (i < sz && c < sz) v = A[(long long)(j0 + i) * l + j0 + c] + (i == c ? shift : 0.0f);
+        a[s] = v;
+        if (i == c) dg[c] = v;
+    }
+    if (t == 0) s_fail = 0;
+    __syncthreads();
+    // pivot sqrt(d) and its reciprocal; a pivot that is not positive and
+    // finite is replaced by 1 and marks the failure
+    auto pivot = [&](float d, float& dj, float& inv) {
+        if (!(d > 0.0f) || !isfinite(d)) {
+            d = 1.0f;
+            s_fail = 1;
         }
-        int bad = 0;
+        dj = sqrtf(d);
+        inv = 1.0f / dj;
+    };
+    if (c == 0) {
+        float dj, inv;
+        pivot(dg[0], dj, inv);
 #pragma unroll
-        for (int j = 0; j < kTriBase; ++j) {
-            float d = __shfl_sync(0xffffffffu, j < 32 ? r0[j] : r1[j], j & 31);
-            if (!(d > 0.0f) || !isfinite(d)) { d = 1.0f; bad = 1; }
-            const float dj = sqrtf(d);
-            const float inv = 1.0f / dj;
-            // column j below the diagonal (entries above it are never read)
-            if (j < 32) {
-                r0[j] = (lane == j) ? dj : r0[j] * inv;
-                r1[j] *= inv;
-            } else {
-                r1[j] = (lane + 32 == j) ? dj : r1[j] * inv;
-            }
-#pragma unroll
-            for (int c = j + 1; c < kTriBase; ++c) {
-                const float lcj = __shfl_sync(0xffffffffu, c < 32 ? r0[j] : r1[j], c & 31);
-                if (c < 32) r0[c] = fmaf(-r0[j], lcj, r0[c]);
-                r1[c] = fmaf(-r1[j], lcj, r1[c]);
-            }
-        }
-#pragma unroll
-        for (int c = 0; c < kTriBase; ++c) {
-            Ls[lane][c] = (c <= lane) ? r0[c] : 0.0f;
-            Ls[lane + 32][c] = (c <= lane + 32) ? r1[c] : 0.0f;
-        }
-        if (lane == 0) s_fail = bad;
+        for (int s = 0; s < RPT; ++s) Lf[g + 4 * s][0] = (g + 4 * s == 0) ? dj : a[s] * inv;
     }
     __syncthreads();
-    // inverse of the block factor by forward substitution; thread c keeps
-    // column c of the inverse in registers (loops fully unrolled) and reads
-    // the rows of the factor as shared-memory broadcasts; then both the
-    // factor and the inverse go back to global memory
-    {
-        const int c = threadIdx.x;
-        float xcol[kTriBase];
+    // Right-looking factorisation: step j subtracts column j's outer product
+    // from the trailing lower triangle; the owners of column j + 1 finish it
+    // in the same step (each recomputes its updated pivot from dg).
+    for (int j = 0; j + 1 < NB; ++j) {
+        if (c > j) {
+            // all shared-memory reads of the step first, then the updates
+            float lij[RPT];
 #pragma unroll
-        for (int i = 0; i < kTriBase; ++i) {
-            float acc = (i == c) ? 1.0f : 0.0f;
+            for (int s = 0; s < RPT; ++s) lij[s] = Lf[g + 4 * s][j];
+            const float lcj = Lf[c][j];
+            const bool next = (c == j + 1);
+            float dj = 0.0f, inv = 0.0f;
+            if (next) pivot(fmaf(-lcj, lcj, dg[c]), dj, inv);
 #pragma unroll
-            for (int k = 0; k < i; ++k) acc = fmaf(-Ls[i][k], xcol[k], acc);
-            xcol[i] = (c <= i) ? acc / Ls[i][i] : 0.0f;
-        }
-        if (c < sz) {
+            for (int s = 0; s < RPT; ++s)
+                if (g + 4 * s >= c) a[s] = fmaf(-lij[s], lcj, a[s]);
+            if (next) {
 #pragma unroll
-            for (int i = 0; i < kTriBase; ++i) {
-                if (i < sz) {
-                    A[(long long)(j0 + i) * l + j0 + c] = Ls[i][c];
-                    X[(long long)(j0 + i) * l + j0 + c] = xcol[i];
-                }
+                for (int s = 0; s < RPT; ++s)
+                    if (g + 4 * s >= c) Lf[g + 4 * s][c] = (g + 4 * s == c) ? dj : a[s] * inv;
+            } else {
+#pragma unroll
+                for (int s = 0; s < RPT; ++s)
+                    if (g + 4 * s == c) dg[c] = a[s];
             }
         }
+        __syncthreads();
     }
-    if (threadIdx.x == 0 && s_fail && b.fail[pi] != nullptr) *b.fail[pi] = 1;
+    // Inverse by forward substitution: step k subtracts multiples of the
+    // finished row k from the rows below; row k + 1 is finished (divided by
+    // its pivot) by the same update.  Right of the diagonal the inverse is
+    // zero, on it 1 / L[i][i].
+    for (int e = t; e < NB * NB; e += NT) {
+        const int i = e / NB, cc = e % NB;
+        Xs[i][cc] = (i == cc) ? 1.0f / Lf[i][i] : 0.0f;
+    }
+    float x[RPT];
+#pragma unroll
+    for (int s = 0; s < RPT; ++s) x[s] = 0.0f;
+    __syncthreads();
+    for (int k = 0; k + 1 < NB; ++k) {
+        if (c <= k) {
+            float lik[RPT];
+#pragma unroll
+            for (int s = 0; s < RPT; ++s) lik[s] = Lf[g + 4 * s][k];
+            const float xkc = Xs[k][c];
+            const float piv = Lf[k + 1][k + 1];
+#pragma unroll
+            for (int s = 0; s < RPT; ++s)
+                if (g + 4 * s > k) x[s] = fmaf(-lik[s], xkc, x[s]);
+#pragma unroll
+            for (int s = 0; s < RPT; ++s)
+                if (g + 4 * s == k + 1) {
+                    x[s] = x[s] / piv;
+                    Xs[k + 1][c] = x[s];
+                }
+        }
+        __syncthreads();
+    }
+    for (int e = t; e < NB * NB; e += NT) {
+        const int i = e / NB, cc = e % NB;
+        if (i < sz && cc < sz) {
+            A[(long long)(j0 + i) * l + j0 + cc] = (cc <= i) ? Lf[i][cc] : 0.0f;
+            X[(long long)(j0 + i) * l + j0 + cc] = Xs[i][cc];
+        }
+    }
+    if (t == 0 && s_fail && b.fail[pi] != nullptr) *b.fail[pi] = 1;
 }
 
 cudaError_t launch_chol_diag(const SmallBatch& b, int j0, cudaStream_t s, int64_t* launches) {
     if (b.count <= 0) return cudaSuccess;
-    k_chol_diag<<<b.count, kTriBase, 0, s>>>(b, j0);
+    k_chol_diag<<<b.count, 256, 0, s>>>(b, j0);
     ++*launches;
     return cudaGetLastError();
 }

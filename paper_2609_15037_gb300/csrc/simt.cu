@@ -247,14 +247,19 @@ __global__ void __launch_bounds__(256, 2) k_gemm(const __grid_constant__ GemmBat
         for (int c = 0; c < 8; ++c) acc[a][c] = 0.0f;
 
     TileLoader<ALAY, ASC, ABF, BLAY, BSC, BBF> ld;
-    const int kend = p.k_tri ? min(p.K, n0 + TN) : p.K;
-    const int ktiles = (kend + TK - 1) / TK;
-    ld.load(p, m0, n0, 0, b.B, b.log2B);
-    ld.store(As[0], Bs[0]);
+    int kbeg = 0, kend = p.K;
+    if (p.k_tri == KTRI_B_UPPER) kend = min(p.K, n0 + TN);
+    else if (p.k_tri == KTRI_B_LOWER) kbeg = min(p.K, n0) & ~(TK - 1);
+    else if (p.k_tri == KTRI_A_LOWER) kend = min(p.K, m0 + TM);
+    const int ktiles = kend > kbeg ? (kend - kbeg + TK - 1) / TK : 0;
+    if (ktiles > 0) {
+        ld.load(p, m0, n0, kbeg, b.B, b.log2B);
+        ld.store(As[0], Bs[0]);
+    }
     __syncthreads();
     for (int kt = 0; kt < ktiles; ++kt) {
         const int cur = kt & 1;
-        if (kt + 1 < ktiles) ld.load(p, m0, n0, (kt + 1) * TK, b.B, b.log2B);
+        if (kt + 1 < ktiles) ld.load(p, m0, n0, kbeg + (kt + 1) * TK, b.B, b.log2B);
 #pragma unroll
         for (int k = 0; k < TK; ++k) {
             float av[8], bv[8];
