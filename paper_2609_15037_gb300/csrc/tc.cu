@@ -97,7 +97,8 @@ template <bool HILO> struct K1Cfg {
 };
 constexpr int K1_WARPS = 12;                            // 0 TMA, 1 MMA, 2 moment loader, 3 moment storer, 4-11 epilogue
 constexpr int K1_THREADS = K1_WARPS * 32;
-constexpr int K1_SMEM = 1024 + (K1Cfg<false>::CTL > K1Cfg<true>::CTL ? K1Cfg<false>::CTL : K1Cfg<true>::CTL) + 2048;
+constexpr int kCtlBytes = 512;                         // barrier block of K1 / K2
+constexpr int K1_SMEM = 1024 + (K1Cfg<false>::CTL > K1Cfg<true>::CTL ? K1Cfg<false>::CTL : K1Cfg<true>::CTL) + kCtlBytes;
 
 struct K1Params {
     CUtensorMap gmap[kTcGroup];        // G of each launch slot (decomposition off): {n, m}, box {64, 64}
@@ -122,7 +123,7 @@ constexpr int K2_WBYTES = K2_BM * K2_WCOLS * 4;         // 16 KB
 constexpr int K2_WARPS = 12;                            // 0 TMA, 1 MMA, 2 W loader, 3 W storer, 4-11 epilogue
 constexpr int K2_THREADS = K2_WARPS * 32;
 constexpr int K2_GUARD = 0;
-constexpr int K2_SMEM = 1024 + K2_STAGES * K2_STAGE_BYTES + K2_WBUF * K2_WBYTES + K2_GUARD + 2048;
+constexpr int K2_SMEM = 1024 + K2_STAGES * K2_STAGE_BYTES + K2_WBUF * K2_WBYTES + K2_GUARD + kCtlBytes;
 
 struct K2Params {
     const int* cta_start;
@@ -146,7 +147,11 @@ struct SmemCtl {
     uint32_t tmem_base;
     int abort;
 };
-static_assert(sizeof(SmemCtl) <= 2048, "the barrier block fits the 2 KB each kernel reserves for it");
+static_assert(sizeof(SmemCtl) <= kCtlBytes, "the barrier block fits the space K1 and K2 reserve for it");
+// K1 and K2 leave room beside them for one K0 CTA (no shared memory of its
+// own, 1 KB reserved by the hardware per CTA) out of the SM's 228 KB.
+static_assert(K1_SMEM + 1024 + 1024 <= 228 * 1024 && K2_SMEM + 1024 + 1024 <= 228 * 1024,
+              "a decomposition CTA fits beside a K1 or K2 CTA");
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
     return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
@@ -766,6 +771,7 @@ k2_backproject(const __grid_constant__ K2Params p) {
         const int ch = ew >> 2;
         const int il = q * 32 + lane;                   // row within the tile
         constexpr int NDM = BLK >= 16 ? 1 : 16 / BLK;   // dM values per thread and chunk
+        constexpr bool HOIST = BLK >= 32 && K2_BN % BLK == 0;
         int buf = 0;
         uint32_t acc_phase = 0;
         uint32_t g = 0;
@@ -779,6 +785,16 @@ k2_backproject(const __grid_constant__ K2Params p) {
             const int i = i0 + il;
             const bool row_ok = i < mm;
             const int nc = min(K2_BN / K2_WCOLS, (nn - n0 + K2_WCOLS - 1) / K2_WCOLS);
+            // blocks of B >= 32 columns: the tile's dM values of this row are
+            // loaded once, before the wait for the accumulator
+            float dmt[HOIST ? K2_BN / BLK : 1];
+            if (HOIST) {
+#pragma unroll
+                for (int d = 0; d < K2_BN / BLK; ++d) {
+                    const int jb = n0 / BLK + d;
+                    dmt[d] = (p.decompose && row_ok && jb < mkb) ? dMp[(long long)i * mkb + jb] : 1.0f;
+                }
+            }
             const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
                                             MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
             if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
@@ -788,10 +804,18 @@ k2_backproject(const __grid_constant__ K2Params p) {
                 const uint32_t ph = (g / K2_WBUF) & 1;
                 const int j0 = n0 + c * K2_WCOLS + ch * 16;
                 float dm[NDM];
+                if (HOIST) {
+                    // the chunk's 16 columns lie in one block
+                    const int cb = c * K2_WCOLS + ch * 16;
+                    dm[0] = dmt[0];
 #pragma unroll
-                for (int d = 0; d < NDM; ++d) {
-                    const int jb = (j0 + 8 * d) / BLK;
-                    dm[d] = (p.decompose && row_ok && jb < mkb) ? dMp[(long long)i * mkb + jb] : 1.0f;
+                    for (int d = 1; d < K2_BN / BLK; ++d) dm[0] = (cb >= d * BLK) ? dmt[d] : dm[0];
+                } else {
+#pragma unroll
+                    for (int d = 0; d < NDM; ++d) {
+                        const int jb = (j0 + 8 * d) / BLK;
+                        dm[d] = (p.decompose && row_ok && jb < mkb) ? dMp[(long long)i * mkb + jb] : 1.0f;
+                    }
                 }
                 float v[16];
                 __syncwarp();
@@ -1282,6 +1306,10 @@ struct TcState {
     bool kr_attrs = false;
     KsParams ps;                           // parameter block of the next split-precision GEMM launch
     bool ks_attrs = false;
+    // decomposition of later module parts, overlapped with K1 / K2 of earlier ones
+    cudaStream_t aux = nullptr;
+    cudaEvent_t ev_start = nullptr;
+    cudaEvent_t ev_part[32] = {};
 };
 
 bool tc_supported(int m, int n, int r, int B, int dtype, int decompose) {
@@ -1322,6 +1350,10 @@ void tc_destroy(TcState* st) {
     if (st->d_maps) cudaFree(st->d_maps);
     for (auto& kv : st->tiles)
         if (kv.second.mem) cudaFree(kv.second.mem);
+    if (st->aux) cudaStreamDestroy(st->aux);
+    if (st->ev_start) cudaEventDestroy(st->ev_start);
+    for (cudaEvent_t e : st->ev_part)
+        if (e) cudaEventDestroy(e);
     delete st;
 }
 
@@ -1478,19 +1510,27 @@ static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
     return &(st->tiles[ids] = t);
 }
 
+// K0 and Optimizer_M of one module part.  `background`: a grid of short
+// CTAs (about four row segments per warp) that fills the room K1 / K2 leave
+// on each SM instead of a persistent grid that would hold SMs they need.
 template <int BLK>
-static cudaError_t launch_blk(TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2, bool decomp,
-                              bool hilo, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+static cudaError_t launch_k0(TcState* st, const K0Params& p0, bool background, cudaStream_t s,
+                             int64_t* launches, const TcProfile& prof) {
+    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, true);
+    const long long items = p0.start[p0.count];
+    const int g0 = background ? static_cast<int>(std::max<long long>(1, std::min<long long>((items + 31) / 32, 1 << 30)))
+                              : st->sms * 3;
+    k0_decompose<BLK><<<g0, 256, 0, s>>>(p0);
+    k0_mag_adam<<<background ? st->sms : st->sms * 4, 256, 0, s>>>(p0);
+    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, false);
+    *launches += 2;
+    return cudaGetLastError();
+}
+
+template <int BLK>
+static cudaError_t launch_k12(TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2, bool hilo,
+                              cudaStream_t s, int64_t* launches, const TcProfile& prof) {
     cudaError_t e;
-    if (decomp) {
-        if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, true);
-        k0_decompose<BLK><<<st->sms * 3, 256, 0, s>>>(st->p0);
-        k0_mag_adam<<<st->sms * 4, 256, 0, s>>>(st->p0);
-        if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, false);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-        *launches += 2;
-    }
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, true);
     if (hilo) k1_project<true><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
     else k1_project<false><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
@@ -1506,6 +1546,36 @@ static cudaError_t launch_blk(TcState* st, const K1Params& p1, const K2Params& p
     ++*launches;
     return cudaSuccess;
 }
+
+static cudaError_t launch_k0_any(int B, TcState* st, const K0Params& p0, bool background, cudaStream_t s,
+                                 int64_t* launches, const TcProfile& prof) {
+    switch (B) {
+        case 8: return launch_k0<8>(st, p0, background, s, launches, prof);
+        case 16: return launch_k0<16>(st, p0, background, s, launches, prof);
+        case 32: return launch_k0<32>(st, p0, background, s, launches, prof);
+        case 64: return launch_k0<64>(st, p0, background, s, launches, prof);
+        default: return launch_k0<128>(st, p0, background, s, launches, prof);
+    }
+}
+
+static cudaError_t launch_k12_any(int B, TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2,
+                                  bool hilo, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+    switch (B) {
+        case 8: return launch_k12<8>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        case 16: return launch_k12<16>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        case 32: return launch_k12<32>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        case 64: return launch_k12<64>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        default: return launch_k12<128>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+    }
+}
+
+// Modules per launch group are split into this many parts (consecutive
+// modules, about equal gradient bytes) when the group has at least
+// kOverlapMin modules: the decomposition of part q + 1 runs on an auxiliary
+// stream while K1 / K2 of part q run.
+constexpr int kOverlapParts = 16;
+constexpr int kOverlapMin = 32;
+static_assert(kOverlapParts <= 32, "one event per part");
 
 int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G, float bc1,
             float bc2, float lr, int first_step, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
@@ -1526,68 +1596,108 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
     const bool dec = hp.decompose != 0;
     const bool hilo = dec && first_step;
     const int B = dec ? hp.block_size : 128;
+    auto fail = [&](const char* what) {
+        st->err = what;
+        return MOARA_ERR_CUDA;
+    };
     for (int c0 = 0; c0 < n_mod; c0 += kTcGroup) {
         const int cnt = std::min(kTcGroup, n_mod - c0);
-        std::vector<int> chunk(ids + c0, ids + c0 + cnt);
-        TcState::Tiles* tl = tc_tiles(st, chunk);
-        if (tl == nullptr) { st->err = "tile list allocation failed"; return MOARA_ERR_CUDA; }
-        K1Params& p1 = st->p1;
-        std::memset(&p1, 0, sizeof(p1));
-        if (dec) {
+        // parts of the group (consecutive modules, about equal G bytes)
+        const int nparts = (dec && cnt >= kOverlapMin) ? kOverlapParts : 1;
+        std::vector<int> pstart{0};
+        if (nparts > 1) {
+            double tot = 0.0;
+            for (int q = 0; q < cnt; ++q) tot += (double)st->mods[ids[c0 + q]].m * st->mods[ids[c0 + q]].n;
+            double acc = 0.0;
+            for (int q = 0; q < cnt; ++q) {
+                acc += (double)st->mods[ids[c0 + q]].m * st->mods[ids[c0 + q]].n;
+                if ((int)pstart.size() < nparts && acc >= tot * pstart.size() / nparts && q + 1 < cnt)
+                    pstart.push_back(q + 1);
+            }
+        }
+        pstart.push_back(cnt);
+        const int np = static_cast<int>(pstart.size()) - 1;
+        if (np > 1) {
+            if (st->aux == nullptr) {
+                cudaError_t e = cudaStreamCreateWithFlags(&st->aux, cudaStreamNonBlocking);
+                if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_start, cudaEventDisableTiming);
+                for (int q = 0; q < 32 && e == cudaSuccess; ++q)
+                    e = cudaEventCreateWithFlags(&st->ev_part[q], cudaEventDisableTiming);
+                if (e != cudaSuccess) return fail("auxiliary stream / events");
+            }
+            // the auxiliary stream starts after everything queued on s so far
+            if (cudaEventRecord(st->ev_start, s) != cudaSuccess ||
+                cudaStreamWaitEvent(st->aux, st->ev_start, 0) != cudaSuccess)
+                return fail("auxiliary stream ordering");
+        }
+        auto build_p0 = [&](int a, int b) {
             K0Params& p0 = st->p0;
             std::memset(&p0, 0, sizeof(p0));
-            p0.count = cnt;
+            p0.count = b - a;
             p0.hilo = hilo ? 1 : 0;
             p0.do_mag = 1;
             p0.decomp_eps = hp.decomp_eps;
             p0.beta1 = hp.beta1; p0.beta2 = hp.beta2; p0.adam_eps = hp.adam_eps;
             p0.bc1 = bc1; p0.bc2 = bc2;
             long long acc = 0, macc = 0;
-            for (int q = 0; q < cnt; ++q) {
-                const TcMod& md = st->mods[chunk[q]];
+            for (int q = 0; q < b - a; ++q) {
+                const TcMod& md = st->mods[ids[c0 + a + q]];
                 const int segs = (md.n + K0_SEG - 1) / K0_SEG;
                 p0.start[q] = acc;
                 p0.mstart[q] = macc;
-                p0.p[q] = K0Item{static_cast<const uint16_t*>(G[c0 + q]), md.Vhi, md.Vlo, md.mag, md.mag_avg,
+                p0.p[q] = K0Item{static_cast<const uint16_t*>(G[c0 + a + q]), md.Vhi, md.Vlo, md.mag, md.mag_avg,
                                  md.mag_avg_sq, md.dM, md.m, md.n, md.kb, segs};
                 acc += static_cast<long long>(md.m) * segs;
                 macc += static_cast<long long>(md.m) * md.kb;
             }
-            p0.start[cnt] = acc;
-            p0.mstart[cnt] = macc;
-        } else {
-            for (int q = 0; q < cnt; ++q) {
-                const TcMod& md = st->mods[chunk[q]];
-                if (!encode_bf16_2d(st->encode, &p1.gmap[q], G[c0 + q], md.n, md.m, 64, 64)) {
-                    st->err = "cuTensorMapEncodeTiled failed for a gradient";
-                    return MOARA_ERR_CUDA;
+            p0.start[b - a] = acc;
+            p0.mstart[b - a] = macc;
+            return &p0;
+        };
+        // decomposition: part 0 on s with the full grid; part q + 1 in the
+        // background on the auxiliary stream, launched after K1 / K2 of part q
+        // so that their persistent CTAs are placed first
+        if (dec && launch_k0_any(B, st, *build_p0(pstart[0], pstart[1]), false, s, launches, prof) != cudaSuccess)
+            return fail("decomposition launch failed");
+        for (int q = 0; q < np; ++q) {
+            const int a = pstart[q], b = pstart[q + 1];
+            std::vector<int> chunk(ids + c0 + a, ids + c0 + b);
+            TcState::Tiles* tl = tc_tiles(st, chunk);
+            if (tl == nullptr) { st->err = "tile list allocation failed"; return MOARA_ERR_CUDA; }
+            if (q > 0 && cudaStreamWaitEvent(s, st->ev_part[q], 0) != cudaSuccess) return fail("part wait");
+            K1Params& p1 = st->p1;
+            std::memset(&p1, 0, sizeof(p1));
+            if (!dec) {
+                for (int k = 0; k < b - a; ++k) {
+                    const TcMod& md = st->mods[chunk[k]];
+                    if (!encode_bf16_2d(st->encode, &p1.gmap[k], G[c0 + a + k], md.n, md.m, 64, 64)) {
+                        st->err = "cuTensorMapEncodeTiled failed for a gradient";
+                        return MOARA_ERR_CUDA;
+                    }
                 }
             }
-        }
-        p1.cta_start = tl->k1_start; p1.tiles = tl->k1;
-        p1.mods = st->d_mods; p1.maps = st->d_maps; p1.status = st->d_status;
-        p1.beta1 = hp.beta1; p1.beta2 = hp.beta2; p1.adam_eps = hp.adam_eps;
-        p1.bc1 = bc1; p1.bc2 = bc2;
-        p1.inv_bc1 = 1.0f / bc1; p1.inv_bc2 = 1.0f / bc2;
-        p1.decompose = dec ? 1 : 0;
-        K2Params p2{};
-        p2.cta_start = tl->k2_start; p2.tiles = tl->k2;
-        p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;
-        p2.step_scale = lr * hp.scale;
-        p2.decompose = hp.decompose;
-        const int g1 = tl->g1;
-        const int g2 = tl->g2;
-        cudaError_t e;
-        switch (B) {
-            case 8: e = launch_blk<8>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
-            case 16: e = launch_blk<16>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
-            case 32: e = launch_blk<32>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
-            case 64: e = launch_blk<64>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
-            default: e = launch_blk<128>(st, p1, p2, g1, g2, dec, hilo, s, launches, prof); break;
-        }
-        if (e != cudaSuccess) {
-            st->err = cudaGetErrorString(e);
-            return MOARA_ERR_CUDA;
+            p1.cta_start = tl->k1_start; p1.tiles = tl->k1;
+            p1.mods = st->d_mods; p1.maps = st->d_maps; p1.status = st->d_status;
+            p1.beta1 = hp.beta1; p1.beta2 = hp.beta2; p1.adam_eps = hp.adam_eps;
+            p1.bc1 = bc1; p1.bc2 = bc2;
+            p1.inv_bc1 = 1.0f / bc1; p1.inv_bc2 = 1.0f / bc2;
+            p1.decompose = dec ? 1 : 0;
+            K2Params p2{};
+            p2.cta_start = tl->k2_start; p2.tiles = tl->k2;
+            p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;
+            p2.step_scale = lr * hp.scale;
+            p2.decompose = hp.decompose;
+            const cudaError_t e = launch_k12_any(B, st, p1, p2, tl->g1, tl->g2, hilo, s, launches, prof);
+            if (e != cudaSuccess) {
+                st->err = cudaGetErrorString(e);
+                return MOARA_ERR_CUDA;
+            }
+            if (dec && q + 1 < np) {
+                if (launch_k0_any(B, st, *build_p0(pstart[q + 1], pstart[q + 2]), true, st->aux, launches, prof) !=
+                        cudaSuccess ||
+                    cudaEventRecord(st->ev_part[q + 1], st->aux) != cudaSuccess)
+                    return fail("background decomposition launch failed");
+            }
         }
     }
     return MOARA_OK;

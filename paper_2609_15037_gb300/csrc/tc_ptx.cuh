@@ -173,6 +173,11 @@ __device__ __forceinline__ void bulk_wait_read_all() {
 }
 
 // Waits until all committed bulk groups have fully completed.
+// all but the most recent bulk async-group have finished reading their source
+__device__ __forceinline__ void bulk_wait_read_1() {
+    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+
 __device__ __forceinline__ void bulk_wait_all() {
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
