@@ -253,12 +253,15 @@ int64_t moara_launch_count(const moara_ctx* ctx);
 #define MOARA_PHASE_TC_BACKPROJECT 5 /* tensor-core back-projection kernel           */
 #define MOARA_PHASE_TC_DECOMPOSE  6  /* tensor-core path: block norms, magnitude Adam, V in bf16 */
 #define MOARA_PHASE_TC_REFRESH    7  /* refresh products V^T Q, V Z on tensor cores (inside REFRESH) */
-#define MOARA_NUM_PHASES          8
+#define MOARA_PHASE_TC_DECOMPOSE_OVERLAP 8  /* decomposition of later module parts on the library's
+                                               auxiliary stream, concurrent with K1 / K2 of earlier
+                                               parts (event time on that stream, not additive)      */
+#define MOARA_NUM_PHASES          9
 int moara_profile_enable(moara_ctx* ctx, int enable);
 
 /* Waits for the recorded events, writes the summed milliseconds and launch
  * counts per phase (arrays of MOARA_NUM_PHASES), and clears the record. */
-int moara_profile_read(moara_ctx* ctx, double ms[8], int64_t launches[8]);
+int moara_profile_read(moara_ctx* ctx, double ms[MOARA_NUM_PHASES], int64_t launches[MOARA_NUM_PHASES]);
 
 /* One optimizer step of a single weight that allocates no device memory.
  *

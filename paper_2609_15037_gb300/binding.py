@@ -241,7 +241,7 @@ def moara_step_static_scratch(hp, m, n, r, grad_dtype, G, W, P, exp_avg, exp_avg
 
 
 PHASES = ["decompose", "project", "backproject", "refresh", "tc_project",
-          "tc_backproject", "tc_decompose", "tc_refresh"]
+          "tc_backproject", "tc_decompose", "tc_refresh", "tc_decompose_overlap"]
 
 
 def moara_profile_enable(ctx, enable=True):
@@ -250,10 +250,10 @@ def moara_profile_enable(ctx, enable=True):
 
 def moara_profile_read(ctx):
     """{phase name: (milliseconds, launches)} since the last read."""
-    ms = (ctypes.c_double * 8)()
-    n = (ctypes.c_int64 * 8)()
+    ms = (ctypes.c_double * len(PHASES))()
+    n = (ctypes.c_int64 * len(PHASES))()
     _check(_lib.moara_profile_read(ctx, ms, n), ctx, "moara_profile_read")
-    return {PHASES[i]: (ms[i], n[i]) for i in range(8)}
+    return {PHASES[i]: (ms[i], n[i]) for i in range(len(PHASES))}
 
 
 EXPORTED = [

@@ -1333,7 +1333,7 @@ int moara_profile_enable(moara_ctx* ctx, int enable) {
     return MOARA_OK;
 }
 
-int moara_profile_read(moara_ctx* ctx, double ms[8], int64_t launches[8]) {
+int moara_profile_read(moara_ctx* ctx, double ms[MOARA_NUM_PHASES], int64_t launches[MOARA_NUM_PHASES]) {
     if (ctx == nullptr || ms == nullptr || launches == nullptr) return MOARA_ERR_INVALID_ARG;
     DeviceGuard g(ctx->device);
     for (auto& r : ctx->recs) {

@@ -1516,13 +1516,14 @@ static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
 template <int BLK>
 static cudaError_t launch_k0(TcState* st, const K0Params& p0, bool background, cudaStream_t s,
                              int64_t* launches, const TcProfile& prof) {
-    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, true);
+    const int phase = background ? MOARA_PHASE_TC_DECOMPOSE_OVERLAP : MOARA_PHASE_TC_DECOMPOSE;
+    if (prof.on) prof.mark(prof.ctx, phase, s, true);
     const long long items = p0.start[p0.count];
     const int g0 = background ? static_cast<int>(std::max<long long>(1, std::min<long long>((items + 31) / 32, 1 << 30)))
                               : st->sms * 3;
     k0_decompose<BLK><<<g0, 256, 0, s>>>(p0);
     k0_mag_adam<<<background ? st->sms : st->sms * 4, 256, 0, s>>>(p0);
-    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, false);
+    if (prof.on) prof.mark(prof.ctx, phase, s, false);
     *launches += 2;
     return cudaGetLastError();
 }
