@@ -266,6 +266,22 @@ def run_gpu(args):
     step_ms = elapsed / args.steps
     status = M.moara_get_device_status(g.ctx, cs)
 
+    # alignment diagnostic S(W, t) over every module (a profiling-step call,
+    # outside the step; it reuses the modules' workspaces, which the next
+    # step rewrites): one untimed call, then the mean of three
+    S_dev = torch.empty(len(ids), dtype=torch.float32, device=dev)
+    M.moara_alignment(g.ctx, ids, gptr, S_dev.data_ptr(), cs)
+    a0 = torch.cuda.Event(enable_timing=True)
+    a1 = torch.cuda.Event(enable_timing=True)
+    a0.record(stream)
+    for _ in range(3):
+        M.moara_alignment(g.ctx, ids, gptr, S_dev.data_ptr(), cs)
+    a1.record(stream)
+    torch.cuda.synchronize()
+    align_ms = a0.elapsed_time(a1) / 3
+    S_host = S_dev.cpu().numpy()
+    status |= M.moara_get_device_status(g.ctx, cs)
+
     # end to end through the C ABI with host buffers: every step uploads its
     # gradients from page-locked host memory (moara_step_grouped_host overlaps
     # the chunked upload with the step kernels) and reads the device status
@@ -382,6 +398,10 @@ def run_gpu(args):
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4,
                 "h2d_gbs_link": round(h2d_gbs, 1),
                 "step_ms_median": round(e2e_median, 3), "steps": e2e_steps},
+        "alignment": {"ms": round(align_ms, 3), "modules": len(ids),
+                      "flops": int(4 * sum(md.m * md.n * md.r for md in mods)),
+                      "tflops": round(4 * sum(md.m * md.n * md.r for md in mods) / (align_ms * 1e-3) / 1e12, 1),
+                      "S_mean": round(float(S_host.mean()), 4)},
         "gpu_launches": int(launches),
         "device_status": status | e2e_status,
         "clocks": clk,

@@ -226,6 +226,27 @@ int moara_step_grouped_host(moara_ctx* ctx, int n_mod, const int* ids,
                             const void* const* G_host, int64_t t, float lr,
                             int auto_refresh, size_t chunk_bytes, void* stream);
 
+/* Alignment diagnostic S(W, t) (§3.2, the module-alignment equation; App. C
+ * "Profiling-based rank allocation"): for each module q of the call,
+ *   S_q = cos(G_q, Rep_B(M) (.) (P P^T V)),  (M, V) = Decompose(G_q, B),
+ * with the module's current projector P (its bf16 copy) and the context's
+ * block size B; the cosine is the Frobenius inner product over ||G|| ||.||
+ * (0 when either norm is 0).  The paper averages S over profiling steps and
+ * matrices of a module type (S_tau) to rank the modules; that average is the
+ * caller's.
+ *
+ * G: device pointers to the modules' gradients (bf16, m x n row-major).
+ * S_out: device array of n_mod floats, written stream-ordered.
+ * Scratch: each module's workspace (its contents are rewritten by the next
+ * step anyway) and three doubles per module owned by the context (allocated
+ * on first use or when a call has more modules than before; growing them
+ * waits for `stream`).
+ * Errors: MOARA_ERR_UNSUPPORTED (nothing launched) when a module is not on
+ * the tensor-core path (bf16 gradient, n and r multiples of 8, B in {8, 16,
+ * 32, 64, 128}); the usual argument errors otherwise. */
+int moara_alignment(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, float* S_out,
+                    void* stream);
+
 /* Reads and clears the device status word (0, or a MOARA_ERR_* code a kernel
  * recorded, e.g. MOARA_ERR_DEVICE_TIMEOUT from a bounded wait).  Synchronizes
  * `stream`.  *status receives the code. */

@@ -86,6 +86,7 @@ def _load():
         "moara_refresh_projector": (i32, [vp, i32, P(i32), P(vp), vp]),
         "moara_step_grouped": (i32, [vp, i32, P(i32), P(vp), i64, f32, i32, vp]),
         "moara_step_grouped_host": (i32, [vp, i32, P(i32), P(vp), i64, f32, i32, sz, vp]),
+        "moara_alignment": (i32, [vp, i32, P(i32), P(vp), vp, vp]),
         "moara_get_device_status": (i32, [vp, P(i32), vp]),
         "moara_last_error": (ctypes.c_char_p, [vp]),
         "moara_status_string": (ctypes.c_char_p, [i32]),
@@ -220,6 +221,12 @@ def moara_step_grouped_host(ctx, ids, host_grads, t, lr, auto_refresh=False,
                                         int(chunk_bytes), stream), ctx, "moara_step_grouped_host")
 
 
+def moara_alignment(ctx, ids, grads, S_out, stream=0):
+    """S_out: device address of len(ids) floats."""
+    n, ia, ga = _arrays(ids, grads)
+    _check(_lib.moara_alignment(ctx, n, ia, ga, S_out, stream), ctx, "moara_alignment")
+
+
 def moara_get_device_status(ctx, stream=0):
     st = ctypes.c_int()
     _check(_lib.moara_get_device_status(ctx, ctypes.byref(st), stream), ctx,
@@ -261,7 +268,7 @@ EXPORTED = [
     "moara_state_bytes", "moara_rank_table", "moara_workspace_bytes", "moara_init_module",
     "moara_load_projector", "moara_refresh_workspace_bytes", "moara_set_refresh_workspace",
     "moara_refresh_projector", "moara_step_grouped", "moara_step_grouped_host",
-    "moara_get_device_status",
+    "moara_get_device_status", "moara_alignment",
     "moara_last_error", "moara_status_string", "moara_launch_count",
     "moara_profile_enable", "moara_profile_read", "moara_step_static_scratch",
 ]

@@ -111,6 +111,13 @@ class MoaraGroup:
         ids = self.ids if ids is None else ids
         B.moara_refresh_projector(self.ctx, ids, [g.data_ptr() for g in grads], stream)
 
+    def alignment(self, grads, ids=None, stream=0):
+        """S(W, t) of each module (a float32 tensor on the group's device)."""
+        ids = self.ids if ids is None else ids
+        out = torch.empty(len(ids), dtype=torch.float32, device=self.device)
+        B.moara_alignment(self.ctx, ids, [g.data_ptr() for g in grads], out.data_ptr(), stream)
+        return out
+
     def step(self, grads, t, lr, auto_refresh=False, ids=None, stream=0):
         ids = self.ids if ids is None else ids
         if auto_refresh:

@@ -43,6 +43,9 @@ struct moara_ctx {
     cudaEvent_t open_event = nullptr;
     double prof_ms[MOARA_NUM_PHASES] = {0};
     int64_t prof_n[MOARA_NUM_PHASES] = {0};
+    // alignment diagnostic: three double accumulators per module of a call
+    double* align_acc = nullptr;
+    int align_cap = 0;
 };
 
 namespace {
@@ -962,6 +965,7 @@ void moara_destroy(moara_ctx* ctx) {
     if (ctx->d_mods) cudaFree(ctx->d_mods);
     if (ctx->d_status) cudaFree(ctx->d_status);
     if (ctx->h_status) cudaFreeHost(ctx->h_status);
+    if (ctx->align_acc) cudaFree(ctx->align_acc);
     delete ctx;
 }
 
@@ -1289,6 +1293,39 @@ int moara_step_grouped_host(moara_ctx* ctx, int n_mod, const int* ids, const voi
         e = cudaEventRecord(ctx->compute_done[b], s);
         if (e != cudaSuccess) return cuda_fail(ctx, e, "step event");
     }
+    return MOARA_OK;
+}
+
+int moara_alignment(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, float* S_out,
+                    void* stream) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    int rc = check_ids(ctx, n_mod, ids, G);
+    if (rc != MOARA_OK) return rc;
+    if (n_mod == 0) return MOARA_OK;
+    if (S_out == nullptr) return fail(ctx, MOARA_ERR_INVALID_ARG, "S_out is null");
+    if ((reinterpret_cast<uintptr_t>(S_out) & 3) != 0) return fail(ctx, MOARA_ERR_ALIGN, "S_out is not 4-byte aligned");
+    for (int i = 0; i < n_mod; ++i)
+        if (!use_tc(ctx, ids[i]))
+            return fail(ctx, MOARA_ERR_UNSUPPORTED,
+                        "alignment: module %d is not on the tensor-core path (bf16 gradient, n and r multiples of 8)",
+                        ids[i]);
+    DeviceGuard g(ctx->device);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (ctx->align_cap < n_mod) {
+        if (ctx->align_acc != nullptr) {
+            // an earlier call may still use the old accumulators
+            cudaError_t e = cudaStreamSynchronize(s);
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "alignment accumulator release");
+            cudaFree(ctx->align_acc);
+            ctx->align_acc = nullptr;
+            ctx->align_cap = 0;
+        }
+        cudaError_t e = cudaMalloc(&ctx->align_acc, sizeof(double) * 3 * (size_t)n_mod);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMalloc of the alignment accumulators");
+        ctx->align_cap = n_mod;
+    }
+    rc = moara::tc_alignment(ctx->tc, ctx->hp, n_mod, ids, G, S_out, ctx->align_acc, s, &ctx->launches);
+    if (rc != MOARA_OK) return fail(ctx, rc, "alignment: %s", moara::tc_last_error(ctx->tc));
     return MOARA_OK;
 }
 

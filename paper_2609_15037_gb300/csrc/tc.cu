@@ -51,6 +51,7 @@ struct TcMod {
     float* mag_avg_sq;
     uint16_t* Nb;     // r x n bf16 Adam update of the direction branch
     float* dM;        // m x kb Adam update of the magnitude branch
+    uint16_t* Pb;     // m x r bf16 projector
 };
 
 struct TcTile {
@@ -891,6 +892,14 @@ struct KrParams {
     CUtensorMap bmap[kKrGroup];        // B ({N, K}), box {64, 64}
     float* out[kKrGroup];              // M x N fp32 or null
     uint16_t* out_bf[kKrGroup];        // M x N bf16 or null
+    uint16_t* out_lo[kKrGroup];        // M x N bf16 residual (out - bf16(out)) or null
+    // alignment reduction (ALIGN): element (j, i) of the product, weighted by
+    // the block norm mag[i][j / al_B], is dotted with G[i][j] (i < al_m)
+    const uint16_t* al_G[kKrGroup];
+    const float* al_mag[kKrGroup];
+    double* al_acc[kKrGroup];          // 3 doubles: <G, a>, <a, a>, <G, G>
+    int al_ld[kKrGroup], al_kb[kKrGroup], al_m[kKrGroup];
+    int al_B;
     int M[kKrGroup], N[kKrGroup], K[kKrGroup];
     int ktri[kKrGroup];
     int tiles_n[kKrGroup];
@@ -899,7 +908,7 @@ struct KrParams {
     int* status;
 };
 
-template <bool KMAJOR, bool LO>
+template <bool KMAJOR, bool LO, bool ALIGN = false>
 __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constant__ KrParams p) {
     constexpr int STAGES = KrCfg<LO>::STAGES;
     constexpr int STAGE_BYTES = KrCfg<LO>::STAGE_BYTES;
@@ -1016,9 +1025,51 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
         const int h = ew >> 2;
         const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[0]), 0, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
-        if (__all_sync(0xffffffffu, got) && h < halves) {
+        if (ALIGN && __all_sync(0xffffffffu, got) && h < halves) {
+            // S(W, t) of §3.2: this thread's row j of the product (P P^T V)^T
+            // against column j of G, weighted by Rep_B(M)
             ptx::tc_fence_after();
             const int row = i0 + h * 128 + q * 32 + lane;
+            const uint16_t* const Gp = p.al_G[pi];
+            const float* const mg = p.al_mag[pi];
+            const int ldg = p.al_ld[pi], kbm = p.al_kb[pi], mm = p.al_m[pi];
+            const int jb = row / p.al_B;
+            float dot = 0.0f, na = 0.0f, gg = 0.0f;
+            for (int c = 0; c < nch * 4; ++c) {
+                const int c0 = n0 + c * 16;
+                if (c0 >= mm) break;                      // warp-uniform
+                float v[16];
+                __syncwarp();
+                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + h * 256 + c * 16, v);
+                if (row >= M) continue;
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const int i = c0 + e;
+                    if (i < mm) {
+                        const float g = __bfloat162float(__ushort_as_bfloat16(Gp[(long long)i * ldg + row]));
+                        const float a = mg[(long long)i * kbm + jb] * v[e];
+                        dot = fmaf(g, a, dot);
+                        na = fmaf(a, a, na);
+                        gg = fmaf(g, g, gg);
+                    }
+                }
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                dot += __shfl_xor_sync(0xffffffffu, dot, o);
+                na += __shfl_xor_sync(0xffffffffu, na, o);
+                gg += __shfl_xor_sync(0xffffffffu, gg, o);
+            }
+            if (lane == 0) {
+                double* acc = p.al_acc[pi];
+                atomicAdd(acc + 0, static_cast<double>(dot));
+                atomicAdd(acc + 1, static_cast<double>(na));
+                atomicAdd(acc + 2, static_cast<double>(gg));
+            }
+        } else if (!ALIGN && __all_sync(0xffffffffu, got) && h < halves) {
+            ptx::tc_fence_after();
+            const int row = i0 + h * 128 + q * 32 + lane;
+            uint16_t* const ol = p.out_lo[pi];
             float* const of = p.out[pi];
             uint16_t* const ob = p.out_bf[pi];
             const long long ro = (long long)row * N;
@@ -1043,14 +1094,27 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
                         b4[1] = make_uint4(pack_bf16x2(v[8], v[9]), pack_bf16x2(v[10], v[11]),
                                            pack_bf16x2(v[12], v[13]), pack_bf16x2(v[14], v[15]));
                     }
+                    if (ol != nullptr) {
+                        float rl[16];
+#pragma unroll
+                        for (int e = 0; e < 16; ++e)
+                            rl[e] = v[e] - __bfloat162float(__float2bfloat16_rn(v[e]));
+                        uint4* l4 = reinterpret_cast<uint4*>(ol + ro + j0);
+                        l4[0] = make_uint4(pack_bf16x2(rl[0], rl[1]), pack_bf16x2(rl[2], rl[3]),
+                                           pack_bf16x2(rl[4], rl[5]), pack_bf16x2(rl[6], rl[7]));
+                        l4[1] = make_uint4(pack_bf16x2(rl[8], rl[9]), pack_bf16x2(rl[10], rl[11]),
+                                           pack_bf16x2(rl[12], rl[13]), pack_bf16x2(rl[14], rl[15]));
+                    }
                 } else {
 #pragma unroll
                     for (int e = 0; e < 16; ++e) {
                         if (j0 + e >= N) continue;
                         if (of != nullptr) of[ro + j0 + e] = v[e];
-                        if (ob != nullptr) {
-                            __nv_bfloat16 hb = __float2bfloat16_rn(v[e]);
-                            ob[ro + j0 + e] = *reinterpret_cast<uint16_t*>(&hb);
+                        const __nv_bfloat16 hb = __float2bfloat16_rn(v[e]);
+                        if (ob != nullptr) ob[ro + j0 + e] = *reinterpret_cast<const uint16_t*>(&hb);
+                        if (ol != nullptr) {
+                            const __nv_bfloat16 lb = __float2bfloat16_rn(v[e] - __bfloat162float(hb));
+                            ol[ro + j0 + e] = *reinterpret_cast<const uint16_t*>(&lb);
                         }
                     }
                 }
@@ -1372,6 +1436,7 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
     t.mag_avg = md.mag_avg; t.mag_avg_sq = md.mag_avg_sq;
     t.Nb = reinterpret_cast<uint16_t*>(md.ws_N);
     t.dM = md.ws_dM;
+    t.Pb = md.Pb;
     CUtensorMap* mp = &st->maps[kMaps * id];
     if (!encode_bf16_2d(st->encode, &mp[0], md.Pb, md.r, md.m, 64, 64) ||
         !encode_bf16_2d(st->encode, &mp[1], md.Pb, md.r, md.m, 64, 128) ||
@@ -1706,13 +1771,17 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
 
 const char* tc_last_error(const TcState* st) { return st ? st->err.c_str() : "no tensor-core state"; }
 
-int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, cudaStream_t s,
-                 int64_t* launches) {
+// Grouped KR launches; with align_B > 0 the alignment epilogue (A K-major
+// with two planes only) replaces the stores.
+static int kr_launch(TcState* st, int a_kmajor, const TcGemmItem* items, int count, int align_B,
+                     const uint16_t* const* al_G, const float* const* al_mag, const int* al_ld, const int* al_kb,
+                     const int* al_m, double* const* al_acc, cudaStream_t s, int64_t* launches) {
     if (!st->kr_attrs) {
         cudaFuncSetAttribute(kr_product<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
         cudaFuncSetAttribute(kr_product<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
         cudaFuncSetAttribute(kr_product<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
         cudaFuncSetAttribute(kr_product<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
+        cudaFuncSetAttribute(kr_product<true, true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
         st->kr_attrs = true;
     }
     for (int i = 0; i < count; ++i) {
@@ -1720,6 +1789,10 @@ int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, 
         const int a_inner = a_kmajor ? x.K : x.M;
         if (x.M < 1 || x.N < 1 || x.K < 1 || (a_inner % 8) != 0 || (x.N % 8) != 0) {
             st->err = "tensor-core refresh GEMM: row pitches must be multiples of 16 bytes";
+            return MOARA_ERR_UNSUPPORTED;
+        }
+        if (align_B > 0 && (!a_kmajor || x.A_lo == nullptr)) {
+            st->err = "alignment product: A must be K-major with two planes";
             return MOARA_ERR_UNSUPPORTED;
         }
     }
@@ -1734,7 +1807,8 @@ int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, 
             std::memset(&kp, 0, sizeof(kp));
             int total = 0;
             for (int q = 0; q < cnt; ++q) {
-                const TcGemmItem& x = items[sel[c0 + q]];
+                const int it = sel[c0 + q];
+                const TcGemmItem& x = items[it];
                 const uint64_t a_cols = a_kmajor ? x.K : x.M, a_rows = a_kmajor ? x.M : x.K;
                 bool ok = encode_bf16_2d(st->encode, &kp.amap[q], x.A, a_cols, a_rows, 64, 64);
                 if (with_lo) ok = ok && encode_bf16_2d(st->encode, &kp.lmap[q], x.A_lo, a_cols, a_rows, 64, 64);
@@ -1745,6 +1819,11 @@ int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, 
                 }
                 kp.out[q] = x.out;
                 kp.out_bf[q] = x.out_bf16;
+                kp.out_lo[q] = x.out_lo;
+                if (align_B > 0) {
+                    kp.al_G[q] = al_G[it]; kp.al_mag[q] = al_mag[it]; kp.al_acc[q] = al_acc[it];
+                    kp.al_ld[q] = al_ld[it]; kp.al_kb[q] = al_kb[it]; kp.al_m[q] = al_m[it];
+                }
                 kp.M[q] = x.M; kp.N[q] = x.N; kp.K[q] = x.K;
                 kp.ktri[q] = x.ktri;
                 kp.tiles_n[q] = (x.N + KR_BN - 1) / KR_BN;
@@ -1754,8 +1833,11 @@ int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, 
             kp.tile_start[cnt] = total;
             kp.count = cnt;
             kp.status = st->d_status;
+            kp.al_B = align_B;
             if (total == 0) continue;
-            if (!a_kmajor) {
+            if (align_B > 0) {
+                kr_product<true, true, true><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
+            } else if (!a_kmajor) {
                 if (with_lo) kr_product<false, true><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
                 else kr_product<false, false><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
             } else {
@@ -1769,6 +1851,144 @@ int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, 
             }
             ++*launches;
         }
+    }
+    return MOARA_OK;
+}
+
+int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, cudaStream_t s,
+                 int64_t* launches) {
+    return kr_launch(st, a_kmajor, items, count, 0, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, s,
+                     launches);
+}
+
+// out (cols x ld_out, bf16) = in^T for in (rows x cols, bf16, row pitch
+// cols); columns rows..ld_out-1 of the output are zero.  32 x 32 tiles.
+__global__ void __launch_bounds__(256) k_transpose_pad_bf16(const uint16_t* __restrict__ in, uint16_t* out,
+                                                           int rows, int cols, int ld_out) {
+    __shared__ uint16_t t[32][33];
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    const int tr = (ld_out + 31) / 32, tc = (cols + 31) / 32;
+    for (int tile = blockIdx.x; tile < tr * tc; tile += gridDim.x) {
+        const int bi = tile / tc, bj = tile - bi * tc;      // input rows 32 bi.., columns 32 bj..
+        for (int r = ty; r < 32; r += 8) {
+            const int i = bi * 32 + r, j = bj * 32 + tx;
+            t[r][tx] = (i < rows && j < cols) ? in[(long long)i * cols + j] : static_cast<uint16_t>(0);
+        }
+        __syncthreads();
+        for (int r = ty; r < 32; r += 8) {
+            const int j = bj * 32 + r, i = bi * 32 + tx;    // output row j, column i
+            if (j < cols && i < ld_out) out[(long long)j * ld_out + i] = t[tx][r];
+        }
+        __syncthreads();
+    }
+}
+
+__global__ void k_align_finish(const double* acc, float* S, int n) {
+    const int q = blockIdx.x * blockDim.x + threadIdx.x;
+    if (q >= n) return;
+    const double dot = acc[3 * q], na = acc[3 * q + 1], gg = acc[3 * q + 2];
+    const double den = sqrt(na) * sqrt(gg);
+    S[q] = den > 0.0 ? static_cast<float>(dot / den) : 0.0f;
+}
+
+int tc_alignment(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G,
+                 float* S_out, double* acc, cudaStream_t s, int64_t* launches) {
+    const int B = hp.block_size;
+    if (!(B == 8 || B == 16 || B == 32 || B == 64 || B == 128)) {
+        st->err = "alignment on tensor cores needs a block size in {8, 16, 32, 64, 128}";
+        return MOARA_ERR_UNSUPPORTED;
+    }
+    for (int q = 0; q < n_mod; ++q) {
+        const int id = ids[q];
+        const TcMod* md = (id >= 0 && id < static_cast<int>(st->mods.size())) ? &st->mods[id] : nullptr;
+        if (md == nullptr || md->Vhi == nullptr || md->Vlo == nullptr || md->Pb == nullptr) {
+            st->err = "alignment: module is not on the tensor-core path";
+            return MOARA_ERR_UNSUPPORTED;
+        }
+        const long long mp = (md->m + 7) / 8 * 8;
+        if ((long long)md->r * mp > 2LL * md->m * md->n) {
+            st->err = "alignment: workspace too small for the transposed projector";
+            return MOARA_ERR_UNSUPPORTED;
+        }
+    }
+    int rc = tc_upload(st);
+    if (rc != MOARA_OK) return rc;
+    // 1. block norms M (into the module's norm buffer) and V = V_hi + V_lo
+    for (int c0 = 0; c0 < n_mod; c0 += kTcGroup) {
+        const int cnt = std::min(kTcGroup, n_mod - c0);
+        K0Params& p0 = st->p0;
+        std::memset(&p0, 0, sizeof(p0));
+        p0.count = cnt;
+        p0.hilo = 1;
+        p0.do_mag = 1;                   // writes the norms; Optimizer_M is not launched
+        p0.decomp_eps = hp.decomp_eps;
+        long long acc_items = 0;
+        for (int q = 0; q < cnt; ++q) {
+            const TcMod& md = st->mods[ids[c0 + q]];
+            const int segs = (md.n + K0_SEG - 1) / K0_SEG;
+            p0.start[q] = acc_items;
+            p0.p[q] = K0Item{static_cast<const uint16_t*>(G[c0 + q]), md.Vhi, md.Vlo, md.mag, nullptr, nullptr,
+                             nullptr, md.m, md.n, md.kb, segs};
+            acc_items += static_cast<long long>(md.m) * segs;
+        }
+        p0.start[cnt] = acc_items;
+        switch (B) {
+            case 8: k0_decompose<8><<<st->sms * 3, 256, 0, s>>>(p0); break;
+            case 16: k0_decompose<16><<<st->sms * 3, 256, 0, s>>>(p0); break;
+            case 32: k0_decompose<32><<<st->sms * 3, 256, 0, s>>>(p0); break;
+            case 64: k0_decompose<64><<<st->sms * 3, 256, 0, s>>>(p0); break;
+            default: k0_decompose<128><<<st->sms * 3, 256, 0, s>>>(p0); break;
+        }
+        ++*launches;
+        if (cudaGetLastError() != cudaSuccess) {
+            st->err = "alignment decomposition launch failed";
+            return MOARA_ERR_CUDA;
+        }
+    }
+    // 2. R^T = V^T P (n x r) as two bf16 planes in the module's N buffer
+    std::vector<TcGemmItem> g1(n_mod);
+    for (int q = 0; q < n_mod; ++q) {
+        const TcMod& md = st->mods[ids[q]];
+        g1[q] = TcGemmItem{md.Vhi, md.Vlo, md.Pb, nullptr, md.Nb, md.n, md.r, md.m, 0,
+                           md.Nb + (size_t)md.n * md.r};
+    }
+    rc = kr_launch(st, 0, g1.data(), n_mod, 0, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, s, launches);
+    if (rc != MOARA_OK) return rc;
+    // 3. P^T (r x mp, zero-padded columns) over the V planes, now free
+    for (int q = 0; q < n_mod; ++q) {
+        const TcMod& md = st->mods[ids[q]];
+        const int mp = (md.m + 7) / 8 * 8;
+        const int tiles = ((mp + 31) / 32) * ((md.r + 31) / 32);
+        k_transpose_pad_bf16<<<std::min(tiles, st->sms * 8), 256, 0, s>>>(md.Pb, md.Vhi, md.m, md.r, mp);
+        ++*launches;
+    }
+    if (cudaMemsetAsync(acc, 0, sizeof(double) * 3 * (size_t)n_mod, s) != cudaSuccess) {
+        st->err = "alignment accumulator reset failed";
+        return MOARA_ERR_CUDA;
+    }
+    // 4. (P R)^T = R^T P^T (n x mp), reduced against G in the epilogue
+    std::vector<TcGemmItem> g2(n_mod);
+    std::vector<const uint16_t*> aG(n_mod);
+    std::vector<const float*> aM(n_mod);
+    std::vector<int> ald(n_mod), akb(n_mod), am(n_mod);
+    std::vector<double*> aacc(n_mod);
+    for (int q = 0; q < n_mod; ++q) {
+        const TcMod& md = st->mods[ids[q]];
+        const int mp = (md.m + 7) / 8 * 8;
+        g2[q] = TcGemmItem{md.Nb, md.Nb + (size_t)md.n * md.r, md.Vhi, nullptr, nullptr, md.n, mp, md.r, 0, nullptr};
+        aG[q] = static_cast<const uint16_t*>(G[q]);
+        aM[q] = md.mag;
+        ald[q] = md.n; akb[q] = md.kb; am[q] = md.m;
+        aacc[q] = acc + 3 * q;
+    }
+    rc = kr_launch(st, 1, g2.data(), n_mod, B, aG.data(), aM.data(), ald.data(), akb.data(), am.data(),
+                   aacc.data(), s, launches);
+    if (rc != MOARA_OK) return rc;
+    k_align_finish<<<(n_mod + 127) / 128, 128, 0, s>>>(acc, S_out, n_mod);
+    ++*launches;
+    if (cudaGetLastError() != cudaSuccess) {
+        st->err = "alignment finish launch failed";
+        return MOARA_ERR_CUDA;
     }
     return MOARA_OK;
 }

@@ -33,6 +33,7 @@ struct TcGemmItem {
     uint16_t* out_bf16;    // M x N row-major bf16, or null
     int M, N, K;
     int ktri;              // B upper triangular: column j needs k <= j only
+    uint16_t* out_lo;      // M x N row-major bf16 residual out - bf16(out), or null
 };
 
 // Grouped launch of TcGemmItems (A read K-major when a_kmajor, else
@@ -40,6 +41,13 @@ struct TcGemmItem {
 // plane 16-byte aligned; returns MOARA_ERR_UNSUPPORTED otherwise.
 int tc_gemm_bf16(TcState* st, int a_kmajor, const TcGemmItem* items, int count, cudaStream_t s,
                  int64_t* launches);
+
+// Alignment diagnostic S(W, t) = cos(G, Rep_B(M) (.) (P P^T V)) of §3.2 for
+// modules on the tensor-core path (bf16 G, B in {8, ..., 128}); uses each
+// module's workspace as scratch and writes S for module q to S_out[q]
+// (device).  acc: device scratch of 3 * n_mod doubles.
+int tc_alignment(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G,
+                 float* S_out, double* acc, cudaStream_t s, int64_t* launches);
 
 // One problem of the split-precision GEMM: out (M x N fp32) = A B with A
 // stored K x M and B stored K x N, each as three consecutive bf16 planes

@@ -358,3 +358,48 @@ def test_alignment_full_rank_projection_is_one():
     assert o.alignment(G, np.eye(6), 3) == pytest.approx(1.0, abs=1e-12)
     P = synth.random_orthonormal(6, 2, seed=1)
     assert o.alignment(G, P, 3) < 0.99
+
+def test_alignment_rank_one_closed_form():
+    """§3.2 with one block per row (B = n) and G = u v^T: V = sign(u) v^T/||v||,
+    so with P = u/||u|| the reconstruction is |u_i| u_i (sum|u|) v_j / ||u||^2 and
+    S = sum|u_i|^3 / (||u|| sqrt(sum u_i^4)); with P along sign(u), S = 1."""
+    rng = _rng(31)
+    u, v = rng.standard_normal(7), rng.standard_normal(5)
+    G = np.outer(u, v)
+    S = o.alignment(G, (u / np.linalg.norm(u))[:, None], 5)
+    closed = np.sum(np.abs(u) ** 3) / (np.linalg.norm(u) * np.sqrt(np.sum(u ** 4)))
+    assert S == pytest.approx(closed, rel=1e-12)
+    sg = np.sign(u)
+    assert o.alignment(G, (sg / np.linalg.norm(sg))[:, None], 5) == pytest.approx(1.0, abs=1e-12)
+
+
+def test_alignment_loop_twin_and_invariances():
+    """The alignment against a pure-loop evaluation of its definition (block
+    norms, V, P P^T V, Rep_B, cosine) on a ragged 5 x 7 case with B = 3, and
+    its invariance under column sign flips of P and positive scaling of G."""
+    rng = _rng(32)
+    m, n, r, B = 5, 7, 2, 3
+    G = rng.standard_normal((m, n))
+    P = synth.random_orthonormal(m, r, seed=4)
+    eps = 1e-12
+    kb = -(-n // B)
+    M = [[0.0] * kb for _ in range(m)]
+    V = [[0.0] * n for _ in range(m)]
+    for i in range(m):
+        for b in range(kb):
+            cols = range(b * B, min(n, (b + 1) * B))
+            M[i][b] = sum(G[i][j] ** 2 for j in cols) ** 0.5
+            for j in cols:
+                V[i][j] = G[i][j] / (M[i][b] + eps)
+    R = [[sum(P[i][a] * V[i][j] for i in range(m)) for j in range(n)] for a in range(r)]
+    num = den_g = den_r = 0.0
+    for i in range(m):
+        for j in range(n):
+            rec = M[i][j // B] * sum(P[i][a] * R[a][j] for a in range(r))
+            num += G[i][j] * rec
+            den_g += G[i][j] ** 2
+            den_r += rec ** 2
+    assert o.alignment(G, P, B) == pytest.approx(num / (den_g * den_r) ** 0.5, rel=1e-12)
+    flip = P * np.array([-1.0, 1.0])
+    assert o.alignment(G, flip, B) == pytest.approx(o.alignment(G, P, B), rel=1e-12)
+    assert o.alignment(3.0 * G, P, B) == pytest.approx(o.alignment(G, P, B), rel=1e-9)
