@@ -203,6 +203,7 @@ def run_gpu(args):
     hp = M.moara_default_hparams()
     hp.block_size = B
     hp.adam_eps = wl["adam_eps"]
+    hp.clip_norm = args.clip_norm
     g = M.MoaraGroup(hp, device=local, refresh_workspace_bytes=int(args.refresh_ws_gb * (1 << 30)))
     stream = torch.cuda.current_stream(dev)
     grads = []
@@ -292,14 +293,26 @@ def run_gpu(args):
     hptr = [h.data_ptr() for h in host]
     e2e_steps = max(1, min(args.steps, 10))
     chunk = int(args.chunk_mb) << 20
-    M.moara_step_grouped_host(g.ctx, ids, hptr, step, LR, False, chunk, cs)   # staging allocation
+    # clipping needs every gradient on the device before the first update, so
+    # the clipped step uploads all of them (plain copies) and then steps
+    via_host_call = args.clip_norm <= 0
+
+    def e2e_step(st):
+        if via_host_call:
+            M.moara_step_grouped_host(g.ctx, ids, hptr, st, LR, False, chunk, cs)
+        else:
+            for h, x in zip(host, grads):
+                x.copy_(h, non_blocking=True)
+            M.moara_step_grouped(g.ctx, ids, gptr, st, LR, False, cs)
+
+    e2e_step(step)   # staging allocation
     step += 1
     torch.cuda.synchronize()
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps + 1)]
     evs[0].record(stream)
     e2e_status = 0
     for k in range(e2e_steps):
-        M.moara_step_grouped_host(g.ctx, ids, hptr, step, LR, False, chunk, cs)
+        e2e_step(step)
         step += 1
         e2e_status |= M.moara_get_device_status(g.ctx, cs)
         evs[k + 1].record(stream)
@@ -384,8 +397,10 @@ def run_gpu(args):
         "config": {"workload": args.workload, "modules": len(mods), "block_size": B,
                    "ranks": "q/k 512, v/o/gate/up 1024, down 2048",
                    "l2": "inputs larger than L2 (no flush needed)",
-                   "parallelism": "replicas" if world > 1 else "single GPU"},
+                   "parallelism": "replicas" if world > 1 else "single GPU",
+                   "clip_norm": args.clip_norm},
         "step_ms_no_refresh": round(step_ms, 4),
+        "clip_norm_ms": round(prof["clip_norm"][0] / args.steps, 4) if prof["clip_norm"][1] else None,
         "refresh_ms": round(refresh_ms, 2), "refresh_amortised_ms": round(refresh_ms / 200.0, 4),
         "hbm_gbs_algorithmic": round(alg_bytes / (step_ms * 1e-3) / 1e9, 1),
         "step_roofline": {"alg_bytes": alg_bytes, "alg_flops": alg_flops,
@@ -397,7 +412,8 @@ def run_gpu(args):
         "e2e": {"value": round(e2e_ms + refresh_ms / 200.0, 4), "unit": "ms",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4,
                 "h2d_gbs_link": round(h2d_gbs, 1),
-                "step_ms_median": round(e2e_median, 3), "steps": e2e_steps},
+                "step_ms_median": round(e2e_median, 3), "steps": e2e_steps,
+                "path": "moara_step_grouped_host" if via_host_call else "host-to-device copies + moara_step_grouped"},
         "alignment": {"ms": round(align_ms, 3), "modules": len(ids),
                       "flops": int(4 * sum(md.m * md.n * md.r for md in mods)),
                       "tflops": round(4 * sum(md.m * md.n * md.r for md in mods) / (align_ms * 1e-3) / 1e12, 1),
@@ -515,6 +531,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--refresh-ws-gb", type=float, default=44.0)
+    ap.add_argument("--clip-norm", type=float, default=0.0,
+                    help="global-norm gradient clipping threshold (0: off, as in the workload's definition)")
     ap.add_argument("--chunk-mb", type=int, default=256,
                     help="gradient chunk of the host-gradient step (e2e)")
     args = ap.parse_args()

@@ -92,6 +92,13 @@ typedef struct moara_hparams {
     int   ritz_iters;       /* orthogonal iterations of the Rayleigh-Ritz stage  */
     int   precision;        /* MOARA_PREC_*                                      */
     uint64_t seed;          /* key of the refresh's Gaussian test matrix         */
+    float clip_norm;        /* global-norm gradient clipping threshold (App. D.2:
+                               1.0 for the 7B runs); <= 0 (default): off.  A step
+                               with clipping scales every gradient of the call by
+                               min(1, clip_norm / (||G||_total + 1e-6)), where
+                               ||G||_total^2 sums the squared entries of all the
+                               call's gradients plus the optional extra term of
+                               moara_set_clip_extra (torch.nn.utils.clip_grad_norm_). */
 } moara_hparams;
 
 /* One registered weight.  All pointers are device pointers, 16-byte aligned,
@@ -226,6 +233,34 @@ int moara_step_grouped_host(moara_ctx* ctx, int n_mod, const int* ids,
                             const void* const* G_host, int64_t t, float lr,
                             int auto_refresh, size_t chunk_bytes, void* stream);
 
+/* Global-norm clipping state (hparams.clip_norm > 0; App. D.2).
+ *
+ * moara_set_clip_extra: `extra_sq` is a device float holding the sum of
+ * squared gradient entries of parameters the library does not own (the
+ * embedding, norms, ...); every clipped step reads it stream-ordered, so the
+ * caller writes it on the step's stream before the step.  NULL (the default)
+ * means 0.  The pointer must stay valid while clipped steps run.
+ *
+ * moara_clip_state: `*state` receives the address of a context-owned device
+ * array {total norm, coefficient} written by every clipped step (before any
+ * of the step's updates), for scaling the caller's other gradients with the
+ * same coefficient.  Valid until moara_destroy.
+ *
+ * Clipping needs every gradient of the step on the device before the first
+ * update: moara_step_grouped_host and moara_step_static_scratch return
+ * MOARA_ERR_UNSUPPORTED when clip_norm > 0.  The refresh is unaffected (the
+ * singular subspace of c G and of V is that of G). */
+int moara_set_clip_extra(moara_ctx* ctx, const float* extra_sq);
+int moara_clip_state(moara_ctx* ctx, const float** state);
+
+/* N-D flatten rule of App. B ("Flattening"): a gradient of shape
+ * (s_0, s_1, ..., s_{k-1}) is treated as the m x n matrix with m = s_0 and
+ * n = s_1 * ... * s_{k-1} (the row axis kept, blocks along the flattened
+ * columns); a 1-D shape gives m = s_0, n = 1.  Host only.  Errors:
+ * MOARA_ERR_INVALID_ARG for ndim < 1, a NULL pointer or a non-positive extent,
+ * MOARA_ERR_SHAPE when m or n exceeds INT_MAX. */
+int moara_flatten_shape(int ndim, const int64_t* shape, int* m, int* n);
+
 /* Alignment diagnostic S(W, t) (§3.2, the module-alignment equation; App. C
  * "Profiling-based rank allocation"): for each module q of the call,
  *   S_q = cos(G_q, Rep_B(M) (.) (P P^T V)),  (M, V) = Decompose(G_q, B),
@@ -277,7 +312,8 @@ int64_t moara_launch_count(const moara_ctx* ctx);
 #define MOARA_PHASE_TC_DECOMPOSE_OVERLAP 8  /* decomposition of later module parts on the library's
                                                auxiliary stream, concurrent with K1 / K2 of earlier
                                                parts (event time on that stream, not additive)      */
-#define MOARA_NUM_PHASES          9
+#define MOARA_PHASE_CLIP_NORM     9  /* global gradient norm and clipping coefficient      */
+#define MOARA_NUM_PHASES          10
 int moara_profile_enable(moara_ctx* ctx, int enable);
 
 /* Waits for the recorded events, writes the summed milliseconds and launch

@@ -19,9 +19,13 @@ follow the paper in its order and notation:
 * ``step``           -- one pass of Algorithm 1's training-phase body for one
                         target weight, with the GaLore scale alpha (App. D.2).
 * ``rank_table``     -- Phase 3 of Algorithm 1 (§3.2, App. C final allocation).
+* ``clip_grads``     -- the global-norm gradient clipping of the 7B runs
+                        (App. D.2), in torch.nn.utils.clip_grad_norm_ form.
+* ``flatten_shape``  -- the N-D flatten rule of App. B (row axis kept, the
+                        remaining axes flattened into columns).
 * ``moment_bytes``   -- optimizer-state memory model of Appendix G.
 
-Readings of the paper where it is silent (each is listed in the design doc):
+Readings of the paper where it is silent:
 
 * Step index: Algorithm 1 refreshes when ``s mod T_SVD == 0``; we take
   s = t - 1 with the 1-based Adam step t, so the first step always computes P.
@@ -252,6 +256,37 @@ def run(state: ModuleState, grads, lr: float, hp: Hparams, t0: int = 1,
         refresh = auto_refresh and is_refresh_step(t, hp.refresh_interval)
         state = step(state, G, t, lr, hp, refresh)
     return state
+
+
+# ---------------------------------------------------------------------------
+# Global-norm gradient clipping (App. D.2) and the N-D flatten rule (App. B)
+# ---------------------------------------------------------------------------
+
+def clip_grads(grads, max_norm: float, extra_sq: float = 0.0):
+    """The 7B runs clip gradients at global norm 1.0 (App. D.2); the paper
+    gives no formula, so this is torch.nn.utils.clip_grad_norm_: the total
+    norm over every gradient (plus the squared norm of gradients outside this
+    list), coefficient min(1, max_norm / (norm + 1e-6)), every gradient scaled
+    by it.  Returns (scaled gradients, total norm, coefficient)."""
+    total_sq = float(extra_sq)
+    for G in grads:
+        G = np.asarray(G, dtype=np.float64)
+        total_sq += float(np.sum(G * G))
+    norm = np.sqrt(total_sq)
+    coef = min(1.0, max_norm / (norm + 1e-6))
+    return [coef * np.asarray(G, dtype=np.float64) for G in grads], norm, coef
+
+
+def flatten_shape(shape):
+    """App. B: a gradient of shape (s_0, ..., s_{k-1}) is treated as the
+    matrix with m = s_0 rows and n = s_1 * ... * s_{k-1} columns."""
+    shape = [int(s) for s in shape]
+    if len(shape) < 1 or min(shape) < 1:
+        raise ValueError("shape must have at least one positive extent")
+    n = 1
+    for s in shape[1:]:
+        n *= s
+    return shape[0], n
 
 
 # ---------------------------------------------------------------------------

@@ -48,6 +48,7 @@ class moara_hparams(ctypes.Structure):
         ("oversample", ctypes.c_int), ("power_iters", ctypes.c_int),
         ("ritz_iters", ctypes.c_int), ("precision", ctypes.c_int),
         ("seed", ctypes.c_uint64),
+        ("clip_norm", ctypes.c_float),
     ]
 
 
@@ -87,6 +88,9 @@ def _load():
         "moara_step_grouped": (i32, [vp, i32, P(i32), P(vp), i64, f32, i32, vp]),
         "moara_step_grouped_host": (i32, [vp, i32, P(i32), P(vp), i64, f32, i32, sz, vp]),
         "moara_alignment": (i32, [vp, i32, P(i32), P(vp), vp, vp]),
+        "moara_set_clip_extra": (i32, [vp, vp]),
+        "moara_clip_state": (i32, [vp, P(vp)]),
+        "moara_flatten_shape": (i32, [i32, P(ctypes.c_int64), P(i32), P(i32)]),
         "moara_get_device_status": (i32, [vp, P(i32), vp]),
         "moara_last_error": (ctypes.c_char_p, [vp]),
         "moara_status_string": (ctypes.c_char_p, [i32]),
@@ -227,6 +231,28 @@ def moara_alignment(ctx, ids, grads, S_out, stream=0):
     _check(_lib.moara_alignment(ctx, n, ia, ga, S_out, stream), ctx, "moara_alignment")
 
 
+def moara_set_clip_extra(ctx, extra_sq_ptr):
+    """extra_sq_ptr: device address of a float (sum of squares of other
+    gradients), or 0 for none."""
+    _check(_lib.moara_set_clip_extra(ctx, extra_sq_ptr or None), ctx, "moara_set_clip_extra")
+
+
+def moara_clip_state(ctx):
+    """Device address of the context's {total norm, coefficient} floats."""
+    out = ctypes.c_void_p()
+    _check(_lib.moara_clip_state(ctx, ctypes.byref(out)), ctx, "moara_clip_state")
+    return out.value
+
+
+def moara_flatten_shape(shape):
+    """(m, n) of the N-D flatten rule for a gradient of this shape."""
+    shp = (ctypes.c_int64 * len(shape))(*[int(x) for x in shape])
+    m, n = ctypes.c_int(), ctypes.c_int()
+    _check(_lib.moara_flatten_shape(len(shape), shp, ctypes.byref(m), ctypes.byref(n)),
+           what="moara_flatten_shape")
+    return m.value, n.value
+
+
 def moara_get_device_status(ctx, stream=0):
     st = ctypes.c_int()
     _check(_lib.moara_get_device_status(ctx, ctypes.byref(st), stream), ctx,
@@ -248,7 +274,7 @@ def moara_step_static_scratch(hp, m, n, r, grad_dtype, G, W, P, exp_avg, exp_avg
 
 
 PHASES = ["decompose", "project", "backproject", "refresh", "tc_project",
-          "tc_backproject", "tc_decompose", "tc_refresh", "tc_decompose_overlap"]
+          "tc_backproject", "tc_decompose", "tc_refresh", "tc_decompose_overlap", "clip_norm"]
 
 
 def moara_profile_enable(ctx, enable=True):
@@ -268,7 +294,8 @@ EXPORTED = [
     "moara_state_bytes", "moara_rank_table", "moara_workspace_bytes", "moara_init_module",
     "moara_load_projector", "moara_refresh_workspace_bytes", "moara_set_refresh_workspace",
     "moara_refresh_projector", "moara_step_grouped", "moara_step_grouped_host",
-    "moara_get_device_status", "moara_alignment",
+    "moara_get_device_status", "moara_alignment", "moara_set_clip_extra", "moara_clip_state",
+    "moara_flatten_shape",
     "moara_last_error", "moara_status_string", "moara_launch_count",
     "moara_profile_enable", "moara_profile_read", "moara_step_static_scratch",
 ]

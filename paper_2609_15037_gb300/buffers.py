@@ -70,6 +70,15 @@ class ModuleBuffers:
             self.P_bf16.copy_(sd["P_bf16"])
 
 
+def _device_floats(ptr, n, device):
+    """A float32 tensor over n floats of library-owned device memory (no copy);
+    valid while the owning context lives."""
+    class _Iface:
+        __cuda_array_interface__ = {"shape": (n,), "typestr": "<f4", "data": (ptr, False), "version": 2}
+    with torch.cuda.device(device):
+        return torch.as_tensor(_Iface(), device=f"cuda:{device}")
+
+
 class MoaraGroup:
     """A context plus the modules registered in it."""
 
@@ -83,6 +92,8 @@ class MoaraGroup:
         self.ids = []
         self._refresh_ws = None
         self._refresh_ws_request = refresh_workspace_bytes
+        self._clip_extra = None
+        self._clip_view = _device_floats(B.moara_clip_state(self.ctx), 2, self.device)
 
     def add(self, m, n, r, grad_dtype="bf16", W0=None):
         buf = ModuleBuffers(m, n, r, self.hp.block_size, grad_dtype,
@@ -110,6 +121,16 @@ class MoaraGroup:
         self.ensure_refresh_workspace()
         ids = self.ids if ids is None else ids
         B.moara_refresh_projector(self.ctx, ids, [g.data_ptr() for g in grads], stream)
+
+    def clip_state(self):
+        """{total norm, coefficient} of the last clipped step (a 2-float tensor
+        view of the context's device array)."""
+        return self._clip_view
+
+    def set_clip_extra(self, extra_sq):
+        """extra_sq: a one-element float32 device tensor (kept alive here), or None."""
+        self._clip_extra = extra_sq
+        B.moara_set_clip_extra(self.ctx, 0 if extra_sq is None else extra_sq.data_ptr())
 
     def alignment(self, grads, ids=None, stream=0):
         """S(W, t) of each module (a float32 tensor on the group's device)."""

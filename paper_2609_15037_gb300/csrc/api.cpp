@@ -2,6 +2,7 @@
 // module table, the memory model and rank table helpers, and the sequencing of
 // the step and refresh kernels.  Declarations and contracts are in moara.h.
 #include <algorithm>
+#include <climits>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -46,6 +47,12 @@ struct moara_ctx {
     // alignment diagnostic: three double accumulators per module of a call
     double* align_acc = nullptr;
     int align_cap = 0;
+    // global-norm clipping: {total norm, coefficient}, per-CTA partial sums,
+    // the caller's extra sum of squares
+    float* d_clip = nullptr;
+    double* d_clip_part = nullptr;
+    int clip_part_cap = 0;
+    const float* clip_extra = nullptr;
 };
 
 namespace {
@@ -104,6 +111,7 @@ int check_hparams(moara_ctx* ctx, const moara_hparams* hp) {
     if (hp->precision != MOARA_PREC_AUTO && hp->precision != MOARA_PREC_FP32 &&
         hp->precision != MOARA_PREC_BF16_TC)
         return fail(ctx, MOARA_ERR_INVALID_ARG, "unknown precision");
+    if (!std::isfinite(hp->clip_norm)) return fail(ctx, MOARA_ERR_INVALID_ARG, "clip_norm must be finite");
     return MOARA_OK;
 }
 
@@ -800,7 +808,7 @@ int do_refresh(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, 
 
 // ------------------------------------------------------------------ step
 int do_step_simt(moara_ctx* ctx, const std::vector<int>& sel, const int* ids, const void* const* G,
-                 int64_t t, float lr, cudaStream_t s) {
+                 int64_t t, float lr, const float* clip, cudaStream_t s) {
     const moara_hparams& hp = ctx->hp;
     const double bc1 = 1.0 - std::pow((double)hp.beta1, (double)t);
     const double bc2 = 1.0 - std::pow((double)hp.beta2, (double)t);
@@ -816,6 +824,7 @@ int do_step_simt(moara_ctx* ctx, const std::vector<int>& sel, const int* ids, co
             db.count = cnt; db.B = hp.block_size; db.do_mag = 1; db.decomp_eps = hp.decomp_eps;
             db.beta1 = hp.beta1; db.beta2 = hp.beta2; db.adam_eps = hp.adam_eps;
             db.bc1 = static_cast<float>(bc1); db.bc2 = static_cast<float>(bc2);
+            db.clip = clip;
             long long acc = 0;
             for (int q = 0; q < cnt; ++q) {
                 const int i = order[c0 + q];
@@ -838,6 +847,7 @@ int do_step_simt(moara_ctx* ctx, const std::vector<int>& sel, const int* ids, co
             moara::GemmBatch b{};
             b.B = hp.block_size; b.beta1 = hp.beta1; b.beta2 = hp.beta2; b.adam_eps = hp.adam_eps;
             b.bc1 = static_cast<float>(bc1); b.bc2 = static_cast<float>(bc2);
+            b.clip = hp.decompose ? nullptr : clip;   // with the decomposition V is unchanged
             for (int q = 0; q < cnt; ++q) {
                 const int i = order[c0 + q];
                 const moara::ModDev& md = ctx->moddev[ids[i]];
@@ -940,7 +950,9 @@ int moara_create(moara_ctx** out, const moara_hparams* hp, int device) {
     if (cudaMalloc(&ctx->d_mods, sizeof(moara::ModDev) * ctx->cap) != cudaSuccess ||
         cudaMalloc(&ctx->d_status, sizeof(int) * 4) != cudaSuccess ||
         cudaMallocHost(&ctx->h_status, sizeof(int) * 4) != cudaSuccess ||
-        cudaMemset(ctx->d_status, 0, sizeof(int) * 4) != cudaSuccess) {
+        cudaMemset(ctx->d_status, 0, sizeof(int) * 4) != cudaSuccess ||
+        cudaMalloc(&ctx->d_clip, sizeof(float) * 2) != cudaSuccess ||
+        cudaMemset(ctx->d_clip, 0, sizeof(float) * 2) != cudaSuccess) {
         moara_destroy(ctx);
         return MOARA_ERR_CUDA;
     }
@@ -966,6 +978,8 @@ void moara_destroy(moara_ctx* ctx) {
     if (ctx->d_status) cudaFree(ctx->d_status);
     if (ctx->h_status) cudaFreeHost(ctx->h_status);
     if (ctx->align_acc) cudaFree(ctx->align_acc);
+    if (ctx->d_clip) cudaFree(ctx->d_clip);
+    if (ctx->d_clip_part) cudaFree(ctx->d_clip_part);
     delete ctx;
 }
 
@@ -1160,6 +1174,46 @@ int step_impl(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, i
         rc = do_refresh(ctx, n_mod, ids, G, s);
         if (rc != MOARA_OK) return rc;
     }
+    // global-norm clipping (App. D.2): the coefficient of this step's
+    // gradients, before any update
+    const float* clip = nullptr;
+    if (ctx->hp.clip_norm > 0.0f) {
+        ProfScope ps(ctx, MOARA_PHASE_CLIP_NORM, s);
+        const int nb = (n_mod + moara::kMaxGroup - 1) / moara::kMaxGroup;
+        if (ctx->clip_part_cap < nb) {
+            if (ctx->d_clip_part != nullptr) {
+                cudaError_t e = cudaStreamSynchronize(s);   // an earlier step may still use them
+                if (e != cudaSuccess) return cuda_fail(ctx, e, "clipping partial sums release");
+                cudaFree(ctx->d_clip_part);
+                ctx->d_clip_part = nullptr;
+                ctx->clip_part_cap = 0;
+            }
+            cudaError_t e = cudaMalloc(&ctx->d_clip_part, sizeof(double) * moara::kNormParts * (size_t)nb);
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMalloc of the clipping partial sums");
+            ctx->clip_part_cap = nb;
+        }
+        for (int c0 = 0, bi = 0; c0 < n_mod; c0 += moara::kMaxGroup, ++bi) {
+            moara::GradNormBatch nbt{};
+            nbt.count = std::min(moara::kMaxGroup, n_mod - c0);
+            long long acc = 0;
+            for (int q = 0; q < nbt.count; ++q) {
+                const moara_module_desc& d = ctx->mods[ids[c0 + q]];
+                nbt.chunk_start[q] = acc;
+                nbt.G[q] = G[c0 + q];
+                nbt.elems[q] = (long long)d.m * d.n;
+                nbt.dtype[q] = d.grad_dtype;
+                acc += (nbt.elems[q] + moara::kNormChunk - 1) / moara::kNormChunk;
+            }
+            nbt.chunk_start[nbt.count] = acc;
+            cudaError_t e = moara::launch_grad_sq(nbt, ctx->d_clip_part + (size_t)bi * moara::kNormParts, s,
+                                                  &ctx->launches);
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "gradient norm launch");
+        }
+        cudaError_t e = moara::launch_clip_finish(ctx->d_clip_part, nb * moara::kNormParts, ctx->clip_extra,
+                                                  ctx->hp.clip_norm, ctx->d_clip, s, &ctx->launches);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "clipping coefficient launch");
+        clip = ctx->d_clip + 1;
+    }
     std::vector<int> simt, tcm;
     for (int i = 0; i < n_mod; ++i) (use_tc(ctx, ids[i]) ? tcm : simt).push_back(i);
     if (!tcm.empty()) {
@@ -1180,12 +1234,12 @@ int step_impl(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, i
             }
         }, ctx};
         rc = moara::tc_step(ctx->tc, ctx->hp, static_cast<int>(mids.size()), mids.data(), gp.data(),
-                            static_cast<float>(bc1), static_cast<float>(bc2), lr, t == 1 ? 1 : 0, s,
+                            static_cast<float>(bc1), static_cast<float>(bc2), lr, t == 1 ? 1 : 0, clip, s,
                             &ctx->launches, tp);
         if (rc != MOARA_OK) return fail(ctx, rc, "tensor-core step launch failed: %s", moara::tc_last_error(ctx->tc));
     }
     if (!simt.empty()) {
-        rc = do_step_simt(ctx, simt, ids, G, t, lr, s);
+        rc = do_step_simt(ctx, simt, ids, G, t, lr, clip, s);
         if (rc != MOARA_OK) return rc;
     }
     return MOARA_OK;
@@ -1245,6 +1299,9 @@ int moara_step_grouped_host(moara_ctx* ctx, int n_mod, const int* ids, const voi
     if (t < 1) return fail(ctx, MOARA_ERR_INVALID_ARG, "step t must be >= 1 (got %lld)", (long long)t);
     if (!std::isfinite(lr)) return fail(ctx, MOARA_ERR_INVALID_ARG, "lr must be finite");
     if (chunk_bytes == 0) return fail(ctx, MOARA_ERR_INVALID_ARG, "chunk_bytes must be > 0");
+    if (ctx->hp.clip_norm > 0.0f)
+        return fail(ctx, MOARA_ERR_UNSUPPORTED,
+                    "global-norm clipping needs all of the step's gradients on the device: use moara_step_grouped");
     if (n_mod == 0) return MOARA_OK;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     DeviceGuard g(ctx->device);
@@ -1293,6 +1350,35 @@ int moara_step_grouped_host(moara_ctx* ctx, int n_mod, const int* ids, const voi
         e = cudaEventRecord(ctx->compute_done[b], s);
         if (e != cudaSuccess) return cuda_fail(ctx, e, "step event");
     }
+    return MOARA_OK;
+}
+
+int moara_set_clip_extra(moara_ctx* ctx, const float* extra_sq) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(extra_sq) & 3) != 0)
+        return fail(ctx, MOARA_ERR_ALIGN, "extra_sq is not 4-byte aligned");
+    ctx->clip_extra = extra_sq;
+    return MOARA_OK;
+}
+
+int moara_clip_state(moara_ctx* ctx, const float** state) {
+    if (ctx == nullptr || state == nullptr) return MOARA_ERR_INVALID_ARG;
+    *state = ctx->d_clip;
+    return MOARA_OK;
+}
+
+int moara_flatten_shape(int ndim, const int64_t* shape, int* m, int* n) {
+    if (ndim < 1 || shape == nullptr || m == nullptr || n == nullptr) return MOARA_ERR_INVALID_ARG;
+    for (int i = 0; i < ndim; ++i)
+        if (shape[i] < 1) return MOARA_ERR_INVALID_ARG;
+    if (shape[0] > INT_MAX) return MOARA_ERR_SHAPE;
+    int64_t cols = 1;
+    for (int i = 1; i < ndim; ++i) {
+        if (cols > INT_MAX / shape[i]) return MOARA_ERR_SHAPE;
+        cols *= shape[i];
+    }
+    *m = static_cast<int>(shape[0]);
+    *n = static_cast<int>(cols);
     return MOARA_OK;
 }
 

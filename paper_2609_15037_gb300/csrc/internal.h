@@ -56,6 +56,7 @@ struct DecompBatch {
     int B;
     int do_mag;
     float decomp_eps, beta1, beta2, adam_eps, bc1, bc2;
+    const float* clip;    // gradient clipping coefficient (device), applied to M before Optimizer_M, or null
     long long item_start[kMaxGroup + 1];
     DecompItem p[kMaxGroup];
 };
@@ -97,6 +98,7 @@ struct GemmBatch {
     int log2B;                    // log2(B) when B is a power of two, else -1 (set at launch)
     float beta1, beta2, adam_eps, bc1, bc2;
     float step_scale;             // lr * alpha (EPI_UPDATE)
+    const float* clip;            // EPI_ADAM: clipping coefficient (device) applied to R, or null
     int tiles_n[kMaxGroup];
     int tile_start[kMaxGroup + 1];
     GemmProb p[kMaxGroup];
@@ -120,6 +122,26 @@ int gemm_tile_n();
 
 cudaError_t launch_f32_to_bf16(const float* src, float* dst_f32, uint16_t* dst_bf16,
                                long long count, cudaStream_t s, int64_t* launches);
+
+// ------------------------------------------------------- gradient clipping
+// Sum of squared gradient entries over a group of gradients, in chunks of
+// kNormChunk elements; chunk c goes to CTA c % kNormParts of the launch, so
+// the partial sums (one double per CTA) and their total are reproducible.
+constexpr int kNormChunk = 16384;
+constexpr int kNormParts = 1216;
+
+struct GradNormBatch {
+    int count;
+    long long chunk_start[kMaxGroup + 1];
+    const void* G[kMaxGroup];
+    long long elems[kMaxGroup];
+    int dtype[kMaxGroup];
+};
+
+cudaError_t launch_grad_sq(const GradNormBatch& b, double* partials, cudaStream_t s, int64_t* launches);
+// state[0] = sqrt(sum of partials[0..n) + *extra), state[1] = min(1, max_norm / (state[0] + 1e-6))
+cudaError_t launch_clip_finish(const double* partials, int n, const float* extra, float max_norm, float* state,
+                               cudaStream_t s, int64_t* launches);
 
 // ------------------------------------------------------------- refresh
 struct RefreshItem {

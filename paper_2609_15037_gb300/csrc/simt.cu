@@ -42,6 +42,8 @@ __device__ __forceinline__ void finish_item(const DecompBatch& b, const DecompIt
     float mag = sqrtf(ss);
     it.inv[local] = 1.0f / (mag + b.decomp_eps);
     if (b.do_mag) {
+        // a clipped gradient c G has block norms c M and the same direction V
+        if (b.clip != nullptr) mag *= *b.clip;
         float ma = b.beta1 * it.mag_avg[local] + (1.0f - b.beta1) * mag;
         float mas = b.beta2 * it.mag_avg_sq[local] + (1.0f - b.beta2) * mag * mag;
         it.mag_avg[local] = ma;
@@ -206,7 +208,9 @@ __device__ __forceinline__ void epilogue(const GemmBatch& b, const GemmProb& p, 
     } else if (EPI == EPI_SUB) {
         p.C[o] = p.C[o] - acc;
     } else if (EPI == EPI_ADAM) {
-        // Optimizer_V (Algorithm 1): Adam on the projected direction R = acc.
+        // Optimizer_V (Algorithm 1): Adam on the projected direction R = acc
+        // (of the clipped gradient when a clipping coefficient is given).
+        if (b.clip != nullptr) acc *= *b.clip;
         float ea = b.beta1 * p.aux0[o] + (1.0f - b.beta1) * acc;
         float eas = b.beta2 * p.aux1[o] + (1.0f - b.beta2) * acc * acc;
         p.aux0[o] = ea;
@@ -392,6 +396,117 @@ cudaError_t launch_gemm(const GemmKind& k, GemmBatch& b, cudaStream_t s, int64_t
     MOARA_GEMM_CASE(A_KCONTIG, false, false, B_KCONTIG, false, false, EPI_SUB)
 #undef MOARA_GEMM_CASE
     return cudaErrorInvalidValue;
+}
+
+// ---------------------------------------------------------------------------
+// Global gradient norm for clipping: sum of squares per chunk in fp32 (at
+// most kNormChunk / 256 terms per thread), chunk sums added in fp64; fixed
+// chunk-to-CTA assignment and reduction order.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ double block_sum_d(double v, double* red) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __syncthreads();
+    if (lane == 0) red[w] = v;
+    __syncthreads();
+    double t = 0.0;
+    if (threadIdx.x == 0)
+        for (int i = 0; i < (int)(blockDim.x >> 5); ++i) t += red[i];
+    return t;
+}
+
+__global__ void __launch_bounds__(256) k_grad_sq(const __grid_constant__ GradNormBatch b, double* partials) {
+    __shared__ double red[8];
+    // a chunk is kNormChunk elements: 8 x 16 bytes per thread for bf16, 16 for
+    // fp32; all of a thread's loads of a chunk are issued before the sums
+    constexpr int VB = kNormChunk / (8 * 256);          // uint4 per thread, bf16
+    constexpr int VF = kNormChunk / (4 * 256);          // float4 per thread, fp32
+    static_assert(VB * 8 * 256 == kNormChunk && VF * 4 * 256 == kNormChunk, "chunk = whole vectors per thread");
+    const long long total = b.chunk_start[b.count];
+    double acc = 0.0;
+    for (long long c = blockIdx.x; c < total; c += gridDim.x) {
+        int lo = 0, hi = b.count - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (b.chunk_start[mid] <= c) lo = mid; else hi = mid - 1;
+        }
+        const long long e0 = (c - b.chunk_start[lo]) * kNormChunk;
+        const long long e1 = min(e0 + (long long)kNormChunk, b.elems[lo]);
+        float ss = 0.0f;
+        if (b.dtype[lo] == MOARA_DTYPE_BF16) {
+            const uint16_t* g = static_cast<const uint16_t*>(b.G[lo]);
+            if (e1 - e0 == kNormChunk) {
+                uint4 w[VB];
+#pragma unroll
+                for (int k = 0; k < VB; ++k)
+                    w[k] = __ldcs(reinterpret_cast<const uint4*>(g + e0 + 8LL * (threadIdx.x + 256 * k)));
+#pragma unroll
+                for (int k = 0; k < VB; ++k) {
+                    const uint32_t ww[4] = {w[k].x, w[k].y, w[k].z, w[k].w};
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const float x = __uint_as_float(ww[q] << 16), y = __uint_as_float(ww[q] & 0xFFFF0000u);
+                        ss = fmaf(x, x, ss);
+                        ss = fmaf(y, y, ss);
+                    }
+                }
+            } else {
+                for (long long k = e0 + threadIdx.x; k < e1; k += blockDim.x) {
+                    const float x = bf16_bits_to_f32(g[k]);
+                    ss = fmaf(x, x, ss);
+                }
+            }
+        } else {
+            const float* g = static_cast<const float*>(b.G[lo]);
+            if (e1 - e0 == kNormChunk) {
+                float4 w[VF];
+#pragma unroll
+                for (int k = 0; k < VF; ++k)
+                    w[k] = __ldcs(reinterpret_cast<const float4*>(g + e0 + 4LL * (threadIdx.x + 256 * k)));
+#pragma unroll
+                for (int k = 0; k < VF; ++k) {
+                    ss = fmaf(w[k].x, w[k].x, ss);
+                    ss = fmaf(w[k].y, w[k].y, ss);
+                    ss = fmaf(w[k].z, w[k].z, ss);
+                    ss = fmaf(w[k].w, w[k].w, ss);
+                }
+            } else {
+                for (long long k = e0 + threadIdx.x; k < e1; k += blockDim.x) ss = fmaf(g[k], g[k], ss);
+            }
+        }
+        acc += static_cast<double>(ss);
+    }
+    const double t = block_sum_d(acc, red);
+    if (threadIdx.x == 0) partials[blockIdx.x] = t;
+}
+
+cudaError_t launch_grad_sq(const GradNormBatch& b, double* partials, cudaStream_t s, int64_t* launches) {
+    k_grad_sq<<<kNormParts, 256, 0, s>>>(b, partials);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+__global__ void __launch_bounds__(256) k_clip_finish(const double* partials, int n, const float* extra,
+                                                     float max_norm, float* state) {
+    __shared__ double red[8];
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) acc += partials[i];
+    double t = block_sum_d(acc, red);
+    if (threadIdx.x == 0) {
+        if (extra != nullptr) t += static_cast<double>(*extra);
+        const double norm = sqrt(t);
+        const double coef = static_cast<double>(max_norm) / (norm + 1e-6);
+        state[0] = static_cast<float>(norm);
+        state[1] = static_cast<float>(coef < 1.0 ? coef : 1.0);
+    }
+}
+
+cudaError_t launch_clip_finish(const double* partials, int n, const float* extra, float max_norm, float* state,
+                               cudaStream_t s, int64_t* launches) {
+    k_clip_finish<<<1, 256, 0, s>>>(partials, n, extra, max_norm, state);
+    ++*launches;
+    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------

@@ -75,6 +75,7 @@ struct K0Params {
     int hilo;                          // also write V_lo = V - V_hi
     int do_mag;                        // run Optimizer_M (off when only V is wanted)
     float decomp_eps, beta1, beta2, adam_eps, bc1, bc2;
+    const float* clip;                 // gradient clipping coefficient (device) for M, or null
     long long start[kTcGroup + 1];     // warp items (row, 1024-column segment) per module
     long long mstart[kTcGroup + 1];    // magnitude entries (m x kb) per module, prefix sums
     K0Item p[kTcGroup];
@@ -111,6 +112,7 @@ struct K1Params {
     float beta1, beta2, adam_eps, bc1, bc2;
     float inv_bc1, inv_bc2;            // 1 / bias corrections
     int decompose;
+    const float* clip;                 // decomposition off: clipping coefficient (device) for R, or null
 };
 
 // ------------------------------------------------------------------- K2
@@ -266,13 +268,15 @@ __global__ void __launch_bounds__(256, 3) k0_decompose(const __grid_constant__ K
 // K0's streaming loop.
 __global__ void __launch_bounds__(256) k0_mag_adam(const __grid_constant__ K0Params p) {
     const long long total = p.mstart[p.count];
+    // a clipped gradient c G has block norms c M and the same direction V
+    const float cf = p.clip != nullptr ? *p.clip : 1.0f;
     int mod = 0;
     for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
          e += (long long)gridDim.x * blockDim.x) {
         while (mod + 1 < p.count && p.mstart[mod + 1] <= e) ++mod;
         const K0Item& it = p.p[mod];
         const long long o = e - p.mstart[mod];
-        const float mag = it.mag[o];
+        const float mag = it.mag[o] * cf;
         const float ma = p.beta1 * it.mag_avg[o] + (1.0f - p.beta1) * mag;
         const float mas = p.beta2 * it.mag_avg_sq[o] + (1.0f - p.beta2) * mag * mag;
         it.mag_avg[o] = ma;
@@ -492,6 +496,8 @@ k1_project(const __grid_constant__ K1Params p) {
         const int q = warp & 3;
         const int ch = ew >> 2;
         const int il = q * 32 + lane;                  // rank row within the tile
+        // R of a clipped gradient (decomposition off; with it V is unchanged)
+        const float cf = p.clip != nullptr ? *p.clip : 1.0f;
         int buf = 0;
         uint32_t acc_phase = 0;
         uint32_t g = 0;
@@ -533,7 +539,7 @@ k1_project(const __grid_constant__ K1Params p) {
                     float es[4] = {sv.x, sv.y, sv.z, sv.w};
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        const float rv = v[4 * u + e];
+                        const float rv = v[4 * u + e] * cf;
                         ea[e] = p.beta1 * ea[e] + (1.0f - p.beta1) * rv;
                         es[e] = p.beta2 * es[e] + (1.0f - p.beta2) * rv * rv;
                         // N goes to K2 in bf16: approximate sqrt / reciprocal
@@ -1644,7 +1650,8 @@ constexpr int kOverlapMin = 32;
 static_assert(kOverlapParts <= 32, "one event per part");
 
 int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G, float bc1,
-            float bc2, float lr, int first_step, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+            float bc2, float lr, int first_step, const float* clip, cudaStream_t s, int64_t* launches,
+            const TcProfile& prof) {
     if (!st->attrs_set) {
         cudaFuncSetAttribute(k1_project<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
         cudaFuncSetAttribute(k1_project<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
@@ -1705,6 +1712,7 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             p0.decomp_eps = hp.decomp_eps;
             p0.beta1 = hp.beta1; p0.beta2 = hp.beta2; p0.adam_eps = hp.adam_eps;
             p0.bc1 = bc1; p0.bc2 = bc2;
+            p0.clip = clip;
             long long acc = 0, macc = 0;
             for (int q = 0; q < b - a; ++q) {
                 const TcMod& md = st->mods[ids[c0 + a + q]];
@@ -1748,6 +1756,7 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             p1.bc1 = bc1; p1.bc2 = bc2;
             p1.inv_bc1 = 1.0f / bc1; p1.inv_bc2 = 1.0f / bc2;
             p1.decompose = dec ? 1 : 0;
+            p1.clip = dec ? nullptr : clip;
             K2Params p2{};
             p2.cta_start = tl->k2_start; p2.tiles = tl->k2;
             p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;

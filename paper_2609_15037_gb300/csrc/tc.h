@@ -20,8 +20,9 @@ struct TcProfile {
 TcState* tc_create(int device, int* d_status);
 void tc_destroy(TcState* st);
 int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp);
+// clip: device clipping coefficient of this step's gradients, or null
 int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G,
-            float bc1, float bc2, float lr, int first_step, cudaStream_t s, int64_t* launches,
+            float bc1, float bc2, float lr, int first_step, const float* clip, cudaStream_t s, int64_t* launches,
             const TcProfile& prof);
 // One problem of the refresh GEMM on tensor cores: out = op(A) B, bf16
 // operands, fp32 accumulation.

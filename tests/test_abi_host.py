@@ -43,6 +43,28 @@ def test_default_hparams_follow_paper(M):
     assert hp.adam_eps == pytest.approx(1e-6) and hp.decomp_eps == pytest.approx(1e-12)
     assert hp.scale == pytest.approx(0.25) and hp.refresh_interval == 200
     assert hp.decompose == 1 and hp.refresh_src == M.MOARA_REFRESH_SRC_V
+    assert hp.clip_norm == 0.0           # clipping off unless asked for (App. D.2: 7B runs only)
+
+
+def test_hparams_struct_matches_header(M):
+    """The binding's struct has the C layout: the library's defaults land in
+    the right fields, including the last one."""
+    hp = M.moara_default_hparams()
+    assert hp.block_size == 128 and hp.power_iters == 2 and hp.oversample == 16
+    assert ctypes.sizeof(M.binding.moara_hparams) == 72
+
+
+def test_flatten_shape_through_the_abi(M):
+    """App. B flatten rule via moara_flatten_shape, against the oracle's."""
+    from oracle import moara_ref as o
+    for shape in [(8, 3, 3, 3), (4096, 11008), (5,), (2, 3, 4, 5, 6)]:
+        assert M.moara_flatten_shape(shape) == o.flatten_shape(shape)
+    with pytest.raises(M.MoaraError) as ei:
+        M.moara_flatten_shape((3, 0))
+    assert ei.value.code == M.MOARA_ERR_INVALID_ARG
+    with pytest.raises(M.MoaraError) as ei:
+        M.moara_flatten_shape((2, 1 << 20, 1 << 12))
+    assert ei.value.code == M.MOARA_ERR_SHAPE
 
 
 def _golden(name):

@@ -403,3 +403,46 @@ def test_alignment_loop_twin_and_invariances():
     flip = P * np.array([-1.0, 1.0])
     assert o.alignment(G, flip, B) == pytest.approx(o.alignment(G, P, B), rel=1e-12)
     assert o.alignment(3.0 * G, P, B) == pytest.approx(o.alignment(G, P, B), rel=1e-9)
+
+
+def test_clip_closed_forms():
+    """App. D.2 clipping: constant gradients with sum of squares 6*9 + 4*4 = 70;
+    below the threshold nothing changes; the extra term of other parameters
+    enters the norm (70 + 30 = 100, norm 10)."""
+    g1, g2 = np.full((2, 3), 3.0), np.full((4, 1), -2.0)
+    out, norm, coef = o.clip_grads([g1, g2], 1.0)
+    assert norm == pytest.approx(np.sqrt(70.0), rel=1e-15)
+    assert coef == pytest.approx(1.0 / (np.sqrt(70.0) + 1e-6), rel=1e-15)
+    assert out[0][0, 0] == pytest.approx(3.0 * coef, rel=1e-15)
+    assert out[1][3, 0] == pytest.approx(-2.0 * coef, rel=1e-15)
+    clipped = np.sqrt(sum(float(np.sum(x * x)) for x in out))
+    assert clipped == pytest.approx(np.sqrt(70.0) / (np.sqrt(70.0) + 1e-6), rel=1e-14)
+    out, norm, coef = o.clip_grads([g1, g2], 100.0)
+    assert coef == 1.0 and np.array_equal(out[0], g1) and np.array_equal(out[1], g2)
+    _, norm, coef = o.clip_grads([g1, g2], 1.0, extra_sq=30.0)
+    assert norm == pytest.approx(10.0, rel=1e-15)
+    assert coef == pytest.approx(1.0 / (10.0 + 1e-6), rel=1e-15)
+
+
+def test_clip_scales_magnitude_not_direction():
+    """§3.1: Decompose(c G) = (c M, V) for c > 0 up to the eps of the block
+    normalisation, so clipping reaches only the magnitude branch when the
+    decomposition is on."""
+    G = _rng(41).standard_normal((6, 10))
+    M, V = o.decompose(G, 4)
+    Mc, Vc = o.decompose(0.3 * G, 4)
+    np.testing.assert_allclose(Mc, 0.3 * M, rtol=1e-14)
+    np.testing.assert_allclose(Vc, V, rtol=1e-10)
+
+
+def test_flatten_rule():
+    """App. B flatten: the row axis is kept and the others are flattened."""
+    assert o.flatten_shape((8, 3, 3, 3)) == (8, 27)
+    assert o.flatten_shape((4096, 11008)) == (4096, 11008)
+    assert o.flatten_shape((5,)) == (5, 1)
+    G = np.arange(2 * 3 * 4, dtype=np.float64).reshape(2, 3, 4)
+    m, n = o.flatten_shape(G.shape)
+    flat = G.reshape(m, n)
+    assert flat[1, 5] == G[1, 1, 1]
+    with pytest.raises(ValueError):
+        o.flatten_shape((3, 0))
