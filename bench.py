@@ -42,9 +42,9 @@ LR = 1e-3
 # kernel source with this code fingerprint (SHA-1 of the source with `//`
 # comments and blank lines removed); after any code change the roofline
 # reports traffic = null until the counters are taken again.
-TRAFFIC = {"source": "paper_2609_15037_gb300/csrc/tc.cu", "sha1": "18c2a29411f1d5b4cfa96e1397f9dc5b7c25e7cd",
+TRAFFIC = {"source": "paper_2609_15037_gb300/csrc/tc.cu", "sha1": "3ee31f04f09f450a3f6f52e63885510ce3074df4",
            "workload": "llama7b_layer",
-           "bytes": {"tc_decompose": 756564992, "tc_project": 1059769344, "tc_backproject": 1739735296}}
+           "bytes": {"tc_decompose": 756953344, "tc_project": 1059397120, "tc_backproject": 1741026304}}
 
 
 def _peaks():
