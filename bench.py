@@ -115,8 +115,9 @@ class Clocks:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
-def _algorithmic(mods, B):
-    """Algorithmic bytes and flops of one step over `mods` (Module list)."""
+def _algorithmic(mods, B, sb=4):
+    """Algorithmic bytes and flops of one step over `mods` (Module list);
+    sb: bytes per element of W and the direction moments (4 or 2)."""
     tot_b = tot_f = 0
     per = {"project": [0, 0], "backproject": [0, 0]}
     for md in mods:
@@ -124,14 +125,14 @@ def _algorithmic(mods, B):
         k = -(-n // B)
         # minimum traffic of one fused pass: G read (bf16), W read+write,
         # direction moments read+write, P read once (bf16), magnitude moments
-        tot_b += 2 * m * n + 8 * m * n + 16 * r * n + 2 * m * r + 16 * m * k
+        tot_b += 2 * m * n + 2 * sb * m * n + 4 * sb * r * n + 2 * m * r + 16 * m * k
         tot_f += 4 * m * r * n
         per["project"][1] += 2 * m * r * n
         per["backproject"][1] += 2 * m * r * n
     return tot_b, tot_f, per
 
 
-def _kernel_bytes(mods, B, tc):
+def _kernel_bytes(mods, B, tc, sb=4):
     """Algorithmic bytes per step of each step kernel as built.
 
     tensor-core path: tc_decompose reads G (bf16), writes V (bf16) and updates
@@ -147,8 +148,8 @@ def _kernel_bytes(mods, B, tc):
         k = -(-n // B)
         if tc:
             add = {"tc_decompose": 2 * m * n + 2 * m * n + 20 * m * k,
-                   "tc_project": 2 * m * n + 2 * m * r + 16 * r * n + 2 * r * n,
-                   "tc_backproject": 8 * m * n + 2 * r * n + 2 * m * r + 4 * m * k}
+                   "tc_project": 2 * m * n + 2 * m * r + 4 * sb * r * n + 2 * r * n,
+                   "tc_backproject": 2 * sb * m * n + 2 * r * n + 2 * m * r + 4 * m * k}
         else:
             add = {"decompose": 2 * m * n + 20 * m * k + 4 * m * k,
                    "project": 2 * m * n + 4 * m * k + 4 * m * r + 16 * r * n + 4 * r * n,
@@ -204,6 +205,8 @@ def run_gpu(args):
     hp.block_size = B
     hp.adam_eps = wl["adam_eps"]
     hp.clip_norm = args.clip_norm
+    hp.state_dtype = M.MOARA_DTYPE_BF16 if args.state_dtype == "bf16" else M.MOARA_DTYPE_F32
+    sbytes = 2 if args.state_dtype == "bf16" else 4
     g = M.MoaraGroup(hp, device=local, refresh_workspace_bytes=int(args.refresh_ws_gb * (1 << 30)))
     stream = torch.cuda.current_stream(dev)
     grads = []
@@ -333,13 +336,13 @@ def run_gpu(args):
     h2d_gbs = h2d / (c0.elapsed_time(c1) * 1e-3) / 1e9
 
     hbm, bf16_peak, bf16_sus, peak_src = _peaks()
-    alg_bytes, alg_flops, _ = _algorithmic(mods, B)
+    alg_bytes, alg_flops, _ = _algorithmic(mods, B, sbytes)
     total_ms = step_ms + refresh_ms / 200.0
     roof_ms = max(alg_bytes / (hbm * 1e9), alg_flops / (bf16_sus * 1e12)) * 1e3
 
     # dominant kernel
     used_tc = prof["tc_project"][1] > 0
-    kbytes = _kernel_bytes(mods, B, used_tc)
+    kbytes = _kernel_bytes(mods, B, used_tc, sbytes)
     names = ["decompose", "project", "backproject", "tc_decompose", "tc_project", "tc_backproject"]
     dom = max(names, key=lambda k: prof[k][0])
     dom_ms = prof[dom][0] / max(prof[dom][1], 1)
@@ -354,7 +357,7 @@ def run_gpu(args):
                 "kernel": dom, "peak_source": "152 SMs x 128 FP32 lanes x 2 x 2.07 GHz"}
     elif dom == "tc_project":
         achieved = flops_dom / (dom_ms * 1e-3) / 1e12
-        tr = _traffic(dom, args.workload)
+        tr = _traffic(dom, args.workload) if sbytes == 4 else None   # counters taken with fp32 states
         roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": bf16_sus,
                 "unit": "TFLOP/s", "frac": round(achieved / bf16_sus, 4),
                 "traffic": None if tr is None else int(tr / n_launch_per_step),
@@ -362,7 +365,7 @@ def run_gpu(args):
     else:
         by = kbytes[dom] / n_launch_per_step
         achieved = by / (dom_ms * 1e-3) / 1e9
-        tr = _traffic(dom, args.workload)
+        tr = _traffic(dom, args.workload) if sbytes == 4 else None   # counters taken with fp32 states
         roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
                 "frac": round(achieved / hbm, 4), "traffic": None if tr is None else int(tr / n_launch_per_step),
                 "kernel": dom, "peak_source": f"hbm_gbs ({peak_src})"}
@@ -392,13 +395,15 @@ def run_gpu(args):
         "metric": METRIC, "value": round(total_ms / world, 4), "unit": "ms",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(total_ms, 4), "higher_is_better": False, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16 G, fp32 W/states" if used_tc else "fp32 (bf16 G)",
+        "vs_baseline": None,
+        "dtype": ("bf16 G, bf16 W/direction states, fp32 magnitude states" if sbytes == 2 else
+                  "bf16 G, fp32 W/states") if used_tc else "fp32 (bf16 G)",
         "data": "synthetic",
         "config": {"workload": args.workload, "modules": len(mods), "block_size": B,
                    "ranks": "q/k 512, v/o/gate/up 1024, down 2048",
                    "l2": "inputs larger than L2 (no flush needed)",
                    "parallelism": "replicas" if world > 1 else "single GPU",
-                   "clip_norm": args.clip_norm},
+                   "clip_norm": args.clip_norm, "state_dtype": args.state_dtype},
         "step_ms_no_refresh": round(step_ms, 4),
         "clip_norm_ms": round(prof["clip_norm"][0] / args.steps, 4) if prof["clip_norm"][1] else None,
         "refresh_ms": round(refresh_ms, 2), "refresh_amortised_ms": round(refresh_ms / 200.0, 4),
@@ -531,6 +536,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--refresh-ws-gb", type=float, default=44.0)
+    ap.add_argument("--state-dtype", default="f32", choices=["f32", "bf16"],
+                    help="W and direction moments in fp32 (the workload's definition) or bf16 (the paper's runs)")
     ap.add_argument("--clip-norm", type=float, default=0.0,
                     help="global-norm gradient clipping threshold (0: off, as in the workload's definition)")
     ap.add_argument("--chunk-mb", type=int, default=256,

@@ -99,6 +99,13 @@ typedef struct moara_hparams {
                                ||G||_total^2 sums the squared entries of all the
                                call's gradients plus the optional extra term of
                                moara_set_clip_extra (torch.nn.utils.clip_grad_norm_). */
+    int   state_dtype;      /* MOARA_DTYPE_F32 (default): W and the direction
+                               moments in fp32; MOARA_DTYPE_BF16: both in bf16
+                               (the paper's runs keep 2-byte states and apply
+                               the update to bf16 weights, App. D.2 / App. G),
+                               updated in fp32 and stored rounded to nearest
+                               even; tensor-core modules only (bf16 G, B >= 32);
+                               the magnitude moments stay fp32. */
 } moara_hparams;
 
 /* One registered weight.  All pointers are device pointers, 16-byte aligned,
@@ -113,6 +120,8 @@ typedef struct moara_hparams {
  *   mag_avg     m x k  fp32 first moment of the magnitude branch (k=ceil(n/B));
  *   mag_avg_sq  m x k  fp32 second moment          unused when decompose = 0
  *   workspace   moara_workspace_bytes() bytes of scratch, private to the module
+ * With hparams.state_dtype = MOARA_DTYPE_BF16, W, exp_avg and exp_avg_sq
+ * point to bf16 arrays of the same shapes (the pointer types stay float*).
  */
 typedef struct moara_module_desc {
     int m, n, r;

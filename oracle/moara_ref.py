@@ -149,6 +149,16 @@ def truncated_svd(X, r: int):
     return fix_signs(U[:, :r]), S
 
 
+def bf16_round(x):
+    """Nearest bf16 value (8 significant bits, ties to even) of each entry,
+    from float64: x = f * 2^e with 0.5 <= |f| < 1, f rounded to a multiple of
+    2^-8.  Zeros, infinities and NaNs pass through; the bf16 range is that
+    of fp32, so no entry here over- or underflows it."""
+    x = np.asarray(x, dtype=np.float64)
+    f, e = np.frexp(x)
+    return np.ldexp(np.rint(f * 256.0), e - 8)
+
+
 def is_refresh_step(t: int, T: int) -> bool:
     """Algorithm 1 refreshes when s mod T_SVD == 0, read with s = t - 1."""
     return (t - 1) % T == 0
@@ -170,6 +180,7 @@ class Hparams:
     refresh_interval: int = 200  # T_SVD
     decompose: bool = True       # False: plain GaLore (no magnitude branch)
     refresh_src: str = "V"       # "V" (Algorithm 1) or "G"
+    state_bf16: bool = False     # W and the direction moments stored in bf16
 
 
 @dataclass
@@ -235,6 +246,11 @@ def step(state: ModuleState, G, t: int, lr: float, hp: Hparams,
     R = s.P.T @ V
     N, s.exp_avg, s.exp_avg_sq = adam(R, s.exp_avg, s.exp_avg_sq, t,
                                       hp.beta1, hp.beta2, hp.adam_eps)
+    if hp.state_bf16:
+        # the paper's runs keep 2-byte direction states (App. G memory model,
+        # App. D.2): the update uses the new moments, which are then stored
+        # rounded to bf16
+        s.exp_avg, s.exp_avg_sq = bf16_round(s.exp_avg), bf16_round(s.exp_avg_sq)
     dV = s.P @ N
     if hp.decompose:
         dM, s.mag_avg, s.mag_avg_sq = adam(M, s.mag_avg, s.mag_avg_sq, t,
@@ -244,6 +260,9 @@ def step(state: ModuleState, G, t: int, lr: float, hp: Hparams,
         dM = None
         U = dV
     s.W = s.W - lr * hp.scale * U
+    if hp.state_bf16:
+        # App. D.2: the recomposed update is applied to bf16 weights
+        s.W = bf16_round(s.W)
     s.extras = {"M": M, "V": V, "R": R, "N": N, "dV": dV, "dM": dM, "U": U}
     return s
 

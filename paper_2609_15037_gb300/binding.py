@@ -49,6 +49,7 @@ class moara_hparams(ctypes.Structure):
         ("ritz_iters", ctypes.c_int), ("precision", ctypes.c_int),
         ("seed", ctypes.c_uint64),
         ("clip_norm", ctypes.c_float),
+        ("state_dtype", ctypes.c_int),
     ]
 
 

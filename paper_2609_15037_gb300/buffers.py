@@ -18,20 +18,22 @@ class ModuleBuffers:
     """Caller-owned buffers of one registered weight (layouts of moara.h)."""
 
     def __init__(self, m, n, r, block_size, grad_dtype="bf16", device="cuda",
-                 W0=None, with_bf16=True):
+                 W0=None, with_bf16=True, state_dtype="f32"):
         self.m, self.n, self.r, self.block_size = m, n, r, block_size
         self.kb = -(-n // block_size)
         self.grad_dtype = grad_dtype
         dev = torch.device(device)
         f32 = dict(dtype=torch.float32, device=dev)
+        # W and the direction moments in fp32, or bf16 (hparams.state_dtype)
+        st = dict(dtype=torch.bfloat16 if state_dtype == "bf16" else torch.float32, device=dev)
         if W0 is None:
-            self.W = torch.zeros(m, n, **f32)
+            self.W = torch.zeros(m, n, **st)
         else:
-            self.W = torch.as_tensor(W0).to(**f32).contiguous().clone()
+            self.W = torch.as_tensor(W0).to(**st).contiguous().clone()
         self.P = torch.zeros(m, r, **f32)
         self.P_bf16 = torch.zeros(m, r, dtype=torch.int16, device=dev) if with_bf16 else None
-        self.exp_avg = torch.zeros(r, n, **f32)
-        self.exp_avg_sq = torch.zeros(r, n, **f32)
+        self.exp_avg = torch.zeros(r, n, **st)
+        self.exp_avg_sq = torch.zeros(r, n, **st)
         self.mag_avg = torch.zeros(m, self.kb, **f32)
         self.mag_avg_sq = torch.zeros(m, self.kb, **f32)
         nbytes = B.moara_workspace_bytes(m, n, r, block_size)
@@ -98,7 +100,8 @@ class MoaraGroup:
     def add(self, m, n, r, grad_dtype="bf16", W0=None):
         buf = ModuleBuffers(m, n, r, self.hp.block_size, grad_dtype,
                             f"cuda:{self.device}", W0=W0,
-                            with_bf16=True)
+                            with_bf16=True,
+                            state_dtype="bf16" if self.hp.state_dtype == B.MOARA_DTYPE_BF16 else "f32")
         mid = B.moara_init_module(self.ctx, buf.desc())
         self.modules.append(buf)
         self.ids.append(mid)

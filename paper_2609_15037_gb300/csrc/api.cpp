@@ -112,6 +112,10 @@ int check_hparams(moara_ctx* ctx, const moara_hparams* hp) {
         hp->precision != MOARA_PREC_BF16_TC)
         return fail(ctx, MOARA_ERR_INVALID_ARG, "unknown precision");
     if (!std::isfinite(hp->clip_norm)) return fail(ctx, MOARA_ERR_INVALID_ARG, "clip_norm must be finite");
+    if (hp->state_dtype != MOARA_DTYPE_F32 && hp->state_dtype != MOARA_DTYPE_BF16)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "state_dtype must be MOARA_DTYPE_F32 or MOARA_DTYPE_BF16");
+    if (hp->state_dtype == MOARA_DTYPE_BF16 && hp->precision == MOARA_PREC_FP32)
+        return fail(ctx, MOARA_ERR_UNSUPPORTED, "bf16 states run on the tensor-core path only");
     return MOARA_OK;
 }
 
@@ -156,7 +160,8 @@ bool use_tc(const moara_ctx* ctx, int mi) {
     const moara_module_desc& d = ctx->mods[mi];
     if (ctx->hp.precision == MOARA_PREC_FP32) return false;
     if (ctx->hp.precision == MOARA_PREC_AUTO && d.grad_dtype != MOARA_DTYPE_BF16) return false;
-    return moara::tc_supported(d.m, d.n, d.r, ctx->hp.block_size, d.grad_dtype, ctx->hp.decompose) &&
+    return moara::tc_supported(d.m, d.n, d.r, ctx->hp.block_size, d.grad_dtype, ctx->hp.decompose,
+                               ctx->hp.state_dtype) &&
            d.P_bf16 != nullptr && ctx->tc != nullptr;
 }
 
@@ -1068,6 +1073,12 @@ int moara_init_module(moara_ctx* ctx, const moara_module_desc* d, int* module_id
         return fail(ctx, MOARA_ERR_ALIGN, "P_bf16 is not 16-byte aligned");
     if (ctx->hp.precision == MOARA_PREC_BF16_TC && d->P_bf16 == nullptr)
         return fail(ctx, MOARA_ERR_INVALID_ARG, "P_bf16 is required with precision BF16_TC");
+    if (ctx->hp.state_dtype == MOARA_DTYPE_BF16 &&
+        (d->grad_dtype != MOARA_DTYPE_BF16 || d->P_bf16 == nullptr || ctx->tc == nullptr ||
+         !moara::tc_supported(d->m, d->n, d->r, ctx->hp.block_size, d->grad_dtype, ctx->hp.decompose,
+                              ctx->hp.state_dtype)))
+        return fail(ctx, MOARA_ERR_UNSUPPORTED,
+                    "bf16 states need the tensor-core path: bf16 gradient, P_bf16, n and r multiples of 8, B >= 32");
     const moara::WsLayout wl = moara::workspace_layout(d->m, d->n, d->r, ctx->hp.block_size);
     if (d->workspace_bytes < wl.total)
         return fail(ctx, MOARA_ERR_WORKSPACE, "workspace of %zu bytes, %zu needed", d->workspace_bytes, wl.total);

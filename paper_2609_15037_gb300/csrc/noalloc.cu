@@ -56,6 +56,7 @@ extern "C" int moara_step_static_scratch(const moara_hparams* hp, int m, int n, 
     if (grad_dtype != MOARA_DTYPE_F32 && grad_dtype != MOARA_DTYPE_BF16) return MOARA_ERR_INVALID_ARG;
     if (t < 1 || !std::isfinite(lr)) return MOARA_ERR_INVALID_ARG;
     if (hp->clip_norm > 0.0f) return MOARA_ERR_UNSUPPORTED;   // global-norm clipping needs the whole step
+    if (hp->state_dtype != MOARA_DTYPE_F32) return MOARA_ERR_UNSUPPORTED;   // fp32 states only here
     if (!aligned16(G) || !aligned16(W) || !aligned16(P) || !aligned16(exp_avg) || !aligned16(exp_avg_sq))
         return G && W && P && exp_avg && exp_avg_sq ? MOARA_ERR_ALIGN : MOARA_ERR_INVALID_ARG;
     if (hp->decompose && (!aligned16(mag_avg) || !aligned16(mag_avg_sq)))

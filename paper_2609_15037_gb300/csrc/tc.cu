@@ -88,8 +88,11 @@ constexpr int K1_B_BYTES = K1_BK * (K1_BN / 2) * 2;     // 16 KB: this CTA's two
 // The Adam moments stream through a ring of slots, each one 32-column chunk
 // of exp_avg and of exp_avg_sq (128 rank rows x 32 fp32, 16 KB each), loaded
 // and stored by TMA.
-constexpr int K1_MCOLS = 32;
-constexpr int K1_MCHUNK = K1_BM * K1_MCOLS * 4;          // 16 KB
+constexpr int K1_MCOLS = 32;                            // fp32 moments: columns per chunk
+constexpr int K1_MCHUNK = K1_BM * K1_MCOLS * 4;          // 16 KB (64 columns of bf16 moments)
+// Chunk width in columns for fp32 (SB false) or bf16 (SB true) states: one
+// 128-byte row of a 128-row chunk either way.
+template <bool SB> struct StateCols { static constexpr int N = SB ? 64 : 32; };
 template <bool HILO> struct K1Cfg {
     static constexpr int STAGES = HILO ? 3 : 5;
     static constexpr int STAGE_BYTES = K1_A_BYTES + (HILO ? 2 : 1) * K1_B_BYTES;
@@ -290,9 +293,11 @@ __global__ void __launch_bounds__(256) k0_mag_adam(const __grid_constant__ K0Par
 // operands), Optimizer_V (Adam) in the epilogue, N written in bf16.  HILO
 // adds the MMA with V_lo (first Adam step).
 // ===========================================================================
-template <bool HILO>
+template <bool HILO, bool SB>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(K1_THREADS, 1)
 k1_project(const __grid_constant__ K1Params p) {
+    constexpr int MC = StateCols<SB>::N;              // moment columns per chunk
+    constexpr int HC = MC / 2;                        // columns per epilogue thread and chunk
     constexpr int STAGES = K1Cfg<HILO>::STAGES;
     constexpr int STAGE_BYTES = K1Cfg<HILO>::STAGE_BYTES;
     constexpr int MSLOTS = K1Cfg<HILO>::MSLOTS;
@@ -439,7 +444,7 @@ k1_project(const __grid_constant__ K1Params p) {
                 const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 6];
                 const CUtensorMap* smap = &p.maps[tl.mod * kMaps + 7];
                 const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
-                const int nc = min(K1_BN / K1_MCOLS, (md.n - n0 + K1_MCOLS - 1) / K1_MCOLS);
+                const int nc = min(K1_BN / MC, (md.n - n0 + MC - 1) / MC);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % MSLOTS;
                     const uint32_t ph = (g / MSLOTS) & 1;
@@ -448,8 +453,8 @@ k1_project(const __grid_constant__ K1Params p) {
                     const uint32_t fb = ptx::smem_u32(&ctl->wfull[b]);
                     ptx::mbar_arrive_expect_tx(fb, 2 * K1_MCHUNK);
                     const uint32_t dst = ptx::smem_u32(mring + b * 2 * K1_MCHUNK);
-                    ptx::tma_load_2d(dst, amap, fb, n0 + c * K1_MCOLS, r0);
-                    ptx::tma_load_2d(dst + K1_MCHUNK, smap, fb, n0 + c * K1_MCOLS, r0);
+                    ptx::tma_load_2d(dst, amap, fb, n0 + c * MC, r0);
+                    ptx::tma_load_2d(dst + K1_MCHUNK, smap, fb, n0 + c * MC, r0);
                     issued |= 1u << b;
                     last_par = (last_par & ~(1u << b)) | (ph << b);
                 }
@@ -470,15 +475,15 @@ k1_project(const __grid_constant__ K1Params p) {
                 const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 6];
                 const CUtensorMap* smap = &p.maps[tl.mod * kMaps + 7];
                 const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
-                const int nc = min(K1_BN / K1_MCOLS, (md.n - n0 + K1_MCOLS - 1) / K1_MCOLS);
+                const int nc = min(K1_BN / MC, (md.n - n0 + MC - 1) / MC);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % MSLOTS;
                     const uint32_t ph = (g / MSLOTS) & 1;
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->wdone[b]), ph, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
                     const uint32_t src = ptx::smem_u32(mring + b * 2 * K1_MCHUNK);
-                    ptx::tma_store_2d(amap, src, n0 + c * K1_MCOLS, r0);
-                    ptx::tma_store_2d(smap, src + K1_MCHUNK, n0 + c * K1_MCOLS, r0);
+                    ptx::tma_store_2d(amap, src, n0 + c * MC, r0);
+                    ptx::tma_store_2d(smap, src + K1_MCHUNK, n0 + c * MC, r0);
                     ptx::bulk_commit_group();
                     ptx::bulk_wait_read_all();            // the slot may be refilled once read
                     ptx::mbar_arrive(ptx::smem_u32(&ctl->wempty[b]));
@@ -510,7 +515,7 @@ k1_project(const __grid_constant__ K1Params p) {
             const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
             const int a = r0 + il;
             const bool row_ok = a < rr;
-            const int nc = min(K1_BN / K1_MCOLS, (nn - n0 + K1_MCOLS - 1) / K1_MCOLS);
+            const int nc = min(K1_BN / MC, (nn - n0 + MC - 1) / MC);
             const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[buf]), acc_phase, abort_flag, p.status,
                                             MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
             if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
@@ -518,58 +523,88 @@ k1_project(const __grid_constant__ K1Params p) {
             for (int c = 0; c < nc; ++c, ++g) {
                 const int b = g % MSLOTS;
                 const uint32_t ph = (g / MSLOTS) & 1;
-                const int j0 = n0 + c * K1_MCOLS + ch * 16;
+                const int j0 = n0 + c * MC + ch * HC;
+                // the thread's HC columns in passes of 16: four 16-byte units
+                // of its row per chunk, 4 fp32 or 8 bf16 moments each
+                constexpr int PU = HC / 4;                  // moments per unit
+                constexpr int UPH = 16 / PU;                // units per pass
+                const uint32_t tcol = tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + c * MC + ch * HC;
                 float v[16];
                 __syncwarp();
-                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + c * K1_MCOLS + ch * 16, v);
+                ptx::tmem_ld16(tcol, v);
                 const bool gotm = ptx::mbar_wait(ptx::smem_u32(&ctl->wfull[b]), ph, abort_flag, p.status,
                                                  MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
                 if (!__all_sync(0xffffffffu, gotm)) { ok = false; break; }
                 uint8_t* arow = mring + b * 2 * K1_MCHUNK + il * 128;
                 uint8_t* srow = arow + K1_MCHUNK;
                 const uint32_t x = static_cast<uint32_t>(il & 7);
-                float nv[16];
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const uint32_t off = ((ch * 4 + u) ^ x) << 4;
-                    float4* a4 = reinterpret_cast<float4*>(arow + off);
-                    float4* s4 = reinterpret_cast<float4*>(srow + off);
-                    const float4 av = *a4, sv = *s4;
-                    float ea[4] = {av.x, av.y, av.z, av.w};
-                    float es[4] = {sv.x, sv.y, sv.z, sv.w};
+                for (int h = 0; h < HC / 16; ++h) {
+                    if (h > 0) ptx::tmem_ld16(tcol + 16 * h, v);
+                    float nv[16];
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float rv = v[4 * u + e] * cf;
-                        ea[e] = p.beta1 * ea[e] + (1.0f - p.beta1) * rv;
-                        es[e] = p.beta2 * es[e] + (1.0f - p.beta2) * rv * rv;
-                        // N goes to K2 in bf16: approximate sqrt / reciprocal
-                        // (relative error ~2^-22) are far below its rounding
-                        nv[4 * u + e] = ea[e] * p.inv_bc1 *
-                                        ptx::rcp_approx(ptx::sqrt_approx(es[e] * p.inv_bc2) + p.adam_eps);
+                    for (int uu = 0; uu < UPH; ++uu) {
+                        const int u = h * UPH + uu;
+                        const uint32_t off = ((ch * 4 + u) ^ x) << 4;
+                        uint4* a4 = reinterpret_cast<uint4*>(arow + off);
+                        uint4* s4 = reinterpret_cast<uint4*>(srow + off);
+                        const uint4 av = *a4, sv = *s4;
+                        const uint32_t aw[4] = {av.x, av.y, av.z, av.w}, sw[4] = {sv.x, sv.y, sv.z, sv.w};
+                        float ea[PU], es[PU];
+                        if constexpr (SB) {
+#pragma unroll
+                            for (int k = 0; k < 4; ++k) {
+                                ea[2 * k] = bf_lo(aw[k]); ea[2 * k + 1] = bf_hi(aw[k]);
+                                es[2 * k] = bf_lo(sw[k]); es[2 * k + 1] = bf_hi(sw[k]);
+                            }
+                        } else {
+#pragma unroll
+                            for (int k = 0; k < PU; ++k) { ea[k] = __uint_as_float(aw[k]); es[k] = __uint_as_float(sw[k]); }
+                        }
+#pragma unroll
+                        for (int e = 0; e < PU; ++e) {
+                            const float rv = v[PU * uu + e] * cf;
+                            ea[e] = p.beta1 * ea[e] + (1.0f - p.beta1) * rv;
+                            es[e] = p.beta2 * es[e] + (1.0f - p.beta2) * rv * rv;
+                            // N goes to K2 in bf16: approximate sqrt / reciprocal
+                            // (relative error ~2^-22) are far below its rounding
+                            nv[PU * uu + e] = ea[e] * p.inv_bc1 *
+                                              ptx::rcp_approx(ptx::sqrt_approx(es[e] * p.inv_bc2) + p.adam_eps);
+                        }
+                        if constexpr (SB) {   // the moments are stored rounded to bf16
+                            *a4 = make_uint4(pack_bf16x2(ea[0], ea[1]), pack_bf16x2(ea[2], ea[3]),
+                                             pack_bf16x2(ea[4], ea[5]), pack_bf16x2(ea[6], ea[7]));
+                            *s4 = make_uint4(pack_bf16x2(es[0], es[1]), pack_bf16x2(es[2], es[3]),
+                                             pack_bf16x2(es[4], es[5]), pack_bf16x2(es[6], es[7]));
+                        } else {
+                            *a4 = make_uint4(__float_as_uint(ea[0]), __float_as_uint(ea[1]),
+                                             __float_as_uint(ea[2]), __float_as_uint(ea[3]));
+                            *s4 = make_uint4(__float_as_uint(es[0]), __float_as_uint(es[1]),
+                                             __float_as_uint(es[2]), __float_as_uint(es[3]));
+                        }
                     }
-                    *a4 = make_float4(ea[0], ea[1], ea[2], ea[3]);
-                    *s4 = make_float4(es[0], es[1], es[2], es[3]);
+                    const int jh = j0 + 16 * h;
+                    if (row_ok && jh < nn) {
+                        const long long o = (long long)a * nn + jh;
+                        if (jh + 16 <= nn) {
+                            uint4* n4 = reinterpret_cast<uint4*>(nb_p + o);
+                            n4[0] = make_uint4(pack_bf16x2(nv[0], nv[1]), pack_bf16x2(nv[2], nv[3]),
+                                               pack_bf16x2(nv[4], nv[5]), pack_bf16x2(nv[6], nv[7]));
+                            n4[1] = make_uint4(pack_bf16x2(nv[8], nv[9]), pack_bf16x2(nv[10], nv[11]),
+                                               pack_bf16x2(nv[12], nv[13]), pack_bf16x2(nv[14], nv[15]));
+                        } else {
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                if (jh + e >= nn) continue;
+                                __nv_bfloat16 hb = __float2bfloat16_rn(nv[e]);
+                                nb_p[o + e] = *reinterpret_cast<uint16_t*>(&hb);
+                            }
+                        }
+                    }
                 }
                 ptx::fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->wdone[b]));
-                if (row_ok && j0 < nn) {
-                    const long long o = (long long)a * nn + j0;
-                    if (j0 + 16 <= nn) {
-                        uint4* n4 = reinterpret_cast<uint4*>(nb_p + o);
-                        n4[0] = make_uint4(pack_bf16x2(nv[0], nv[1]), pack_bf16x2(nv[2], nv[3]),
-                                           pack_bf16x2(nv[4], nv[5]), pack_bf16x2(nv[6], nv[7]));
-                        n4[1] = make_uint4(pack_bf16x2(nv[8], nv[9]), pack_bf16x2(nv[10], nv[11]),
-                                           pack_bf16x2(nv[12], nv[13]), pack_bf16x2(nv[14], nv[15]));
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            if (j0 + e >= nn) continue;
-                            __nv_bfloat16 hb = __float2bfloat16_rn(nv[e]);
-                            nb_p[o + e] = *reinterpret_cast<uint16_t*>(&hb);
-                        }
-                    }
-                }
             }
             if (!ok) break;
             ptx::tc_fence_before();
@@ -594,9 +629,12 @@ k1_project(const __grid_constant__ K1Params p) {
 // ===========================================================================
 // K2: back-projection dV = P N and the weight update in the epilogue.
 // ===========================================================================
-template <int BLK>
+template <int BLK, bool SB>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(K2_THREADS, 1)
 k2_backproject(const __grid_constant__ K2Params p) {
+    constexpr int WC = StateCols<SB>::N;              // W columns per ring chunk
+    constexpr int HC = WC / 2;                        // columns per epilogue thread and chunk
+    static_assert(!SB || BLK >= 32, "bf16 states: a thread's 32 columns lie in one block");
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
     uint8_t* wring = smem + K2_STAGES * K2_STAGE_BYTES;
@@ -726,7 +764,7 @@ k2_backproject(const __grid_constant__ K2Params p) {
                 const TcMod& md = p.mods[tl.mod];
                 const CUtensorMap* wmap = &p.maps[tl.mod * kMaps + 3];
                 const int i0 = (2 * tl.t0 + crank) * K2_BM, n0 = tl.t1 * K2_BN;
-                const int nc = min(K2_BN / K2_WCOLS, (md.n - n0 + K2_WCOLS - 1) / K2_WCOLS);
+                const int nc = min(K2_BN / WC, (md.n - n0 + WC - 1) / WC);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % K2_WBUF;
                     const uint32_t ph = (g / K2_WBUF) & 1;
@@ -734,7 +772,7 @@ k2_backproject(const __grid_constant__ K2Params p) {
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
                     const uint32_t fb = ptx::smem_u32(&ctl->wfull[b]);
                     ptx::mbar_arrive_expect_tx(fb, K2_WBYTES);
-                    ptx::tma_load_2d(ptx::smem_u32(wring + b * K2_WBYTES), wmap, fb, n0 + c * K2_WCOLS, i0);
+                    ptx::tma_load_2d(ptx::smem_u32(wring + b * K2_WBYTES), wmap, fb, n0 + c * WC, i0);
                     issued |= 1u << b;
                     last_par = (last_par & ~(1u << b)) | (ph << b);
                 }
@@ -754,13 +792,13 @@ k2_backproject(const __grid_constant__ K2Params p) {
                 const TcMod& md = p.mods[tl.mod];
                 const CUtensorMap* wmap = &p.maps[tl.mod * kMaps + 3];
                 const int i0 = (2 * tl.t0 + crank) * K2_BM, n0 = tl.t1 * K2_BN;
-                const int nc = min(K2_BN / K2_WCOLS, (md.n - n0 + K2_WCOLS - 1) / K2_WCOLS);
+                const int nc = min(K2_BN / WC, (md.n - n0 + WC - 1) / WC);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % K2_WBUF;
                     const uint32_t ph = (g / K2_WBUF) & 1;
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->wdone[b]), ph, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
-                    ptx::tma_store_2d(wmap, ptx::smem_u32(wring + b * K2_WBYTES), n0 + c * K2_WCOLS, i0);
+                    ptx::tma_store_2d(wmap, ptx::smem_u32(wring + b * K2_WBYTES), n0 + c * WC, i0);
                     ptx::bulk_commit_group();
                     ptx::bulk_wait_read_all();            // the chunk may be refilled once read
                     ptx::mbar_arrive(ptx::smem_u32(&ctl->wempty[b]));
@@ -771,8 +809,9 @@ k2_backproject(const __grid_constant__ K2Params p) {
     } else {
         // ------------------------------------------------- epilogue warps
         // 8 warps: TMEM lane quarter q = warp % 4, column half ch of each
-        // 32-column chunk; each thread updates 16 values of its W row in the
-        // swizzled shared-memory chunk: W -= lr * alpha * dM * (P N).
+        // chunk (32 fp32 / 64 bf16 columns); each thread updates 16 / 32
+        // values of its W row in the swizzled shared-memory chunk:
+        // W -= lr * alpha * dM * (P N), rounded to bf16 for bf16 weights.
         const int ew = warp - 4;                        // 0..7
         const int q = warp & 3;
         const int ch = ew >> 2;
@@ -791,7 +830,7 @@ k2_backproject(const __grid_constant__ K2Params p) {
             const int i0 = (2 * tl.t0 + crank) * K2_BM, n0 = tl.t1 * K2_BN;
             const int i = i0 + il;
             const bool row_ok = i < mm;
-            const int nc = min(K2_BN / K2_WCOLS, (nn - n0 + K2_WCOLS - 1) / K2_WCOLS);
+            const int nc = min(K2_BN / WC, (nn - n0 + WC - 1) / WC);
             // blocks of B >= 32 columns: the tile's dM values of this row are
             // loaded once, before the wait for the accumulator
             float dmt[HOIST ? K2_BN / BLK : 1];
@@ -809,11 +848,11 @@ k2_backproject(const __grid_constant__ K2Params p) {
             for (int c = 0; c < nc; ++c, ++g) {
                 const int b = g % K2_WBUF;
                 const uint32_t ph = (g / K2_WBUF) & 1;
-                const int j0 = n0 + c * K2_WCOLS + ch * 16;
+                const int j0 = n0 + c * WC + ch * HC;
                 float dm[NDM];
                 if (HOIST) {
-                    // the chunk's 16 columns lie in one block
-                    const int cb = c * K2_WCOLS + ch * 16;
+                    // the thread's 16 (32) columns of the chunk lie in one block
+                    const int cb = c * WC + ch * HC;
                     dm[0] = dmt[0];
 #pragma unroll
                     for (int d = 1; d < K2_BN / BLK; ++d) dm[0] = (cb >= d * BLK) ? dmt[d] : dm[0];
@@ -824,9 +863,12 @@ k2_backproject(const __grid_constant__ K2Params p) {
                         dm[d] = (p.decompose && row_ok && jb < mkb) ? dMp[(long long)i * mkb + jb] : 1.0f;
                     }
                 }
-                float v[16];
+                float v[HC];
                 __syncwarp();
-                ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + c * K2_WCOLS + ch * 16, v);
+#pragma unroll
+                for (int h = 0; h < HC / 16; ++h)
+                    ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + c * WC + ch * HC + 16 * h,
+                                   *reinterpret_cast<float(*)[16]>(v + 16 * h));
                 const bool gotw = ptx::mbar_wait(ptx::smem_u32(&ctl->wfull[b]), ph, abort_flag, p.status,
                                                  MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
                 if (!__all_sync(0xffffffffu, gotw)) { ok = false; break; }
@@ -834,14 +876,30 @@ k2_backproject(const __grid_constant__ K2Params p) {
                 const uint32_t x = static_cast<uint32_t>(il & 7);
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    float4* w4 = reinterpret_cast<float4*>(wrow + (((ch * 4 + u) ^ x) << 4));
-                    float4 w = *w4;
-                    const float d0 = dm[NDM == 1 ? 0 : (u * 4) / BLK];
-                    w.x -= p.step_scale * (d0 * v[4 * u + 0]);
-                    w.y -= p.step_scale * (d0 * v[4 * u + 1]);
-                    w.z -= p.step_scale * (d0 * v[4 * u + 2]);
-                    w.w -= p.step_scale * (d0 * v[4 * u + 3]);
-                    *w4 = w;
+                    uint4* w4 = reinterpret_cast<uint4*>(wrow + (((ch * 4 + u) ^ x) << 4));
+                    const uint4 wv = *w4;
+                    if constexpr (SB) {
+                        const float d0 = dm[0];
+                        const uint32_t ww[4] = {wv.x, wv.y, wv.z, wv.w};
+                        uint32_t out[4];
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const float lo = bf_lo(ww[k]) - p.step_scale * (d0 * v[8 * u + 2 * k]);
+                            const float hi = bf_hi(ww[k]) - p.step_scale * (d0 * v[8 * u + 2 * k + 1]);
+                            out[k] = pack_bf16x2(lo, hi);
+                        }
+                        *w4 = make_uint4(out[0], out[1], out[2], out[3]);
+                    } else {
+                        float4 w = make_float4(__uint_as_float(wv.x), __uint_as_float(wv.y), __uint_as_float(wv.z),
+                                               __uint_as_float(wv.w));
+                        const float d0 = dm[NDM == 1 ? 0 : (u * 4) / BLK];
+                        w.x -= p.step_scale * (d0 * v[4 * u + 0]);
+                        w.y -= p.step_scale * (d0 * v[4 * u + 1]);
+                        w.z -= p.step_scale * (d0 * v[4 * u + 2]);
+                        w.w -= p.step_scale * (d0 * v[4 * u + 3]);
+                        *w4 = make_uint4(__float_as_uint(w.x), __float_as_uint(w.y), __float_as_uint(w.z),
+                                         __float_as_uint(w.w));
+                    }
                 }
                 ptx::fence_proxy_async_smem();
                 __syncwarp();
@@ -1344,7 +1402,9 @@ int max_clusters(const void* fn, int threads, int smem, int cap) {
 
 template <int BLK>
 void set_smem_attrs() {
-    cudaFuncSetAttribute(k2_backproject<BLK>, cudaFuncAttributeMaxDynamicSharedMemorySize, K2_SMEM);
+    cudaFuncSetAttribute(k2_backproject<BLK, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K2_SMEM);
+    if constexpr (BLK >= 32)
+        cudaFuncSetAttribute(k2_backproject<BLK, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K2_SMEM);
 }
 
 }  // namespace
@@ -1382,7 +1442,8 @@ struct TcState {
     cudaEvent_t ev_part[32] = {};
 };
 
-bool tc_supported(int m, int n, int r, int B, int dtype, int decompose) {
+bool tc_supported(int m, int n, int r, int B, int dtype, int decompose, int state_dtype) {
+    if (state_dtype == MOARA_DTYPE_BF16 && decompose && B < 32) return false;
     if (dtype != MOARA_DTYPE_BF16) return false;
     if (m < 1 || n < 8 || r < 8) return false;
     if ((n % 8) != 0 || (r % 8) != 0) return false;
@@ -1433,7 +1494,13 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
         st->mods.resize(id + 1, TcMod{});
         st->maps.resize(kMaps * (id + 1));
     }
-    if (!tc_supported(md.m, md.n, md.r, hp.block_size, md.dtype, hp.decompose) || md.Pb == nullptr) return MOARA_OK;
+    if (!tc_supported(md.m, md.n, md.r, hp.block_size, md.dtype, hp.decompose, hp.state_dtype) || md.Pb == nullptr)
+        return MOARA_OK;
+    // W and the direction moments: fp32, or bf16 (state_dtype); a ring chunk
+    // is one 128-byte row wide either way
+    const bool sb = hp.state_dtype == MOARA_DTYPE_BF16;
+    const CUtensorMapDataType sdt = sb ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    const int ses = sb ? 2 : 4, scols = sb ? StateCols<true>::N : StateCols<false>::N;
     TcMod t{};
     t.m = md.m; t.n = md.n; t.r = md.r; t.kb = md.kb;
     t.Vhi = md.ws_Vhi; t.Vlo = md.ws_Vlo;
@@ -1447,12 +1514,11 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
     if (!encode_bf16_2d(st->encode, &mp[0], md.Pb, md.r, md.m, 64, 64) ||
         !encode_bf16_2d(st->encode, &mp[1], md.Pb, md.r, md.m, 64, 128) ||
         !encode_bf16_2d(st->encode, &mp[2], t.Nb, md.n, md.r, 64, 64) ||
-        !encode_2d(st->encode, &mp[3], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, md.W, md.n, md.m, K2_WCOLS, K2_BM) ||
+        !encode_2d(st->encode, &mp[3], sdt, ses, md.W, md.n, md.m, scols, K2_BM) ||
         !encode_bf16_2d(st->encode, &mp[4], t.Vhi, md.n, md.m, 64, 64) ||
         !encode_bf16_2d(st->encode, &mp[5], t.Vlo, md.n, md.m, 64, 64) ||
-        !encode_2d(st->encode, &mp[6], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, md.exp_avg, md.n, md.r, K1_MCOLS, K1_BM) ||
-        !encode_2d(st->encode, &mp[7], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, md.exp_avg_sq, md.n, md.r, K1_MCOLS,
-                   K1_BM)) {
+        !encode_2d(st->encode, &mp[6], sdt, ses, md.exp_avg, md.n, md.r, scols, K1_BM) ||
+        !encode_2d(st->encode, &mp[7], sdt, ses, md.exp_avg_sq, md.n, md.r, scols, K1_BM)) {
         st->err = "cuTensorMapEncodeTiled failed";
         return MOARA_ERR_CUDA;
     }
@@ -1599,19 +1665,19 @@ static cudaError_t launch_k0(TcState* st, const K0Params& p0, bool background, c
     return cudaGetLastError();
 }
 
-template <int BLK>
+template <int BLK, bool SB>
 static cudaError_t launch_k12(TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2, bool hilo,
                               cudaStream_t s, int64_t* launches, const TcProfile& prof) {
     cudaError_t e;
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, true);
-    if (hilo) k1_project<true><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
-    else k1_project<false><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+    if (hilo) k1_project<true, SB><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+    else k1_project<false, SB><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, false);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     ++*launches;
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_BACKPROJECT, s, true);
-    k2_backproject<BLK><<<2 * g2, K2_THREADS, K2_SMEM, s>>>(p2);
+    k2_backproject<BLK, SB><<<2 * g2, K2_THREADS, K2_SMEM, s>>>(p2);
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_BACKPROJECT, s, false);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -1630,14 +1696,21 @@ static cudaError_t launch_k0_any(int B, TcState* st, const K0Params& p0, bool ba
     }
 }
 
-static cudaError_t launch_k12_any(int B, TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2,
-                                  bool hilo, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+static cudaError_t launch_k12_any(int B, bool sb, TcState* st, const K1Params& p1, const K2Params& p2, int g1,
+                                  int g2, bool hilo, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+    if (sb) {   // bf16 states: B >= 32 (tc_supported)
+        switch (B) {
+            case 32: return launch_k12<32, true>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+            case 64: return launch_k12<64, true>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+            default: return launch_k12<128, true>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        }
+    }
     switch (B) {
-        case 8: return launch_k12<8>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-        case 16: return launch_k12<16>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-        case 32: return launch_k12<32>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-        case 64: return launch_k12<64>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-        default: return launch_k12<128>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        case 8: return launch_k12<8, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        case 16: return launch_k12<16, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        case 32: return launch_k12<32, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        case 64: return launch_k12<64, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        default: return launch_k12<128, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
     }
 }
 
@@ -1653,14 +1726,16 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             float bc2, float lr, int first_step, const float* clip, cudaStream_t s, int64_t* launches,
             const TcProfile& prof) {
     if (!st->attrs_set) {
-        cudaFuncSetAttribute(k1_project<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
-        cudaFuncSetAttribute(k1_project<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
+        cudaFuncSetAttribute(k1_project<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
+        cudaFuncSetAttribute(k1_project<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
+        cudaFuncSetAttribute(k1_project<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
+        cudaFuncSetAttribute(k1_project<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
         set_smem_attrs<8>(); set_smem_attrs<16>(); set_smem_attrs<32>(); set_smem_attrs<64>();
         set_smem_attrs<128>();
         // clusters of two that fit on the GPU at once (persistent grids)
-        st->k1_clusters = max_clusters(reinterpret_cast<const void*>(k1_project<false>), K1_THREADS, K1_SMEM,
+        st->k1_clusters = max_clusters(reinterpret_cast<const void*>(k1_project<false, false>), K1_THREADS, K1_SMEM,
                                        st->sms / 2);
-        st->k2_clusters = max_clusters(reinterpret_cast<const void*>(k2_backproject<128>), K2_THREADS, K2_SMEM,
+        st->k2_clusters = max_clusters(reinterpret_cast<const void*>(k2_backproject<128, false>), K2_THREADS, K2_SMEM,
                                        st->sms / 2);
         st->attrs_set = true;
     }
@@ -1762,7 +1837,8 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;
             p2.step_scale = lr * hp.scale;
             p2.decompose = hp.decompose;
-            const cudaError_t e = launch_k12_any(B, st, p1, p2, tl->g1, tl->g2, hilo, s, launches, prof);
+            const cudaError_t e = launch_k12_any(B, hp.state_dtype == MOARA_DTYPE_BF16, st, p1, p2, tl->g1, tl->g2,
+                                                 hilo, s, launches, prof);
             if (e != cudaSuccess) {
                 st->err = cudaGetErrorString(e);
                 return MOARA_ERR_CUDA;

@@ -8,7 +8,7 @@ namespace moara {
 struct TcState;
 
 // Whether a module of this shape can run on the tensor-core kernels.
-bool tc_supported(int m, int n, int r, int B, int dtype, int decompose);
+bool tc_supported(int m, int n, int r, int B, int dtype, int decompose, int state_dtype);
 
 // Hook used to time the tensor-core launches with CUDA events.
 struct TcProfile {

@@ -446,3 +446,35 @@ def test_flatten_rule():
     assert flat[1, 5] == G[1, 1, 1]
     with pytest.raises(ValueError):
         o.flatten_shape((3, 0))
+
+
+def test_bf16_round_matches_torch_and_ties_to_even():
+    """bf16_round against torch's float32 -> bfloat16 conversion (a library
+    routine) on fp32-representable inputs, and the tie rule by hand:
+    1 + 2^-8 lies halfway between 1 and 1 + 2^-7 and rounds to the even 1;
+    1 + 3 * 2^-8 rounds up to 1 + 2^-6."""
+    torch = pytest.importorskip("torch")
+    x = (_rng(51).standard_normal(10000) * np.exp(_rng(52).uniform(-20, 20, 10000))).astype(np.float32)
+    ref = torch.tensor(x).to(torch.bfloat16).to(torch.float64).numpy()
+    assert np.array_equal(o.bf16_round(x.astype(np.float64)), ref)
+    assert o.bf16_round(np.array([1.0 + 2.0 ** -8]))[0] == 1.0
+    assert o.bf16_round(np.array([1.0 + 3 * 2.0 ** -8]))[0] == 1.0 + 2.0 ** -6
+    assert o.bf16_round(np.array([-(1.0 + 2.0 ** -8)]))[0] == -1.0
+    assert o.bf16_round(np.array([0.0]))[0] == 0.0
+
+
+def test_bf16_state_step_stores_rounded_states():
+    """With bf16 states the step's W and direction moments are bf16 values
+    and differ from the fp32-state step by rounding only."""
+    rng = _rng(53)
+    m, n, r, B = 16, 24, 4, 8
+    G = rng.standard_normal((m, n))
+    W0 = o.bf16_round(rng.standard_normal((m, n)) * 0.02)
+    P = np.linalg.qr(rng.standard_normal((m, r)))[0]
+    hp32, hp16 = o.Hparams(block_size=B), o.Hparams(block_size=B, state_bf16=True)
+    s32 = o.step(o.init_state(W0, r, B, P=P), G, 1, 1e-3, hp32, False)
+    s16 = o.step(o.init_state(W0, r, B, P=P), G, 1, 1e-3, hp16, False)
+    for x in (s16.W, s16.exp_avg, s16.exp_avg_sq):
+        assert np.array_equal(o.bf16_round(x), x)
+    np.testing.assert_array_equal(s16.W, o.bf16_round(s32.W))
+    np.testing.assert_array_equal(s16.exp_avg, o.bf16_round(s32.exp_avg))
