@@ -355,13 +355,17 @@ def run_gpu(args):
         roof = {"bound": "alu", "achieved": round(achieved, 2), "peak": round(alu_peak, 1),
                 "unit": "TFLOP/s", "frac": round(achieved / alu_peak, 4), "traffic": None,
                 "kernel": dom, "peak_source": "152 SMs x 128 FP32 lanes x 2 x 2.07 GHz"}
-    elif dom == "tc_project":
+    elif dom in ("tc_project", "tc_backproject") and \
+            flops_dom / (bf16_sus * 1e12) >= kbytes[dom] / n_launch_per_step / (hbm * 1e9):
+        # the kernel's own roof is the tensor pipe: its flops at the sustained
+        # bf16 rate take longer than its bytes at the copy bandwidth
         achieved = flops_dom / (dom_ms * 1e-3) / 1e12
         tr = _traffic(dom, args.workload) if sbytes == 4 else None   # counters taken with fp32 states
         roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": bf16_sus,
                 "unit": "TFLOP/s", "frac": round(achieved / bf16_sus, 4),
                 "traffic": None if tr is None else int(tr / n_launch_per_step),
-                "kernel": dom, "peak_source": f"bf16_tflops_sustained ({peak_src})"}
+                "kernel": dom, "peak_source": f"bf16_tflops_sustained ({peak_src})",
+                "hbm_frac": round(kbytes[dom] / n_launch_per_step / (dom_ms * 1e-3) / 1e9 / hbm, 4)}
     else:
         by = kbytes[dom] / n_launch_per_step
         achieved = by / (dom_ms * 1e-3) / 1e9
