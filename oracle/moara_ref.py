@@ -181,6 +181,8 @@ class Hparams:
     decompose: bool = True       # False: plain GaLore (no magnitude branch)
     refresh_src: str = "V"       # "V" (Algorithm 1) or "G"
     state_bf16: bool = False     # W and the direction moments stored in bf16
+    proj_rule: str = "left"      # "left": P (m x r) for every weight; "smaller":
+                                 # GaLore's rule, a right projector Q (n x r) when m > n
 
 
 @dataclass
@@ -202,18 +204,30 @@ class ModuleState:
                        mag_avg_sq=self.mag_avg_sq.copy(), extras={})
 
 
-def init_state(W, r: int, B: int, P=None) -> ModuleState:
-    """Zero Adam moments (r x n and m x k) for weight W (m x n)."""
+def is_right(m: int, n: int, proj_rule: str) -> bool:
+    """GaLore's smaller-side rule: project the column space (right projector
+    Q, n x r) of a tall weight (m > n); the paper's memory numbers assume it
+    (App. G, d_W = max(m, n))."""
+    return proj_rule == "smaller" and m > n
+
+
+def init_state(W, r: int, B: int, P=None, proj_rule: str = "left") -> ModuleState:
+    """Zero Adam moments for weight W (m x n): r x n with a left projector P
+    (m x r), m x r with a right projector Q (n x r, stored in ``P``); m x k
+    magnitude moments."""
     W = np.array(W, dtype=np.float64, copy=True)
     m, n = W.shape
     k = num_blocks(n, B)
+    right = is_right(m, n, proj_rule)
+    shape = (n, r) if right else (m, r)
     if P is None:
-        P = np.zeros((m, r), dtype=np.float64)
+        P = np.zeros(shape, dtype=np.float64)
     P = np.array(P, dtype=np.float64, copy=True)
-    if P.shape != (m, r):
-        raise ValueError("P must be m x r")
+    if P.shape != shape:
+        raise ValueError(f"projector must be {shape[0]} x {shape[1]}")
+    mom = (m, r) if right else (r, n)
     return ModuleState(W=W, P=P,
-                       exp_avg=np.zeros((r, n)), exp_avg_sq=np.zeros((r, n)),
+                       exp_avg=np.zeros(mom), exp_avg_sq=np.zeros(mom),
                        mag_avg=np.zeros((m, k)), mag_avg_sq=np.zeros((m, k)))
 
 
@@ -240,10 +254,12 @@ def step(state: ModuleState, G, t: int, lr: float, hp: Hparams,
         M, V = decompose(G, B, hp.decomp_eps)
     else:
         M, V = None, G
+    right = is_right(m, n, hp.proj_rule)
     if refresh:
         src = V if hp.refresh_src == "V" else G
-        s.P, _ = truncated_svd(src, r)
-    R = s.P.T @ V
+        # right projector: the top-r right singular vectors of the source
+        s.P, _ = truncated_svd(src.T if right else src, r)
+    R = V @ s.P if right else s.P.T @ V
     N, s.exp_avg, s.exp_avg_sq = adam(R, s.exp_avg, s.exp_avg_sq, t,
                                       hp.beta1, hp.beta2, hp.adam_eps)
     if hp.state_bf16:
@@ -251,7 +267,7 @@ def step(state: ModuleState, G, t: int, lr: float, hp: Hparams,
         # App. D.2): the update uses the new moments, which are then stored
         # rounded to bf16
         s.exp_avg, s.exp_avg_sq = bf16_round(s.exp_avg), bf16_round(s.exp_avg_sq)
-    dV = s.P @ N
+    dV = N @ s.P.T if right else s.P @ N
     if hp.decompose:
         dM, s.mag_avg, s.mag_avg_sq = adam(M, s.mag_avg, s.mag_avg_sq, t,
                                            hp.beta1, hp.beta2, hp.adam_eps)

@@ -478,3 +478,42 @@ def test_bf16_state_step_stores_rounded_states():
         assert np.array_equal(o.bf16_round(x), x)
     np.testing.assert_array_equal(s16.W, o.bf16_round(s32.W))
     np.testing.assert_array_equal(s16.exp_avg, o.bf16_round(s32.exp_avg))
+
+
+def test_right_projection_is_the_transposed_left_step():
+    """GaLore's rule for a tall weight: without the decomposition the step
+    with the right projector Q on G (m x n) is the left-projector step on
+    G^T (n x m) with P = Q, transposed back (same Adam moments, transposed)."""
+    rng = _rng(61)
+    m, n, r = 12, 7, 3
+    hpR = o.Hparams(block_size=4, decompose=False, proj_rule="smaller")
+    hpL = o.Hparams(block_size=4, decompose=False)
+    W0 = rng.standard_normal((m, n)) * 0.02
+    Q = np.linalg.qr(rng.standard_normal((n, r)))[0]
+    sR, sL = o.init_state(W0, r, 4, P=Q, proj_rule="smaller"), o.init_state(W0.T, r, 4, P=Q)
+    for t in range(1, 4):
+        G = rng.standard_normal((m, n))
+        sR = o.step(sR, G, t, 1e-3, hpR, False)
+        sL = o.step(sL, G.T, t, 1e-3, hpL, False)
+    np.testing.assert_allclose(sR.W, sL.W.T, rtol=0, atol=1e-15)
+    np.testing.assert_allclose(sR.exp_avg, sL.exp_avg.T, rtol=0, atol=1e-15)
+
+
+def test_right_projector_refresh_and_full_rank():
+    """The smaller-side refresh takes the top-r right singular vectors (the
+    row space of V); with r = n the projector spans everything and, as with
+    P = I for the left rule, the direction branch is Adam on V itself."""
+    rng = _rng(62)
+    m, n, B = 10, 6, 3
+    G = rng.standard_normal((m, n))
+    hp = o.Hparams(block_size=B, proj_rule="smaller")
+    st = o.step(o.init_state(np.zeros((m, n)), 2, B, proj_rule="smaller"), G, 1, 1e-3, hp, True)
+    V = o.decompose(G, B)[1]
+    _, S, Vt = np.linalg.svd(V)
+    cos = np.abs(np.sum(st.P * Vt[:2].T, axis=0))
+    np.testing.assert_allclose(cos, 1.0, atol=1e-12)
+    # full rank, Q = I: R = V, so the step equals the P = I left-rule step on V's rows
+    st_r = o.step(o.init_state(np.zeros((m, n)), n, B, P=np.eye(n), proj_rule="smaller"), G, 1, 1e-3, hp, False)
+    np.testing.assert_allclose(st_r.extras["R"], V, atol=1e-15)
+    # square and wide weights keep the left projector under the smaller-side rule
+    assert not o.is_right(6, 6, "smaller") and not o.is_right(4, 9, "smaller") and o.is_right(9, 4, "smaller")
