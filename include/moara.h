@@ -54,6 +54,9 @@ extern "C" {
 #define MOARA_ERR_UNSUPPORTED     -9  /* valid request this build cannot serve    */
 
 /* ---- enums ------------------------------------------------------------- */
+#define MOARA_PROJ_LEFT    0
+#define MOARA_PROJ_SMALLER 1
+
 #define MOARA_DTYPE_F32    0   /* 32-bit IEEE float gradient                     */
 #define MOARA_DTYPE_BF16   1   /* bfloat16 gradient                              */
 
@@ -106,6 +109,12 @@ typedef struct moara_hparams {
                                updated in fp32 and stored rounded to nearest
                                even; tensor-core modules only (bf16 G, B >= 32);
                                the magnitude moments stay fp32. */
+    int   proj_rule;        /* MOARA_PROJ_LEFT (default): projector P (m x r) on
+                               the left of every weight; MOARA_PROJ_SMALLER:
+                               GaLore's rule, a right projector Q (n x r) for
+                               tall weights (m > n), R = V Q (m x r), dV = N Q^T;
+                               tensor-core modules only (the paper's memory
+                               model counts r * max(m, n) state entries, App. G). */
 } moara_hparams;
 
 /* One registered weight.  All pointers are device pointers, 16-byte aligned,
@@ -122,6 +131,8 @@ typedef struct moara_hparams {
  *   workspace   moara_workspace_bytes() bytes of scratch, private to the module
  * With hparams.state_dtype = MOARA_DTYPE_BF16, W, exp_avg and exp_avg_sq
  * point to bf16 arrays of the same shapes (the pointer types stay float*).
+ * With hparams.proj_rule = MOARA_PROJ_SMALLER and m > n, P and P_bf16 hold
+ * the right projector Q (n x r) and exp_avg / exp_avg_sq are m x r.
  */
 typedef struct moara_module_desc {
     int m, n, r;

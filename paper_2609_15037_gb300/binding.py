@@ -33,6 +33,8 @@ MOARA_REFRESH_SRC_G = 1
 MOARA_PREC_AUTO = 0
 MOARA_PREC_FP32 = 1
 MOARA_PREC_BF16_TC = 2
+MOARA_PROJ_LEFT = 0
+MOARA_PROJ_SMALLER = 1
 MOARA_DRULE_N = 0
 MOARA_DRULE_MAX = 1
 MODULE_BITS = {"q": 0, "k": 1, "v": 2, "o": 3, "gate": 4, "up": 5, "down": 6}
@@ -50,6 +52,7 @@ class moara_hparams(ctypes.Structure):
         ("seed", ctypes.c_uint64),
         ("clip_norm", ctypes.c_float),
         ("state_dtype", ctypes.c_int),
+        ("proj_rule", ctypes.c_int),
     ]
 
 

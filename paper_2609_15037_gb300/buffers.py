@@ -18,7 +18,7 @@ class ModuleBuffers:
     """Caller-owned buffers of one registered weight (layouts of moara.h)."""
 
     def __init__(self, m, n, r, block_size, grad_dtype="bf16", device="cuda",
-                 W0=None, with_bf16=True, state_dtype="f32"):
+                 W0=None, with_bf16=True, state_dtype="f32", right=False):
         self.m, self.n, self.r, self.block_size = m, n, r, block_size
         self.kb = -(-n // block_size)
         self.grad_dtype = grad_dtype
@@ -30,10 +30,15 @@ class ModuleBuffers:
             self.W = torch.zeros(m, n, **st)
         else:
             self.W = torch.as_tensor(W0).to(**st).contiguous().clone()
-        self.P = torch.zeros(m, r, **f32)
-        self.P_bf16 = torch.zeros(m, r, dtype=torch.int16, device=dev) if with_bf16 else None
-        self.exp_avg = torch.zeros(r, n, **st)
-        self.exp_avg_sq = torch.zeros(r, n, **st)
+        # left projector P (m x r) with r x n moments, or a right projector
+        # Q (n x r) with m x r moments
+        self.right = right
+        pr = n if right else m
+        mom = (m, r) if right else (r, n)
+        self.P = torch.zeros(pr, r, **f32)
+        self.P_bf16 = torch.zeros(pr, r, dtype=torch.int16, device=dev) if with_bf16 else None
+        self.exp_avg = torch.zeros(*mom, **st)
+        self.exp_avg_sq = torch.zeros(*mom, **st)
         self.mag_avg = torch.zeros(m, self.kb, **f32)
         self.mag_avg_sq = torch.zeros(m, self.kb, **f32)
         nbytes = B.moara_workspace_bytes(m, n, r, block_size)
@@ -101,7 +106,8 @@ class MoaraGroup:
         buf = ModuleBuffers(m, n, r, self.hp.block_size, grad_dtype,
                             f"cuda:{self.device}", W0=W0,
                             with_bf16=True,
-                            state_dtype="bf16" if self.hp.state_dtype == B.MOARA_DTYPE_BF16 else "f32")
+                            state_dtype="bf16" if self.hp.state_dtype == B.MOARA_DTYPE_BF16 else "f32",
+                            right=self.hp.proj_rule == B.MOARA_PROJ_SMALLER and m > n)
         mid = B.moara_init_module(self.ctx, buf.desc())
         self.modules.append(buf)
         self.ids.append(mid)

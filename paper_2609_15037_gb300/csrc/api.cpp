@@ -114,6 +114,8 @@ int check_hparams(moara_ctx* ctx, const moara_hparams* hp) {
     if (!std::isfinite(hp->clip_norm)) return fail(ctx, MOARA_ERR_INVALID_ARG, "clip_norm must be finite");
     if (hp->state_dtype != MOARA_DTYPE_F32 && hp->state_dtype != MOARA_DTYPE_BF16)
         return fail(ctx, MOARA_ERR_INVALID_ARG, "state_dtype must be MOARA_DTYPE_F32 or MOARA_DTYPE_BF16");
+    if (hp->proj_rule != MOARA_PROJ_LEFT && hp->proj_rule != MOARA_PROJ_SMALLER)
+        return fail(ctx, MOARA_ERR_INVALID_ARG, "unknown proj_rule");
     if (hp->state_dtype == MOARA_DTYPE_BF16 && hp->precision == MOARA_PREC_FP32)
         return fail(ctx, MOARA_ERR_UNSUPPORTED, "bf16 states run on the tensor-core path only");
     return MOARA_OK;
@@ -173,11 +175,14 @@ WsLayout workspace_layout(int m, int n, int r, int B) {
     const int kb = blocks_of(n, B);
     WsLayout w{};
     size_t off = 0;
-    w.off_N = off;   off = align_up(off + sizeof(float) * (size_t)r * n, 256);
+    // N: r x n, or m x r for a right projector (sized for either on a tall weight)
+    w.off_N = off;   off = align_up(off + sizeof(float) * (size_t)r * std::max(n, m), 256);
     w.off_dM = off;  off = align_up(off + sizeof(float) * (size_t)m * kb, 256);
     w.off_inv = off; off = align_up(off + sizeof(float) * (size_t)m * kb, 256);
     w.off_Vhi = off; off = align_up(off + sizeof(uint16_t) * (size_t)m * n, 256);
     w.off_Vlo = off; off = align_up(off + sizeof(uint16_t) * (size_t)m * n, 256);
+    w.off_Qt = 0;
+    if (m > n) { w.off_Qt = off; off = align_up(off + sizeof(uint16_t) * (size_t)r * n, 256); }   // Q^T
     w.total = off;
     return w;
 }
@@ -428,23 +433,27 @@ struct RefreshRunner {
     // out (n x l) = V^T X with X (m x l) in bf16; fp32 and/or bf16 output
     void tc_vt_times(const std::vector<uint16_t*>& X, const std::vector<float*>& out,
                      const std::vector<uint16_t*>& out_bf) {
-        std::vector<moara::TcGemmItem> g;
+        // V stored m x n is read MN-major; for a transposed item (V^T) the
+        // same product is V X with V read K-major
+        std::vector<moara::TcGemmItem> g[2];
         for (size_t i = 0; i < it.size(); ++i) {
             const auto& x = it[i];
-            g.push_back({x.Vhi, x.Vlo, X[i], out[i], out_bf[i], x.n, x.l, x.m, 0});
+            g[x.trans ? 1 : 0].push_back({x.Vhi, x.Vlo, X[i], out[i], out_bf[i], x.n, x.l, x.m, 0});
         }
-        tc_gemm(0, g);
+        tc_gemm(0, g[0]);
+        tc_gemm(1, g[1]);
     }
 
     // out (m x l) = V Z with Z (n x l) in bf16
     void tc_v_times(const std::vector<uint16_t*>& Z, const std::vector<float*>& out,
                     const std::vector<uint16_t*>& out_bf) {
-        std::vector<moara::TcGemmItem> g;
+        std::vector<moara::TcGemmItem> g[2];
         for (size_t i = 0; i < it.size(); ++i) {
             const auto& x = it[i];
-            g.push_back({x.Vhi, x.Vlo, Z[i], out[i], out_bf[i], x.m, x.l, x.n, 0});
+            g[x.trans ? 1 : 0].push_back({x.Vhi, x.Vlo, Z[i], out[i], out_bf[i], x.m, x.l, x.n, 0});
         }
-        tc_gemm(1, g);
+        tc_gemm(1, g[0]);
+        tc_gemm(0, g[1]);
     }
 
     // One shifted CholeskyQR pass on tensor cores: X_out = X_in R^-1 with
@@ -543,7 +552,7 @@ struct RefreshRunner {
         }
         if (src_v && tc) {
             std::vector<moara::TcSplitItem> sp;
-            for (auto& x : it) sp.push_back({x.G, x.Vhi_w, x.Vlo, x.m, x.n});
+            for (auto& x : it) sp.push_back({x.G, x.Vhi_w, x.Vlo, x.trans ? x.n : x.m, x.trans ? x.m : x.n});
             if (moara::tc_split_v(ctx->tc, sp.data(), n_it, hp.block_size, hp.decomp_eps, s, &ctx->launches) !=
                 MOARA_OK)
                 chk(cudaErrorLaunchFailure);
@@ -768,8 +777,14 @@ int do_refresh(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, 
                 const int gi = sel[end];
                 const int id = ids[gi];
                 const moara_module_desc& d = ctx->mods[id];
+                const bool tr = ctx->moddev[id].right != 0;   // right projector: the refresh of V^T
+                if (tr && kind == 0)
+                    return fail(ctx, MOARA_ERR_UNSUPPORTED,
+                                "module %d: a right projector is refreshed on tensor cores only (r + p a multiple of 8)",
+                                id);
+                const int rm = tr ? d.n : d.m, rn = tr ? d.m : d.n;
                 const int l = refresh_l(ctx, d.m, d.n, d.r);
-                const size_t need = align_up(moara::refresh_ws_bytes(d.m, d.n, d.r, l, hp.block_size, src_v), 256);
+                const size_t need = align_up(moara::refresh_ws_bytes(rm, rn, d.r, l, hp.block_size, src_v), 256);
                 if (used + need > ctx->refresh_ws_bytes) {
                     if (rr.it.empty())
                         return fail(ctx, MOARA_ERR_WORKSPACE,
@@ -778,9 +793,10 @@ int do_refresh(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, 
                     break;
                 }
                 moara::RefreshItem x{};
-                x.m = d.m; x.n = d.n; x.r = d.r; x.l = l; x.kb = blocks_of(d.n, hp.block_size);
+                x.m = rm; x.n = rn; x.r = d.r; x.l = l; x.kb = blocks_of(d.n, hp.block_size);
+                x.trans = tr ? 1 : 0;
                 x.dtype = d.grad_dtype; x.G = G[gi];
-                moara::refresh_carve(x, static_cast<char*>(ctx->refresh_ws) + used, d.m, d.n, d.r, l,
+                moara::refresh_carve(x, static_cast<char*>(ctx->refresh_ws) + used, rm, rn, d.r, l,
                                      hp.block_size, src_v);
                 x.P = d.P; x.Pb = d.P_bf16;
                 const uint64_t cnt = static_cast<uint64_t>(ctx->refresh_count[id]++);
@@ -800,6 +816,11 @@ int do_refresh(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, 
                 ++end;
             }
             rr.run();
+            // a right projector's K2 operand is Q^T
+            for (size_t q = start; q < end && rr.err == cudaSuccess; ++q) {
+                const moara::ModDev& md = ctx->moddev[ids[sel[q]]];
+                if (md.right) rr.chk(moara::tc_transpose_bf16(md.Pb, md.ws_Qt, md.n, md.r, s, &ctx->launches));
+            }
             if (rr.err != cudaSuccess) {
                 if (kind == 1 && ctx->tc != nullptr)
                     return fail(ctx, MOARA_ERR_CUDA, "tensor-core refresh: %s", moara::tc_last_error(ctx->tc));
@@ -1073,6 +1094,14 @@ int moara_init_module(moara_ctx* ctx, const moara_module_desc* d, int* module_id
         return fail(ctx, MOARA_ERR_ALIGN, "P_bf16 is not 16-byte aligned");
     if (ctx->hp.precision == MOARA_PREC_BF16_TC && d->P_bf16 == nullptr)
         return fail(ctx, MOARA_ERR_INVALID_ARG, "P_bf16 is required with precision BF16_TC");
+    const bool right = ctx->hp.proj_rule == MOARA_PROJ_SMALLER && d->m > d->n;
+    if (right && (d->grad_dtype != MOARA_DTYPE_BF16 || d->P_bf16 == nullptr || ctx->tc == nullptr ||
+                  ctx->hp.precision == MOARA_PREC_FP32 ||
+                  !moara::tc_supported(d->m, d->n, d->r, ctx->hp.block_size, d->grad_dtype, ctx->hp.decompose,
+                                       ctx->hp.state_dtype)))
+        return fail(ctx, MOARA_ERR_UNSUPPORTED,
+                    "a right projector (m > n under MOARA_PROJ_SMALLER) needs the tensor-core path: bf16 gradient, "
+                    "P_bf16, n and r multiples of 8");
     if (ctx->hp.state_dtype == MOARA_DTYPE_BF16 &&
         (d->grad_dtype != MOARA_DTYPE_BF16 || d->P_bf16 == nullptr || ctx->tc == nullptr ||
          !moara::tc_supported(d->m, d->n, d->r, ctx->hp.block_size, d->grad_dtype, ctx->hp.decompose,
@@ -1103,6 +1132,7 @@ int moara_init_module(moara_ctx* ctx, const moara_module_desc* d, int* module_id
     moara::ModDev md{};
     md.m = d->m; md.n = d->n; md.r = d->r; md.kb = blocks_of(d->n, ctx->hp.block_size);
     md.dtype = d->grad_dtype;
+    md.right = right ? 1 : 0;
     md.W = d->W; md.P = d->P; md.Pb = d->P_bf16;
     md.exp_avg = d->exp_avg; md.exp_avg_sq = d->exp_avg_sq;
     md.mag_avg = d->mag_avg; md.mag_avg_sq = d->mag_avg_sq;
@@ -1112,6 +1142,7 @@ int moara_init_module(moara_ctx* ctx, const moara_module_desc* d, int* module_id
     md.ws_inv = reinterpret_cast<float*>(ws + wl.off_inv);
     md.ws_Vhi = reinterpret_cast<uint16_t*>(ws + wl.off_Vhi);
     md.ws_Vlo = reinterpret_cast<uint16_t*>(ws + wl.off_Vlo);
+    md.ws_Qt = wl.off_Qt != 0 ? reinterpret_cast<uint16_t*>(ws + wl.off_Qt) : nullptr;
     const int id = static_cast<int>(ctx->mods.size());
     cudaError_t e = cudaMemcpy(ctx->d_mods + id, &md, sizeof(md), cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "module table copy");
@@ -1135,8 +1166,10 @@ int moara_load_projector(moara_ctx* ctx, int module_id, const float* P_src, void
     if (!aligned16(P_src)) return fail(ctx, MOARA_ERR_ALIGN, "P_src is not 16-byte aligned");
     DeviceGuard g(ctx->device);
     const moara::ModDev& md = ctx->moddev[module_id];
-    cudaError_t e = moara::launch_f32_to_bf16(P_src, md.P, md.Pb, (long long)md.m * md.r,
-                                              static_cast<cudaStream_t>(stream), &ctx->launches);
+    const int rows = md.right ? md.n : md.m;      // P (m x r) or the right projector Q (n x r)
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = moara::launch_f32_to_bf16(P_src, md.P, md.Pb, (long long)rows * md.r, s, &ctx->launches);
+    if (e == cudaSuccess && md.right) e = moara::tc_transpose_bf16(md.Pb, md.ws_Qt, md.n, md.r, s, &ctx->launches);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "projector copy");
     return MOARA_OK;
 }
@@ -1146,7 +1179,9 @@ int moara_refresh_workspace_bytes(const moara_ctx* ctx, int m, int n, int r, siz
     if (m < 1 || n < 1) return MOARA_ERR_SHAPE;
     if (r < 1 || r > std::min(m, n)) return MOARA_ERR_RANK;
     const int src_v = (ctx->hp.refresh_src == MOARA_REFRESH_SRC_V && ctx->hp.decompose) ? 1 : 0;
-    *out = align_up(moara::refresh_ws_bytes(m, n, r, refresh_l(ctx, m, n, r), ctx->hp.block_size, src_v), 256);
+    const bool tr = ctx->hp.proj_rule == MOARA_PROJ_SMALLER && m > n;   // refresh of V^T
+    *out = align_up(moara::refresh_ws_bytes(tr ? n : m, tr ? m : n, r, refresh_l(ctx, m, n, r), ctx->hp.block_size,
+                                            src_v), 256);
     return MOARA_OK;
 }
 

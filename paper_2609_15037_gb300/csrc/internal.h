@@ -20,7 +20,7 @@ constexpr int kMaxGroup = 224;
 struct ModDev {
     int m, n, r, kb;        // kb = ceil(n / B)
     int dtype;              // MOARA_DTYPE_*
-    int pad_;
+    int right;              // 1: right projector Q (n x r) in P / Pb, moments m x r
     float* W;
     float* P;
     uint16_t* Pb;
@@ -33,11 +33,12 @@ struct ModDev {
     float* ws_inv;          // m x kb inverse block scales 1 / (||g|| + eps)
     uint16_t* ws_Vhi;       // m x n direction matrix V in bf16 (tensor-core path)
     uint16_t* ws_Vlo;       // m x n bf16 residual V - V_hi (first Adam step)
+    uint16_t* ws_Qt;        // r x n bf16 transpose of a right projector (tall modules), or null
 };
 
 // Workspace carve-up of one module (byte offsets, 256-byte aligned).
 struct WsLayout {
-    size_t off_N, off_dM, off_inv, off_Vhi, off_Vlo, total;
+    size_t off_N, off_dM, off_inv, off_Vhi, off_Vlo, off_Qt, total;   // off_Qt = 0: none
 };
 WsLayout workspace_layout(int m, int n, int r, int B);
 
@@ -164,6 +165,7 @@ struct RefreshItem {
     uint16_t* Pb;     // m x r bf16 destination (may be null)
     uint64_t key;     // RNG key (seed, module, refresh count)
     int tc;           // products with V on tensor cores
+    int trans;        // right projector: the refresh runs on V^T (m, n above are V's n, m)
     const uint16_t* Vhi;    // m x n bf16 planes of V (or G) for the tensor-core products
     uint16_t* Vhi_w;        // writable view of Vhi when V is formed here (null otherwise)
     uint16_t* Vlo;          // residual plane, or null when Vhi is exact

@@ -41,6 +41,7 @@ constexpr int kMaps = 8;                      // tensor maps per module
 
 struct TcMod {
     int m, n, r, kb;
+    int right;        // right projector Q (n x r): K1 computes R = V Q (m x r)
     uint16_t* Vhi;    // m x n bf16 direction matrix (written by K0)
     uint16_t* Vlo;    // m x n bf16 residual (first Adam step)
     float* W;
@@ -357,7 +358,8 @@ k1_project(const __grid_constant__ K1Params p) {
                 const CUtensorMap* vmap = p.decompose ? &p.maps[tl.mod * kMaps + 4] : &p.gmap[tl.slot];
                 const CUtensorMap* lmap = &p.maps[tl.mod * kMaps + 5];
                 const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
-                const int nk = (md.m + K1_BK - 1) / K1_BK;
+                const bool right = md.right != 0;
+                const int nk = ((right ? md.n : md.m) + K1_BK - 1) / K1_BK;
                 for (int kb = 0; kb < nk; ++kb) {
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
@@ -366,13 +368,24 @@ k1_project(const __grid_constant__ K1Params p) {
                     if (crank == 0) ptx::mbar_arrive_expect_tx(own, 2 * STAGE_BYTES);
                     const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
                     const uint32_t b = a + K1_A_BYTES;
+                    if (!right) {
 #pragma unroll
-                    for (int c = 0; c < 2; ++c) ptx::tma_load_2d_pair(a + c * 8192, pmap, fb, r0 + 64 * c, kb * K1_BK);
+                        for (int c = 0; c < 2; ++c) ptx::tma_load_2d_pair(a + c * 8192, pmap, fb, r0 + 64 * c, kb * K1_BK);
 #pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        const int c = 2 * crank + h;
-                        ptx::tma_load_2d_pair(b + h * 8192, vmap, fb, n0 + 64 * c, kb * K1_BK);
-                        if (HILO) ptx::tma_load_2d_pair(b + K1_B_BYTES + h * 8192, lmap, fb, n0 + 64 * c, kb * K1_BK);
+                        for (int h = 0; h < 2; ++h) {
+                            const int c = 2 * crank + h;
+                            ptx::tma_load_2d_pair(b + h * 8192, vmap, fb, n0 + 64 * c, kb * K1_BK);
+                            if (HILO) ptx::tma_load_2d_pair(b + K1_B_BYTES + h * 8192, lmap, fb, n0 + 64 * c, kb * K1_BK);
+                        }
+                    } else {
+                        // A: this CTA's 128 rows of V (64 columns, K-major; V_lo
+                        // in the third slot at the first step); B: this CTA's
+                        // 128 ranks of Q, two 64-rank chunks (MN-major)
+                        ptx::tma_load_2d_pair(a, vmap, fb, kb * K1_BK, r0);
+                        if (HILO) ptx::tma_load_2d_pair(b + K1_B_BYTES, lmap, fb, kb * K1_BK, r0);
+#pragma unroll
+                        for (int h = 0; h < 2; ++h)
+                            ptx::tma_load_2d_pair(b + h * 8192, pmap, fb, n0 + 64 * (2 * crank + h), kb * K1_BK);
                     }
                     issued |= 1u << stage;
                     last_par = (last_par & ~(1u << stage)) | (phase << stage);
@@ -390,7 +403,8 @@ k1_project(const __grid_constant__ K1Params p) {
             // M = 256 (both CTAs' rank tiles), N = 256, K = 16 per MMA; the
             // full barrier of a stage counts both CTAs' copies
             if (lane == 0) {
-                constexpr uint32_t idesc = ptx::idesc_bf16(256, K1_BN, 1, 1);
+                constexpr uint32_t idesc_l = ptx::idesc_bf16(256, K1_BN, 1, 1);   // A MN-major (P^T)
+                constexpr uint32_t idesc_r = ptx::idesc_bf16(256, K1_BN, 0, 1);   // A K-major (V rows)
                 int stage = 0;
                 uint32_t phase = 0;
                 int buf = 0;
@@ -399,7 +413,9 @@ k1_project(const __grid_constant__ K1Params p) {
                 for (int t = t_begin; t < t_end && ok; ++t) {
                     const TcTile tl = p.tiles[t];
                     const TcMod& md = p.mods[tl.mod];
-                    const int nk = (md.m + K1_BK - 1) / K1_BK;
+                    const bool right = md.right != 0;
+                    const uint32_t idesc = right ? idesc_r : idesc_l;
+                    const int nk = ((right ? md.n : md.m) + K1_BK - 1) / K1_BK;
                     if (!ptx::mbar_wait_cluster(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
                                                 MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
                     ptx::tc_fence_after();
@@ -412,12 +428,21 @@ k1_project(const __grid_constant__ K1Params p) {
                         const uint32_t b = a + K1_A_BYTES;
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk) {
-                            const uint64_t adesc = ptx::smem_desc_sw128(a + kk * 2048, 8192, 1024);
                             const uint64_t bdesc = ptx::smem_desc_sw128(b + kk * 2048, 8192, 1024);
-                            ptx::mma2_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
-                            if (HILO) {   // P^T V_lo: the bf16 rounding residual of V
-                                const uint64_t ldesc = ptx::smem_desc_sw128(b + K1_B_BYTES + kk * 2048, 8192, 1024);
-                                ptx::mma2_f16(d0, adesc, ldesc, idesc, 1);
+                            if (!right) {
+                                const uint64_t adesc = ptx::smem_desc_sw128(a + kk * 2048, 8192, 1024);
+                                ptx::mma2_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
+                                if (HILO) {   // P^T V_lo: the bf16 rounding residual of V
+                                    const uint64_t ldesc = ptx::smem_desc_sw128(b + K1_B_BYTES + kk * 2048, 8192, 1024);
+                                    ptx::mma2_f16(d0, adesc, ldesc, idesc, 1);
+                                }
+                            } else {
+                                const uint64_t adesc = ptx::smem_desc_sw128(a + kk * 32, 16, 1024);
+                                ptx::mma2_f16(d0, adesc, bdesc, idesc, (kb | kk) != 0);
+                                if (HILO) {   // V_lo Q
+                                    const uint64_t ldesc = ptx::smem_desc_sw128(b + K1_B_BYTES + kk * 32, 16, 1024);
+                                    ptx::mma2_f16(d0, ldesc, bdesc, idesc, 1);
+                                }
                             }
                         }
                         ptx::mma2_commit_mc(ptx::smem_u32(&ctl->empty[stage]), 0x3);
@@ -444,7 +469,8 @@ k1_project(const __grid_constant__ K1Params p) {
                 const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 6];
                 const CUtensorMap* smap = &p.maps[tl.mod * kMaps + 7];
                 const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
-                const int nc = min(K1_BN / MC, (md.n - n0 + MC - 1) / MC);
+                const int cols = md.right ? md.r : md.n;    // R is r x n, or m x r (right projector)
+                const int nc = min(K1_BN / MC, (cols - n0 + MC - 1) / MC);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % MSLOTS;
                     const uint32_t ph = (g / MSLOTS) & 1;
@@ -475,7 +501,8 @@ k1_project(const __grid_constant__ K1Params p) {
                 const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 6];
                 const CUtensorMap* smap = &p.maps[tl.mod * kMaps + 7];
                 const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
-                const int nc = min(K1_BN / MC, (md.n - n0 + MC - 1) / MC);
+                const int cols = md.right ? md.r : md.n;    // R is r x n, or m x r (right projector)
+                const int nc = min(K1_BN / MC, (cols - n0 + MC - 1) / MC);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % MSLOTS;
                     const uint32_t ph = (g / MSLOTS) & 1;
@@ -510,7 +537,8 @@ k1_project(const __grid_constant__ K1Params p) {
         for (int t = t_begin; t < t_end && ok; ++t) {
             const TcTile tl = p.tiles[t];
             const TcMod& md = p.mods[tl.mod];
-            const int rr = md.r, nn = md.n;
+            // R (and the moments, N) is r x n, or m x r with a right projector
+            const int rr = md.right ? md.m : md.r, nn = md.right ? md.r : md.n;
             uint16_t* const nb_p = md.Nb;
             const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
             const int a = r0 + il;
@@ -1510,15 +1538,35 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
     t.Nb = reinterpret_cast<uint16_t*>(md.ws_N);
     t.dM = md.ws_dM;
     t.Pb = md.Pb;
+    t.right = md.right;
     CUtensorMap* mp = &st->maps[kMaps * id];
-    if (!encode_bf16_2d(st->encode, &mp[0], md.Pb, md.r, md.m, 64, 64) ||
-        !encode_bf16_2d(st->encode, &mp[1], md.Pb, md.r, md.m, 64, 128) ||
-        !encode_bf16_2d(st->encode, &mp[2], t.Nb, md.n, md.r, 64, 64) ||
-        !encode_2d(st->encode, &mp[3], sdt, ses, md.W, md.n, md.m, scols, K2_BM) ||
-        !encode_bf16_2d(st->encode, &mp[4], t.Vhi, md.n, md.m, 64, 64) ||
-        !encode_bf16_2d(st->encode, &mp[5], t.Vlo, md.n, md.m, 64, 64) ||
-        !encode_2d(st->encode, &mp[6], sdt, ses, md.exp_avg, md.n, md.r, scols, K1_BM) ||
-        !encode_2d(st->encode, &mp[7], sdt, ses, md.exp_avg_sq, md.n, md.r, scols, K1_BM)) {
+    bool ok;
+    if (!md.right) {
+        // K1: A = P^T (MN-major chunks of P), B = V (MN-major), moments r x n;
+        // K2: A = P rows (K-major), B = N (MN-major)
+        ok = encode_bf16_2d(st->encode, &mp[0], md.Pb, md.r, md.m, 64, 64) &&
+             encode_bf16_2d(st->encode, &mp[1], md.Pb, md.r, md.m, 64, 128) &&
+             encode_bf16_2d(st->encode, &mp[2], t.Nb, md.n, md.r, 64, 64) &&
+             encode_bf16_2d(st->encode, &mp[4], t.Vhi, md.n, md.m, 64, 64) &&
+             encode_bf16_2d(st->encode, &mp[5], t.Vlo, md.n, md.m, 64, 64) &&
+             encode_2d(st->encode, &mp[6], sdt, ses, md.exp_avg, md.n, md.r, scols, K1_BM) &&
+             encode_2d(st->encode, &mp[7], sdt, ses, md.exp_avg_sq, md.n, md.r, scols, K1_BM);
+    } else {
+        // right projector Q (n x r): K1 computes R = V Q with A = V rows
+        // (K-major, 128 rows x 64 columns) and B = Q (MN-major chunks), moments
+        // m x r; K2 computes dV = N Q^T with A = N rows (K-major) and
+        // B = Q^T (r x n, MN-major)
+        ok = md.ws_Qt != nullptr &&
+             encode_bf16_2d(st->encode, &mp[0], md.Pb, md.r, md.n, 64, 64) &&
+             encode_bf16_2d(st->encode, &mp[1], t.Nb, md.r, md.m, 64, 128) &&
+             encode_bf16_2d(st->encode, &mp[2], md.ws_Qt, md.n, md.r, 64, 64) &&
+             encode_bf16_2d(st->encode, &mp[4], t.Vhi, md.n, md.m, 64, 128) &&
+             encode_bf16_2d(st->encode, &mp[5], t.Vlo, md.n, md.m, 64, 128) &&
+             encode_2d(st->encode, &mp[6], sdt, ses, md.exp_avg, md.r, md.m, scols, K1_BM) &&
+             encode_2d(st->encode, &mp[7], sdt, ses, md.exp_avg_sq, md.r, md.m, scols, K1_BM);
+    }
+    ok = ok && encode_2d(st->encode, &mp[3], sdt, ses, md.W, md.n, md.m, scols, K2_BM);
+    if (!ok) {
         st->err = "cuTensorMapEncodeTiled failed";
         return MOARA_ERR_CUDA;
     }
@@ -1601,12 +1649,14 @@ static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
         const TcMod& md = st->mods[ids[slot]];
         // column tiles outer, rank pairs inner: clusters that start together
         // share the V panel of one column tile in L2
-        const int nt = (md.n + K1_BN - 1) / K1_BN, rt = (md.r + K1_BM - 1) / K1_BM;
+        // R: r x n (K = m), or m x r (K = n) with a right projector
+        const int Rr = md.right ? md.m : md.r, Rc = md.right ? md.r : md.n, Rk = md.right ? md.n : md.m;
+        const int nt = (Rc + K1_BN - 1) / K1_BN, rt = (Rr + K1_BM - 1) / K1_BM;
         for (int j = 0; j < nt; ++j)
             for (int i = 0; i < (rt + 1) / 2; ++i) {
-                const int rows = std::min(K1_BM, md.r - 2 * i * K1_BM);
-                const double mma = 8.0 * md.m;
-                const double epi = 0.66 * rows * std::min(K1_BN, md.n - j * K1_BN);
+                const int rows = std::min(K1_BM, Rr - 2 * i * K1_BM);
+                const double mma = 8.0 * Rk;
+                const double epi = 0.66 * rows * std::min(K1_BN, Rc - j * K1_BN);
                 k1.push_back({ids[slot], static_cast<int>(slot), i, j});
                 c1.push_back(std::max(mma, epi));
             }
@@ -1819,7 +1869,9 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             if (!dec) {
                 for (int k = 0; k < b - a; ++k) {
                     const TcMod& md = st->mods[chunk[k]];
-                    if (!encode_bf16_2d(st->encode, &p1.gmap[k], G[c0 + a + k], md.n, md.m, 64, 64)) {
+                    // G as K1's B operand (64 x 64 chunks), or as its A operand
+                    // (128 rows x 64 columns) for a right projector
+                    if (!encode_bf16_2d(st->encode, &p1.gmap[k], G[c0 + a + k], md.n, md.m, 64, md.right ? 128 : 64)) {
                         st->err = "cuTensorMapEncodeTiled failed for a gradient";
                         return MOARA_ERR_CUDA;
                     }
@@ -1968,6 +2020,14 @@ __global__ void __launch_bounds__(256) k_transpose_pad_bf16(const uint16_t* __re
     }
 }
 
+cudaError_t tc_transpose_bf16(const uint16_t* in, uint16_t* out, int rows, int cols, cudaStream_t s,
+                              int64_t* launches) {
+    const int tiles = ((rows + 31) / 32) * ((cols + 31) / 32);
+    k_transpose_pad_bf16<<<std::max(1, std::min(tiles, 152 * 8)), 256, 0, s>>>(in, out, rows, cols, rows);
+    ++*launches;
+    return cudaGetLastError();
+}
+
 __global__ void k_align_finish(const double* acc, float* S, int n) {
     const int q = blockIdx.x * blockDim.x + threadIdx.x;
     if (q >= n) return;
@@ -1986,7 +2046,7 @@ int tc_alignment(TcState* st, const moara_hparams& hp, int n_mod, const int* ids
     for (int q = 0; q < n_mod; ++q) {
         const int id = ids[q];
         const TcMod* md = (id >= 0 && id < static_cast<int>(st->mods.size())) ? &st->mods[id] : nullptr;
-        if (md == nullptr || md->Vhi == nullptr || md->Vlo == nullptr || md->Pb == nullptr) {
+        if (md == nullptr || md->Vhi == nullptr || md->Vlo == nullptr || md->Pb == nullptr || md->right) {
             st->err = "alignment: module is not on the tensor-core path";
             return MOARA_ERR_UNSUPPORTED;
         }

@@ -77,6 +77,10 @@ struct TcSplitItem {
 int tc_split_v(TcState* st, const TcSplitItem* items, int count, int B, float decomp_eps, cudaStream_t s,
                int64_t* launches);
 
+// out (cols x rows, bf16) = in^T for in (rows x cols, bf16, row-major)
+cudaError_t tc_transpose_bf16(const uint16_t* in, uint16_t* out, int rows, int cols, cudaStream_t s,
+                              int64_t* launches);
+
 const char* tc_last_error(const TcState* st);
 
 }  // namespace moara

@@ -51,7 +51,8 @@ def test_hparams_struct_matches_header(M):
     the right fields, including the last one."""
     hp = M.moara_default_hparams()
     assert hp.block_size == 128 and hp.power_iters == 2 and hp.oversample == 16
-    assert ctypes.sizeof(M.binding.moara_hparams) == 72
+    assert ctypes.sizeof(M.binding.moara_hparams) == 80
+    assert hp.proj_rule == M.MOARA_PROJ_LEFT and hp.state_dtype == M.MOARA_DTYPE_F32
 
 
 def test_flatten_shape_through_the_abi(M):
