@@ -115,24 +115,32 @@ class Clocks:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
-def _algorithmic(mods, B, sb=4):
+def _right(md, rule):
+    """GaLore's smaller-side rule: a right projector for a tall weight."""
+    return rule == "smaller" and md.m > md.n
+
+
+def _algorithmic(mods, B, sb=4, rule="left"):
     """Algorithmic bytes and flops of one step over `mods` (Module list);
-    sb: bytes per element of W and the direction moments (4 or 2)."""
+    sb: bytes per element of W and the direction moments (4 or 2); rule:
+    projection side ("left", or "smaller": right projector when m > n)."""
     tot_b = tot_f = 0
     per = {"project": [0, 0], "backproject": [0, 0]}
     for md in mods:
         m, n, r = md.m, md.n, md.r
         k = -(-n // B)
+        # R is r x n, or m x r with a right projector (n x r)
+        rc, pr = (m, n) if _right(md, rule) else (n, m)
         # minimum traffic of one fused pass: G read (bf16), W read+write,
         # direction moments read+write, P read once (bf16), magnitude moments
-        tot_b += 2 * m * n + 2 * sb * m * n + 4 * sb * r * n + 2 * m * r + 16 * m * k
+        tot_b += 2 * m * n + 2 * sb * m * n + 4 * sb * r * rc + 2 * pr * r + 16 * m * k
         tot_f += 4 * m * r * n
         per["project"][1] += 2 * m * r * n
         per["backproject"][1] += 2 * m * r * n
     return tot_b, tot_f, per
 
 
-def _kernel_bytes(mods, B, tc, sb=4):
+def _kernel_bytes(mods, B, tc, sb=4, rule="left"):
     """Algorithmic bytes per step of each step kernel as built.
 
     tensor-core path: tc_decompose reads G (bf16), writes V (bf16) and updates
@@ -147,9 +155,10 @@ def _kernel_bytes(mods, B, tc, sb=4):
         m, n, r = md.m, md.n, md.r
         k = -(-n // B)
         if tc:
+            rc, pr = (m, n) if _right(md, rule) else (n, m)   # R: r x rc; projector: pr x r
             add = {"tc_decompose": 2 * m * n + 2 * m * n + 20 * m * k,
-                   "tc_project": 2 * m * n + 2 * m * r + 4 * sb * r * n + 2 * r * n,
-                   "tc_backproject": 2 * sb * m * n + 2 * r * n + 2 * m * r + 4 * m * k}
+                   "tc_project": 2 * m * n + 2 * pr * r + 4 * sb * r * rc + 2 * r * rc,
+                   "tc_backproject": 2 * sb * m * n + 2 * r * rc + 2 * pr * r + 4 * m * k}
         else:
             add = {"decompose": 2 * m * n + 20 * m * k + 4 * m * k,
                    "project": 2 * m * n + 4 * m * k + 4 * m * r + 16 * r * n + 4 * r * n,
@@ -207,6 +216,7 @@ def run_gpu(args):
     hp.clip_norm = args.clip_norm
     hp.state_dtype = M.MOARA_DTYPE_BF16 if args.state_dtype == "bf16" else M.MOARA_DTYPE_F32
     sbytes = 2 if args.state_dtype == "bf16" else 4
+    hp.proj_rule = M.MOARA_PROJ_SMALLER if args.proj_rule == "smaller" else M.MOARA_PROJ_LEFT
     g = M.MoaraGroup(hp, device=local, refresh_workspace_bytes=int(args.refresh_ws_gb * (1 << 30)))
     stream = torch.cuda.current_stream(dev)
     grads = []
@@ -273,13 +283,16 @@ def run_gpu(args):
     # alignment diagnostic S(W, t) over every module (a profiling-step call,
     # outside the step; it reuses the modules' workspaces, which the next
     # step rewrites): one untimed call, then the mean of three
-    S_dev = torch.empty(len(ids), dtype=torch.float32, device=dev)
-    M.moara_alignment(g.ctx, ids, gptr, S_dev.data_ptr(), cs)
+    # (modules with a left projector: the diagnostic is defined for P P^T V)
+    a_sel = [k for k, md in enumerate(mods) if not _right(md, args.proj_rule)]
+    a_ids, a_ptr = [ids[k] for k in a_sel], [gptr[k] for k in a_sel]
+    S_dev = torch.empty(max(1, len(a_ids)), dtype=torch.float32, device=dev)
+    M.moara_alignment(g.ctx, a_ids, a_ptr, S_dev.data_ptr(), cs)
     a0 = torch.cuda.Event(enable_timing=True)
     a1 = torch.cuda.Event(enable_timing=True)
     a0.record(stream)
     for _ in range(3):
-        M.moara_alignment(g.ctx, ids, gptr, S_dev.data_ptr(), cs)
+        M.moara_alignment(g.ctx, a_ids, a_ptr, S_dev.data_ptr(), cs)
     a1.record(stream)
     torch.cuda.synchronize()
     align_ms = a0.elapsed_time(a1) / 3
@@ -336,13 +349,13 @@ def run_gpu(args):
     h2d_gbs = h2d / (c0.elapsed_time(c1) * 1e-3) / 1e9
 
     hbm, bf16_peak, bf16_sus, peak_src = _peaks()
-    alg_bytes, alg_flops, _ = _algorithmic(mods, B, sbytes)
+    alg_bytes, alg_flops, _ = _algorithmic(mods, B, sbytes, args.proj_rule)
     total_ms = step_ms + refresh_ms / 200.0
     roof_ms = max(alg_bytes / (hbm * 1e9), alg_flops / (bf16_sus * 1e12)) * 1e3
 
     # dominant kernel
     used_tc = prof["tc_project"][1] > 0
-    kbytes = _kernel_bytes(mods, B, used_tc, sbytes)
+    kbytes = _kernel_bytes(mods, B, used_tc, sbytes, args.proj_rule)
     names = ["decompose", "project", "backproject", "tc_decompose", "tc_project", "tc_backproject"]
     dom = max(names, key=lambda k: prof[k][0])
     dom_ms = prof[dom][0] / max(prof[dom][1], 1)
@@ -360,7 +373,8 @@ def run_gpu(args):
         # the kernel's own roof is the tensor pipe: its flops at the sustained
         # bf16 rate take longer than its bytes at the copy bandwidth
         achieved = flops_dom / (dom_ms * 1e-3) / 1e12
-        tr = _traffic(dom, args.workload) if sbytes == 4 else None   # counters taken with fp32 states
+        # the counters were taken with fp32 states and left projectors
+        tr = _traffic(dom, args.workload) if (sbytes == 4 and args.proj_rule == "left") else None
         roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": bf16_sus,
                 "unit": "TFLOP/s", "frac": round(achieved / bf16_sus, 4),
                 "traffic": None if tr is None else int(tr / n_launch_per_step),
@@ -369,7 +383,8 @@ def run_gpu(args):
     else:
         by = kbytes[dom] / n_launch_per_step
         achieved = by / (dom_ms * 1e-3) / 1e9
-        tr = _traffic(dom, args.workload) if sbytes == 4 else None   # counters taken with fp32 states
+        # the counters were taken with fp32 states and left projectors
+        tr = _traffic(dom, args.workload) if (sbytes == 4 and args.proj_rule == "left") else None
         roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
                 "frac": round(achieved / hbm, 4), "traffic": None if tr is None else int(tr / n_launch_per_step),
                 "kernel": dom, "peak_source": f"hbm_gbs ({peak_src})"}
@@ -407,7 +422,8 @@ def run_gpu(args):
                    "ranks": "q/k 512, v/o/gate/up 1024, down 2048",
                    "l2": "inputs larger than L2 (no flush needed)",
                    "parallelism": "replicas" if world > 1 else "single GPU",
-                   "clip_norm": args.clip_norm, "state_dtype": args.state_dtype},
+                   "clip_norm": args.clip_norm, "state_dtype": args.state_dtype,
+                   "proj_rule": args.proj_rule},
         "step_ms_no_refresh": round(step_ms, 4),
         "clip_norm_ms": round(prof["clip_norm"][0] / args.steps, 4) if prof["clip_norm"][1] else None,
         "refresh_ms": round(refresh_ms, 2), "refresh_amortised_ms": round(refresh_ms / 200.0, 4),
@@ -423,10 +439,11 @@ def run_gpu(args):
                 "h2d_gbs_link": round(h2d_gbs, 1),
                 "step_ms_median": round(e2e_median, 3), "steps": e2e_steps,
                 "path": "moara_step_grouped_host" if via_host_call else "host-to-device copies + moara_step_grouped"},
-        "alignment": {"ms": round(align_ms, 3), "modules": len(ids),
-                      "flops": int(4 * sum(md.m * md.n * md.r for md in mods)),
-                      "tflops": round(4 * sum(md.m * md.n * md.r for md in mods) / (align_ms * 1e-3) / 1e12, 1),
-                      "S_mean": round(float(S_host.mean()), 4)},
+        "alignment": {"ms": round(align_ms, 3), "modules": len(a_ids),
+                      "flops": int(4 * sum(mods[k].m * mods[k].n * mods[k].r for k in a_sel)),
+                      "tflops": round(4 * sum(mods[k].m * mods[k].n * mods[k].r for k in a_sel)
+                                      / max(align_ms * 1e-3, 1e-9) / 1e12, 1),
+                      "S_mean": round(float(S_host[:len(a_ids)].mean()), 4) if a_ids else None},
         "gpu_launches": int(launches),
         "device_status": status | e2e_status,
         "clocks": clk,
@@ -440,17 +457,18 @@ def run_gpu(args):
         torch.distributed.destroy_process_group()
 
 
-def _oracle_layer_sample(wl, layer_modules, seed=0):
+def _oracle_layer_sample(wl, layer_modules, seed=0, rule="left", state_bf16=False):
     """Oracle step on the seven modules of one decoder layer (float64)."""
     import numpy as np
     from oracle import moara_ref as o
-    hp = o.Hparams(block_size=wl["block_size"], adam_eps=wl["adam_eps"])
+    hp = o.Hparams(block_size=wl["block_size"], adam_eps=wl["adam_eps"], proj_rule=rule, state_bf16=state_bf16)
     rng = np.random.default_rng(seed)
     states, grads = [], []
     for md in layer_modules:
         W = rng.standard_normal((md.m, md.n)) * 0.02
-        P = np.linalg.qr(rng.standard_normal((md.m, md.r)))[0]
-        states.append(o.init_state(W, md.r, wl["block_size"], P=P))
+        right = _right(md, rule)
+        P = np.linalg.qr(rng.standard_normal((md.n if right else md.m, md.r)))[0]
+        states.append(o.init_state(W, md.r, wl["block_size"], P=P, proj_rule=rule))
         grads.append(rng.standard_normal((md.m, md.n)) * 1e-3)
     return states, grads, hp
 
@@ -464,7 +482,8 @@ def cpu_baseline(args, budget_s=20.0):
     wl = synth.workload(args.workload)
     layer = [md for md in wl["modules"] if md.name.startswith("layer0.")]
     layers = len(wl["modules"]) // len(layer)
-    states, grads, hp = _oracle_layer_sample(wl, layer)
+    states, grads, hp = _oracle_layer_sample(wl, layer, rule=getattr(args, "proj_rule", "left"),
+                                             state_bf16=getattr(args, "state_dtype", "f32") == "bf16")
     times = []
     t_start = time.time()
     t = 1
@@ -498,7 +517,8 @@ def run_reference(args):
     wl = synth.workload(args.workload)
     layer = [md for md in wl["modules"] if md.name.startswith("layer0.")]
     layers = len(wl["modules"]) // len(layer)
-    states, grads, hp = _oracle_layer_sample(wl, layer)
+    states, grads, hp = _oracle_layer_sample(wl, layer, rule=getattr(args, "proj_rule", "left"),
+                                             state_bf16=getattr(args, "state_dtype", "f32") == "bf16")
     t = 1
     for _ in range(args.warmup):
         for i in range(len(layer)):
@@ -542,6 +562,8 @@ def main():
     ap.add_argument("--refresh-ws-gb", type=float, default=44.0)
     ap.add_argument("--state-dtype", default="f32", choices=["f32", "bf16"],
                     help="W and direction moments in fp32 (the workload's definition) or bf16 (the paper's runs)")
+    ap.add_argument("--proj-rule", default="left", choices=["left", "smaller"],
+                    help="left projector for every weight (the workload's definition) or GaLore's smaller-side rule")
     ap.add_argument("--clip-norm", type=float, default=0.0,
                     help="global-norm gradient clipping threshold (0: off, as in the workload's definition)")
     ap.add_argument("--chunk-mb", type=int, default=256,
