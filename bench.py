@@ -283,8 +283,7 @@ def run_gpu(args):
     # alignment diagnostic S(W, t) over every module (a profiling-step call,
     # outside the step; it reuses the modules' workspaces, which the next
     # step rewrites): one untimed call, then the mean of three
-    # (modules with a left projector: the diagnostic is defined for P P^T V)
-    a_sel = [k for k, md in enumerate(mods) if not _right(md, args.proj_rule)]
+    a_sel = list(range(len(mods)))
     a_ids, a_ptr = [ids[k] for k in a_sel], [gptr[k] for k in a_sel]
     S_dev = torch.empty(max(1, len(a_ids)), dtype=torch.float32, device=dev)
     M.moara_alignment(g.ctx, a_ids, a_ptr, S_dev.data_ptr(), cs)

@@ -285,7 +285,7 @@ int moara_flatten_shape(int ndim, const int64_t* shape, int* m, int* n);
  * "Profiling-based rank allocation"): for each module q of the call,
  *   S_q = cos(G_q, Rep_B(M) (.) (P P^T V)),  (M, V) = Decompose(G_q, B),
  * with the module's current projector P (its bf16 copy) and the context's
- * block size B; the cosine is the Frobenius inner product over ||G|| ||.||
+ * block size B (V Q Q^T for a module with a right projector Q); the cosine is the Frobenius inner product over ||G|| ||.||
  * (0 when either norm is 0).  The paper averages S over profiling steps and
  * matrices of a module type (S_tau) to rank the modules; that average is the
  * caller's.

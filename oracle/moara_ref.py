@@ -328,11 +328,14 @@ def flatten_shape(shape):
 # Alignment diagnostic S(W, t) (§3.2)
 # ---------------------------------------------------------------------------
 
-def alignment(G, P, B: int, eps: float = DECOMP_EPS) -> float:
-    """S(W,t) = cos(G, G_recon) with G_recon = Rep_B(M) (.) (P P^T V)  (§3.2)."""
+def alignment(G, P, B: int, eps: float = DECOMP_EPS, right: bool = False) -> float:
+    """S(W,t) = cos(G, G_recon) with G_recon = Rep_B(M) (.) (P P^T V)  (§3.2);
+    with a right projector Q (n x r, passed as P) the projected direction is
+    V Q Q^T."""
     G = np.asarray(G, dtype=np.float64)
     M, V = decompose(G, B, eps)
-    G_recon = rep_b(M, B, G.shape[1]) * (P @ (P.T @ V))
+    proj = (V @ P) @ P.T if right else P @ (P.T @ V)
+    G_recon = rep_b(M, B, G.shape[1]) * proj
     num = float(np.sum(G * G_recon))
     den = float(np.sqrt(np.sum(G * G)) * np.sqrt(np.sum(G_recon * G_recon)))
     return num / den if den > 0 else 0.0

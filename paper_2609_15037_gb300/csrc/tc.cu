@@ -42,6 +42,7 @@ constexpr int kMaps = 8;                      // tensor maps per module
 struct TcMod {
     int m, n, r, kb;
     int right;        // right projector Q (n x r): K1 computes R = V Q (m x r)
+    uint16_t* Qt;     // r x n bf16 transpose of a right projector (K2's B operand)
     uint16_t* Vhi;    // m x n bf16 direction matrix (written by K0)
     uint16_t* Vlo;    // m x n bf16 residual (first Adam step)
     float* W;
@@ -985,12 +986,13 @@ struct KrParams {
     float* out[kKrGroup];              // M x N fp32 or null
     uint16_t* out_bf[kKrGroup];        // M x N bf16 or null
     uint16_t* out_lo[kKrGroup];        // M x N bf16 residual (out - bf16(out)) or null
-    // alignment reduction (ALIGN): element (j, i) of the product, weighted by
-    // the block norm mag[i][j / al_B], is dotted with G[i][j] (i < al_m)
+    // alignment reduction (ALIGN): element (j, i) of the product (al_tr) or
+    // element (i, j), weighted by the block norm mag[i][j / al_B], is dotted
+    // with G[i][j]; al_m is the number of valid product columns
     const uint16_t* al_G[kKrGroup];
     const float* al_mag[kKrGroup];
     double* al_acc[kKrGroup];          // 3 doubles: <G, a>, <a, a>, <G, G>
-    int al_ld[kKrGroup], al_kb[kKrGroup], al_m[kKrGroup];
+    int al_ld[kKrGroup], al_kb[kKrGroup], al_m[kKrGroup], al_tr[kKrGroup];
     int al_B;
     int M[kKrGroup], N[kKrGroup], K[kKrGroup];
     int ktri[kKrGroup];
@@ -1118,13 +1120,15 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
         const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[0]), 0, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
         if (ALIGN && __all_sync(0xffffffffu, got) && h < halves) {
-            // S(W, t) of §3.2: this thread's row j of the product (P P^T V)^T
-            // against column j of G, weighted by Rep_B(M)
+            // S(W, t) of §3.2: this thread's row of the product -- row j of
+            // (P P^T V)^T against column j of G, or row i of V Q Q^T against
+            // row i of G -- weighted by Rep_B(M)
             ptx::tc_fence_after();
             const int row = i0 + h * 128 + q * 32 + lane;
             const uint16_t* const Gp = p.al_G[pi];
             const float* const mg = p.al_mag[pi];
             const int ldg = p.al_ld[pi], kbm = p.al_kb[pi], mm = p.al_m[pi];
+            const bool tr = p.al_tr[pi] != 0;
             const int jb = row / p.al_B;
             float dot = 0.0f, na = 0.0f, gg = 0.0f;
             for (int c = 0; c < nch * 4; ++c) {
@@ -1136,10 +1140,12 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
                 if (row >= M) continue;
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
-                    const int i = c0 + e;
-                    if (i < mm) {
-                        const float g = __bfloat162float(__ushort_as_bfloat16(Gp[(long long)i * ldg + row]));
-                        const float a = mg[(long long)i * kbm + jb] * v[e];
+                    const int ci = c0 + e;
+                    if (ci < mm) {
+                        const long long go = tr ? (long long)ci * ldg + row : (long long)row * ldg + ci;
+                        const long long mo = tr ? (long long)ci * kbm + jb : (long long)row * kbm + ci / p.al_B;
+                        const float g = __bfloat162float(__ushort_as_bfloat16(Gp[go]));
+                        const float a = mg[mo] * v[e];
                         dot = fmaf(g, a, dot);
                         na = fmaf(a, a, na);
                         gg = fmaf(g, g, gg);
@@ -1539,6 +1545,7 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
     t.dM = md.ws_dM;
     t.Pb = md.Pb;
     t.right = md.right;
+    t.Qt = md.ws_Qt;
     CUtensorMap* mp = &st->maps[kMaps * id];
     bool ok;
     if (!md.right) {
@@ -1912,7 +1919,8 @@ const char* tc_last_error(const TcState* st) { return st ? st->err.c_str() : "no
 // with two planes only) replaces the stores.
 static int kr_launch(TcState* st, int a_kmajor, const TcGemmItem* items, int count, int align_B,
                      const uint16_t* const* al_G, const float* const* al_mag, const int* al_ld, const int* al_kb,
-                     const int* al_m, double* const* al_acc, cudaStream_t s, int64_t* launches) {
+                     const int* al_m, double* const* al_acc, cudaStream_t s, int64_t* launches,
+                     const int* al_tr = nullptr) {
     if (!st->kr_attrs) {
         cudaFuncSetAttribute(kr_product<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
         cudaFuncSetAttribute(kr_product<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, KR_SMEM);
@@ -1960,6 +1968,7 @@ static int kr_launch(TcState* st, int a_kmajor, const TcGemmItem* items, int cou
                 if (align_B > 0) {
                     kp.al_G[q] = al_G[it]; kp.al_mag[q] = al_mag[it]; kp.al_acc[q] = al_acc[it];
                     kp.al_ld[q] = al_ld[it]; kp.al_kb[q] = al_kb[it]; kp.al_m[q] = al_m[it];
+                    kp.al_tr[q] = al_tr != nullptr ? al_tr[it] : 1;
                 }
                 kp.M[q] = x.M; kp.N[q] = x.N; kp.K[q] = x.K;
                 kp.ktri[q] = x.ktri;
@@ -2046,7 +2055,7 @@ int tc_alignment(TcState* st, const moara_hparams& hp, int n_mod, const int* ids
     for (int q = 0; q < n_mod; ++q) {
         const int id = ids[q];
         const TcMod* md = (id >= 0 && id < static_cast<int>(st->mods.size())) ? &st->mods[id] : nullptr;
-        if (md == nullptr || md->Vhi == nullptr || md->Vlo == nullptr || md->Pb == nullptr || md->right) {
+        if (md == nullptr || md->Vhi == nullptr || md->Vlo == nullptr || md->Pb == nullptr) {
             st->err = "alignment: module is not on the tensor-core path";
             return MOARA_ERR_UNSUPPORTED;
         }
@@ -2090,18 +2099,29 @@ int tc_alignment(TcState* st, const moara_hparams& hp, int n_mod, const int* ids
             return MOARA_ERR_CUDA;
         }
     }
-    // 2. R^T = V^T P (n x r) as two bf16 planes in the module's N buffer
-    std::vector<TcGemmItem> g1(n_mod);
+    // 2. left projector: R^T = V^T P (n x r); right projector: R = V Q
+    //    (m x r); as two bf16 planes in the module's N buffer
+    std::vector<TcGemmItem> g1[2];
     for (int q = 0; q < n_mod; ++q) {
         const TcMod& md = st->mods[ids[q]];
-        g1[q] = TcGemmItem{md.Vhi, md.Vlo, md.Pb, nullptr, md.Nb, md.n, md.r, md.m, 0,
-                           md.Nb + (size_t)md.n * md.r};
+        if (!md.right)
+            g1[0].push_back(TcGemmItem{md.Vhi, md.Vlo, md.Pb, nullptr, md.Nb, md.n, md.r, md.m, 0,
+                                       md.Nb + (size_t)md.n * md.r});
+        else
+            g1[1].push_back(TcGemmItem{md.Vhi, md.Vlo, md.Pb, nullptr, md.Nb, md.m, md.r, md.n, 0,
+                                       md.Nb + (size_t)md.m * md.r});
     }
-    rc = kr_launch(st, 0, g1.data(), n_mod, 0, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, s, launches);
-    if (rc != MOARA_OK) return rc;
-    // 3. P^T (r x mp, zero-padded columns) over the V planes, now free
+    for (int side = 0; side < 2; ++side) {
+        if (g1[side].empty()) continue;
+        rc = kr_launch(st, side, g1[side].data(), static_cast<int>(g1[side].size()), 0, nullptr, nullptr, nullptr,
+                       nullptr, nullptr, nullptr, s, launches);
+        if (rc != MOARA_OK) return rc;
+    }
+    // 3. left projector: P^T (r x mp, zero-padded columns) over the V planes,
+    //    now free (a right projector's Q^T is kept in the workspace)
     for (int q = 0; q < n_mod; ++q) {
         const TcMod& md = st->mods[ids[q]];
+        if (md.right) continue;
         const int mp = (md.m + 7) / 8 * 8;
         const int tiles = ((mp + 31) / 32) * ((md.r + 31) / 32);
         k_transpose_pad_bf16<<<std::min(tiles, st->sms * 8), 256, 0, s>>>(md.Pb, md.Vhi, md.m, md.r, mp);
@@ -2111,23 +2131,32 @@ int tc_alignment(TcState* st, const moara_hparams& hp, int n_mod, const int* ids
         st->err = "alignment accumulator reset failed";
         return MOARA_ERR_CUDA;
     }
-    // 4. (P R)^T = R^T P^T (n x mp), reduced against G in the epilogue
+    // 4. left: (P R)^T = R^T P^T (n x mp); right: V Q Q^T = R Q^T (m x n);
+    //    reduced against G in the epilogue
     std::vector<TcGemmItem> g2(n_mod);
     std::vector<const uint16_t*> aG(n_mod);
     std::vector<const float*> aM(n_mod);
-    std::vector<int> ald(n_mod), akb(n_mod), am(n_mod);
+    std::vector<int> ald(n_mod), akb(n_mod), am(n_mod), atr(n_mod);
     std::vector<double*> aacc(n_mod);
     for (int q = 0; q < n_mod; ++q) {
         const TcMod& md = st->mods[ids[q]];
-        const int mp = (md.m + 7) / 8 * 8;
-        g2[q] = TcGemmItem{md.Nb, md.Nb + (size_t)md.n * md.r, md.Vhi, nullptr, nullptr, md.n, mp, md.r, 0, nullptr};
+        if (!md.right) {
+            const int mp = (md.m + 7) / 8 * 8;
+            g2[q] = TcGemmItem{md.Nb, md.Nb + (size_t)md.n * md.r, md.Vhi, nullptr, nullptr, md.n, mp, md.r, 0, nullptr};
+            am[q] = md.m;
+            atr[q] = 1;
+        } else {
+            g2[q] = TcGemmItem{md.Nb, md.Nb + (size_t)md.m * md.r, md.Qt, nullptr, nullptr, md.m, md.n, md.r, 0, nullptr};
+            am[q] = md.n;
+            atr[q] = 0;
+        }
         aG[q] = static_cast<const uint16_t*>(G[q]);
         aM[q] = md.mag;
-        ald[q] = md.n; akb[q] = md.kb; am[q] = md.m;
+        ald[q] = md.n; akb[q] = md.kb;
         aacc[q] = acc + 3 * q;
     }
     rc = kr_launch(st, 1, g2.data(), n_mod, B, aG.data(), aM.data(), ald.data(), akb.data(), am.data(),
-                   aacc.data(), s, launches);
+                   aacc.data(), s, launches, atr.data());
     if (rc != MOARA_OK) return rc;
     k_align_finish<<<(n_mod + 127) / 128, 128, 0, s>>>(acc, S_out, n_mod);
     ++*launches;

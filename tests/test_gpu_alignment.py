@@ -82,6 +82,28 @@ def test_alignment_full_size_module(M):
     assert abs(S[0] - ref[0]) <= TOL, (S, ref)
 
 
+def test_alignment_right_projectors(M):
+    """Under the smaller-side rule a tall module's S uses V Q Q^T (its right
+    projector); a wide one keeps P P^T V; both in one call."""
+    B = 64
+    shapes = [(640, 256, 64), (256, 640, 64), (392, 136, 40)]
+    g = M.MoaraGroup(block_size=B, precision=M.MOARA_PREC_BF16_TC, proj_rule=M.MOARA_PROJ_SMALLER)
+    grads, refs = [], []
+    for i, (m, n, r) in enumerate(shapes):
+        right = m > n
+        G = synth.to_bf16_exact(synth.lowrank_grad(m, n, 16, 10.0, 0.01, 0, seed=9, module=i, noise_rel=True))
+        V = o.decompose(G, B)[1]
+        P = synth.to_bf16_exact(o.truncated_svd(V.T if right else V, r)[0])
+        mid = g.add(m, n, r, "bf16")
+        g.load_projector(mid, P)
+        grads.append(_dev(G))
+        refs.append(o.alignment(G, P, B, right=right))
+    S = g.alignment(grads).cpu().numpy()
+    assert g.status() == 0
+    g.close()
+    assert np.max(np.abs(S - np.array(refs))) <= TOL, (S, refs)
+
+
 def test_alignment_errors(M):
     g = M.MoaraGroup(block_size=64)
     mid = g.add(64, 64, 8, "f32")

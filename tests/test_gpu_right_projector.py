@@ -139,8 +139,4 @@ def test_right_projector_refusals(M):
     with pytest.raises(M.MoaraError) as ei:
         g.add(128, 64, 8, "f32")
     assert ei.value.code == M.MOARA_ERR_UNSUPPORTED
-    g.add(128, 64, 8, "bf16")
-    with pytest.raises(M.MoaraError) as ei:
-        g.alignment([torch.zeros(128, 64, dtype=torch.bfloat16, device="cuda")])
-    assert ei.value.code == M.MOARA_ERR_UNSUPPORTED
     g.close()

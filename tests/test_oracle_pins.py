@@ -517,3 +517,17 @@ def test_right_projector_refresh_and_full_rank():
     np.testing.assert_allclose(st_r.extras["R"], V, atol=1e-15)
     # square and wide weights keep the left projector under the smaller-side rule
     assert not o.is_right(6, 6, "smaller") and not o.is_right(4, 9, "smaller") and o.is_right(9, 4, "smaller")
+
+
+def test_alignment_right_projector_is_the_transposed_case_without_blocks():
+    """With one block per row and a rank-one G = u v^T, V = sign(u) v^T / ||v||
+    lies in the row space span(v): a right projector along v reconstructs V
+    exactly (S = 1), one orthogonal to v gives S = 0."""
+    rng = _rng(63)
+    u, v = rng.standard_normal(7), rng.standard_normal(5)
+    G = np.outer(u, v)
+    q = (v / np.linalg.norm(v))[:, None]
+    assert o.alignment(G, q, 5, right=True) == pytest.approx(1.0, abs=1e-12)
+    w = rng.standard_normal(5)
+    w -= q[:, 0] * (q[:, 0] @ w)
+    assert o.alignment(G, (w / np.linalg.norm(w))[:, None], 5, right=True) == pytest.approx(0.0, abs=1e-12)
