@@ -1221,12 +1221,19 @@ int step_impl(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, i
         if (rc != MOARA_OK) return rc;
     }
     // global-norm clipping (App. D.2): the coefficient of this step's
-    // gradients, before any update
+    // gradients, before any update.  When every module runs on tensor cores
+    // with the decomposition, the step takes it from the block norms of its
+    // own decomposition (no extra pass over G); otherwise a norm pass first.
     const float* clip = nullptr;
+    moara::TcClipFuse fuse{};
+    bool fused = false;
+    if (ctx->hp.clip_norm > 0.0f && ctx->hp.decompose && n_mod <= moara::tc_group_limit()) {
+        fused = true;
+        for (int i = 0; i < n_mod && fused; ++i) fused = use_tc(ctx, ids[i]);
+    }
     if (ctx->hp.clip_norm > 0.0f) {
-        ProfScope ps(ctx, MOARA_PHASE_CLIP_NORM, s);
-        const int nb = (n_mod + moara::kMaxGroup - 1) / moara::kMaxGroup;
-        if (ctx->clip_part_cap < nb) {
+        const int need = fused ? 1 : (n_mod + moara::kMaxGroup - 1) / moara::kMaxGroup;
+        if (ctx->clip_part_cap < need) {
             if (ctx->d_clip_part != nullptr) {
                 cudaError_t e = cudaStreamSynchronize(s);   // an earlier step may still use them
                 if (e != cudaSuccess) return cuda_fail(ctx, e, "clipping partial sums release");
@@ -1234,10 +1241,15 @@ int step_impl(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, i
                 ctx->d_clip_part = nullptr;
                 ctx->clip_part_cap = 0;
             }
-            cudaError_t e = cudaMalloc(&ctx->d_clip_part, sizeof(double) * moara::kNormParts * (size_t)nb);
+            cudaError_t e = cudaMalloc(&ctx->d_clip_part, sizeof(double) * moara::kNormParts * (size_t)need);
             if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMalloc of the clipping partial sums");
-            ctx->clip_part_cap = nb;
+            ctx->clip_part_cap = need;
         }
+        fuse = moara::TcClipFuse{ctx->d_clip, ctx->d_clip_part, ctx->clip_extra, ctx->hp.clip_norm};
+    }
+    if (ctx->hp.clip_norm > 0.0f && !fused) {
+        ProfScope ps(ctx, MOARA_PHASE_CLIP_NORM, s);
+        const int nb = (n_mod + moara::kMaxGroup - 1) / moara::kMaxGroup;
         for (int c0 = 0, bi = 0; c0 < n_mod; c0 += moara::kMaxGroup, ++bi) {
             moara::GradNormBatch nbt{};
             nbt.count = std::min(moara::kMaxGroup, n_mod - c0);
@@ -1280,8 +1292,8 @@ int step_impl(moara_ctx* ctx, int n_mod, const int* ids, const void* const* G, i
             }
         }, ctx};
         rc = moara::tc_step(ctx->tc, ctx->hp, static_cast<int>(mids.size()), mids.data(), gp.data(),
-                            static_cast<float>(bc1), static_cast<float>(bc2), lr, t == 1 ? 1 : 0, clip, s,
-                            &ctx->launches, tp);
+                            static_cast<float>(bc1), static_cast<float>(bc2), lr, t == 1 ? 1 : 0, clip,
+                            fused ? &fuse : nullptr, s, &ctx->launches, tp);
         if (rc != MOARA_OK) return fail(ctx, rc, "tensor-core step launch failed: %s", moara::tc_last_error(ctx->tc));
     }
     if (!simt.empty()) {

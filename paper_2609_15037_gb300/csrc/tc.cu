@@ -290,6 +290,38 @@ __global__ void __launch_bounds__(256) k0_mag_adam(const __grid_constant__ K0Par
     }
 }
 
+// Sum of the squared block norms K0 wrote (= ||G||_F^2 of the group, up to
+// their rounding) for global-norm clipping: chunks of kNormChunk entries,
+// chunk c on CTA c mod gridDim, fp32 per chunk and fp64 across chunks in a
+// fixed order, one partial sum per CTA.
+__global__ void __launch_bounds__(256) k0_mag_sq(const __grid_constant__ K0Params p, double* partials) {
+    __shared__ double red[8];
+    const long long total = p.mstart[p.count];
+    const long long nchunks = (total + kNormChunk - 1) / kNormChunk;
+    double acc = 0.0;
+    int mod = 0;
+    for (long long c = blockIdx.x; c < nchunks; c += gridDim.x) {
+        const long long e0 = c * kNormChunk, e1 = min(e0 + (long long)kNormChunk, total);
+        float ss = 0.0f;
+        for (long long e = e0 + threadIdx.x; e < e1; e += blockDim.x) {
+            while (mod + 1 < p.count && p.mstart[mod + 1] <= e) ++mod;
+            while (mod > 0 && p.mstart[mod] > e) --mod;
+            const float x = p.p[mod].mag[e - p.mstart[mod]];
+            ss = fmaf(x, x, ss);
+        }
+        acc += static_cast<double>(ss);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < 8; ++w) t += red[w];
+        partials[blockIdx.x] = t;
+    }
+}
+
 // ===========================================================================
 // K1: projection R = P^T V (tile 128 ranks x 256 columns x 64 rows, MN-major
 // operands), Optimizer_V (Adam) in the epilogue, N written in bf16.  HILO
@@ -1709,30 +1741,34 @@ static TcState::Tiles* tc_tiles(TcState* st, const std::vector<int>& ids) {
 // on each SM instead of a persistent grid that would hold SMs they need.
 template <int BLK>
 static cudaError_t launch_k0(TcState* st, const K0Params& p0, bool background, cudaStream_t s,
-                             int64_t* launches, const TcProfile& prof) {
+                             int64_t* launches, const TcProfile& prof, bool mag_adam = true) {
     const int phase = background ? MOARA_PHASE_TC_DECOMPOSE_OVERLAP : MOARA_PHASE_TC_DECOMPOSE;
     if (prof.on) prof.mark(prof.ctx, phase, s, true);
     const long long items = p0.start[p0.count];
     const int g0 = background ? static_cast<int>(std::max<long long>(1, std::min<long long>((items + 31) / 32, 1 << 30)))
                               : st->sms * 3;
     k0_decompose<BLK><<<g0, 256, 0, s>>>(p0);
-    k0_mag_adam<<<background ? st->sms : st->sms * 4, 256, 0, s>>>(p0);
+    if (mag_adam) k0_mag_adam<<<background ? st->sms : st->sms * 4, 256, 0, s>>>(p0);
     if (prof.on) prof.mark(prof.ctx, phase, s, false);
-    *launches += 2;
+    *launches += mag_adam ? 2 : 1;
     return cudaGetLastError();
 }
 
+// which: 1 = K1 only, 2 = K2 only, 3 = both
 template <int BLK, bool SB>
 static cudaError_t launch_k12(TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2, bool hilo,
-                              cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+                              cudaStream_t s, int64_t* launches, const TcProfile& prof, int which) {
     cudaError_t e;
-    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, true);
-    if (hilo) k1_project<true, SB><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
-    else k1_project<false, SB><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
-    if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, false);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    ++*launches;
+    if (which & 1) {
+        if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, true);
+        if (hilo) k1_project<true, SB><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+        else k1_project<false, SB><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+        if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, false);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        ++*launches;
+    }
+    if (!(which & 2)) return cudaSuccess;
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_BACKPROJECT, s, true);
     k2_backproject<BLK, SB><<<2 * g2, K2_THREADS, K2_SMEM, s>>>(p2);
     if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_BACKPROJECT, s, false);
@@ -1743,31 +1779,32 @@ static cudaError_t launch_k12(TcState* st, const K1Params& p1, const K2Params& p
 }
 
 static cudaError_t launch_k0_any(int B, TcState* st, const K0Params& p0, bool background, cudaStream_t s,
-                                 int64_t* launches, const TcProfile& prof) {
+                                 int64_t* launches, const TcProfile& prof, bool mag_adam = true) {
     switch (B) {
-        case 8: return launch_k0<8>(st, p0, background, s, launches, prof);
-        case 16: return launch_k0<16>(st, p0, background, s, launches, prof);
-        case 32: return launch_k0<32>(st, p0, background, s, launches, prof);
-        case 64: return launch_k0<64>(st, p0, background, s, launches, prof);
-        default: return launch_k0<128>(st, p0, background, s, launches, prof);
+        case 8: return launch_k0<8>(st, p0, background, s, launches, prof, mag_adam);
+        case 16: return launch_k0<16>(st, p0, background, s, launches, prof, mag_adam);
+        case 32: return launch_k0<32>(st, p0, background, s, launches, prof, mag_adam);
+        case 64: return launch_k0<64>(st, p0, background, s, launches, prof, mag_adam);
+        default: return launch_k0<128>(st, p0, background, s, launches, prof, mag_adam);
     }
 }
 
 static cudaError_t launch_k12_any(int B, bool sb, TcState* st, const K1Params& p1, const K2Params& p2, int g1,
-                                  int g2, bool hilo, cudaStream_t s, int64_t* launches, const TcProfile& prof) {
+                                  int g2, bool hilo, cudaStream_t s, int64_t* launches, const TcProfile& prof,
+                                  int which = 3) {
     if (sb) {   // bf16 states: B >= 32 (tc_supported)
         switch (B) {
-            case 32: return launch_k12<32, true>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-            case 64: return launch_k12<64, true>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-            default: return launch_k12<128, true>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+            case 32: return launch_k12<32, true>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
+            case 64: return launch_k12<64, true>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
+            default: return launch_k12<128, true>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
         }
     }
     switch (B) {
-        case 8: return launch_k12<8, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-        case 16: return launch_k12<16, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-        case 32: return launch_k12<32, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-        case 64: return launch_k12<64, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
-        default: return launch_k12<128, false>(st, p1, p2, g1, g2, hilo, s, launches, prof);
+        case 8: return launch_k12<8, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
+        case 16: return launch_k12<16, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
+        case 32: return launch_k12<32, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
+        case 64: return launch_k12<64, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
+        default: return launch_k12<128, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
     }
 }
 
@@ -1779,9 +1816,11 @@ constexpr int kOverlapParts = 16;
 constexpr int kOverlapMin = 32;
 static_assert(kOverlapParts <= 32, "one event per part");
 
+int tc_group_limit() { return kTcGroup; }
+
 int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G, float bc1,
-            float bc2, float lr, int first_step, const float* clip, cudaStream_t s, int64_t* launches,
-            const TcProfile& prof) {
+            float bc2, float lr, int first_step, const float* clip, const TcClipFuse* fuse, cudaStream_t s,
+            int64_t* launches, const TcProfile& prof) {
     if (!st->attrs_set) {
         cudaFuncSetAttribute(k1_project<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
         cudaFuncSetAttribute(k1_project<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
@@ -1805,6 +1844,13 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
         st->err = what;
         return MOARA_ERR_CUDA;
     };
+    // clipping from the block norms: Optimizer_M and K2 wait for the norm of
+    // every module, so they run once after all decompositions and K1s
+    const bool fused = fuse != nullptr && dec;
+    if (fused && n_mod > kTcGroup) {
+        st->err = "fused clipping takes at most tc_group_limit() modules";
+        return MOARA_ERR_UNSUPPORTED;
+    }
     for (int c0 = 0; c0 < n_mod; c0 += kTcGroup) {
         const int cnt = std::min(kTcGroup, n_mod - c0);
         // parts of the group (consecutive modules, about equal G bytes)
@@ -1863,7 +1909,8 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
         // decomposition: part 0 on s with the full grid; part q + 1 in the
         // background on the auxiliary stream, launched after K1 / K2 of part q
         // so that their persistent CTAs are placed first
-        if (dec && launch_k0_any(B, st, *build_p0(pstart[0], pstart[1]), false, s, launches, prof) != cudaSuccess)
+        if (dec && launch_k0_any(B, st, *build_p0(pstart[0], pstart[1]), false, s, launches, prof, !fused) !=
+                       cudaSuccess)
             return fail("decomposition launch failed");
         for (int q = 0; q < np; ++q) {
             const int a = pstart[q], b = pstart[q + 1];
@@ -1897,16 +1944,47 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             p2.step_scale = lr * hp.scale;
             p2.decompose = hp.decompose;
             const cudaError_t e = launch_k12_any(B, hp.state_dtype == MOARA_DTYPE_BF16, st, p1, p2, tl->g1, tl->g2,
-                                                 hilo, s, launches, prof);
+                                                 hilo, s, launches, prof, fused ? 1 : 3);
             if (e != cudaSuccess) {
                 st->err = cudaGetErrorString(e);
                 return MOARA_ERR_CUDA;
             }
             if (dec && q + 1 < np) {
-                if (launch_k0_any(B, st, *build_p0(pstart[q + 1], pstart[q + 2]), true, st->aux, launches, prof) !=
-                        cudaSuccess ||
+                if (launch_k0_any(B, st, *build_p0(pstart[q + 1], pstart[q + 2]), true, st->aux, launches, prof,
+                                  !fused) != cudaSuccess ||
                     cudaEventRecord(st->ev_part[q + 1], st->aux) != cudaSuccess)
                     return fail("background decomposition launch failed");
+            }
+        }
+        if (fused) {
+            // total norm from every module's block norms, the coefficient,
+            // Optimizer_M of the clipped magnitudes, then K2 over the group
+            K0Params* pall = build_p0(0, cnt);
+            pall->clip = fuse->state + 1;
+            if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_CLIP_NORM, s, true);
+            k0_mag_sq<<<kNormParts, 256, 0, s>>>(*pall, fuse->partials);
+            ++*launches;
+            if (launch_clip_finish(fuse->partials, kNormParts, fuse->extra, fuse->max_norm, fuse->state, s,
+                                   launches) != cudaSuccess)
+                return fail("clipping coefficient launch failed");
+            if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_CLIP_NORM, s, false);
+            if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, true);
+            k0_mag_adam<<<st->sms * 4, 256, 0, s>>>(*pall);
+            ++*launches;
+            if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_DECOMPOSE, s, false);
+            std::vector<int> all(ids + c0, ids + c0 + cnt);
+            TcState::Tiles* tl = tc_tiles(st, all);
+            if (tl == nullptr) { st->err = "tile list allocation failed"; return MOARA_ERR_CUDA; }
+            K2Params p2{};
+            p2.cta_start = tl->k2_start; p2.tiles = tl->k2;
+            p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;
+            p2.step_scale = lr * hp.scale;
+            p2.decompose = hp.decompose;
+            const cudaError_t e = launch_k12_any(B, hp.state_dtype == MOARA_DTYPE_BF16, st, st->p1, p2, tl->g1, tl->g2,
+                                                 hilo, s, launches, prof, 2);
+            if (e != cudaSuccess) {
+                st->err = cudaGetErrorString(e);
+                return MOARA_ERR_CUDA;
             }
         }
     }

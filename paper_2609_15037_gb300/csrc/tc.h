@@ -20,10 +20,24 @@ struct TcProfile {
 TcState* tc_create(int device, int* d_status);
 void tc_destroy(TcState* st);
 int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp);
-// clip: device clipping coefficient of this step's gradients, or null
+// Global-norm clipping computed inside the step from the decomposition's
+// block norms (no extra pass over G): the step writes {norm, coefficient} to
+// state after every module's decomposition and before Optimizer_M.
+struct TcClipFuse {
+    float* state;           // device {total norm, coefficient}
+    double* partials;       // device scratch of kNormParts doubles
+    const float* extra;     // device sum of squares of other gradients, or null
+    float max_norm;
+};
+// Largest number of modules one fused-clipping step takes.
+int tc_group_limit();
+
+// clip: device clipping coefficient of this step's gradients, or null;
+// fuse: clipping from the block norms (decomposition on, at most
+// tc_group_limit() modules), or null
 int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, const void* const* G,
-            float bc1, float bc2, float lr, int first_step, const float* clip, cudaStream_t s, int64_t* launches,
-            const TcProfile& prof);
+            float bc1, float bc2, float lr, int first_step, const float* clip, const TcClipFuse* fuse,
+            cudaStream_t s, int64_t* launches, const TcProfile& prof);
 // One problem of the refresh GEMM on tensor cores: out = op(A) B, bf16
 // operands, fp32 accumulation.
 struct TcGemmItem {
