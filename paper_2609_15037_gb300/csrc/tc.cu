@@ -327,7 +327,9 @@ __global__ void __launch_bounds__(256) k0_mag_sq(const __grid_constant__ K0Param
 // operands), Optimizer_V (Adam) in the epilogue, N written in bf16.  HILO
 // adds the MMA with V_lo (first Adam step).
 // ===========================================================================
-template <bool HILO, bool SB>
+// RT: the launch may hold modules with a right projector (per-tile operand
+// roles); without it those branches are compiled out.
+template <bool HILO, bool SB, bool RT>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(K1_THREADS, 1)
 k1_project(const __grid_constant__ K1Params p) {
     constexpr int MC = StateCols<SB>::N;              // moment columns per chunk
@@ -391,7 +393,7 @@ k1_project(const __grid_constant__ K1Params p) {
                 const CUtensorMap* vmap = p.decompose ? &p.maps[tl.mod * kMaps + 4] : &p.gmap[tl.slot];
                 const CUtensorMap* lmap = &p.maps[tl.mod * kMaps + 5];
                 const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
-                const bool right = md.right != 0;
+                const bool right = RT && md.right != 0;
                 const int nk = ((right ? md.n : md.m) + K1_BK - 1) / K1_BK;
                 for (int kb = 0; kb < nk; ++kb) {
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
@@ -446,7 +448,7 @@ k1_project(const __grid_constant__ K1Params p) {
                 for (int t = t_begin; t < t_end && ok; ++t) {
                     const TcTile tl = p.tiles[t];
                     const TcMod& md = p.mods[tl.mod];
-                    const bool right = md.right != 0;
+                    const bool right = RT && md.right != 0;
                     const uint32_t idesc = right ? idesc_r : idesc_l;
                     const int nk = ((right ? md.n : md.m) + K1_BK - 1) / K1_BK;
                     if (!ptx::mbar_wait_cluster(ptx::smem_u32(&ctl->acce[buf]), acc_phase ^ 1, abort_flag, p.status,
@@ -502,7 +504,7 @@ k1_project(const __grid_constant__ K1Params p) {
                 const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 6];
                 const CUtensorMap* smap = &p.maps[tl.mod * kMaps + 7];
                 const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
-                const int cols = md.right ? md.r : md.n;    // R is r x n, or m x r (right projector)
+                const int cols = (RT && md.right) ? md.r : md.n;    // R is r x n, or m x r (right projector)
                 const int nc = min(K1_BN / MC, (cols - n0 + MC - 1) / MC);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % MSLOTS;
@@ -534,7 +536,7 @@ k1_project(const __grid_constant__ K1Params p) {
                 const CUtensorMap* amap = &p.maps[tl.mod * kMaps + 6];
                 const CUtensorMap* smap = &p.maps[tl.mod * kMaps + 7];
                 const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
-                const int cols = md.right ? md.r : md.n;    // R is r x n, or m x r (right projector)
+                const int cols = (RT && md.right) ? md.r : md.n;    // R is r x n, or m x r (right projector)
                 const int nc = min(K1_BN / MC, (cols - n0 + MC - 1) / MC);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % MSLOTS;
@@ -571,7 +573,7 @@ k1_project(const __grid_constant__ K1Params p) {
             const TcTile tl = p.tiles[t];
             const TcMod& md = p.mods[tl.mod];
             // R (and the moments, N) is r x n, or m x r with a right projector
-            const int rr = md.right ? md.m : md.r, nn = md.right ? md.r : md.n;
+            const int rr = (RT && md.right) ? md.m : md.r, nn = (RT && md.right) ? md.r : md.n;
             uint16_t* const nb_p = md.Nb;
             const int r0 = (2 * tl.t0 + crank) * K1_BM, n0 = tl.t1 * K1_BN;
             const int a = r0 + il;
@@ -1757,12 +1759,17 @@ static cudaError_t launch_k0(TcState* st, const K0Params& p0, bool background, c
 // which: 1 = K1 only, 2 = K2 only, 3 = both
 template <int BLK, bool SB>
 static cudaError_t launch_k12(TcState* st, const K1Params& p1, const K2Params& p2, int g1, int g2, bool hilo,
-                              cudaStream_t s, int64_t* launches, const TcProfile& prof, int which) {
+                              cudaStream_t s, int64_t* launches, const TcProfile& prof, int which, bool rt) {
     cudaError_t e;
     if (which & 1) {
         if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, true);
-        if (hilo) k1_project<true, SB><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
-        else k1_project<false, SB><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+        if (rt) {
+            if (hilo) k1_project<true, SB, true><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+            else k1_project<false, SB, true><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+        } else {
+            if (hilo) k1_project<true, SB, false><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+            else k1_project<false, SB, false><<<2 * g1, K1_THREADS, K1_SMEM, s>>>(p1);
+        }
         if (prof.on) prof.mark(prof.ctx, MOARA_PHASE_TC_PROJECT, s, false);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
@@ -1791,20 +1798,20 @@ static cudaError_t launch_k0_any(int B, TcState* st, const K0Params& p0, bool ba
 
 static cudaError_t launch_k12_any(int B, bool sb, TcState* st, const K1Params& p1, const K2Params& p2, int g1,
                                   int g2, bool hilo, cudaStream_t s, int64_t* launches, const TcProfile& prof,
-                                  int which = 3) {
+                                  int which = 3, bool rt = false) {
     if (sb) {   // bf16 states: B >= 32 (tc_supported)
         switch (B) {
-            case 32: return launch_k12<32, true>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
-            case 64: return launch_k12<64, true>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
-            default: return launch_k12<128, true>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
+            case 32: return launch_k12<32, true>(st, p1, p2, g1, g2, hilo, s, launches, prof, which, rt);
+            case 64: return launch_k12<64, true>(st, p1, p2, g1, g2, hilo, s, launches, prof, which, rt);
+            default: return launch_k12<128, true>(st, p1, p2, g1, g2, hilo, s, launches, prof, which, rt);
         }
     }
     switch (B) {
-        case 8: return launch_k12<8, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
-        case 16: return launch_k12<16, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
-        case 32: return launch_k12<32, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
-        case 64: return launch_k12<64, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
-        default: return launch_k12<128, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which);
+        case 8: return launch_k12<8, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which, rt);
+        case 16: return launch_k12<16, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which, rt);
+        case 32: return launch_k12<32, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which, rt);
+        case 64: return launch_k12<64, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which, rt);
+        default: return launch_k12<128, false>(st, p1, p2, g1, g2, hilo, s, launches, prof, which, rt);
     }
 }
 
@@ -1822,14 +1829,15 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             float bc2, float lr, int first_step, const float* clip, const TcClipFuse* fuse, cudaStream_t s,
             int64_t* launches, const TcProfile& prof) {
     if (!st->attrs_set) {
-        cudaFuncSetAttribute(k1_project<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
-        cudaFuncSetAttribute(k1_project<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
-        cudaFuncSetAttribute(k1_project<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
-        cudaFuncSetAttribute(k1_project<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
+        for (auto fn : {k1_project<true, false, false>, k1_project<false, false, false>, k1_project<true, true, false>,
+                        k1_project<false, true, false>, k1_project<true, false, true>, k1_project<false, false, true>,
+                        k1_project<true, true, true>, k1_project<false, true, true>})
+            cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, K1_SMEM);
         set_smem_attrs<8>(); set_smem_attrs<16>(); set_smem_attrs<32>(); set_smem_attrs<64>();
         set_smem_attrs<128>();
         // clusters of two that fit on the GPU at once (persistent grids)
-        st->k1_clusters = max_clusters(reinterpret_cast<const void*>(k1_project<false, false>), K1_THREADS, K1_SMEM,
+        st->k1_clusters = max_clusters(reinterpret_cast<const void*>(k1_project<false, false, false>), K1_THREADS,
+                                       K1_SMEM,
                                        st->sms / 2);
         st->k2_clusters = max_clusters(reinterpret_cast<const void*>(k2_backproject<128, false>), K2_THREADS, K2_SMEM,
                                        st->sms / 2);
@@ -1943,8 +1951,10 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             p2.mods = st->d_mods; p2.maps = st->d_maps; p2.status = st->d_status;
             p2.step_scale = lr * hp.scale;
             p2.decompose = hp.decompose;
+            bool rt = false;
+            for (int k = 0; k < b - a; ++k) rt = rt || st->mods[chunk[k]].right != 0;
             const cudaError_t e = launch_k12_any(B, hp.state_dtype == MOARA_DTYPE_BF16, st, p1, p2, tl->g1, tl->g2,
-                                                 hilo, s, launches, prof, fused ? 1 : 3);
+                                                 hilo, s, launches, prof, fused ? 1 : 3, rt);
             if (e != cudaSuccess) {
                 st->err = cudaGetErrorString(e);
                 return MOARA_ERR_CUDA;
