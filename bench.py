@@ -39,12 +39,14 @@ LR = 1e-3
 # (profiles/step_kernels_llama7b_layer.md).  A full-model launch processes the
 # same kinds of tiles, so its traffic is scaled by the ratio of the kernel's
 # algorithmic bytes (full model / captured workload).  Valid only for the
-# kernel source with this code fingerprint (SHA-1 of the source with `//`
-# comments and blank lines removed); after any code change the roofline
-# reports traffic = null until the counters are taken again.
-TRAFFIC = {"source": "paper_2609_15037_gb300/csrc/tc.cu", "sha1": "3ee31f04f09f450a3f6f52e63885510ce3074df4",
+# kernel code with this fingerprint (SHA-1 of the step kernels' part of the
+# source -- everything before the refresh GEMMs -- with `//` comments and
+# blank lines removed); after any change there the roofline reports
+# traffic = null until the counters are taken again.
+TRAFFIC = {"source": "paper_2609_15037_gb300/csrc/tc.cu", "until": "// KR: bf16 tensor-core GEMM of the projector refresh",
+           "sha1": "6edf3139deaa69d28e942a7082282ab87cc2f8ee",
            "workload": "llama7b_layer",
-           "bytes": {"tc_decompose": 756953344, "tc_project": 1059397120, "tc_backproject": 1741026304}}
+           "bytes": {"tc_decompose": 757951488, "tc_project": 1057314560, "tc_backproject": 1736570368}}
 
 
 def _peaks():
@@ -168,13 +170,16 @@ def _kernel_bytes(mods, B, tc, sb=4, rule="left"):
     return kb
 
 
-def _code_sha1(path):
-    """SHA-1 of a C++/CUDA source with `//` comments and blank lines removed."""
+def _code_sha1(path, until=None):
+    """SHA-1 of a C++/CUDA source (up to the first line that starts with
+    `until`, if given) with `//` comments and blank lines removed."""
     import hashlib
     lines = []
     with open(path, encoding="utf-8") as f:
-        for ln in f:
-            ln = ln.split("//", 1)[0].strip()
+        for raw in f:
+            if until is not None and raw.startswith(until):
+                break
+            ln = raw.split("//", 1)[0].strip()
             if ln:
                 lines.append(ln)
     return hashlib.sha1("\n".join(lines).encode()).hexdigest()
@@ -187,7 +192,7 @@ def _traffic(kernel, workload):
     import synth
     if TRAFFIC["sha1"] is None or kernel not in TRAFFIC["bytes"]:
         return None
-    if _code_sha1(os.path.join(ROOT, TRAFFIC["source"])) != TRAFFIC["sha1"]:
+    if _code_sha1(os.path.join(ROOT, TRAFFIC["source"]), TRAFFIC["until"]) != TRAFFIC["sha1"]:
         return None
     cap = synth.workload(TRAFFIC["workload"])
     cur = synth.workload(workload)

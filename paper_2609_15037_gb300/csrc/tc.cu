@@ -1027,7 +1027,7 @@ struct KrParams {
     const float* al_mag[kKrGroup];
     double* al_acc[kKrGroup];          // 3 doubles: <G, a>, <a, a>, <G, G>
     int al_ld[kKrGroup], al_kb[kKrGroup], al_m[kKrGroup], al_tr[kKrGroup];
-    int al_B;
+    int al_B, al_log2B;                // block size (a power of two) and its log2
     int M[kKrGroup], N[kKrGroup], K[kKrGroup];
     int ktri[kKrGroup];
     int tiles_n[kKrGroup];
@@ -1163,7 +1163,8 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
             const float* const mg = p.al_mag[pi];
             const int ldg = p.al_ld[pi], kbm = p.al_kb[pi], mm = p.al_m[pi];
             const bool tr = p.al_tr[pi] != 0;
-            const int jb = row / p.al_B;
+            const int lgB = p.al_log2B;
+            const int jb = row >> lgB;
             float dot = 0.0f, na = 0.0f, gg = 0.0f;
             for (int c = 0; c < nch * 4; ++c) {
                 const int c0 = n0 + c * 16;
@@ -1172,17 +1173,31 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
                 __syncwarp();
                 ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + h * 256 + c * 16, v);
                 if (row >= M) continue;
+                if (tr) {                                 // product entry (j, i): G[i][j], M[i][j / B]
 #pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    const int ci = c0 + e;
-                    if (ci < mm) {
-                        const long long go = tr ? (long long)ci * ldg + row : (long long)row * ldg + ci;
-                        const long long mo = tr ? (long long)ci * kbm + jb : (long long)row * kbm + ci / p.al_B;
-                        const float g = __bfloat162float(__ushort_as_bfloat16(Gp[go]));
-                        const float a = mg[mo] * v[e];
-                        dot = fmaf(g, a, dot);
-                        na = fmaf(a, a, na);
-                        gg = fmaf(g, g, gg);
+                    for (int e = 0; e < 16; ++e) {
+                        const int ci = c0 + e;
+                        if (ci < mm) {
+                            const float g = __bfloat162float(__ushort_as_bfloat16(Gp[(long long)ci * ldg + row]));
+                            const float a = mg[(long long)ci * kbm + jb] * v[e];
+                            dot = fmaf(g, a, dot);
+                            na = fmaf(a, a, na);
+                            gg = fmaf(g, g, gg);
+                        }
+                    }
+                } else {                                  // product entry (i, j): G[i][j], M[i][j / B]
+                    const uint16_t* grow = Gp + (long long)row * ldg;
+                    const float* mrow = mg + (long long)row * kbm;
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const int ci = c0 + e;
+                        if (ci < mm) {
+                            const float g = __bfloat162float(__ushort_as_bfloat16(grow[ci]));
+                            const float a = mrow[ci >> lgB] * v[e];
+                            dot = fmaf(g, a, dot);
+                            na = fmaf(a, a, na);
+                            gg = fmaf(g, g, gg);
+                        }
                     }
                 }
             }
@@ -2068,6 +2083,8 @@ static int kr_launch(TcState* st, int a_kmajor, const TcGemmItem* items, int cou
             kp.count = cnt;
             kp.status = st->d_status;
             kp.al_B = align_B;
+            kp.al_log2B = 0;
+            while ((1 << kp.al_log2B) < align_B) ++kp.al_log2B;
             if (total == 0) continue;
             if (align_B > 0) {
                 kr_product<true, true, true><<<total, KR_THREADS, KR_SMEM, s>>>(kp);
