@@ -321,8 +321,8 @@ struct RefreshRunner {
         }
         chk(moara::launch_trace_shift(sb, s, &ctx->launches));
         const int nb = moara::kTriBase;
-        moara::GemmKind solve{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
-        moara::GemmKind upd{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_SUB};
+        moara::GemmKind solve{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_STORE, 1};
+        moara::GemmKind upd{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_SUB, 1};
         for (int j0 = 0; j0 < lmax; j0 += nb) {
             chk(moara::launch_chol_diag(sb, j0, s, &ctx->launches));
             std::vector<int> act;

@@ -113,6 +113,7 @@ enum BLayout { B_NCONTIG = 0, B_KCONTIG = 1 };
 
 struct GemmKind {
     int a_layout, b_layout, a_scale, b_scale, a_bf16, b_bf16, epi;
+    int narrow = 0;       // 128 x 64 output tiles, four CTAs per SM (plain fp32 operands, short K)
 };
 
 // Host launchers (return cudaError_t of the launch).

@@ -342,6 +342,151 @@ __global__ void __launch_bounds__(256, 2) k_gemm(const __grid_constant__ GemmBat
     }
 }
 
+// ---------------------------------------------------------------------------
+// Narrow variant for the blocked Cholesky's panel solve and trailing update
+// (K = 64): 128 x 64 output tiles, 8 x 4 per thread, plain fp32 operands,
+// four CTAs per SM, so more tiles are in flight to hide the short K loop's
+// load and store latency.
+// ---------------------------------------------------------------------------
+constexpr int TN2 = 64;
+
+template <int ALAY, int BLAY, int EPI>
+__global__ void __launch_bounds__(256, 4) k_gemm_n64(const __grid_constant__ GemmBatch b) {
+    __shared__ __align__(16) float As[2][TK][TM + TPAD];
+    __shared__ __align__(16) float Bs[2][TK][TN2 + TPAD];
+    const int tile = blockIdx.x;
+    int lo = 0, hi = b.count - 1;
+    while (lo < hi) {
+        int mid = (lo + hi + 1) >> 1;
+        if (b.tile_start[mid] <= tile) lo = mid; else hi = mid - 1;
+    }
+    const GemmProb& p = b.p[lo];
+    const int local = tile - b.tile_start[lo];
+    const int tn = b.tiles_n[lo];
+    const int m0 = (local / tn) * TM;
+    const int n0 = (local % tn) * TN2;
+    if (p.lower_only && n0 >= m0 + TM) return;
+
+    const int t = threadIdx.x;
+    const int tx = t & 15, ty = t >> 4;
+    float acc[8][4];
+#pragma unroll
+    for (int a = 0; a < 8; ++a)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[a][c] = 0.0f;
+
+    int kbeg = 0, kend = p.K;
+    if (p.k_tri == KTRI_B_UPPER) kend = min(p.K, n0 + TN2);
+    else if (p.k_tri == KTRI_B_LOWER) kbeg = min(p.K, n0) & ~(TK - 1);
+    else if (p.k_tri == KTRI_A_LOWER) kend = min(p.K, m0 + TM);
+    const int ktiles = kend > kbeg ? (kend - kbeg + TK - 1) / TK : 0;
+    const float* A = static_cast<const float*>(p.A);
+    const float* Bm = static_cast<const float*>(p.Bm);
+    float ra[NQ], rb[4];
+    auto load = [&](int k0) {
+#pragma unroll
+        for (int q = 0; q < NQ; ++q) {
+            int i, k;
+            if (ALAY == A_KCONTIG) { k = t & (TK - 1); i = (t / TK) + (256 / TK) * q; }
+            else                   { i = t & 127; k = (t >> 7) + 2 * q; }
+            const int gi = m0 + i, gk = k0 + k;
+            ra[q] = (gi < p.M && gk < p.K)
+                        ? __ldg(A + (ALAY == A_KCONTIG ? (long long)gi * p.lda + gk : (long long)gk * p.lda + gi))
+                        : 0.0f;
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            int j, k;
+            if (BLAY == B_NCONTIG) { j = t & 63; k = (t >> 6) + 4 * q; }
+            else                   { k = t & (TK - 1); j = (t / TK) + 16 * q; }
+            const int gj = n0 + j, gk = k0 + k;
+            rb[q] = (gj < p.N && gk < p.K)
+                        ? __ldg(Bm + (BLAY == B_NCONTIG ? (long long)gk * p.ldb + gj : (long long)gj * p.ldb + gk))
+                        : 0.0f;
+        }
+    };
+    auto store = [&](int buf) {
+#pragma unroll
+        for (int q = 0; q < NQ; ++q) {
+            int i, k;
+            if (ALAY == A_KCONTIG) { k = t & (TK - 1); i = (t / TK) + (256 / TK) * q; }
+            else                   { i = t & 127; k = (t >> 7) + 2 * q; }
+            As[buf][k][i] = ra[q];
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            int j, k;
+            if (BLAY == B_NCONTIG) { j = t & 63; k = (t >> 6) + 4 * q; }
+            else                   { k = t & (TK - 1); j = (t / TK) + 16 * q; }
+            Bs[buf][k][j] = rb[q];
+        }
+    };
+    if (ktiles > 0) {
+        load(kbeg);
+        store(0);
+    }
+    __syncthreads();
+    for (int kt = 0; kt < ktiles; ++kt) {
+        const int cur = kt & 1;
+        if (kt + 1 < ktiles) load(kbeg + (kt + 1) * TK);
+#pragma unroll
+        for (int k = 0; k < TK; ++k) {
+            const float4 a0 = *reinterpret_cast<const float4*>(&As[cur][k][ty * 4]);
+            const float4 a1 = *reinterpret_cast<const float4*>(&As[cur][k][64 + ty * 4]);
+            const float4 b0 = *reinterpret_cast<const float4*>(&Bs[cur][k][tx * 4]);
+            const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            const float bv[4] = {b0.x, b0.y, b0.z, b0.w};
+#pragma unroll
+            for (int a = 0; a < 8; ++a)
+#pragma unroll
+                for (int c = 0; c < 4; ++c) acc[a][c] = fmaf(av[a], bv[c], acc[a][c]);
+        }
+        if (kt + 1 < ktiles) store(cur ^ 1);
+        __syncthreads();
+    }
+    const bool vec = (p.ldc & 3) == 0 && (reinterpret_cast<uintptr_t>(p.C) & 15) == 0 &&
+                     (EPI != EPI_STORE || p.c_bf16 == nullptr);
+#pragma unroll
+    for (int a = 0; a < 8; ++a) {
+        const int i = m0 + (a < 4 ? ty * 4 + a : 64 + ty * 4 + (a - 4));
+        if (i >= p.M) continue;
+        const int j = n0 + tx * 4;
+        if (vec && j + 3 < p.N) {
+            float4* dst = reinterpret_cast<float4*>(p.C + (long long)i * p.ldc + j);
+            float4 v = make_float4(acc[a][0], acc[a][1], acc[a][2], acc[a][3]);
+            if (EPI == EPI_SUB) {
+                const float4 c = *dst;
+                v = make_float4(c.x - v.x, c.y - v.y, c.z - v.z, c.w - v.w);
+            } else if (EPI == EPI_STORE_NEG) {
+                v = make_float4(-v.x, -v.y, -v.z, -v.w);
+            }
+            *dst = v;
+        } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (j + c < p.N) epilogue<EPI>(b, p, i, j + c, acc[a][c]);
+        }
+    }
+}
+
+template <int ALAY, int BLAY, int EPI>
+static cudaError_t launch_n64(GemmBatch& b, cudaStream_t s, int64_t* launches) {
+    int total = 0;
+    for (int i = 0; i < b.count; ++i) {
+        const GemmProb& p = b.p[i];
+        const int tm = (p.M + TM - 1) / TM;
+        const int tn = (p.N + TN2 - 1) / TN2;
+        b.tiles_n[i] = tn;
+        b.tile_start[i] = total;
+        total += tm * tn;
+    }
+    b.tile_start[b.count] = total;
+    if (total == 0) return cudaSuccess;
+    k_gemm_n64<ALAY, BLAY, EPI><<<total, 256, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
 template <int ALAY, bool ASC, bool ABF, int BLAY, bool BSC, bool BBF, int EPI>
 static cudaError_t launch_one(GemmBatch& b, cudaStream_t s, int64_t* launches) {
     b.log2B = -1;
@@ -369,6 +514,12 @@ static cudaError_t launch_one(GemmBatch& b, cudaStream_t s, int64_t* launches) {
 // Dispatch over the operand/epilogue combinations the library uses.
 cudaError_t launch_gemm(const GemmKind& k, GemmBatch& b, cudaStream_t s, int64_t* launches) {
     if (b.count <= 0) return cudaSuccess;
+    if (k.narrow && !k.a_scale && !k.b_scale && !k.a_bf16 && !k.b_bf16 && k.a_layout == A_KCONTIG &&
+        k.b_layout == B_KCONTIG) {
+        b.log2B = -1;
+        if (k.epi == EPI_STORE) return launch_n64<A_KCONTIG, B_KCONTIG, EPI_STORE>(b, s, launches);
+        if (k.epi == EPI_SUB) return launch_n64<A_KCONTIG, B_KCONTIG, EPI_SUB>(b, s, launches);
+    }
 #define MOARA_GEMM_CASE(AL, AS, AB, BL, BS, BB, EP)                                         \
     if (k.a_layout == AL && !!k.a_scale == AS && !!k.a_bf16 == AB && k.b_layout == BL &&   \
         !!k.b_scale == BS && !!k.b_bf16 == BB && k.epi == EP)                               \
