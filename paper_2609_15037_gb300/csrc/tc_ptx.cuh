@@ -172,12 +172,13 @@ __device__ __forceinline__ void bulk_wait_read_all() {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 
-// Waits until all committed bulk groups have fully completed.
-// all but the most recent bulk async-group have finished reading their source
+// Waits until all committed bulk groups but the most recent one have finished
+// reading their shared-memory source.
 __device__ __forceinline__ void bulk_wait_read_1() {
     asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
 }
 
+// Waits until all committed bulk groups have fully completed.
 __device__ __forceinline__ void bulk_wait_all() {
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
