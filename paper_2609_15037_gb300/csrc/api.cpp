@@ -196,8 +196,7 @@ size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v) {
     add(sizeof(float) * (size_t)n * l);  // Za (also Omega)
     add(sizeof(float) * (size_t)n * l);  // Zb
     add(sizeof(float) * (size_t)m * l);  // Qa
-    add(sizeof(float) * (size_t)m * l);  // Qb
-    add(sizeof(uint16_t) * (size_t)m * l);  // Qbf
+    add((sizeof(float) + sizeof(uint16_t)) * (size_t)m * l);  // Qb, then Qbf (also 3 bf16 planes of Q)
     add(sizeof(uint16_t) * (size_t)n * l);  // Zbf
     for (int i = 0; i < 3; ++i) add(3 * sizeof(uint16_t) * (size_t)l * l);   // Cp, P1, P2
     for (int i = 0; i < 6; ++i) add(sizeof(float) * (size_t)l * l);
@@ -219,8 +218,10 @@ void refresh_carve(RefreshItem& it, void* base, int m, int n, int r, int l, int 
     it.Omega = it.Za;
     it.Zb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)n * l));
     it.Qa = reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * l));
-    it.Qb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * l));
-    it.Qbf = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * (size_t)m * l));
+    // Qbf follows Qb without padding: the pair holds the three bf16 planes
+    // of a tall Q for the tensor-core CholeskyQR pass
+    it.Qb = reinterpret_cast<float*>(take((sizeof(float) + sizeof(uint16_t)) * (size_t)m * l));
+    it.Qbf = reinterpret_cast<uint16_t*>(it.Qb + (size_t)m * l);
     it.Zbf = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * (size_t)n * l));
     it.Cp = reinterpret_cast<uint16_t*>(take(3 * sizeof(uint16_t) * (size_t)l * l));
     it.P1 = reinterpret_cast<uint16_t*>(take(3 * sizeof(uint16_t) * (size_t)l * l));
@@ -496,6 +497,12 @@ struct RefreshRunner {
         chk(moara::launch_split3(sb, transpose, s, &ctx->launches));
     }
 
+    void ks_run(const std::vector<moara::TcSplitGemmItem>& g) {
+        ProfScope ps(ctx, MOARA_PHASE_TC_REFRESH, s);
+        if (moara::tc_gemm_split3(ctx->tc, g.data(), static_cast<int>(g.size()), s, &ctx->launches) != MOARA_OK)
+            chk(cudaErrorLaunchFailure);
+    }
+
     // out = A B (l x l) from three-plane operands (A stored K x M, B K x N)
     void ks_gemm(const std::vector<uint16_t*>& A, const std::vector<uint16_t*>& B, const std::vector<float*>& out,
                  int ktri) {
@@ -505,9 +512,45 @@ struct RefreshRunner {
             const size_t pl = (size_t)l * l;
             g.push_back({A[i], B[i], pl, pl, out[i], l, l, l, ktri});
         }
-        ProfScope ps(ctx, MOARA_PHASE_TC_REFRESH, s);
-        if (moara::tc_gemm_split3(ctx->tc, g.data(), static_cast<int>(g.size()), s, &ctx->launches) != MOARA_OK)
-            chk(cudaErrorLaunchFailure);
+        ks_run(g);
+    }
+
+    // Shifted CholeskyQR pass of a tall X (rows x l, rows % 8 == 0) with the
+    // Gram matrix X^T X (K = rows) and the triangular apply X R^-1 as
+    // split-precision tensor-core products; X is replaced in place (the apply
+    // reads only the planes).  `pl` holds 3 * rows * l bf16 entries: the
+    // planes of X for the Gram matrix, then those of X^T for the apply.
+    void ks_cholqr_tall(std::vector<float*>& X, const std::vector<uint16_t*>& pl, const std::vector<int>& rows,
+                        float shift_rel) {
+        const size_t n_it = it.size();
+        auto split_rows = [&](int transpose) {
+            moara::SmallBatch sb = small();
+            for (size_t i = 0; i < n_it; ++i) {
+                sb.a[i] = X[i]; sb.h[i] = pl[i]; sb.rows[i] = rows[i]; sb.l[i] = it[i].l;
+            }
+            chk(moara::launch_split3(sb, transpose, s, &ctx->launches));
+        };
+        split_rows(0);                      // X stored K x M (and K x N): rows x l
+        std::vector<moara::TcSplitGemmItem> g;
+        for (size_t i = 0; i < n_it; ++i) {
+            const int l = it[i].l;
+            const size_t pm = (size_t)rows[i] * l;
+            g.push_back({pl[i], pl[i], pm, pm, it[i].Cg, l, l, rows[i], 0});
+        }
+        ks_run(g);                          // Gram X^T X
+        cholesky_blocked(rows, shift_rel);
+        tri_inverse(/*have_diag=*/true);
+        std::vector<float*> linv(n_it);
+        std::vector<uint16_t*> p2(n_it);
+        for (size_t i = 0; i < n_it; ++i) { linv[i] = it[i].Linv; p2[i] = it[i].P2; }
+        split3(linv, p2, 1);                // B = Linv^T (upper triangular)
+        split_rows(1);                      // A = X stored K x M: its transpose, l x rows
+        g.clear();
+        for (size_t i = 0; i < n_it; ++i) {
+            const int l = it[i].l;
+            g.push_back({pl[i], p2[i], (size_t)rows[i] * l, (size_t)l * l, X[i], rows[i], l, l, 1});
+        }
+        ks_run(g);
     }
 
     // One CholeskyQR pass on an l x l matrix with the Gram matrix and the
@@ -605,7 +648,19 @@ struct RefreshRunner {
                     }
                 }
             }
-            cholqr2s(Qa, Qb, rows_m, &qbf);     // Q in Qb (fp32) and qbf
+            bool tall_ks = true;
+            for (int i = 0; i < n_it; ++i) tall_ks = tall_ks && rows_m[i] % 8 == 0;
+            if (tall_ks) {
+                // shifted first pass on tensor cores (the planes of Q fill the
+                // Qb / Qbf pair), the pass that fixes Q's orthonormality on the
+                // fp32 units
+                std::vector<uint16_t*> qpl(n_it);
+                for (int i = 0; i < n_it; ++i) qpl[i] = reinterpret_cast<uint16_t*>(it[i].Qb);
+                ks_cholqr_tall(Qa, qpl, rows_m, 2.0f * u_rnd);
+                cholqr_pass(Qa, Qb, rows_m, 0.0f, &qbf);    // Q in Qb (fp32) and qbf
+            } else {
+                cholqr2s(Qa, Qb, rows_m, &qbf);             // Q in Qb (fp32) and qbf
+            }
             // Rayleigh-Ritz matrix C = Z^T Z with Z = V^T Q (bf16 operands)
             tc_vt_times(qbf, nof, zraw);
             std::vector<moara::TcGemmItem> gram;

@@ -475,43 +475,59 @@ cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* lau
 // set, which leaves the previous projector in place.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_sign_fix_store(const __grid_constant__ SmallBatch b) {
+    // a CTA owns 32 columns: lane = column, the 8 warps split the rows, so
+    // every row segment is one coalesced 128-byte load
+    __shared__ float s_best[8][32];
+    __shared__ int s_bi[8][32];
+    __shared__ float s_sgn[32];
     const int pi = blockIdx.y;
     const int rows = b.rows[pi], r = b.l[pi];
     if (b.fail[pi] != nullptr && *b.fail[pi] != 0) return;
     const float* Pt = b.a[pi];
     float* P = b.c[pi];
     uint16_t* Pb = b.h[pi];
-    const int lane = threadIdx.x & 31;
-    const int wpb = blockDim.x >> 5;
-    for (int q = blockIdx.x * wpb + (threadIdx.x >> 5); q < r; q += gridDim.x * wpb) {
-        // one warp per column: largest |entry| (lowest row on ties)
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int q0 = blockIdx.x * 32; q0 < r; q0 += gridDim.x * 32) {
+        const int q = q0 + lane;
+        const bool col = q < r;
+        // largest |entry| of the column over this warp's rows (ascending, so
+        // the lowest row wins ties)
         float best = -1.0f;
         int bi = 0x7fffffff;
-        for (int i = lane; i < rows; i += 32) {
-            const float a = fabsf(Pt[(long long)i * r + q]);
-            if (a > best) { best = a; bi = i; }
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float ob = __shfl_xor_sync(0xffffffffu, best, o);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-            if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
-        }
-        const float sgnv = (bi < rows && Pt[(long long)bi * r + q] < 0.0f) ? -1.0f : 1.0f;
-        for (int i = lane; i < rows; i += 32) {
-            const float v = Pt[(long long)i * r + q] * sgnv;
-            P[(long long)i * r + q] = v;
-            if (Pb != nullptr) {
-                __nv_bfloat16 h = __float2bfloat16_rn(v);
-                Pb[(long long)i * r + q] = *reinterpret_cast<uint16_t*>(&h);
+        if (col)
+            for (int i = warp; i < rows; i += 8) {
+                const float a = fabsf(Pt[(long long)i * r + q]);
+                if (a > best) { best = a; bi = i; }
             }
+        s_best[warp][lane] = best;
+        s_bi[warp][lane] = bi;
+        __syncthreads();
+        if (warp == 0) {
+            for (int w = 1; w < 8; ++w) {
+                const float ob = s_best[w][lane];
+                const int oi = s_bi[w][lane];
+                if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
+            }
+            s_sgn[lane] = (col && bi < rows && Pt[(long long)bi * r + q] < 0.0f) ? -1.0f : 1.0f;
         }
+        __syncthreads();
+        const float sgnv = s_sgn[lane];
+        if (col)
+            for (int i = warp; i < rows; i += 8) {
+                const float v = Pt[(long long)i * r + q] * sgnv;
+                P[(long long)i * r + q] = v;
+                if (Pb != nullptr) {
+                    __nv_bfloat16 h = __float2bfloat16_rn(v);
+                    Pb[(long long)i * r + q] = *reinterpret_cast<uint16_t*>(&h);
+                }
+            }
+        __syncthreads();   // the shared arrays are reused by the next column group
     }
 }
 
 cudaError_t launch_sign_fix_store(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
     if (b.count <= 0) return cudaSuccess;
-    k_sign_fix_store<<<dim3(32, b.count), 256, 0, s>>>(b);
+    k_sign_fix_store<<<dim3(64, b.count), 256, 0, s>>>(b);
     ++*launches;
     return cudaGetLastError();
 }
