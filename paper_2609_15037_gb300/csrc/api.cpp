@@ -195,8 +195,7 @@ size_t refresh_ws_bytes(int m, int n, int r, int l, int B, int src_v) {
     if (src_v) add(sizeof(float) * (size_t)m * kb);
     add(sizeof(float) * (size_t)n * l);  // Za (also Omega)
     add(sizeof(float) * (size_t)n * l);  // Zb
-    add(sizeof(float) * (size_t)m * l);  // Qa
-    add((sizeof(float) + sizeof(uint16_t)) * (size_t)m * l);  // Qb, then Qbf (also 3 bf16 planes of Q)
+    add(2 * sizeof(float) * (size_t)m * l + align_up(sizeof(uint16_t) * (size_t)m * l, 16));  // Qa, Qbf, Qb
     add(sizeof(uint16_t) * (size_t)n * l);  // Zbf
     for (int i = 0; i < 3; ++i) add(3 * sizeof(uint16_t) * (size_t)l * l);   // Cp, P1, P2
     for (int i = 0; i < 6; ++i) add(sizeof(float) * (size_t)l * l);
@@ -217,11 +216,13 @@ void refresh_carve(RefreshItem& it, void* base, int m, int n, int r, int l, int 
     it.Za = reinterpret_cast<float*>(take(sizeof(float) * (size_t)n * l));
     it.Omega = it.Za;
     it.Zb = reinterpret_cast<float*>(take(sizeof(float) * (size_t)n * l));
-    it.Qa = reinterpret_cast<float*>(take(sizeof(float) * (size_t)m * l));
-    // Qbf follows Qb without padding: the pair holds the three bf16 planes
-    // of a tall Q for the tensor-core CholeskyQR pass
-    it.Qb = reinterpret_cast<float*>(take((sizeof(float) + sizeof(uint16_t)) * (size_t)m * l));
-    it.Qbf = reinterpret_cast<uint16_t*>(it.Qb + (size_t)m * l);
+    // Qa, Qbf, Qb back to back (Qb 16-byte aligned after Qbf): Qbf + Qb
+    // hold the three bf16 planes of a tall Q (3 m l entries) for the
+    // tensor-core CholeskyQR pass
+    const size_t qbf_bytes = align_up(sizeof(uint16_t) * (size_t)m * l, 16);
+    it.Qa = reinterpret_cast<float*>(take(2 * sizeof(float) * (size_t)m * l + qbf_bytes));
+    it.Qbf = reinterpret_cast<uint16_t*>(it.Qa + (size_t)m * l);
+    it.Qb = reinterpret_cast<float*>(reinterpret_cast<char*>(it.Qbf) + qbf_bytes);
     it.Zbf = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * (size_t)n * l));
     it.Cp = reinterpret_cast<uint16_t*>(take(3 * sizeof(uint16_t) * (size_t)l * l));
     it.P1 = reinterpret_cast<uint16_t*>(take(3 * sizeof(uint16_t) * (size_t)l * l));
@@ -624,6 +625,10 @@ struct RefreshRunner {
             zraw[i] = reinterpret_cast<uint16_t*>(it[i].Za);
         }
         const float u_rnd = 5.9604645e-08f;   // fp32 unit roundoff
+        // split-precision tensor-core products with the tall Q need its row
+        // count to be a multiple of 8 (TMA row pitch of Q^T)
+        bool tall_ks = tc;
+        for (int i = 0; i < n_it; ++i) tall_ks = tall_ks && rows_m[i] % 8 == 0;
         if (tc) {
             // Subspace iteration with every product and every intermediate
             // orthonormalisation on tensor cores; only the last Y gets the
@@ -648,14 +653,12 @@ struct RefreshRunner {
                     }
                 }
             }
-            bool tall_ks = true;
-            for (int i = 0; i < n_it; ++i) tall_ks = tall_ks && rows_m[i] % 8 == 0;
             if (tall_ks) {
                 // shifted first pass on tensor cores (the planes of Q fill the
-                // Qb / Qbf pair), the pass that fixes Q's orthonormality on the
+                // Qbf / Qb pair), the pass that fixes Q's orthonormality on the
                 // fp32 units
                 std::vector<uint16_t*> qpl(n_it);
-                for (int i = 0; i < n_it; ++i) qpl[i] = reinterpret_cast<uint16_t*>(it[i].Qb);
+                for (int i = 0; i < n_it; ++i) qpl[i] = it[i].Qbf;
                 ks_cholqr_tall(Qa, qpl, rows_m, 2.0f * u_rnd);
                 cholqr_pass(Qa, Qb, rows_m, 0.0f, &qbf);    // Q in Qb (fp32) and qbf
             } else {
@@ -793,15 +796,18 @@ struct RefreshRunner {
             }
             chk(moara::launch_gather_cols(sb, s, &ctx->launches));
         }
-        // P_tmp (m x r) = Q * Xs into Qa
+        // P_tmp (m x r) = Q * Xs into Qa, on the fp32 units: the final
+        // projector's orthonormality is fixed here (a split-precision
+        // tensor-core product leaves column norms ~1e-5 short)
         gemm(prod, [&](int i, moara::GemmProb& p) {
             p.A = Qb[i]; p.Bm = Xb[i]; p.C = Qa[i];
             p.M = it[i].m; p.N = it[i].r; p.K = it[i].l; p.lda = it[i].l; p.ldb = it[i].r; p.ldc = it[i].r;
         });
+        const std::vector<float*>& ptmp = Qa;
         {
             moara::SmallBatch sb = small();
             for (int i = 0; i < n_it; ++i) {
-                sb.a[i] = Qa[i]; sb.c[i] = it[i].P; sb.h[i] = it[i].Pb; sb.fail[i] = it[i].fail;
+                sb.a[i] = ptmp[i]; sb.c[i] = it[i].P; sb.h[i] = it[i].Pb; sb.fail[i] = it[i].fail;
                 sb.rows[i] = it[i].m; sb.l[i] = it[i].r;
             }
             chk(moara::launch_sign_fix_store(sb, s, &ctx->launches));
