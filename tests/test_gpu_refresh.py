@@ -163,13 +163,15 @@ def test_refresh_workspace_too_small(M):
     g.close()
 
 
+@pytest.mark.parametrize("m", [384, 390])
 @pytest.mark.parametrize("src", ["V", "G"])
-def test_refresh_clear_gap_bf16_tensor_cores(M, src):
+def test_refresh_clear_gap_bf16_tensor_cores(M, src, m):
     """bf16 gradient: the refresh products run on tensor cores (V = V_hi + V_lo
     in bf16, Q and Z in bf16).  Same clear-gap spectrum as above, exact in
     bf16; all r directions and each singular vector individually, in order and
-    with the oracle's sign convention."""
-    m, n, r, B = 384, 512, 16, 64
+    with the oracle's sign convention.  m = 390 (not a multiple of 8) takes
+    the fp32 CholeskyQR2 of the tall Q instead of the split-precision pass."""
+    n, r, B = 512, 16, 64
     u, v = synth.lowrank_factors(m, n, r + 8, seed=5)
     sig = np.concatenate([10.0 * 0.7 ** np.arange(r), 0.01 * 0.7 ** np.arange(8)])
     G = (u * sig) @ v.T + 1e-4 * np.random.default_rng(1).standard_normal((m, n))
