@@ -495,6 +495,37 @@ def _oracle_layer_sample(wl, layer_modules, seed=0, rule="left", state_bf16=Fals
     return states, grads, hp
 
 
+def _oracle_module_ms(args, threads):
+    """Oracle step time (best of two) of layer 0's first module, in a child
+    process whose BLAS runs `threads` threads (the thread count is fixed when
+    NumPy loads its BLAS, hence the child)."""
+    rule = getattr(args, "proj_rule", "left")
+    sb = getattr(args, "state_dtype", "f32") == "bf16"
+    code = "\n".join([
+        "import sys, time, json",
+        f"sys.path.insert(0, {ROOT!r})",
+        "import bench, synth",
+        "from oracle import moara_ref as o",
+        f"wl = synth.workload({args.workload!r})",
+        "md = [m for m in wl['modules'] if m.name.startswith('layer0.')][0]",
+        f"st, gr, hp = bench._oracle_layer_sample(wl, [md], rule={rule!r}, state_bf16={sb!r})",
+        "best = 1e30",
+        "for t in (1, 2):",
+        "    t0 = time.perf_counter()",
+        "    st[0] = o.step(st[0], gr[0], t, bench.LR, hp, refresh=False)",
+        "    best = min(best, time.perf_counter() - t0)",
+        "print(json.dumps({'ms': best * 1e3, 'shape': f'{md.m}x{md.n} r {md.r}'}))",
+    ])
+    env = dict(os.environ, OMP_NUM_THREADS=str(threads), OPENBLAS_NUM_THREADS=str(threads),
+               MKL_NUM_THREADS=str(threads))
+    try:
+        res = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                             timeout=300, cwd=ROOT)
+        return json.loads(res.stdout.strip().splitlines()[-1])
+    except Exception:
+        return None
+
+
 def cpu_baseline(args, budget_s=20.0):
     """The oracle as it stands, one 7B decoder layer per sample, scaled to the
     full model (x layers).  Runs in this process on the host cores."""
@@ -523,10 +554,17 @@ def cpu_baseline(args, budget_s=20.0):
     except Exception:
         cores = os.cpu_count()
     threads = os.environ.get("OMP_NUM_THREADS") or os.environ.get("OPENBLAS_NUM_THREADS") or str(cores)
-    return {"value": round(per_layer * layers * 1e3, 1), "unit": "ms", "cores": int(threads),
-            "kind": "oracle",
-            "sample": f"one decoder layer (7 modules) of the {len(wl['modules'])}-matrix model, "
-                      f"float64 NumPy step without refresh, best of {len(times)}, x{layers} layers"}
+    out = {"value": round(per_layer * layers * 1e3, 1), "unit": "ms", "cores": int(threads),
+           "kind": "oracle",
+           "sample": f"one decoder layer (7 modules) of the {len(wl['modules'])}-matrix model, "
+                     f"float64 NumPy step without refresh, best of {len(times)}, x{layers} layers"}
+    # the same oracle on one module at one BLAS thread and at all of them
+    one = _oracle_module_ms(args, 1)
+    allc = _oracle_module_ms(args, int(threads))
+    if one is not None and allc is not None:
+        out["one_module"] = {"shape": one["shape"], "ms_1_thread": round(one["ms"], 1),
+                             "ms_all_threads": round(allc["ms"], 1), "threads": int(threads)}
+    return out
 
 
 def run_reference(args):
