@@ -339,8 +339,9 @@ def run_gpu(args):
                 x.copy_(h, non_blocking=True)
             M.moara_step_grouped(g.ctx, ids, gptr, st, LR, False, cs)
 
-    e2e_step(step)   # staging allocation
-    step += 1
+    for _ in range(max(1, args.warmup)):   # staging allocation, then the same warm-up as the device timing
+        e2e_step(step)
+        step += 1
     torch.cuda.synchronize()
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps + 1)]
     evs[0].record(stream)
