@@ -433,14 +433,16 @@ struct RefreshRunner {
     }
 
     // out (n x l) = V^T X with X (m x l) in bf16; fp32 and/or bf16 output
+    // (`lo` false: V_hi alone, for products whose output is rounded to bf16
+    // anyway, the intermediate iterates of the subspace iteration)
     void tc_vt_times(const std::vector<uint16_t*>& X, const std::vector<float*>& out,
-                     const std::vector<uint16_t*>& out_bf) {
+                     const std::vector<uint16_t*>& out_bf, bool lo = true) {
         // V stored m x n is read MN-major; for a transposed item (V^T) the
         // same product is V X with V read K-major
         std::vector<moara::TcGemmItem> g[2];
         for (size_t i = 0; i < it.size(); ++i) {
             const auto& x = it[i];
-            g[x.trans ? 1 : 0].push_back({x.Vhi, x.Vlo, X[i], out[i], out_bf[i], x.n, x.l, x.m, 0});
+            g[x.trans ? 1 : 0].push_back({x.Vhi, lo ? x.Vlo : nullptr, X[i], out[i], out_bf[i], x.n, x.l, x.m, 0});
         }
         tc_gemm(0, g[0]);
         tc_gemm(1, g[1]);
@@ -448,11 +450,11 @@ struct RefreshRunner {
 
     // out (m x l) = V Z with Z (n x l) in bf16
     void tc_v_times(const std::vector<uint16_t*>& Z, const std::vector<float*>& out,
-                    const std::vector<uint16_t*>& out_bf) {
+                    const std::vector<uint16_t*>& out_bf, bool lo = true) {
         std::vector<moara::TcGemmItem> g[2];
         for (size_t i = 0; i < it.size(); ++i) {
             const auto& x = it[i];
-            g[x.trans ? 1 : 0].push_back({x.Vhi, x.Vlo, Z[i], out[i], out_bf[i], x.m, x.l, x.n, 0});
+            g[x.trans ? 1 : 0].push_back({x.Vhi, lo ? x.Vlo : nullptr, Z[i], out[i], out_bf[i], x.m, x.l, x.n, 0});
         }
         tc_gemm(1, g[0]);
         tc_gemm(0, g[1]);
@@ -640,13 +642,15 @@ struct RefreshRunner {
             if (q_it == 0) {
                 tc_v_times(zbf, Qa, nob);
             } else {
-                tc_v_times(zbf, nof, ybf);
+                // the iterates rounded to bf16 take V_hi alone; the last Y and
+                // the Rayleigh-Ritz product take V_hi + V_lo
+                tc_v_times(zbf, nof, ybf, false);
                 tc_cholqr_pass(ybf, qbf, rows_m, 2.0f * u_rnd);
                 for (int q = 0; q < q_it; ++q) {
-                    tc_vt_times(qbf, nof, zraw);
+                    tc_vt_times(qbf, nof, zraw, false);
                     tc_cholqr_pass(zraw, zbf, rows_n, 2.0f * u_rnd);
                     if (q + 1 < q_it) {
-                        tc_v_times(zbf, nof, ybf);
+                        tc_v_times(zbf, nof, ybf, false);
                         tc_cholqr_pass(ybf, qbf, rows_m, 2.0f * u_rnd);
                     } else {
                         tc_v_times(zbf, Qa, nob);
