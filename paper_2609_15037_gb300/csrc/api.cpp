@@ -500,22 +500,25 @@ struct RefreshRunner {
         chk(moara::launch_split3(sb, transpose, s, &ctx->launches));
     }
 
-    void ks_run(const std::vector<moara::TcSplitGemmItem>& g) {
+    // planes = 3: fp32-accurate operands; 2: hi + mid (16 bits), for iterates
+    // that a later fp32-accurate pass corrects
+    void ks_run(const std::vector<moara::TcSplitGemmItem>& g, int planes) {
         ProfScope ps(ctx, MOARA_PHASE_TC_REFRESH, s);
-        if (moara::tc_gemm_split3(ctx->tc, g.data(), static_cast<int>(g.size()), s, &ctx->launches) != MOARA_OK)
+        if (moara::tc_gemm_split3(ctx->tc, g.data(), static_cast<int>(g.size()), planes, s, &ctx->launches) !=
+            MOARA_OK)
             chk(cudaErrorLaunchFailure);
     }
 
     // out = A B (l x l) from three-plane operands (A stored K x M, B K x N)
     void ks_gemm(const std::vector<uint16_t*>& A, const std::vector<uint16_t*>& B, const std::vector<float*>& out,
-                 int ktri) {
+                 int ktri, int planes) {
         std::vector<moara::TcSplitGemmItem> g;
         for (size_t i = 0; i < it.size(); ++i) {
             const int l = it[i].l;
             const size_t pl = (size_t)l * l;
             g.push_back({A[i], B[i], pl, pl, out[i], l, l, l, ktri});
         }
-        ks_run(g);
+        ks_run(g, planes);
     }
 
     // Shifted CholeskyQR pass of a tall X (rows x l, rows % 8 == 0) with the
@@ -524,7 +527,7 @@ struct RefreshRunner {
     // reads only the planes).  `pl` holds 3 * rows * l bf16 entries: the
     // planes of X for the Gram matrix, then those of X^T for the apply.
     void ks_cholqr_tall(std::vector<float*>& X, const std::vector<uint16_t*>& pl, const std::vector<int>& rows,
-                        float shift_rel) {
+                        float shift_rel, int planes) {
         const size_t n_it = it.size();
         auto split_rows = [&](int transpose) {
             moara::SmallBatch sb = small();
@@ -540,7 +543,7 @@ struct RefreshRunner {
             const size_t pm = (size_t)rows[i] * l;
             g.push_back({pl[i], pl[i], pm, pm, it[i].Cg, l, l, rows[i], 0});
         }
-        ks_run(g);                          // Gram X^T X
+        ks_run(g, planes);                  // Gram X^T X
         cholesky_blocked(rows, shift_rel);
         tri_inverse(/*have_diag=*/true);
         std::vector<float*> linv(n_it);
@@ -553,27 +556,27 @@ struct RefreshRunner {
             const int l = it[i].l;
             g.push_back({pl[i], p2[i], (size_t)rows[i] * l, (size_t)l * l, X[i], rows[i], l, l, 1});
         }
-        ks_run(g);
+        ks_run(g, planes);
     }
 
     // One CholeskyQR pass on an l x l matrix with the Gram matrix and the
     // triangular apply as split-precision tensor-core products (fp32-accurate):
     // Xout = Win R^-1, R^T R = Win^T Win + shift.
     void ks_cholqr_pass(std::vector<float*>& Win, std::vector<float*>& Xout, const std::vector<int>& rows_l,
-                        float shift_rel) {
+                        float shift_rel, int planes) {
         std::vector<uint16_t*> p1(it.size()), p2(it.size());
         for (size_t i = 0; i < it.size(); ++i) { p1[i] = it[i].P1; p2[i] = it[i].P2; }
         std::vector<float*> cg(it.size());
         for (size_t i = 0; i < it.size(); ++i) cg[i] = it[i].Cg;
         split3(Win, p1, 0);                 // W (as A = W^T, MN-major, and as B)
-        ks_gemm(p1, p1, cg, 0);             // Gram W^T W
+        ks_gemm(p1, p1, cg, 0, planes);     // Gram W^T W
         cholesky_blocked(rows_l, shift_rel);
         tri_inverse(/*have_diag=*/true);
         std::vector<float*> linv(it.size());
         for (size_t i = 0; i < it.size(); ++i) linv[i] = it[i].Linv;
         split3(linv, p2, 1);                // B = Linv^T (upper triangular)
         split3(Win, p1, 1);                 // A = W read MN-major: its transpose
-        ks_gemm(p1, p2, Xout, 1);
+        ks_gemm(p1, p2, Xout, 1, planes);
     }
 
     void run() {
@@ -663,7 +666,7 @@ struct RefreshRunner {
                 // fp32 units
                 std::vector<uint16_t*> qpl(n_it);
                 for (int i = 0; i < n_it; ++i) qpl[i] = it[i].Qbf;
-                ks_cholqr_tall(Qa, qpl, rows_m, 2.0f * u_rnd);
+                ks_cholqr_tall(Qa, qpl, rows_m, 2.0f * u_rnd, 2);
                 cholqr_pass(Qa, Qb, rows_m, 0.0f, &qbf);    // Q in Qb (fp32) and qbf
             } else {
                 cholqr2s(Qa, Qb, rows_m, &qbf);             // Q in Qb (fp32) and qbf
@@ -754,13 +757,17 @@ struct RefreshRunner {
         if (tc) split3(cr, cp, 0);          // C is symmetric: read MN-major as A
         for (int q = 0; q < hp.ritz_iters; ++q) {
             if (tc) {
+                // the iterations before the last carry hi + mid planes (16
+                // bits): the later iterations correct them
+                const bool last = q + 1 == hp.ritz_iters;
+                const int planes = last ? 3 : 2;
                 split3(Xa, p1, 0);
-                ks_gemm(cp, p1, Xb, 0);                  // W = C X
-                ks_cholqr_pass(Xb, Xa, rows_l, 2.0f * u_rnd);
+                ks_gemm(cp, p1, Xb, 0, planes);          // W = C X
+                ks_cholqr_pass(Xb, Xa, rows_l, 2.0f * u_rnd, planes);
                 // the tensor cores accumulate long sums less tightly than
                 // fp32 FMAs: the pass that fixes the final orthonormality of
                 // X runs on the fp32 units
-                if (q + 1 < hp.ritz_iters) ks_cholqr_pass(Xa, Xb, rows_l, 0.0f);
+                if (!last) ks_cholqr_pass(Xa, Xb, rows_l, 0.0f, planes);
                 else cholqr_pass(Xa, Xb, rows_l, 0.0f);
                 std::swap(Xa, Xb);                       // X in Xa
             } else {
@@ -776,7 +783,7 @@ struct RefreshRunner {
         // W = C X into Xb
         if (tc) {
             split3(Xa, p1, 0);
-            ks_gemm(cp, p1, Xb, 0);
+            ks_gemm(cp, p1, Xb, 0, 3);
         } else {
             gemm(prod, [&](int i, moara::GemmProb& p) {
                 const int l = it[i].l;

@@ -1288,9 +1288,16 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
 // ===========================================================================
 constexpr int KS_BM = 256, KS_BN = 256, KS_BK = 32;
 constexpr int KS_PLANE = KS_BM * KS_BK * 2;               // 16 KB: one plane of A (or B)
-constexpr int KS_STAGE = 6 * KS_PLANE;                    // 96 KB
-constexpr int KS_STAGES = 2;
-constexpr int KS_SMEM = 1024 + KS_STAGES * KS_STAGE + 2048;
+constexpr int KS_RING = 12 * KS_PLANE;                    // 192 KB of stages
+constexpr int KS_SMEM = 1024 + KS_RING + 2048;
+// NP = 3 planes: six products per k-step, two stages of 96 KB.  NP = 2
+// (hi + mid, 16 significant bits; for iterates that a later fp32-accurate
+// pass corrects): three products (hi.hi, hi.mid, mid.hi), three stages of 64 KB.
+template <int NP> struct KsCfg {
+    static constexpr int STAGE = 2 * NP * KS_PLANE;
+    static constexpr int STAGES = KS_RING / STAGE;
+    static constexpr int PRODUCTS = NP == 3 ? 6 : 3;
+};
 constexpr int kKsGroup = 36;                              // problems per launch (six maps each in the parameters)
 
 struct KsParams {
@@ -1305,10 +1312,12 @@ struct KsParams {
     int* status;
 };
 
+template <int NP>
 __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constant__ KsParams p) {
+    constexpr int KS_STAGE = KsCfg<NP>::STAGE, KS_STAGES = KsCfg<NP>::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
-    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + KS_STAGES * KS_STAGE);
+    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + KS_RING);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int* abort_flag = &ctl->abort;
 
@@ -1352,7 +1361,7 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued = 0, last_par = 0;
-            const uint32_t bytes = 3 * KS_PLANE + 3 * nch * 4096;
+            const uint32_t bytes = NP * KS_PLANE + NP * nch * 4096;
             for (int kb = 0; kb < nk; ++kb) {
                 if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
                                     MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) {
@@ -1363,9 +1372,9 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
                 const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
                 ptx::mbar_arrive_expect_tx(fb, bytes);
                 const uint32_t a = ptx::smem_u32(smem + stage * KS_STAGE);
-                const uint32_t b = a + 3 * KS_PLANE;
+                const uint32_t b = a + NP * KS_PLANE;
 #pragma unroll
-                for (int q = 0; q < 3; ++q) {
+                for (int q = 0; q < NP; ++q) {
 #pragma unroll
                     for (int c = 0; c < 4; ++c)
                         ptx::tma_load_2d(a + q * KS_PLANE + c * 4096, &p.amap[pi][q], fb, i0 + 64 * c, kb * KS_BK);
@@ -1390,11 +1399,11 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
                                     MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) break;
                 ptx::tc_fence_after();
                 const uint32_t a = ptx::smem_u32(smem + stage * KS_STAGE);
-                const uint32_t b = a + 3 * KS_PLANE;
+                const uint32_t b = a + NP * KS_PLANE;
 #pragma unroll
                 for (int kk = 0; kk < 2; ++kk) {
 #pragma unroll
-                    for (int e = 0; e < 6; ++e) {
+                    for (int e = 0; e < KsCfg<NP>::PRODUCTS; ++e) {
                         const uint64_t bdesc = ptx::smem_desc_sw128(b + PB[e] * KS_PLANE + kk * 2048, 4096, 1024);
                         for (int h = 0; h < halves; ++h) {
                             const uint64_t adesc =
@@ -2310,10 +2319,16 @@ int tc_split_v(TcState* st, const TcSplitItem* items, int count, int B, float de
     return MOARA_OK;
 }
 
-int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, cudaStream_t s, int64_t* launches) {
+int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, int planes, cudaStream_t s,
+                   int64_t* launches) {
     if (!st->ks_attrs) {
-        cudaFuncSetAttribute(ks_product, cudaFuncAttributeMaxDynamicSharedMemorySize, KS_SMEM);
+        cudaFuncSetAttribute(ks_product<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, KS_SMEM);
+        cudaFuncSetAttribute(ks_product<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, KS_SMEM);
         st->ks_attrs = true;
+    }
+    if (planes != 2 && planes != 3) {
+        st->err = "split-precision GEMM: 2 or 3 planes";
+        return MOARA_ERR_INVALID_ARG;
     }
     for (int i = 0; i < count; ++i) {
         const TcSplitGemmItem& x = items[i];
@@ -2349,7 +2364,8 @@ int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, cudaStr
         kp.count = cnt;
         kp.status = st->d_status;
         if (total == 0) continue;
-        ks_product<<<total, KR_THREADS, KS_SMEM, s>>>(kp);
+        if (planes == 3) ks_product<3><<<total, KR_THREADS, KS_SMEM, s>>>(kp);
+        else ks_product<2><<<total, KR_THREADS, KS_SMEM, s>>>(kp);
         const cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) {
             st->err = cudaGetErrorString(e);

@@ -78,7 +78,10 @@ struct TcSplitGemmItem {
 };
 
 // Grouped launch; M and N multiples of 8, planes 16-byte aligned.
-int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, cudaStream_t s, int64_t* launches);
+// planes = 3: hi + mid + lo (fp32-accurate); planes = 2: hi + mid only
+// (16 significant bits, three products per k-step).
+int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, int planes, cudaStream_t s,
+                   int64_t* launches);
 
 // V = Decompose(G, B) direction as two bf16 planes (V_hi, V_lo) for the
 // refresh products; G bf16 m x n, B in {8, ..., 128}.
