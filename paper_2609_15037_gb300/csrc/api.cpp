@@ -250,6 +250,9 @@ int refresh_l(const moara_ctx* ctx, int m, int n, int r) {
 }
 
 // ------------------------------------------------------------------ refresh
+// Panel width of the fast blocked Cholesky (tensor-core trailing updates).
+constexpr int kFastPanel = 256;
+
 struct RefreshRunner {
     moara_ctx* ctx;
     cudaStream_t s;
@@ -311,7 +314,7 @@ struct RefreshRunner {
     // Lower Cholesky factor of Cg (+ shift on the diagonal) in place, by 64-wide
     // panels: factor the diagonal block (its inverse goes to the diagonal block
     // of Linv), solve the panel below it, update the trailing matrix.
-    void cholesky_blocked(const std::vector<int>& rows, float shift_rel) {
+    void cholesky_blocked(const std::vector<int>& rows, float shift_rel, bool fast = false) {
         int lmax = 0;
         moara::SmallBatch sb = small();
         sb.shift_rel = shift_rel;
@@ -327,19 +330,21 @@ struct RefreshRunner {
         moara::GemmKind upd{moara::A_KCONTIG, moara::B_KCONTIG, 0, 0, 0, 0, moara::EPI_SUB, 1};
         for (int j0 = 0; j0 < lmax; j0 += nb) {
             chk(moara::launch_chol_diag(sb, j0, s, &ctx->launches));
-            std::vector<int> act;
-            for (int i = 0; i < static_cast<int>(it.size()); ++i)
-                if (j0 + nb < it[i].l) act.push_back(i);
-            if (act.empty()) continue;
+            // fast: the 64-wide steps update only the rest of their
+            // kFastPanel-wide panel; the trailing matrix past the panel gets
+            // one tensor-core update per panel
+            const int pend = fast ? (j0 / kFastPanel + 1) * kFastPanel : lmax;
             for (int pass = 0; pass < 2; ++pass) {
                 moara::GemmBatch b{};
-                b.count = static_cast<int>(act.size());
                 b.B = 1;
-                for (int q = 0; q < b.count; ++q) {
-                    const auto& x = it[act[q]];
+                for (int i = 0; i < static_cast<int>(it.size()); ++i) {
+                    const auto& x = it[i];
                     const long long l = x.l;
                     const int j1 = j0 + nb;
-                    moara::GemmProb& p = b.p[q];
+                    if (j1 >= x.l) continue;
+                    const int cend = std::min(x.l, pend);
+                    if (pass == 1 && cend <= j1) continue;
+                    moara::GemmProb& p = b.p[b.count++];
                     p = moara::GemmProb{};
                     p.lda = p.ldb = p.ldc = x.l;
                     if (pass == 0) {      // L[j1:, panel] = A[j1:, panel] * Ljj^-T (in place)
@@ -347,17 +352,46 @@ struct RefreshRunner {
                         p.Bm = x.Linv + j0 * l + j0;
                         p.C = x.Cg + j1 * l + j0;
                         p.M = x.l - j1; p.N = nb; p.K = nb;
-                    } else {              // A[j1:, j1:] -= L[j1:, panel] L[j1:, panel]^T (lower tiles)
+                    } else {              // A[j1:, j1:cend] -= L[j1:, panel] L[j1:cend, panel]^T (lower tiles)
                         p.A = x.Cg + j1 * l + j0;
                         p.Bm = x.Cg + j1 * l + j0;
                         p.C = x.Cg + j1 * l + j1;
-                        p.M = x.l - j1; p.N = x.l - j1; p.K = nb;
+                        p.M = x.l - j1; p.N = cend - j1; p.K = nb;
                         p.lower_only = 1;
                     }
                 }
-                chk(moara::launch_gemm(pass == 0 ? solve : upd, b, s, &ctx->launches));
+                if (b.count > 0) chk(moara::launch_gemm(pass == 0 ? solve : upd, b, s, &ctx->launches));
             }
+            if (fast && j0 + nb == pend) trailing_update_tc(pend);
         }
+    }
+
+    // A[pe:, pe:] -= L[pe:, pe - kFastPanel : pe] L[pe:, ...]^T (lower tiles)
+    // for every item with l > pe, as a two-plane split-precision product
+    // (16 significant bits): the panel's transposed planes go to P1.
+    void trailing_update_tc(int pe) {
+        moara::SmallBatch sq{};
+        std::vector<moara::TcSplitGemmItem> g;
+        for (size_t i = 0; i < it.size(); ++i) {
+            const auto& x = it[i];
+            if (x.l <= pe) continue;
+            const int rest = x.l - pe;
+            const int q = sq.count++;
+            sq.a[q] = x.Cg + (size_t)pe * x.l + (pe - kFastPanel);
+            sq.h[q] = x.P1;
+            sq.rows[q] = rest;
+            sq.l[q] = kFastPanel;
+            sq.ld[q] = x.l;
+            const size_t pl = (size_t)rest * kFastPanel;
+            moara::TcSplitGemmItem item{x.P1, x.P1, pl, pl, x.Cg + (size_t)pe * x.l + pe, rest, rest, kFastPanel, 0};
+            item.ldo = x.l;
+            item.sub = 1;
+            item.lower = 1;
+            g.push_back(item);
+        }
+        if (g.empty()) return;
+        chk(moara::launch_split3(sq, 1, s, &ctx->launches));
+        ks_run(g, 2);
     }
 
     void tri_inverse(bool have_diag) {
@@ -473,7 +507,7 @@ struct RefreshRunner {
             gram.push_back({Xin[i], nullptr, Xin[i], it[i].Cg, nullptr, l, l, rows[i], 0});
         }
         tc_gemm(0, gram);
-        cholesky_blocked(rows, shift_rel);
+        cholesky_blocked(rows, shift_rel, /*fast=*/true);
         tri_inverse(/*have_diag=*/true);
         {   // (R^-1) in bf16: the transpose of the lower-triangular Linv, into Tt
             moara::SmallBatch sb = small();
@@ -544,7 +578,7 @@ struct RefreshRunner {
             g.push_back({pl[i], pl[i], pm, pm, it[i].Cg, l, l, rows[i], 0});
         }
         ks_run(g, planes);                  // Gram X^T X
-        cholesky_blocked(rows, shift_rel);
+        cholesky_blocked(rows, shift_rel, /*fast=*/true);
         tri_inverse(/*have_diag=*/true);
         std::vector<float*> linv(n_it);
         std::vector<uint16_t*> p2(n_it);
@@ -570,7 +604,7 @@ struct RefreshRunner {
         for (size_t i = 0; i < it.size(); ++i) cg[i] = it[i].Cg;
         split3(Win, p1, 0);                 // W (as A = W^T, MN-major, and as B)
         ks_gemm(p1, p1, cg, 0, planes);     // Gram W^T W
-        cholesky_blocked(rows_l, shift_rel);
+        cholesky_blocked(rows_l, shift_rel, /*fast=*/true);
         tri_inverse(/*have_diag=*/true);
         std::vector<float*> linv(it.size());
         for (size_t i = 0; i < it.size(); ++i) linv[i] = it[i].Linv;

@@ -191,6 +191,7 @@ struct SmallBatch {
     int* fail[kMaxGroup];
     int* iaux[kMaxGroup];
     uint16_t* h[kMaxGroup];
+    int ld[kMaxGroup];    // row pitch of a (split3), 0: l
     float shift_rel;      // diagonal shift: shift_rel * sqrt(rows) * trace
     uint64_t key[kMaxGroup];
 };

@@ -331,9 +331,9 @@ cudaError_t launch_transpose_bf16(const SmallBatch& b, cudaStream_t s, int64_t* 
 }
 
 // ---------------------------------------------------------------------------
-// Three bf16 planes of an fp32 matrix (rows x l, row-major): hi = bf16(x),
-// mid = bf16(x - hi), lo = bf16(x - hi - mid), so hi + mid + lo carries 24
-// significant bits.  With `transpose` the planes hold the l x rows transpose.
+// Three bf16 planes of an fp32 matrix (rows x l, row-major, row pitch ld or
+// l): hi = bf16(x), mid = bf16(x - hi), lo = bf16(x - hi - mid), so
+// hi + mid + lo carries 24 significant bits.  With `transpose` the planes hold the l x rows transpose.
 // Planes are consecutive at h, each rows * l elements.  32 x 32 tiles through
 // shared memory keep both sides coalesced.
 // ---------------------------------------------------------------------------
@@ -341,6 +341,7 @@ __global__ void __launch_bounds__(256) k_split3(const __grid_constant__ SmallBat
     __shared__ float t[32][33];
     const int pi = blockIdx.z;
     const int rows = b.rows[pi], cols = b.l[pi];
+    const long long lds = b.ld[pi] > 0 ? b.ld[pi] : cols;
     const float* src = b.a[pi];
     uint16_t* dst = b.h[pi];
     const long long plane = (long long)rows * cols;
@@ -350,7 +351,7 @@ __global__ void __launch_bounds__(256) k_split3(const __grid_constant__ SmallBat
         const int ti = tile / tc, tj = tile - ti * tc;
         for (int r = ty; r < 32; r += 8) {
             const int i = ti * 32 + r, j = tj * 32 + tx;
-            t[r][tx] = (i < rows && j < cols) ? src[(long long)i * cols + j] : 0.0f;
+            t[r][tx] = (i < rows && j < cols) ? src[(long long)i * lds + j] : 0.0f;
         }
         __syncthreads();
         for (int r = ty; r < 32; r += 8) {

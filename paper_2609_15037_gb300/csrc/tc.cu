@@ -1306,6 +1306,9 @@ struct KsParams {
     float* out[kKsGroup];
     int M[kKsGroup], N[kKsGroup], K[kKsGroup];
     int ktri[kKsGroup];
+    int ldo[kKsGroup];                 // row pitch of out
+    int sub[kKsGroup];                 // out -= A B
+    int lower[kKsGroup];               // tiles above the diagonal are skipped
     int tiles_n[kKsGroup];
     int tile_start[kKsGroup + 1];
     int count;
@@ -1332,6 +1335,7 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
     const int M = p.M[pi], N = p.N[pi], K = p.K[pi];
     const int i0 = (local / p.tiles_n[pi]) * KS_BM;
     const int n0 = (local % p.tiles_n[pi]) * KS_BN;
+    if (p.lower[pi] && n0 >= i0 + KS_BM) return;     // whole CTA, before any barrier or TMEM
     const int nch = min(4, (N - n0 + 63) / 64);
     const int halves = (M - i0) > 128 ? 2 : 1;
     const int kend = p.ktri[pi] ? min(K, n0 + KS_BN) : K;
@@ -1429,7 +1433,8 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
             ptx::tc_fence_after();
             const int row = i0 + h * 128 + q * 32 + lane;
             float* const of = p.out[pi];
-            const long long ro = (long long)row * N;
+            const long long ro = (long long)row * p.ldo[pi];
+            const bool sub = p.sub[pi] != 0;
             for (int c = 0; c < nch * 4; ++c) {
                 const int j0 = n0 + c * 16;
                 if (j0 >= N) break;                       // warp-uniform
@@ -1440,11 +1445,18 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
                 if (j0 + 16 <= N) {
                     float4* o4 = reinterpret_cast<float4*>(of + ro + j0);
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) o4[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+                    for (int e = 0; e < 4; ++e) {
+                        float4 w = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+                        if (sub) {
+                            const float4 o = o4[e];
+                            w = make_float4(o.x - w.x, o.y - w.y, o.z - w.z, o.w - w.w);
+                        }
+                        o4[e] = w;
+                    }
                 } else {
 #pragma unroll
                     for (int e = 0; e < 16; ++e)
-                        if (j0 + e < N) of[ro + j0 + e] = v[e];
+                        if (j0 + e < N) of[ro + j0 + e] = sub ? of[ro + j0 + e] - v[e] : v[e];
                 }
             }
         }
@@ -2336,6 +2348,11 @@ int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, int pla
             st->err = "split-precision GEMM: M and N must be multiples of 8";
             return MOARA_ERR_UNSUPPORTED;
         }
+        const int ldo = x.ldo > 0 ? x.ldo : x.N;
+        if (ldo < x.N || (ldo % 4) != 0 || (reinterpret_cast<uintptr_t>(x.out) & 15) != 0) {
+            st->err = "split-precision GEMM: out must be 16-byte aligned with a row pitch >= N, a multiple of 4";
+            return MOARA_ERR_UNSUPPORTED;
+        }
     }
     for (int c0 = 0; c0 < count; c0 += kKsGroup) {
         const int cnt = std::min(kKsGroup, count - c0);
@@ -2356,6 +2373,9 @@ int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, int pla
             kp.out[q] = x.out;
             kp.M[q] = x.M; kp.N[q] = x.N; kp.K[q] = x.K;
             kp.ktri[q] = x.ktri;
+            kp.ldo[q] = x.ldo > 0 ? x.ldo : x.N;
+            kp.sub[q] = x.sub;
+            kp.lower[q] = x.lower;
             kp.tiles_n[q] = (x.N + KS_BN - 1) / KS_BN;
             kp.tile_start[q] = total;
             total += ((x.M + KS_BM - 1) / KS_BM) * kp.tiles_n[q];

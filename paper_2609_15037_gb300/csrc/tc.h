@@ -75,6 +75,9 @@ struct TcSplitGemmItem {
     float* out;
     int M, N, K;
     int ktri;              // B upper triangular: column j needs k <= j only
+    int ldo;               // row pitch of out (elements); 0: N
+    int sub;               // 1: out -= A B instead of out = A B
+    int lower;             // 1: only output tiles on or below the diagonal
 };
 
 // Grouped launch; M and N multiples of 8, planes 16-byte aligned.
