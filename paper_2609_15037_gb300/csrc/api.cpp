@@ -841,14 +841,37 @@ struct RefreshRunner {
             }
             chk(moara::launch_gather_cols(sb, s, &ctx->launches));
         }
-        // P_tmp (m x r) = Q * Xs into Qa, on the fp32 units: the final
-        // projector's orthonormality is fixed here (a split-precision
-        // tensor-core product leaves column norms ~1e-5 short)
-        gemm(prod, [&](int i, moara::GemmProb& p) {
-            p.A = Qb[i]; p.Bm = Xb[i]; p.C = Qa[i];
-            p.M = it[i].m; p.N = it[i].r; p.K = it[i].l; p.lda = it[i].l; p.ldb = it[i].r; p.ldc = it[i].r;
-        });
-        const std::vector<float*>& ptmp = Qa;
+        // P_tmp (m x r) = Q * Xs; the store below scales every column to unit
+        // length
+        std::vector<float*> ptmp(n_it);
+        if (tall_ks) {
+            // three-plane split-precision product: the planes of Q^T fill the
+            // Qa / Qbf pair (Q itself is in Qb), those of Xs the P1 region;
+            // P_tmp overwrites Q, which the product no longer reads.  The
+            // tensor cores' accumulation leaves the column norms ~1e-5 short;
+            // the unit-length store removes that.
+            moara::SmallBatch sq = small(), sx = small();
+            for (int i = 0; i < n_it; ++i) {
+                sq.a[i] = Qb[i]; sq.h[i] = reinterpret_cast<uint16_t*>(it[i].Qa); sq.rows[i] = it[i].m;
+                sq.l[i] = it[i].l;
+                sx.a[i] = Xb[i]; sx.h[i] = it[i].P1; sx.rows[i] = it[i].l; sx.l[i] = it[i].r;
+            }
+            chk(moara::launch_split3(sq, 1, s, &ctx->launches));
+            chk(moara::launch_split3(sx, 0, s, &ctx->launches));
+            std::vector<moara::TcSplitGemmItem> g;
+            for (int i = 0; i < n_it; ++i) {
+                g.push_back({reinterpret_cast<uint16_t*>(it[i].Qa), it[i].P1, (size_t)it[i].m * it[i].l,
+                             (size_t)it[i].l * it[i].r, Qb[i], it[i].m, it[i].r, it[i].l, 0});
+                ptmp[i] = Qb[i];
+            }
+            ks_run(g, 3);
+        } else {
+            gemm(prod, [&](int i, moara::GemmProb& p) {
+                p.A = Qb[i]; p.Bm = Xb[i]; p.C = Qa[i];
+                p.M = it[i].m; p.N = it[i].r; p.K = it[i].l; p.lda = it[i].l; p.ldb = it[i].r; p.ldc = it[i].r;
+            });
+            ptmp = Qa;
+        }
         {
             moara::SmallBatch sb = small();
             for (int i = 0; i < n_it; ++i) {

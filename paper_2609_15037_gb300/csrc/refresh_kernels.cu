@@ -470,16 +470,17 @@ cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* lau
 }
 
 // ---------------------------------------------------------------------------
-// Final projector: each column of a (rows x l, here l = r columns) is signed
-// so that its largest-magnitude entry is positive (lowest row wins ties), then
-// stored to c (fp32) and h (bf16).  Skipped when the problem's fail flag is
-// set, which leaves the previous projector in place.
+// Final projector: each column of a (rows x l, here l = r columns) is scaled
+// to unit length and signed so that its largest-magnitude entry is positive
+// (lowest row wins ties), then stored to c (fp32) and h (bf16).  Skipped when
+// the problem's fail flag is set, which leaves the previous projector in place.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_sign_fix_store(const __grid_constant__ SmallBatch b) {
     // a CTA owns 32 columns: lane = column, the 8 warps split the rows, so
     // every row segment is one coalesced 128-byte load
     __shared__ float s_best[8][32];
     __shared__ int s_bi[8][32];
+    __shared__ float s_ss[8][32];
     __shared__ float s_sgn[32];
     const int pi = blockIdx.y;
     const int rows = b.rows[pi], r = b.l[pi];
@@ -493,23 +494,30 @@ __global__ void __launch_bounds__(256) k_sign_fix_store(const __grid_constant__ 
         const bool col = q < r;
         // largest |entry| of the column over this warp's rows (ascending, so
         // the lowest row wins ties)
-        float best = -1.0f;
+        float best = -1.0f, ss = 0.0f;
         int bi = 0x7fffffff;
         if (col)
             for (int i = warp; i < rows; i += 8) {
-                const float a = fabsf(Pt[(long long)i * r + q]);
+                const float v = Pt[(long long)i * r + q];
+                const float a = fabsf(v);
+                ss = fmaf(v, v, ss);
                 if (a > best) { best = a; bi = i; }
             }
         s_best[warp][lane] = best;
         s_bi[warp][lane] = bi;
+        s_ss[warp][lane] = ss;
         __syncthreads();
         if (warp == 0) {
             for (int w = 1; w < 8; ++w) {
                 const float ob = s_best[w][lane];
                 const int oi = s_bi[w][lane];
+                ss += s_ss[w][lane];
                 if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
             }
-            s_sgn[lane] = (col && bi < rows && Pt[(long long)bi * r + q] < 0.0f) ? -1.0f : 1.0f;
+            const float sg = (col && bi < rows && Pt[(long long)bi * r + q] < 0.0f) ? -1.0f : 1.0f;
+            // unit length (a zero or non-finite column is left unscaled)
+            const float nrm = sqrtf(ss);
+            s_sgn[lane] = (nrm > 0.0f && isfinite(nrm)) ? sg / nrm : sg;
         }
         __syncthreads();
         const float sgnv = s_sgn[lane];
