@@ -228,6 +228,27 @@ def test_projector_rotation_changes_update():
 
 # ---------------------------------------------------------------- refresh
 
+def test_fix_signs_convention_by_hand():
+    """Singular vectors are defined up to sign; the projector fixes it so that
+    each column's largest-magnitude entry is positive, the lowest row winning
+    a tie of magnitudes.  Checked on hand-made columns."""
+    P = np.array([[-0.5, 0.5, 0.0, -0.25],
+                  [0.5, -0.5, 0.0, 0.75],
+                  [0.1, 0.2, 0.0, -0.75]])
+    F = o.fix_signs(P)
+    # column 0: tie of 0.5 between rows 0 (negative) and 1: row 0 wins, flip
+    np.testing.assert_array_equal(F[:, 0], [0.5, -0.5, -0.1])
+    # column 1: the same tie, row 0 positive: unchanged
+    np.testing.assert_array_equal(F[:, 1], P[:, 1])
+    # column 2: all zero stays zero
+    np.testing.assert_array_equal(F[:, 2], P[:, 2])
+    # column 3: tie of 0.75 between rows 1 (positive) and 2: unchanged
+    np.testing.assert_array_equal(F[:, 3], P[:, 3])
+    # idempotent, and a sign flip of the input gives the same output
+    np.testing.assert_array_equal(o.fix_signs(F), F)
+    np.testing.assert_array_equal(o.fix_signs(-P), F)
+
+
 def test_refresh_orthonormal_and_eckart_young():
     """TruncatedSVD: P^T P = I, and the captured energy ||P^T V||_F^2 equals
     the sum of the top-r squared singular values (Eckart-Young), more than
