@@ -218,8 +218,9 @@ int moara_set_refresh_workspace(moara_ctx* ctx, void* ptr, size_t bytes);
  * computed by randomized subspace iteration (Gaussian sketch with p extra
  * columns, q power iterations, CholeskyQR orthonormalisation, Rayleigh-Ritz
  * on the sketch).  Columns come in descending singular-value order, each
- * signed so that its largest-magnitude entry is positive.  Writes P and
- * P_bf16.  G[i] is the m x n gradient of module ids[i] (device, dtype of the
+ * of unit length and signed so that its largest-magnitude entry is positive
+ * (the lowest row on ties).  Writes P and P_bf16; a module whose
+ * factorisation meets a non-positive pivot keeps its previous P.  G[i] is the m x n gradient of module ids[i] (device, dtype of the
  * module).  MOARA_ERR_WORKSPACE if one module does not fit the workspace. */
 int moara_refresh_projector(moara_ctx* ctx, int n_mod, const int* ids,
                             const void* const* G, void* stream);
