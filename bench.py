@@ -219,6 +219,14 @@ def _traffic(kernel, workload):
     return int(TRAFFIC["bytes"][kernel] * scale)
 
 
+def _rank_summary(mods):
+    """Ranks by module type, e.g. 'q 512, k 512, v 1024, ...' (first layer)."""
+    seen = {}
+    for md in mods:
+        seen.setdefault(md.mtype, md.r)
+    return ", ".join(f"{t} {r}" for t, r in seen.items())
+
+
 def run_gpu(args):
     import torch
     import paper_2609_15037_gb300 as M
@@ -437,11 +445,14 @@ def run_gpu(args):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(total_ms, 4), "higher_is_better": False, "scaling": "weak",
         "vs_baseline": None,
-        "dtype": ("bf16 G, bf16 W/direction states, fp32 magnitude states" if sbytes == 2 else
-                  "bf16 G, fp32 W/states") if used_tc else "fp32 (bf16 G)",
+        "dtype": "bf16" if used_tc else "f32",
         "data": "synthetic",
         "config": {"workload": args.workload, "modules": len(mods), "block_size": B,
-                   "ranks": "q/k 512, v/o/gate/up 1024, down 2048",
+                   "ranks": _rank_summary(mods),
+                   "precision": (("bf16 MMA operands (G, V, P, N), fp32 accumulation and elementwise; "
+                                  + ("bf16 W and direction states, fp32 magnitude states" if sbytes == 2
+                                     else "fp32 W and states")) if used_tc
+                                 else "fp32 SIMT (bf16 G read as is)"),
                    "l2": "inputs larger than L2 (no flush needed)",
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "clip_norm": args.clip_norm, "state_dtype": args.state_dtype,
