@@ -318,6 +318,21 @@ const char* moara_status_string(int code);
 /* Number of kernel launches the context has enqueued since creation. */
 int64_t moara_launch_count(const moara_ctx* ctx);
 
+/* Failure-detection hook (the paper has no counterpart).  Every wait of the
+ * library's kernels on an mbarrier is bounded; when the bound passes without
+ * progress the kernel records MOARA_ERR_DEVICE_TIMEOUT in the device status
+ * word, waits (with the default bound) for its own copies and tensor-core
+ * work in flight, frees its tensor memory and returns, leaving the context
+ * usable.  This call sets the bound, in SM clock cycles, of the waits of the
+ * tensor-core products of the projector refresh and of moara_alignment (the
+ * single-CTA kernels) for launches enqueued afterwards; cycles <= 0 restores
+ * the default (2^32 cycles, about 2 s).  A bound shorter than the kernels'
+ * own latency (a few hundred cycles) makes them give up on purpose, which is
+ * how the failure path is tested; their outputs are then undefined until the
+ * next call with the default bound.  The step kernels' two-CTA pairs keep the
+ * default bound.  Returns MOARA_ERR_UNSUPPORTED without tensor-core state. */
+int moara_set_wait_limit(moara_ctx* ctx, int64_t cycles);
+
 /* Per-kernel timing with CUDA events recorded on the launching stream around
  * every launch of the step and refresh kernels (enable != 0 turns it on).
  * Phases: MOARA_PHASE_*.  Adds two event records per launch; no effect on
@@ -368,11 +383,21 @@ int moara_profile_read(moara_ctx* ctx, double ms[MOARA_NUM_PHASES], int64_t laun
  * 16-byte aligned.  Returns MOARA_ERR_WORKSPACE when
  * 4*(r*n + 2*m*ceil(n/B)) bytes (each part rounded up to 256 bytes) exceed
  * the 16 MiB array; nothing is launched then.  The first call on a device
- * looks up the array's device address (once per device) and should come
- * before any stream capture.  All calls share the one array: calls whose
- * kernels overlap on the GPU (different streams, or different host threads
- * on the same device) race on it and must be serialised by the caller.  No
- * scratch value is carried from one call to the next. */
+ * looks up the array's device address (once per device, then cached).  With
+ * lazy module loading, the CUDA default, that first call is also what loads
+ * the library's module holding the array onto the device and so reserves the
+ * 16 MiB there: a caller whose memory pool takes the GPU's free memory should
+ * make one accepted call before reserving its pool, and before any stream
+ * capture.  Later calls on that device allocate nothing.  The cached address
+ * is that of the device's primary context; after cudaDeviceReset it is stale
+ * and this entry point must not be called again in the process.  All calls
+ * share the one array: calls whose kernels overlap on the GPU (different
+ * streams, or different host threads on the same device) race on it and must
+ * be serialised by the caller.  No scratch value is carried from one call to
+ * the next.  Only the left projector is taken: with proj_rule =
+ * MOARA_PROJ_SMALLER and m > n the call returns MOARA_ERR_UNSUPPORTED.
+ * hp->precision is ignored (the fp32 path always runs), and so are the
+ * refresh fields; clip_norm > 0 and bf16 states return MOARA_ERR_UNSUPPORTED. */
 int moara_step_static_scratch(const moara_hparams* hp, int m, int n, int r, int grad_dtype,
                               const void* G, float* W, const float* P, float* exp_avg,
                               float* exp_avg_sq, float* mag_avg, float* mag_avg_sq, int64_t t,

@@ -99,6 +99,7 @@ def _load():
         "moara_last_error": (ctypes.c_char_p, [vp]),
         "moara_status_string": (ctypes.c_char_p, [i32]),
         "moara_launch_count": (i64, [vp]),
+        "moara_set_wait_limit": (i32, [vp, i64]),
         "moara_profile_enable": (i32, [vp, i32]),
         "moara_profile_read": (i32, [vp, P(ctypes.c_double), P(i64)]),
         "moara_step_static_scratch": (i32, [P(moara_hparams), i32, i32, i32, i32, vp, vp, vp, vp,
@@ -268,6 +269,10 @@ def moara_launch_count(ctx):
     return int(_lib.moara_launch_count(ctx))
 
 
+def moara_set_wait_limit(ctx, cycles):
+    _check(_lib.moara_set_wait_limit(ctx, int(cycles)), ctx, "moara_set_wait_limit")
+
+
 def moara_step_static_scratch(hp, m, n, r, grad_dtype, G, W, P, exp_avg, exp_avg_sq,
                               mag_avg, mag_avg_sq, t, lr, stream=0):
     """Single-module step with the library's built-in scratch (no device
@@ -300,6 +305,6 @@ EXPORTED = [
     "moara_refresh_projector", "moara_step_grouped", "moara_step_grouped_host",
     "moara_get_device_status", "moara_alignment", "moara_set_clip_extra", "moara_clip_state",
     "moara_flatten_shape",
-    "moara_last_error", "moara_status_string", "moara_launch_count",
+    "moara_last_error", "moara_status_string", "moara_launch_count", "moara_set_wait_limit",
     "moara_profile_enable", "moara_profile_read", "moara_step_static_scratch",
 ]

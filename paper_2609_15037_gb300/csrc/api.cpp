@@ -1637,6 +1637,13 @@ const char* moara_status_string(int code) {
 
 int64_t moara_launch_count(const moara_ctx* ctx) { return ctx ? ctx->launches : -1; }
 
+int moara_set_wait_limit(moara_ctx* ctx, int64_t cycles) {
+    if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
+    if (ctx->tc == nullptr) return fail(ctx, MOARA_ERR_UNSUPPORTED, "no tensor-core state on this device");
+    moara::tc_set_wait_limit(ctx->tc, static_cast<long long>(cycles));
+    return MOARA_OK;
+}
+
 int moara_profile_enable(moara_ctx* ctx, int enable) {
     if (ctx == nullptr) return MOARA_ERR_INVALID_ARG;
     ctx->prof = enable != 0;

@@ -22,7 +22,13 @@ float* g_scratch_addr[kMaxDevices] = {};
 
 // Device address of the array on the current device.  In host code the
 // array's name is only a host-side stand-in, so the address is looked up once
-// per device (the first call on that device) with that device current.
+// per device (the first call on that device) with that device current.  With
+// lazy module loading (the CUDA default) that first lookup is also what loads
+// this file's module on the device and reserves the 16 MiB there.  The cached
+// address belongs to the device's primary context: after cudaDeviceReset (or
+// any reset of the primary context) the module is loaded again, possibly at
+// another address, and the cached one is stale -- such a caller must not use
+// this entry point again in the same process.
 int scratch_address(float** out) {
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MOARA_ERR_CUDA;
@@ -47,12 +53,20 @@ extern "C" int moara_step_static_scratch(const moara_hparams* hp, int m, int n, 
                                          float* exp_avg_sq, float* mag_avg, float* mag_avg_sq, int64_t t,
                                          float lr, void* stream) {
     if (hp == nullptr) return MOARA_ERR_INVALID_ARG;
+    // the same hyper-parameter checks as moara_create
     if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f) || !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f) ||
-        !(hp->adam_eps >= 0.0f) || !(hp->decomp_eps >= 0.0f) || !std::isfinite(hp->scale) ||
+        !(hp->adam_eps >= 0.0f) || !std::isfinite(hp->adam_eps) || !(hp->decomp_eps >= 0.0f) ||
+        !std::isfinite(hp->decomp_eps) || !std::isfinite(hp->scale) || !std::isfinite(hp->clip_norm) ||
         (hp->decompose != 0 && hp->decompose != 1))
+        return MOARA_ERR_INVALID_ARG;
+    if (hp->proj_rule != MOARA_PROJ_LEFT && hp->proj_rule != MOARA_PROJ_SMALLER) return MOARA_ERR_INVALID_ARG;
+    if (hp->precision != MOARA_PREC_AUTO && hp->precision != MOARA_PREC_FP32 && hp->precision != MOARA_PREC_BF16_TC)
         return MOARA_ERR_INVALID_ARG;
     if (m < 1 || n < 1 || hp->block_size < 1) return MOARA_ERR_SHAPE;
     if (r < 1 || r > (m < n ? m : n)) return MOARA_ERR_RANK;
+    // only the left projector P (m x r) is taken here; the smaller-side rule
+    // would give a tall weight a right projector
+    if (hp->proj_rule == MOARA_PROJ_SMALLER && m > n) return MOARA_ERR_UNSUPPORTED;
     if (grad_dtype != MOARA_DTYPE_F32 && grad_dtype != MOARA_DTYPE_BF16) return MOARA_ERR_INVALID_ARG;
     if (t < 1 || !std::isfinite(lr)) return MOARA_ERR_INVALID_ARG;
     if (hp->clip_norm > 0.0f) return MOARA_ERR_UNSUPPORTED;   // global-norm clipping needs the whole step

@@ -121,17 +121,27 @@ struct K1Params {
 };
 
 // ------------------------------------------------------------------- K2
-constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64, K2_STAGES = 5;
+constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64;
 constexpr int K2_A_BYTES = K2_BM * K2_BK * 2;           // 16 KB: P rows, K-major
 constexpr int K2_B_BYTES = K2_BK * (K2_BN / 2) * 2;     // 16 KB: this CTA's two 64-column chunks of N
 constexpr int K2_STAGE_BYTES = K2_A_BYTES + K2_B_BYTES;
-// W streams through a ring of 128-row x 32-column fp32 chunks (TMA in and out)
-constexpr int K2_WCOLS = 32, K2_WBUF = 4;
+// W moves in chunks of 128 rows x one 128-byte row (32 fp32 / 64 bf16 columns).
+// fp32 W (SB false): the epilogue writes the update dW = -lr*alpha*(Rep_B(dM)
+// (.) dV) into a staging chunk and a TMA reduce-add applies it to W in L2, so
+// W never enters the SM: two staging chunks, six operand stages.  bf16 W (SB
+// true; the fp32 update is rounded once, which an L2 add of a bf16 dW would
+// not reproduce): a four-chunk ring, TMA in and out, five operand stages.
+constexpr int K2_WCOLS = 32;
 constexpr int K2_WBYTES = K2_BM * K2_WCOLS * 4;         // 16 KB
+template <bool SB> struct K2Cfg {
+    static constexpr int STAGES = SB ? 5 : 6;
+    static constexpr int WBUF = SB ? 4 : 2;
+    static constexpr int BYTES = STAGES * K2_STAGE_BYTES + WBUF * K2_WBYTES;
+};
 constexpr int K2_WARPS = 12;                            // 0 TMA, 1 MMA, 2 W loader, 3 W storer, 4-11 epilogue
 constexpr int K2_THREADS = K2_WARPS * 32;
-constexpr int K2_GUARD = 0;
-constexpr int K2_SMEM = 1024 + K2_STAGES * K2_STAGE_BYTES + K2_WBUF * K2_WBYTES + K2_GUARD + kCtlBytes;
+constexpr int K2_SMEM = 1024 + (K2Cfg<true>::BYTES > K2Cfg<false>::BYTES ? K2Cfg<true>::BYTES : K2Cfg<false>::BYTES) +
+                        kCtlBytes;
 
 struct K2Params {
     const int* cta_start;
@@ -698,10 +708,11 @@ k2_backproject(const __grid_constant__ K2Params p) {
     constexpr int WC = StateCols<SB>::N;              // W columns per ring chunk
     constexpr int HC = WC / 2;                        // columns per epilogue thread and chunk
     static_assert(!SB || BLK >= 32, "bf16 states: a thread's 32 columns lie in one block");
+    constexpr int K2_STAGES = K2Cfg<SB>::STAGES, K2_WBUF = K2Cfg<SB>::WBUF;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = align1024(smem_raw);
     uint8_t* wring = smem + K2_STAGES * K2_STAGE_BYTES;
-    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(wring + K2_WBUF * K2_WBYTES + K2_GUARD);
+    SmemCtl* ctl = reinterpret_cast<SmemCtl*>(wring + K2_WBUF * K2_WBYTES);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int crank = static_cast<int>(ptx::cluster_ctarank());   // row tile 2 t0 + crank of each pair tile
     const int cluster = blockIdx.x >> 1;
@@ -818,7 +829,8 @@ k2_backproject(const __grid_constant__ K2Params p) {
         }
     } else if (warp == 2) {
         // ------------------------------------------- W chunk loader (TMA in)
-        if (lane == 0) {
+        // (bf16 W only: an fp32 W is updated by reduce-add, never loaded)
+        if (SB && lane == 0) {
             uint32_t g = 0;
             uint32_t issued = 0, last_par = 0;
             bool ok = true;
@@ -846,7 +858,7 @@ k2_backproject(const __grid_constant__ K2Params p) {
             }
         }
     } else if (warp == 3) {
-        // ------------------------------------------ W chunk storer (TMA out)
+        // ------------------------------ W chunk storer (TMA store / reduce-add)
         if (lane == 0) {
             uint32_t g = 0;
             bool ok = true;
@@ -861,7 +873,8 @@ k2_backproject(const __grid_constant__ K2Params p) {
                     const uint32_t ph = (g / K2_WBUF) & 1;
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->wdone[b]), ph, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
-                    ptx::tma_store_2d(wmap, ptx::smem_u32(wring + b * K2_WBYTES), n0 + c * WC, i0);
+                    if constexpr (SB) ptx::tma_store_2d(wmap, ptx::smem_u32(wring + b * K2_WBYTES), n0 + c * WC, i0);
+                    else ptx::tma_reduce_add_2d(wmap, ptx::smem_u32(wring + b * K2_WBYTES), n0 + c * WC, i0);
                     ptx::bulk_commit_group();
                     ptx::bulk_wait_read_all();            // the chunk may be refilled once read
                     ptx::mbar_arrive(ptx::smem_u32(&ctl->wempty[b]));
@@ -872,9 +885,10 @@ k2_backproject(const __grid_constant__ K2Params p) {
     } else {
         // ------------------------------------------------- epilogue warps
         // 8 warps: TMEM lane quarter q = warp % 4, column half ch of each
-        // chunk (32 fp32 / 64 bf16 columns); each thread updates 16 / 32
-        // values of its W row in the swizzled shared-memory chunk:
-        // W -= lr * alpha * dM * (P N), rounded to bf16 for bf16 weights.
+        // chunk (32 fp32 / 64 bf16 columns); each thread handles 16 / 32
+        // values of its W row in the swizzled shared-memory chunk: the update
+        // dW = -lr * alpha * dM * (P N) for an fp32 W (added to W by the
+        // storer's reduce), or W - lr * alpha * dM * (P N) rounded to bf16.
         const int ew = warp - 4;                        // 0..7
         const int q = warp & 3;
         const int ch = ew >> 2;
@@ -932,16 +946,19 @@ k2_backproject(const __grid_constant__ K2Params p) {
                 for (int h = 0; h < HC / 16; ++h)
                     ptx::tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + c * WC + ch * HC + 16 * h,
                                    *reinterpret_cast<float(*)[16]>(v + 16 * h));
-                const bool gotw = ptx::mbar_wait(ptx::smem_u32(&ctl->wfull[b]), ph, abort_flag, p.status,
-                                                 MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+                // bf16 W: the loaded chunk; fp32 W: a free staging chunk
+                const bool gotw = SB ? ptx::mbar_wait(ptx::smem_u32(&ctl->wfull[b]), ph, abort_flag, p.status,
+                                                      MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)
+                                     : ptx::mbar_wait(ptx::smem_u32(&ctl->wempty[b]), ph ^ 1, abort_flag, p.status,
+                                                      MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
                 if (!__all_sync(0xffffffffu, gotw)) { ok = false; break; }
                 uint8_t* wrow = wring + b * K2_WBYTES + il * 128;
                 const uint32_t x = static_cast<uint32_t>(il & 7);
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     uint4* w4 = reinterpret_cast<uint4*>(wrow + (((ch * 4 + u) ^ x) << 4));
-                    const uint4 wv = *w4;
                     if constexpr (SB) {
+                        const uint4 wv = *w4;
                         const float d0 = dm[0];
                         const uint32_t ww[4] = {wv.x, wv.y, wv.z, wv.w};
                         uint32_t out[4];
@@ -953,15 +970,12 @@ k2_backproject(const __grid_constant__ K2Params p) {
                         }
                         *w4 = make_uint4(out[0], out[1], out[2], out[3]);
                     } else {
-                        float4 w = make_float4(__uint_as_float(wv.x), __uint_as_float(wv.y), __uint_as_float(wv.z),
-                                               __uint_as_float(wv.w));
                         const float d0 = dm[NDM == 1 ? 0 : (u * 4) / BLK];
-                        w.x -= p.step_scale * (d0 * v[4 * u + 0]);
-                        w.y -= p.step_scale * (d0 * v[4 * u + 1]);
-                        w.z -= p.step_scale * (d0 * v[4 * u + 2]);
-                        w.w -= p.step_scale * (d0 * v[4 * u + 3]);
-                        *w4 = make_uint4(__float_as_uint(w.x), __float_as_uint(w.y), __float_as_uint(w.z),
-                                         __float_as_uint(w.w));
+                        const float ms = -p.step_scale;
+                        *w4 = make_uint4(__float_as_uint(ms * (d0 * v[4 * u + 0])),
+                                         __float_as_uint(ms * (d0 * v[4 * u + 1])),
+                                         __float_as_uint(ms * (d0 * v[4 * u + 2])),
+                                         __float_as_uint(ms * (d0 * v[4 * u + 3])));
                     }
                 }
                 ptx::fence_proxy_async_smem();
@@ -990,8 +1004,10 @@ k2_backproject(const __grid_constant__ K2Params p) {
 
 // ---------------------------------------------------------------- host side
 // ===========================================================================
-// KR: bf16 tensor-core GEMM of the projector refresh (randomized subspace
-// iteration, §3.3 / App. B.2): out (M x N) = op(A) B with fp32 accumulation,
+// KR: bf16 tensor-core GEMM of the projector refresh (the TruncatedSVD of
+// Algorithm 1, computed by randomized subspace iteration after Halko,
+// Martinsson and Tropp, 2011 -- this library's choice of method, not the
+// paper's): out (M x N) = op(A) B with fp32 accumulation,
 // written in fp32 and/or bf16.  A is read K-major (stored M x K) or MN-major
 // (stored K x M), optionally as two planes A_hi + A_lo (two MMAs per k-step
 // keep ~16 significant bits of A, used for V); B is stored K x N (MN-major).
@@ -1034,6 +1050,7 @@ struct KrParams {
     int tile_start[kKrGroup + 1];
     int count;
     int* status;
+    long long wait_limit;              // clock cycles of a bounded wait before it gives up
 };
 
 template <bool KMAJOR, bool LO, bool ALIGN = false>
@@ -1090,11 +1107,8 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
             const uint32_t bytes = (LO ? 2 : 1) * KR_PLANE + nch * 8192;
             for (int kb = 0; kb < nk; ++kb) {
                 if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
-                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) {
-                    for (int s = 0; s < STAGES; ++s)
-                        if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
+                                    MOARA_ERR_DEVICE_TIMEOUT, p.wait_limit))
                     break;
-                }
                 const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
                 ptx::mbar_arrive_expect_tx(fb, bytes);
                 const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
@@ -1111,6 +1125,10 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
                 last_par = (last_par & ~(1u << stage)) | (phase << stage);
                 if (++stage == STAGES) { stage = 0; phase ^= 1; }
             }
+            // every copy issued has landed before the CTA may leave (after a
+            // wait that gave up elsewhere the MMA may not have consumed them)
+            for (int s = 0; s < STAGES; ++s)
+                if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -1119,7 +1137,7 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
             uint32_t phase = 0;
             for (int kb = 0; kb < nk; ++kb) {
                 if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
-                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) break;
+                                    MOARA_ERR_DEVICE_TIMEOUT, p.wait_limit)) break;
                 ptx::tc_fence_after();
                 const uint32_t a = ptx::smem_u32(smem + stage * STAGE_BYTES);
                 const uint32_t b = a + (LO ? 2 : 1) * KR_PLANE;
@@ -1152,7 +1170,7 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
         const int q = warp & 3;
         const int h = ew >> 2;
         const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[0]), 0, abort_flag, p.status,
-                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+                                        MOARA_ERR_DEVICE_TIMEOUT, p.wait_limit);
         if (ALIGN && __all_sync(0xffffffffu, got) && h < halves) {
             // S(W, t) of §3.2: this thread's row of the product -- row j of
             // (P P^T V)^T against column j of G, or row i of V Q Q^T against
@@ -1313,6 +1331,7 @@ struct KsParams {
     int tile_start[kKsGroup + 1];
     int count;
     int* status;
+    long long wait_limit;              // clock cycles of a bounded wait before it gives up
 };
 
 template <int NP>
@@ -1368,11 +1387,8 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
             const uint32_t bytes = NP * KS_PLANE + NP * nch * 4096;
             for (int kb = 0; kb < nk; ++kb) {
                 if (!ptx::mbar_wait(ptx::smem_u32(&ctl->empty[stage]), phase ^ 1, abort_flag, p.status,
-                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) {
-                    for (int s = 0; s < KS_STAGES; ++s)
-                        if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
+                                    MOARA_ERR_DEVICE_TIMEOUT, p.wait_limit))
                     break;
-                }
                 const uint32_t fb = ptx::smem_u32(&ctl->full[stage]);
                 ptx::mbar_arrive_expect_tx(fb, bytes);
                 const uint32_t a = ptx::smem_u32(smem + stage * KS_STAGE);
@@ -1389,6 +1405,10 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
                 last_par = (last_par & ~(1u << stage)) | (phase << stage);
                 if (++stage == KS_STAGES) { stage = 0; phase ^= 1; }
             }
+            // every copy issued has landed before the CTA may leave (after a
+            // wait that gave up elsewhere the MMA may not have consumed them)
+            for (int s = 0; s < KS_STAGES; ++s)
+                if (issued & (1u << s)) wait_drain(ptx::smem_u32(&ctl->full[s]), (last_par >> s) & 1);
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -1400,7 +1420,7 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
             uint32_t phase = 0;
             for (int kb = 0; kb < nk; ++kb) {
                 if (!ptx::mbar_wait(ptx::smem_u32(&ctl->full[stage]), phase, abort_flag, p.status,
-                                    MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) break;
+                                    MOARA_ERR_DEVICE_TIMEOUT, p.wait_limit)) break;
                 ptx::tc_fence_after();
                 const uint32_t a = ptx::smem_u32(smem + stage * KS_STAGE);
                 const uint32_t b = a + NP * KS_PLANE;
@@ -1428,7 +1448,7 @@ __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constan
         const int q = warp & 3;
         const int h = ew >> 2;
         const bool got = ptx::mbar_wait(ptx::smem_u32(&ctl->accf[0]), 0, abort_flag, p.status,
-                                        MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+                                        MOARA_ERR_DEVICE_TIMEOUT, p.wait_limit);
         if (__all_sync(0xffffffffu, got) && h < halves) {
             ptx::tc_fence_after();
             const int row = i0 + h * 128 + q * 32 + lane;
@@ -1544,6 +1564,7 @@ struct TcState {
     cudaStream_t aux = nullptr;
     cudaEvent_t ev_start = nullptr;
     cudaEvent_t ev_part[32] = {};
+    long long wait_limit = kWaitLimit;     // bounded waits of the refresh / alignment products (KR, KS)
 };
 
 bool tc_supported(int m, int n, int r, int B, int dtype, int decompose, int state_dtype) {
@@ -2039,6 +2060,10 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
 
 const char* tc_last_error(const TcState* st) { return st ? st->err.c_str() : "no tensor-core state"; }
 
+void tc_set_wait_limit(TcState* st, long long cycles) {
+    if (st != nullptr) st->wait_limit = cycles > 0 ? cycles : kWaitLimit;
+}
+
 // Grouped KR launches; with align_B > 0 the alignment epilogue (A K-major
 // with two planes only) replaces the stores.
 static int kr_launch(TcState* st, int a_kmajor, const TcGemmItem* items, int count, int align_B,
@@ -2103,6 +2128,7 @@ static int kr_launch(TcState* st, int a_kmajor, const TcGemmItem* items, int cou
             kp.tile_start[cnt] = total;
             kp.count = cnt;
             kp.status = st->d_status;
+            kp.wait_limit = st->wait_limit;
             kp.al_B = align_B;
             kp.al_log2B = 0;
             while ((1 << kp.al_log2B) < align_B) ++kp.al_log2B;
@@ -2383,6 +2409,7 @@ int tc_gemm_split3(TcState* st, const TcSplitGemmItem* items, int count, int pla
         kp.tile_start[cnt] = total;
         kp.count = cnt;
         kp.status = st->d_status;
+        kp.wait_limit = st->wait_limit;
         if (total == 0) continue;
         if (planes == 3) ks_product<3><<<total, KR_THREADS, KS_SMEM, s>>>(kp);
         else ks_product<2><<<total, KR_THREADS, KS_SMEM, s>>>(kp);

@@ -103,4 +103,9 @@ cudaError_t tc_transpose_bf16(const uint16_t* in, uint16_t* out, int rows, int c
 
 const char* tc_last_error(const TcState* st);
 
+// Clock cycles a bounded wait of the refresh / alignment product kernels (KR,
+// KS) spins before it gives up and records MOARA_ERR_DEVICE_TIMEOUT; <= 0
+// restores the default (~2 s).
+void tc_set_wait_limit(TcState* st, long long cycles);
+
 }  // namespace moara

@@ -1,8 +1,9 @@
 """The bench's multi-GPU path on CPU: the step shards by module with no
-exchange, so N > 1 runs N replicas; the job's time is the maximum over ranks
-(barrier and all-reduce MAX, here over gloo, world size 2) and the job's
-value is ms per full-model step of the whole job; the reference arm runs on
-rank 0 only and the other ranks exit without output."""
+exchange, so with N > 1 each rank owns every N-th module and steps only
+those; the job's time is the maximum over ranks (barrier and all-reduce MAX,
+here over gloo, world size 2) and the job's value is ms per full-model step
+(the slowest shard's step plus its refresh amortised over 200 steps); the
+reference arm runs on rank 0 only and the other ranks exit without output."""
 
 import io
 import os
@@ -40,11 +41,11 @@ def _worker(rank, world, port, out):
         if rank != 0:
             bench.run_reference(type("A", (), dict(workload="llama7b_layer", steps=1, warmup=0, gpus=world,
                                                   cpu_seconds=1.0, proj_rule="left", state_dtype="f32"))())
-    out.put((rank, t, bench.job_value(t, 200.0, world), buf.getvalue()))
+    out.put((rank, t, bench.job_value(t, 200.0), buf.getvalue(), bench.shard_modules(224, rank, world)))
     dist.destroy_process_group()
 
 
-def test_replicas_take_the_slowest_rank_and_report_job_throughput():
+def test_shards_take_the_slowest_rank_and_cover_every_module_once():
     world = 2
     ctx = mp.get_context("spawn")
     q = ctx.Queue()
@@ -56,8 +57,14 @@ def test_replicas_take_the_slowest_rank_and_report_job_throughput():
     for p in procs:
         p.join(timeout=60)
         assert p.exitcode == 0
-    for rank, t, value, printed in res:
+    owned = []
+    for rank, t, value, printed, shard in res:
         assert t == 15.0                      # max over ranks
-        assert value == pytest.approx((15.0 + 1.0) / 2)   # (step + refresh / 200) / replicas
+        assert value == pytest.approx(15.0 + 1.0)   # slowest shard's step + refresh / 200
         if rank != 0:
             assert printed == ""              # non-zero ranks of the reference arm stay silent
+        owned += shard
+        # each shard holds every module type of the 7-per-layer model equally often
+        types = [i % 7 for i in shard]
+        assert all(types.count(k) == 16 for k in range(7))
+    assert sorted(owned) == list(range(224))
