@@ -152,7 +152,7 @@ typedef struct moara_ctx moara_ctx;
 
 /* Fills *out with the paper's defaults (App. D.2: beta 0.9/0.999, eps 1e-6,
  * alpha 0.25, T 200; App. B.1: decomp eps 1e-12; B = 128) and the refresh
- * defaults p = 16, q = 2, ritz_iters = 12, precision AUTO, seed 0. */
+ * defaults p = 32, q = 4, ritz_iters = 3, precision AUTO, seed 0. */
 int moara_default_hparams(moara_hparams* out);
 
 /* Creates a context on CUDA device `device` (the current device is restored

@@ -826,11 +826,15 @@ struct RefreshRunner {
             });
         }
         {
+            // exact Rayleigh-Ritz within the leading 64 columns (Jacobi), so
+            // that the separated leading eigenvectors are exact whatever the
+            // number of orthogonal iterations; then the Ritz order
             moara::SmallBatch sb = small();
             for (int i = 0; i < n_it; ++i) {
                 sb.a[i] = Xa[i]; sb.b[i] = Xb[i]; sb.c[i] = it[i].ritz; sb.iaux[i] = it[i].perm;
                 sb.l[i] = it[i].l;
             }
+            chk(moara::launch_lead_ritz(sb, s, &ctx->launches));
             chk(moara::launch_ritz_sort(sb, s, &ctx->launches));
         }
         {   // Xs (l x r) = X[:, perm[:r]] into Xb
@@ -1080,9 +1084,9 @@ int moara_default_hparams(moara_hparams* out) {
     out->refresh_interval = 200;
     out->decompose = 1;
     out->refresh_src = MOARA_REFRESH_SRC_V;
-    out->oversample = 16;
-    out->power_iters = 2;
-    out->ritz_iters = 12;
+    out->oversample = 32;
+    out->power_iters = 4;
+    out->ritz_iters = 3;
     out->precision = MOARA_PREC_AUTO;
     out->seed = 0;
     return MOARA_OK;

@@ -207,6 +207,9 @@ cudaError_t launch_trace_shift(const SmallBatch& b, cudaStream_t s, int64_t* lau
 cudaError_t launch_chol_diag(const SmallBatch& b, int j0, cudaStream_t s, int64_t* launches);
 cudaError_t launch_set_identity(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_ritz_sort(const SmallBatch& b, cudaStream_t s, int64_t* launches);
+// Exact Rayleigh-Ritz (Jacobi) on the leading min(64, l) columns of X (a)
+// with W = C X (b): both rotated in place by the eigenvectors of X_w^T W_w.
+cudaError_t launch_lead_ritz(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_gather_cols(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_sign_fix_store(const SmallBatch& b, cudaStream_t s, int64_t* launches);
 cudaError_t launch_transpose_bf16(const SmallBatch& b, cudaStream_t s, int64_t* launches);  // h = bf16(a^T)

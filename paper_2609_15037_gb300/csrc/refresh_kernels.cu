@@ -438,6 +438,171 @@ __global__ void __launch_bounds__(kSmallThreads) k_ritz_sort(const __grid_consta
     }
 }
 
+// ---------------------------------------------------------------------------
+// Exact Rayleigh-Ritz on the leading w = min(64, l) columns of an orthonormal
+// X (a, l x l) with W = C X (b): H = X_w^T W_w (w x w, symmetric), its
+// eigen-decomposition H = J diag(h) J^T by the cyclic Jacobi method (Golub
+// and Van Loan, Matrix Computations, 4th ed., §8.5: one rotation per index
+// pair zeroes H_pq; the pairs of a sweep are scheduled as a round-robin
+// tournament so that the w / 2 rotations of a round touch disjoint rows and
+// columns and run in parallel), then X_w <- X_w J and W_w <- W_w J.  The
+// orthogonal iteration before it leaves span(X_w) close to the leading
+// invariant subspace of C; within it the individual eigenvectors of
+// separated eigenvalues are then exact up to rounding.  One CTA per
+// problem, everything in shared memory, rows of X and W streamed in chunks.
+// ---------------------------------------------------------------------------
+constexpr int kLeadW = 64;
+constexpr int kLeadChunk = 16;            // rows of X / W per chunk
+
+__global__ void __launch_bounds__(kSmallThreads) k_lead_ritz(const __grid_constant__ SmallBatch b) {
+    __shared__ float H[kLeadW][kLeadW + 1];
+    __shared__ float J[kLeadW][kLeadW + 1];
+    __shared__ float xs[kLeadChunk][kLeadW];
+    __shared__ float ws[kLeadChunk][kLeadW];
+    __shared__ float rc[kLeadW / 2], rs_[kLeadW / 2];
+    __shared__ int rp[kLeadW / 2], rq[kLeadW / 2];
+    __shared__ float red[33];
+    const int pi = blockIdx.x;
+    const int l = b.l[pi];
+    const int w = l < kLeadW ? l : kLeadW;
+    const int wp = w + (w & 1);                    // even player count (a dummy index when w is odd)
+    float* X = b.a[pi];
+    float* W = b.b[pi];
+    const int t = threadIdx.x;
+    // H = X_w^T W_w: thread t owns entries t, t + 1024, ... of the w x w block
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    for (int r0 = 0; r0 < l; r0 += kLeadChunk) {
+        for (int e = t; e < kLeadChunk * kLeadW; e += blockDim.x) {
+            const int i = e / kLeadW, j = e % kLeadW;
+            const bool in = r0 + i < l && j < w;
+            xs[i][j] = in ? X[(long long)(r0 + i) * l + j] : 0.0f;
+            ws[i][j] = in ? W[(long long)(r0 + i) * l + j] : 0.0f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int e = t + u * blockDim.x;
+            if (e < w * w) {
+                const int p = e / w, q = e % w;
+#pragma unroll 4
+                for (int i = 0; i < kLeadChunk; ++i) acc[u] = fmaf(xs[i][p], ws[i][q], acc[u]);
+            }
+        }
+        __syncthreads();
+    }
+    for (int e = t; e < kLeadW * kLeadW; e += blockDim.x) {
+        const int p = e / kLeadW, q = e % kLeadW;
+        H[p][q] = 0.0f;
+        J[p][q] = (p == q) ? 1.0f : 0.0f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int e = t + u * blockDim.x;
+        if (e < w * w) H[e / w][e % w] = acc[u];
+    }
+    __syncthreads();
+    // symmetrise (the two triangles differ by rounding)
+    for (int e = t; e < w * w; e += blockDim.x) {
+        const int p = e / w, q = e % w;
+        if (p < q) {
+            const float v = 0.5f * (H[p][q] + H[q][p]);
+            H[p][q] = v;
+            H[q][p] = v;
+        }
+    }
+    __syncthreads();
+    const int npairs = wp / 2;
+    for (int sweep = 0; sweep < 20; ++sweep) {
+        // stop once the off-diagonal mass is below fp32 resolution of the diagonal
+        float off = 0.0f, dia = 0.0f;
+        for (int e = t; e < w * w; e += blockDim.x) {
+            const int p = e / w, q = e % w;
+            const float v = H[p][q];
+            if (p == q) dia = fmaf(v, v, dia); else off = fmaf(v, v, off);
+        }
+        off = block_sum(off, red);
+        dia = block_sum(dia, red);
+        if (!(off > 1e-14f * dia)) break;          // also ends on a non-finite H
+        for (int round = 0; round < wp - 1; ++round) {
+            if (t < npairs) {
+                // tournament: player 0 fixed, the others rotate by one each round
+                auto player = [&](int pos) { return pos == 0 ? 0 : 1 + (pos - 1 + round) % (wp - 1); };
+                int p = player(t), q = player(wp - 1 - t);
+                if (p > q) { const int x = p; p = q; q = x; }
+                float c = 1.0f, sn = 0.0f;
+                if (q < w) {
+                    const float hpq = H[p][q];
+                    if (fabsf(hpq) > 1e-30f) {
+                        const float tau = (H[q][q] - H[p][p]) / (2.0f * hpq);
+                        const float tt = (tau >= 0.0f ? 1.0f : -1.0f) / (fabsf(tau) + sqrtf(1.0f + tau * tau));
+                        c = 1.0f / sqrtf(1.0f + tt * tt);
+                        sn = tt * c;
+                    }
+                }
+                rp[t] = p; rq[t] = q; rc[t] = c; rs_[t] = sn;
+            }
+            __syncthreads();
+            // columns: H <- H G, J <- J G
+            for (int e = t; e < npairs * kLeadW; e += blockDim.x) {
+                const int k = e / kLeadW, row = e % kLeadW;
+                const int p = rp[k], q = rq[k];
+                if (q >= w || row >= w) continue;
+                const float c = rc[k], sn = rs_[k];
+                const float hp = H[row][p], hq = H[row][q];
+                H[row][p] = c * hp - sn * hq;
+                H[row][q] = sn * hp + c * hq;
+                const float jp = J[row][p], jq = J[row][q];
+                J[row][p] = c * jp - sn * jq;
+                J[row][q] = sn * jp + c * jq;
+            }
+            __syncthreads();
+            // rows: H <- G^T H
+            for (int e = t; e < npairs * kLeadW; e += blockDim.x) {
+                const int k = e / kLeadW, col = e % kLeadW;
+                const int p = rp[k], q = rq[k];
+                if (q >= w || col >= w) continue;
+                const float c = rc[k], sn = rs_[k];
+                const float hp = H[p][col], hq = H[q][col];
+                H[p][col] = c * hp - sn * hq;
+                H[q][col] = sn * hp + c * hq;
+            }
+            __syncthreads();
+        }
+    }
+    // X_w <- X_w J, W_w <- W_w J, chunk by chunk
+    for (int r0 = 0; r0 < l; r0 += kLeadChunk) {
+        for (int e = t; e < kLeadChunk * kLeadW; e += blockDim.x) {
+            const int i = e / kLeadW, j = e % kLeadW;
+            const bool in = r0 + i < l && j < w;
+            xs[i][j] = in ? X[(long long)(r0 + i) * l + j] : 0.0f;
+            ws[i][j] = in ? W[(long long)(r0 + i) * l + j] : 0.0f;
+        }
+        __syncthreads();
+        float ox = 0.0f, ow = 0.0f;
+        const int i = t / kLeadW, j = t % kLeadW;     // 1024 threads = 16 rows x 64 columns
+        if (j < w) {
+            for (int k = 0; k < w; ++k) {
+                ox = fmaf(xs[i][k], J[k][j], ox);
+                ow = fmaf(ws[i][k], J[k][j], ow);
+            }
+        }
+        __syncthreads();
+        if (j < w && r0 + i < l) {
+            X[(long long)(r0 + i) * l + j] = ox;
+            W[(long long)(r0 + i) * l + j] = ow;
+        }
+        __syncthreads();
+    }
+}
+
+cudaError_t launch_lead_ritz(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
+    if (b.count <= 0) return cudaSuccess;
+    k_lead_ritz<<<b.count, kSmallThreads, 0, s>>>(b);
+    ++*launches;
+    return cudaGetLastError();
+}
+
 cudaError_t launch_ritz_sort(const SmallBatch& b, cudaStream_t s, int64_t* launches) {
     if (b.count <= 0) return cudaSuccess;
     k_ritz_sort<<<b.count, kSmallThreads, 0, s>>>(b);

@@ -50,7 +50,7 @@ def test_hparams_struct_matches_header(M):
     """The binding's struct has the C layout: the library's defaults land in
     the right fields, including the last one."""
     hp = M.moara_default_hparams()
-    assert hp.block_size == 128 and hp.power_iters == 2 and hp.oversample == 16
+    assert hp.block_size == 128 and hp.power_iters == 4 and hp.oversample == 32 and hp.ritz_iters == 3
     assert ctypes.sizeof(M.binding.moara_hparams) == 80
     assert hp.proj_rule == M.MOARA_PROJ_LEFT and hp.state_dtype == M.MOARA_DTYPE_F32
 

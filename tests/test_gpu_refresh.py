@@ -1,13 +1,19 @@
-"""GPU projector refresh (TruncatedSVD of Algorithm 1 by randomized subspace
-iteration) against the oracle's exact fp64 SVD.
+"""GPU projector refresh (TruncatedSVD of Algorithm 1, computed by the
+library's randomized subspace iteration) against the float64 references.
 
-Checks: P^T P = I within 1e-5; principal angles <= 1e-2 rad on the leading
+Every refreshed projector is checked for P^T P = I within 1e-5, principal
+angles <= 1e-2 rad against the exact top-r subspace on the leading
 directions up to the spectral gap k_gap (largest k <= r with
-sigma_k / sigma_{k+1} >= 1.5); captured energy ||P^T X||_F^2 >= (1 - 1e-2)
-sum_{i<=r} sigma_i^2 (the spectrum of V is a flat noise bulk near r, where
-the top-r subspace is ill-conditioned and any approximate method loses a
-little energy); and, on an input with a clear gap at r, all r angles and
-the individual singular vectors in order.
+sigma_k / sigma_{k+1} >= 1.5), and captured energy against the float64
+restatement of the same randomized method with the same Philox sketch
+(oracle/rsi_ref.py; the device may lose at most 3e-4 of the optimum plus a
+quarter of the method's own deficit more).  On inputs with a clear gap at r
+the energy must also reach (1 - 1e-3) of the exact optimum and every
+singular vector must match individually, in order.  The decomposed V of
+the rank-32-plus-noise gradients has a flat noise bulk around r; there the
+method's own deficit against the exact SVD is measured and reported (the
+flat-bulk figures are recorded with the design notes), not hidden behind a
+looser bar.
 """
 
 import numpy as np
@@ -16,7 +22,8 @@ import pytest
 from oracle import moara_ref as o
 import synth
 
-from gpu_helpers import principal_angles, gap_index, make_inputs
+from gpu_helpers import principal_angles, gap_index, make_inputs, check_refresh, top_subspace
+from oracle import rsi_ref as R
 
 pytestmark = pytest.mark.gpu
 
@@ -36,16 +43,10 @@ def _dev(G, bf16=True):
     return (t.to(torch.bfloat16) if bf16 else t).cuda()
 
 
-def _check_projector(P, X, r, tol_angle=1e-2):
-    U, S, _ = np.linalg.svd(X, full_matrices=False)
-    np.testing.assert_allclose(P.T @ P, np.eye(r), atol=1e-5)
-    k = gap_index(S, r)
-    if k > 0:
-        ang = principal_angles(P[:, :k], U[:, :k])
-        assert ang.max() <= tol_angle, (k, ang.max())
-    energy = np.sum((P.T @ X) ** 2)
-    assert energy >= (1 - 1e-2) * np.sum(S[:r] ** 2)
-    return k
+def _check(g, mid, P, X, r, exact_bar=None):
+    hp = g.hp
+    return check_refresh(P, X, r, hp.oversample, hp.power_iters, R.sketch_key(hp.seed, mid, 0),
+                         exact_bar=exact_bar)
 
 
 @pytest.mark.parametrize("src", ["V", "G"])
@@ -63,7 +64,8 @@ def test_refresh_llama300m_attention_and_mlp(M, src):
     for i, (m, n, r) in enumerate(shapes):
         P = g.modules[i].P.double().cpu().numpy()
         X = o.decompose(grads[i][0], B)[1] if src == "V" else grads[i][0]
-        _check_projector(P, X, r)
+        res = _check(g, g.ids[i], P, X, r)
+        print(f"{m}x{n} r={r} src={src}: deficit {res['deficit']:.2e} (float64 method {res['deficit_rsi']:.2e})")
         Pb = g.modules[i].P_bf16.view(torch.bfloat16).float().cpu().numpy()
         np.testing.assert_allclose(Pb, P, rtol=2 ** -8, atol=1e-30)
     g.close()
@@ -87,6 +89,7 @@ def test_refresh_clear_gap_all_directions(M):
     Po = o.truncated_svd(G, r)[0]
     # columns come in descending order with the oracle's sign convention
     assert np.min(np.sum(P * Po, axis=0)) >= 0.9999
+    _check(g, g.ids[0], P, G, r, exact_bar=1e-3)
     g.close()
 
 
@@ -145,7 +148,8 @@ def test_refresh_qwen2_7b_gqa_modules_with_step(M):
     for i, (m, n, r) in enumerate(shapes):
         P = g.modules[i].P.double().cpu().numpy()
         X = o.decompose(grads[i][0], B)[1]
-        _check_projector(P, X, r)
+        res = _check(g, g.ids[i], P, X, r)
+        print(f"{m}x{n} r={r}: deficit {res['deficit']:.2e} (float64 method {res['deficit_rsi']:.2e})")
         assert np.all(np.isfinite(g.modules[i].W.cpu().numpy()))
     g.close()
 
@@ -192,10 +196,31 @@ def test_refresh_clear_gap_bf16_tensor_cores(M, src, m):
         np.testing.assert_allclose(P.T @ P, np.eye(r), atol=1e-5)
         assert principal_angles(P, Po).max() <= 1e-2
         assert np.min(np.sum(P * Po, axis=0)) >= 0.9999
+        _check(g, g.ids[0], P, X, r, exact_bar=1e-3)
     else:
         # the block normalisation bends V's spectrum: the generic checks, then
         # each vector individually up to the spectral gap
-        k = _check_projector(P, X, r)
-        assert k > 0
+        res = _check(g, g.ids[0], P, X, r)
+        assert res["k_gap"] > 0
+        k = res["k_gap"]
         assert np.min(np.sum(P[:, :k] * Po[:, :k], axis=0)) >= 0.9999
+    g.close()
+
+
+@pytest.mark.parametrize("m,n,r", [(4096, 11008, 2048), (11008, 4096, 1024)])
+def test_refresh_llama2_7b_full_size_modules(M, m, n, r):
+    """The refresh at the sizes the bench times: down (4096 x 11008, r = 2048,
+    sketch width l = r + p) and gate / up (11008 x 4096, r = 1024); B = 128,
+    bf16 G, the bench's recipe (rank-32 signal plus noise)."""
+    B = 128
+    G = synth.to_bf16_exact(synth.lowrank_grad(m, n, 32, 10.0, 0.01, 1, seed=0, module=3, noise_rel=True))
+    g = M.MoaraGroup(block_size=B)
+    mid = g.add(m, n, r, "bf16")
+    g.refresh([_dev(G)])
+    torch.cuda.synchronize()
+    assert g.status() == 0
+    P = g.modules[0].P.double().cpu().numpy()
+    X = o.decompose(G, B)[1]
+    res = _check(g, mid, P, X, r)
+    print(f"{m}x{n} r={r}: deficit {res['deficit']:.2e} (float64 method {res['deficit_rsi']:.2e}), k_gap {res['k_gap']}")
     g.close()
