@@ -173,11 +173,16 @@ cudaError_t launch_trace_shift(const SmallBatch& b, cudaStream_t s, int64_t* lau
     return cudaGetLastError();
 }
 
-__global__ void __launch_bounds__(256) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
-    constexpr int NB = kTriBase, NT = 256, RPT = NB * NB / NT;   // 16 rows per thread
-    __shared__ float Lf[NB][NB + 1];   // the factor, one finished column per step
-    __shared__ float Xs[NB][NB + 1];   // the inverse, one finished row per step
-    __shared__ float dg[NB];           // current diagonal of the trailing matrix
+// 64 threads, thread i keeps row i of the block (and later row i of its
+// inverse) in registers; the finished column j of the factor, and later the
+// finished row k of the inverse, is broadcast through shared memory, so each
+// of the 64 steps costs two barriers of two warps and one pass of predicated
+// register FMAs.  The block moves between global and shared memory coalesced.
+__global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
+    constexpr int NB = kTriBase;
+    __shared__ float tile[NB][NB + 1];   // coalesced staging of the block
+    __shared__ float bc[NB];             // broadcast column / row
+    __shared__ float piv;
     __shared__ int s_fail;
     const int pi = blockIdx.x;
     const int l = b.l[pi];
@@ -186,110 +191,85 @@ __global__ void __launch_bounds__(256) k_chol_diag(const __grid_constant__ Small
     float* A = b.a[pi];
     float* X = b.c[pi];
     const float shift = b.b[pi][0];
-    const int t = threadIdx.x;
-    // thread t keeps column c, rows i = g + 4s (s < 16), of the block in
-    // registers; rows and columns past sz are padded with the identity
-    const int c = t % NB, g = t / NB;
-    float a[RPT];
-#pragma unroll
-    for (int s = 0; s < RPT; ++s) {
-        const int i = g + 4 * s;
-        float v = (i == c) ? 1.0f : 0.0f;
-        if (i < sz && c < sz) v = A[(long long)(j0 + i) * l + j0 + c] + (i == c ? shift : 0.0f);
-        a[s] = v;
-        if (i == c) dg[c] = v;
-    }
-    if (t == 0) s_fail = 0;
+    const int i = threadIdx.x;
+    // rows and columns past sz are padded with the identity
+    for (int r = 0; r < NB; ++r)
+        tile[r][i] = (r < sz && i < sz) ? A[(long long)(j0 + r) * l + j0 + i] + (r == i ? shift : 0.0f)
+                                        : (r == i ? 1.0f : 0.0f);
+    if (i == 0) s_fail = 0;
     __syncthreads();
-    // pivot sqrt(d) and its reciprocal; a pivot that is not positive and
-    // finite is replaced by 1 and marks the failure
-    auto pivot = [&](float d, float& dj, float& inv) {
-        if (!(d > 0.0f) || !isfinite(d)) {
-            d = 1.0f;
-            s_fail = 1;
+    float a[NB];
+#pragma unroll
+    for (int k = 0; k < NB; ++k) a[k] = tile[i][k];
+    // right-looking factorisation: step j finishes column j (pivot sqrt(d);
+    // a pivot that is not positive and finite is replaced by 1 and marks the
+    // failure) and subtracts its outer product from the trailing lower part
+#pragma unroll
+    for (int j = 0; j < NB; ++j) {
+        if (i == j) {
+            float d = a[j];
+            if (!(d > 0.0f) || !isfinite(d)) {
+                d = 1.0f;
+                s_fail = 1;
+            }
+            a[j] = sqrtf(d);
+            piv = a[j];
         }
-        dj = sqrtf(d);
-        inv = 1.0f / dj;
-    };
-    if (c == 0) {
-        float dj, inv;
-        pivot(dg[0], dj, inv);
+        __syncthreads();
+        if (i > j) {
+            a[j] = a[j] / piv;
+            bc[i] = a[j];
+        }
+        __syncthreads();
+        if (i > j) {
+            const float lij = a[j];
 #pragma unroll
-        for (int s = 0; s < RPT; ++s) Lf[g + 4 * s][0] = (g + 4 * s == 0) ? dj : a[s] * inv;
+            for (int k = j + 1; k < NB; ++k)
+                if (k <= i) a[k] = fmaf(-lij, bc[k], a[k]);
+        }
     }
-    __syncthreads();
-    // Right-looking factorisation: step j subtracts column j's outer product
-    // from the trailing lower triangle; the owners of column j + 1 finish it
-    // in the same step (each recomputes its updated pivot from dg).
-    for (int j = 0; j + 1 < NB; ++j) {
-        if (c > j) {
-            // all shared-memory reads of the step first, then the updates
-            float lij[RPT];
+    // inverse by forward substitution: row k of the inverse is finished at
+    // step k (divided by the pivot) and broadcast; rows below subtract
+    // L[i][k] times it
+    float x[NB];
 #pragma unroll
-            for (int s = 0; s < RPT; ++s) lij[s] = Lf[g + 4 * s][j];
-            const float lcj = Lf[c][j];
-            const bool next = (c == j + 1);
-            float dj = 0.0f, inv = 0.0f;
-            if (next) pivot(fmaf(-lcj, lcj, dg[c]), dj, inv);
+    for (int c = 0; c < NB; ++c) x[c] = (c == i) ? 1.0f : 0.0f;
 #pragma unroll
-            for (int s = 0; s < RPT; ++s)
-                if (g + 4 * s >= c) a[s] = fmaf(-lij[s], lcj, a[s]);
-            if (next) {
+    for (int k = 0; k < NB; ++k) {
+        if (i == k) {
+            const float inv = 1.0f / a[k];
 #pragma unroll
-                for (int s = 0; s < RPT; ++s)
-                    if (g + 4 * s >= c) Lf[g + 4 * s][c] = (g + 4 * s == c) ? dj : a[s] * inv;
-            } else {
-#pragma unroll
-                for (int s = 0; s < RPT; ++s)
-                    if (g + 4 * s == c) dg[c] = a[s];
+            for (int c = 0; c <= k; ++c) {
+                x[c] *= inv;
+                bc[c] = x[c];
             }
         }
         __syncthreads();
-    }
-    // Inverse by forward substitution: step k subtracts multiples of the
-    // finished row k from the rows below; row k + 1 is finished (divided by
-    // its pivot) by the same update.  Right of the diagonal the inverse is
-    // zero, on it 1 / L[i][i].
-    for (int e = t; e < NB * NB; e += NT) {
-        const int i = e / NB, cc = e % NB;
-        Xs[i][cc] = (i == cc) ? 1.0f / Lf[i][i] : 0.0f;
-    }
-    float x[RPT];
+        if (i > k) {
+            const float lik = a[k];
 #pragma unroll
-    for (int s = 0; s < RPT; ++s) x[s] = 0.0f;
-    __syncthreads();
-    for (int k = 0; k + 1 < NB; ++k) {
-        if (c <= k) {
-            float lik[RPT];
-#pragma unroll
-            for (int s = 0; s < RPT; ++s) lik[s] = Lf[g + 4 * s][k];
-            const float xkc = Xs[k][c];
-            const float piv = Lf[k + 1][k + 1];
-#pragma unroll
-            for (int s = 0; s < RPT; ++s)
-                if (g + 4 * s > k) x[s] = fmaf(-lik[s], xkc, x[s]);
-#pragma unroll
-            for (int s = 0; s < RPT; ++s)
-                if (g + 4 * s == k + 1) {
-                    x[s] = x[s] / piv;
-                    Xs[k + 1][c] = x[s];
-                }
+            for (int c = 0; c <= k; ++c) x[c] = fmaf(-lik, bc[c], x[c]);
         }
         __syncthreads();
     }
-    for (int e = t; e < NB * NB; e += NT) {
-        const int i = e / NB, cc = e % NB;
-        if (i < sz && cc < sz) {
-            A[(long long)(j0 + i) * l + j0 + cc] = (cc <= i) ? Lf[i][cc] : 0.0f;
-            X[(long long)(j0 + i) * l + j0 + cc] = Xs[i][cc];
-        }
-    }
-    if (t == 0 && s_fail && b.fail[pi] != nullptr) *b.fail[pi] = 1;
+    // the factor (zeros above the diagonal) in place, the inverse into c
+#pragma unroll
+    for (int k = 0; k < NB; ++k) tile[i][k] = (k <= i) ? a[k] : 0.0f;
+    __syncthreads();
+    for (int r = 0; r < sz; ++r)
+        if (i < sz) A[(long long)(j0 + r) * l + j0 + i] = tile[r][i];
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < NB; ++k) tile[i][k] = (k <= i) ? x[k] : 0.0f;
+    __syncthreads();
+    for (int r = 0; r < sz; ++r)
+        if (i < sz) X[(long long)(j0 + r) * l + j0 + i] = tile[r][i];
+    if (i == 0 && s_fail && b.fail[pi] != nullptr) *b.fail[pi] = 1;
 }
 
 cudaError_t launch_chol_diag(const SmallBatch& b, int j0, cudaStream_t s, int64_t* launches) {
     if (b.count <= 0) return cudaSuccess;
-    k_chol_diag<<<b.count, 256, 0, s>>>(b, j0);
+    k_chol_diag<<<b.count, 64, 0, s>>>(b, j0);
     ++*launches;
     return cudaGetLastError();
 }
