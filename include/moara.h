@@ -51,7 +51,7 @@ extern "C" {
 #define MOARA_ERR_CUDA            -6  /* a CUDA runtime call failed               */
 #define MOARA_ERR_DEVICE_TIMEOUT  -7  /* a bounded device-side wait ran out       */
 #define MOARA_ERR_WORKSPACE       -8  /* workspace missing or too small           */
-#define MOARA_ERR_UNSUPPORTED     -9  /* valid request this build cannot serve    */
+#define MOARA_ERR_UNSUPPORTED     -9  /* valid request the library cannot serve   */
 
 /* ---- enums ------------------------------------------------------------- */
 #define MOARA_PROJ_LEFT    0
