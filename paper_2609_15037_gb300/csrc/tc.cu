@@ -1563,7 +1563,8 @@ struct TcState {
     // decomposition of later module parts, overlapped with K1 / K2 of earlier ones
     cudaStream_t aux = nullptr;
     cudaEvent_t ev_start = nullptr;
-    cudaEvent_t ev_part[32] = {};
+    cudaEvent_t ev_part[32] = {};          // decomposition of part q done (auxiliary stream)
+    cudaEvent_t ev_k1[32] = {};            // K1 of part q about to start (launching stream)
     long long wait_limit = kWaitLimit;     // bounded waits of the refresh / alignment products (KR, KS)
 };
 
@@ -1609,6 +1610,8 @@ void tc_destroy(TcState* st) {
     if (st->aux) cudaStreamDestroy(st->aux);
     if (st->ev_start) cudaEventDestroy(st->ev_start);
     for (cudaEvent_t e : st->ev_part)
+        if (e) cudaEventDestroy(e);
+    for (cudaEvent_t e : st->ev_k1)
         if (e) cudaEventDestroy(e);
     delete st;
 }
@@ -1937,8 +1940,10 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             if (st->aux == nullptr) {
                 cudaError_t e = cudaStreamCreateWithFlags(&st->aux, cudaStreamNonBlocking);
                 if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_start, cudaEventDisableTiming);
-                for (int q = 0; q < 32 && e == cudaSuccess; ++q)
+                for (int q = 0; q < 32 && e == cudaSuccess; ++q) {
                     e = cudaEventCreateWithFlags(&st->ev_part[q], cudaEventDisableTiming);
+                    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st->ev_k1[q], cudaEventDisableTiming);
+                }
                 if (e != cudaSuccess) return fail("auxiliary stream / events");
             }
             // the auxiliary stream starts after everything queued on s so far
@@ -2010,17 +2015,32 @@ int tc_step(TcState* st, const moara_hparams& hp, int n_mod, const int* ids, con
             p2.decompose = hp.decompose;
             bool rt = false;
             for (int k = 0; k < b - a; ++k) rt = rt || st->mods[chunk[k]].right != 0;
-            const cudaError_t e = launch_k12_any(B, hp.state_dtype == MOARA_DTYPE_BF16, st, p1, p2, tl->g1, tl->g2,
-                                                 hilo, s, launches, prof, fused ? 1 : 3, rt);
+            const bool sb = hp.state_dtype == MOARA_DTYPE_BF16;
+            // The decomposition of part q + 1 starts when K1 of part q does:
+            // K1 runs tensor-bound with HBM to spare, while K2, whose W
+            // stream keeps HBM busy, loses most when it shares the memory
+            // system.  (Also holding K2 back until the decomposition ends
+            // left a gap after each K1 and was slower.)
+            const bool bg = dec && q + 1 < np;
+            if (bg && cudaEventRecord(st->ev_k1[q], s) != cudaSuccess) return fail("part event");
+            cudaError_t e = launch_k12_any(B, sb, st, p1, p2, tl->g1, tl->g2, hilo, s, launches, prof, 1, rt);
             if (e != cudaSuccess) {
                 st->err = cudaGetErrorString(e);
                 return MOARA_ERR_CUDA;
             }
-            if (dec && q + 1 < np) {
-                if (launch_k0_any(B, st, *build_p0(pstart[q + 1], pstart[q + 2]), true, st->aux, launches, prof,
+            if (bg) {
+                if (cudaStreamWaitEvent(st->aux, st->ev_k1[q], 0) != cudaSuccess ||
+                    launch_k0_any(B, st, *build_p0(pstart[q + 1], pstart[q + 2]), true, st->aux, launches, prof,
                                   !fused) != cudaSuccess ||
                     cudaEventRecord(st->ev_part[q + 1], st->aux) != cudaSuccess)
                     return fail("background decomposition launch failed");
+            }
+            if (!fused) {
+                e = launch_k12_any(B, sb, st, p1, p2, tl->g1, tl->g2, hilo, s, launches, prof, 2, rt);
+                if (e != cudaSuccess) {
+                    st->err = cudaGetErrorString(e);
+                    return MOARA_ERR_CUDA;
+                }
             }
         }
         if (fused) {
