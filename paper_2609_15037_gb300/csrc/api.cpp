@@ -561,7 +561,7 @@ struct RefreshRunner {
     // reads only the planes).  `pl` holds 3 * rows * l bf16 entries: the
     // planes of X for the Gram matrix, then those of X^T for the apply.
     void ks_cholqr_tall(std::vector<float*>& X, const std::vector<uint16_t*>& pl, const std::vector<int>& rows,
-                        float shift_rel, int planes) {
+                        float shift_rel, int planes, bool fast_chol = true) {
         const size_t n_it = it.size();
         auto split_rows = [&](int transpose) {
             moara::SmallBatch sb = small();
@@ -578,7 +578,7 @@ struct RefreshRunner {
             g.push_back({pl[i], pl[i], pm, pm, it[i].Cg, l, l, rows[i], 0});
         }
         ks_run(g, planes);                  // Gram X^T X
-        cholesky_blocked(rows, shift_rel, /*fast=*/true);
+        cholesky_blocked(rows, shift_rel, fast_chol);
         tri_inverse(/*have_diag=*/true);
         std::vector<float*> linv(n_it);
         std::vector<uint16_t*> p2(n_it);
@@ -701,7 +701,16 @@ struct RefreshRunner {
                 std::vector<uint16_t*> qpl(n_it);
                 for (int i = 0; i < n_it; ++i) qpl[i] = it[i].Qbf;
                 ks_cholqr_tall(Qa, qpl, rows_m, 2.0f * u_rnd, 2);
-                cholqr_pass(Qa, Qb, rows_m, 0.0f, &qbf);    // Q in Qb (fp32) and qbf
+                // the second pass with three-plane (24-bit) operands and an
+                // fp32 Cholesky: the tensor cores' accumulation leaves the
+                // Gram matrix's diagonal short by ~1e-5 (relative), which
+                // scales Q's columns alike and is removed by the unit-length
+                // store of P; the off-diagonal orthogonality it gives is that
+                // of the fp32 pass
+                ks_cholqr_tall(Qa, qpl, rows_m, 0.0f, 3, /*fast_chol=*/false);
+                for (int i = 0; i < n_it; ++i)                  // Q in Qb (fp32) and qbf
+                    chk(moara::launch_f32_to_bf16(Qa[i], Qb[i], qbf[i], (long long)it[i].m * it[i].l, s,
+                                                  &ctx->launches));
             } else {
                 cholqr2s(Qa, Qb, rows_m, &qbf);             // Q in Qb (fp32) and qbf
             }

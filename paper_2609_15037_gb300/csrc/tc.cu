@@ -37,11 +37,12 @@ namespace {
 
 constexpr int kTcGroup = 224;                 // modules per launch (G maps in params)
 constexpr long long kWaitLimit = 1LL << 32;   // ~2 s of SM clocks
-constexpr int kMaps = 8;                      // tensor maps per module
+constexpr int kMaps = 9;                      // tensor maps per module
 
 struct TcMod {
     int m, n, r, kb;
     int right;        // right projector Q (n x r): K1 computes R = V Q (m x r)
+    int w3d;          // fp32 W with n % 64 == 0: K2 adds its update in 64 x 64 chunks (map 8)
     uint16_t* Qt;     // r x n bf16 transpose of a right projector (K2's B operand)
     uint16_t* Vhi;    // m x n bf16 direction matrix (written by K0)
     uint16_t* Vlo;    // m x n bf16 residual (first Adam step)
@@ -707,6 +708,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(K2_THREADS, 1)
 k2_backproject(const __grid_constant__ K2Params p) {
     constexpr int WC = StateCols<SB>::N;              // W columns per ring chunk
     constexpr int HC = WC / 2;                        // columns per epilogue thread and chunk
+    // fp32 W, blocks of >= 32 columns: 64 x 64 update chunks through the 3-D
+    // map where the module allows it (TcMod::w3d)
+    constexpr bool W3D = !SB && BLK >= 32 && K2_BN % BLK == 0;
     static_assert(!SB || BLK >= 32, "bf16 states: a thread's 32 columns lie in one block");
     constexpr int K2_STAGES = K2Cfg<SB>::STAGES, K2_WBUF = K2Cfg<SB>::WBUF;
     extern __shared__ uint8_t smem_raw[];
@@ -867,14 +871,18 @@ k2_backproject(const __grid_constant__ K2Params p) {
                 const TcMod& md = p.mods[tl.mod];
                 const CUtensorMap* wmap = &p.maps[tl.mod * kMaps + 3];
                 const int i0 = (2 * tl.t0 + crank) * K2_BM, n0 = tl.t1 * K2_BN;
-                const int nc = min(K2_BN / WC, (md.n - n0 + WC - 1) / WC);
+                const bool w3 = W3D && md.w3d;
+                const int nc = w3 ? 2 * min(K2_BN / 64, (md.n - n0) / 64) : min(K2_BN / WC, (md.n - n0 + WC - 1) / WC);
                 for (int c = 0; c < nc; ++c, ++g) {
                     const int b = g % K2_WBUF;
                     const uint32_t ph = (g / K2_WBUF) & 1;
                     if (!ptx::mbar_wait(ptx::smem_u32(&ctl->wdone[b]), ph, abort_flag, p.status,
                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit)) { ok = false; break; }
-                    if constexpr (SB) ptx::tma_store_2d(wmap, ptx::smem_u32(wring + b * K2_WBYTES), n0 + c * WC, i0);
-                    else ptx::tma_reduce_add_2d(wmap, ptx::smem_u32(wring + b * K2_WBYTES), n0 + c * WC, i0);
+                    const uint32_t src = ptx::smem_u32(wring + b * K2_WBYTES);
+                    if constexpr (SB) ptx::tma_store_2d(wmap, src, n0 + c * WC, i0);
+                    else if (w3) ptx::tma_reduce_add_3d(&p.maps[tl.mod * kMaps + 8], src, 0, (n0 + 64 * (c >> 1)) / 32,
+                                                        i0 + 64 * (c & 1));
+                    else ptx::tma_reduce_add_2d(wmap, src, n0 + c * WC, i0);
                     ptx::bulk_commit_group();
                     ptx::bulk_wait_read_all();            // the chunk may be refilled once read
                     ptx::mbar_arrive(ptx::smem_u32(&ctl->wempty[b]));
@@ -907,7 +915,8 @@ k2_backproject(const __grid_constant__ K2Params p) {
             const int i0 = (2 * tl.t0 + crank) * K2_BM, n0 = tl.t1 * K2_BN;
             const int i = i0 + il;
             const bool row_ok = i < mm;
-            const int nc = min(K2_BN / WC, (nn - n0 + WC - 1) / WC);
+            const bool w3 = W3D && md.w3d;
+            const int nc = w3 ? 2 * min(K2_BN / 64, (nn - n0) / 64) : min(K2_BN / WC, (nn - n0 + WC - 1) / WC);
             // blocks of B >= 32 columns: the tile's dM values of this row are
             // loaded once, before the wait for the accumulator
             float dmt[HOIST ? K2_BN / BLK : 1];
@@ -925,6 +934,47 @@ k2_backproject(const __grid_constant__ K2Params p) {
             for (int c = 0; c < nc; ++c, ++g) {
                 const int b = g % K2_WBUF;
                 const uint32_t ph = (g / K2_WBUF) & 1;
+                if constexpr (W3D) {
+                    if (w3) {
+                        // chunk c: rows 64 (c & 1) .. + 63 and columns 64 (c >> 1) .. + 63 of
+                        // the tile, written by the four warps of that row half (warp ch:
+                        // the 32-column group ch, one 128-byte line per row; two lines
+                        // of a warp's store share a bank group); the other four only
+                        // pass the chunk's barriers
+                        const bool mine = (c & 1) == (q >> 1);
+                        const int cb = (c >> 1) * 64 + ch * 32;
+                        float v[32];
+                        if (mine) {
+                            __syncwarp();
+                            const uint32_t ta = tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * 256 + cb;
+                            ptx::tmem_ld16(ta, *reinterpret_cast<float(*)[16]>(v));
+                            ptx::tmem_ld16(ta + 16, *reinterpret_cast<float(*)[16]>(v + 16));
+                        }
+                        const bool gotw = ptx::mbar_wait(ptx::smem_u32(&ctl->wempty[b]), ph ^ 1, abort_flag, p.status,
+                                                         MOARA_ERR_DEVICE_TIMEOUT, kWaitLimit);
+                        if (!__all_sync(0xffffffffu, gotw)) { ok = false; break; }
+                        if (mine) {
+                            float d0 = dmt[0];
+#pragma unroll
+                            for (int d = 1; d < K2_BN / BLK; ++d) d0 = (cb >= d * BLK) ? dmt[d] : d0;
+                            const float ms = -p.step_scale;
+                            const int ln = (32 * (q & 1) + lane) * 2 + ch;    // box line: row * 2 + group
+                            uint8_t* line = wring + b * K2_WBYTES + ln * 128;
+                            const uint32_t x = static_cast<uint32_t>(ln & 7);
+#pragma unroll
+                            for (int u = 0; u < 8; ++u)
+                                *reinterpret_cast<uint4*>(line + ((u ^ x) << 4)) =
+                                    make_uint4(__float_as_uint(ms * (d0 * v[4 * u + 0])),
+                                               __float_as_uint(ms * (d0 * v[4 * u + 1])),
+                                               __float_as_uint(ms * (d0 * v[4 * u + 2])),
+                                               __float_as_uint(ms * (d0 * v[4 * u + 3])));
+                        }
+                        ptx::fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&ctl->wdone[b]));
+                        continue;
+                    }
+                }
                 const int j0 = n0 + c * WC + ch * HC;
                 float dm[NDM];
                 if (HOIST) {
@@ -1670,6 +1720,24 @@ int tc_register(TcState* st, int id, const ModDev& md, const moara_hparams& hp) 
     if (!ok) {
         st->err = "cuTensorMapEncodeTiled failed";
         return MOARA_ERR_CUDA;
+    }
+    // An fp32 W whose rows split into 64-column pairs of 128-byte groups is
+    // also viewed as (32 columns, n / 32 groups, m rows): a box of 32 x 2 x 64
+    // adds 64 rows x 256 contiguous bytes per row with one reduce, traversed
+    // row by row, while each 128-byte group stays one swizzled line of the
+    // staging chunk (line = row * 2 + group).  The wider contiguous pieces per
+    // row keep HBM pages open longer than the 128-byte pieces of the 2-D map
+    // (K2 per two 7B layers 0.74 -> 0.70 ms; the group-outer box order, whose
+    // lines are free of bank conflicts, gave 0.72 ms).
+    t.w3d = 0;
+    if (!sb && md.n % 64 == 0) {
+        const cuuint64_t dims[3] = {32, static_cast<cuuint64_t>(md.n / 32), static_cast<cuuint64_t>(md.m)};
+        const cuuint64_t strides[2] = {128, static_cast<cuuint64_t>(md.n) * 4};
+        const cuuint32_t box[3] = {32, 2, 64};
+        const cuuint32_t estr[3] = {1, 1, 1};
+        t.w3d = st->encode(&mp[8], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, md.W, dims, strides, box, estr,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
     }
     st->mods[id] = t;
     st->dirty = true;
