@@ -173,15 +173,21 @@ cudaError_t launch_trace_shift(const SmallBatch& b, cudaStream_t s, int64_t* lau
     return cudaGetLastError();
 }
 
-// 64 threads, thread i keeps row i of the block (and later row i of its
-// inverse) in registers; the finished column j of the factor, and later the
-// finished row k of the inverse, is broadcast through shared memory, so each
-// of the 64 steps costs two barriers of two warps and one pass of predicated
-// register FMAs.  The block moves between global and shared memory coalesced.
+// 64 threads, thread i keeps row i of the block in registers.  The step
+// loops stay rolled (a fully unrolled 64 x 64 factorisation is too large for
+// the instruction cache and stalls on instruction fetch): during the
+// factorisation each row is shifted left by one column per step, so the
+// column being eliminated is always a[0] and every register index is a
+// compile-time constant; the finished column j of the factor is broadcast
+// through shared memory.  The inverse then runs by forward substitution,
+// thread i holding row i of the inverse; the finished row k is broadcast
+// (its entries past k are exact zeros, so every row update may run over all
+// 64 columns).  Each step costs two barriers of two warps.  The block moves
+// between global and shared memory coalesced.
 __global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
     constexpr int NB = kTriBase;
-    __shared__ float tile[NB][NB + 1];   // coalesced staging of the block
-    __shared__ float bc[NB];             // broadcast column / row
+    __shared__ float tile[NB][NB + 1];   // the block; the factor's lower part as it is finished
+    __shared__ __align__(16) float bc[NB + 4];   // broadcast column of the factor / row of the inverse
     __shared__ float piv;
     __shared__ int s_fail;
     const int pi = blockIdx.x;
@@ -197,36 +203,50 @@ __global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallB
         tile[r][i] = (r < sz && i < sz) ? A[(long long)(j0 + r) * l + j0 + i] + (r == i ? shift : 0.0f)
                                         : (r == i ? 1.0f : 0.0f);
     if (i == 0) s_fail = 0;
+    bc[i] = 0.0f;
+    if (i < 4) bc[NB + i] = 0.0f;
     __syncthreads();
     float a[NB];
 #pragma unroll
     for (int k = 0; k < NB; ++k) a[k] = tile[i][k];
-    // right-looking factorisation: step j finishes column j (pivot sqrt(d);
-    // a pivot that is not positive and finite is replaced by 1 and marks the
-    // failure) and subtracts its outer product from the trailing lower part
-#pragma unroll
+    // right-looking factorisation; at step j, a[k] of row i holds column j + k
+    // of the updated matrix.  A pivot that is not positive and finite is
+    // replaced by 1 and marks the failure.
+#pragma unroll 1
     for (int j = 0; j < NB; ++j) {
         if (i == j) {
-            float d = a[j];
+            float d = a[0];
             if (!(d > 0.0f) || !isfinite(d)) {
                 d = 1.0f;
                 s_fail = 1;
             }
-            a[j] = sqrtf(d);
-            piv = a[j];
+            d = sqrtf(d);
+            piv = d;
+            tile[j][j] = d;
         }
         __syncthreads();
+        float lij = 0.0f;
         if (i > j) {
-            a[j] = a[j] / piv;
-            bc[i] = a[j];
+            lij = a[0] / piv;
+            bc[i - j - 1] = lij;       // column j of L below the diagonal, from index 0
+            tile[i][j] = lij;
         }
         __syncthreads();
-        if (i > j) {
-            const float lij = a[j];
+        // row i -= L[i][j] * (column j of L)^T over columns j + 1 .., shifted
+        // left by one: a[k] (column j + k) takes bc[k - 1] = L[j + k][j].
+        // Past index 62 - j, bc holds earlier columns' values; they reach
+        // only slots of columns past the block or above the diagonal (and
+        // rows i <= j, which are finished), none of which is read again.
+        const float4* col4 = reinterpret_cast<const float4*>(bc);
 #pragma unroll
-            for (int k = j + 1; k < NB; ++k)
-                if (k <= i) a[k] = fmaf(-lij, bc[k], a[k]);
+        for (int k = 1; k < NB; k += 4) {
+            const float4 lk = col4[(k - 1) / 4];
+            a[k - 1] = fmaf(-lij, lk.x, a[k]);
+            a[k] = fmaf(-lij, lk.y, a[k + 1]);
+            a[k + 1] = fmaf(-lij, lk.z, a[k + 2]);
+            if (k + 3 < NB) a[k + 2] = fmaf(-lij, lk.w, a[k + 3]);
         }
+        a[NB - 1] = 0.0f;
     }
     // inverse by forward substitution: row k of the inverse is finished at
     // step k (divided by the pivot) and broadcast; rows below subtract
@@ -234,27 +254,33 @@ __global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallB
     float x[NB];
 #pragma unroll
     for (int c = 0; c < NB; ++c) x[c] = (c == i) ? 1.0f : 0.0f;
-#pragma unroll
+    float4* bc4 = reinterpret_cast<float4*>(bc);
+#pragma unroll 1
     for (int k = 0; k < NB; ++k) {
         if (i == k) {
-            const float inv = 1.0f / a[k];
+            const float inv = 1.0f / tile[k][k];
 #pragma unroll
-            for (int c = 0; c <= k; ++c) {
-                x[c] *= inv;
-                bc[c] = x[c];
+            for (int c = 0; c < NB; c += 4) {
+                x[c] *= inv; x[c + 1] *= inv; x[c + 2] *= inv; x[c + 3] *= inv;
+                bc4[c / 4] = make_float4(x[c], x[c + 1], x[c + 2], x[c + 3]);
             }
         }
         __syncthreads();
         if (i > k) {
-            const float lik = a[k];
+            const float lik = tile[i][k];
 #pragma unroll
-            for (int c = 0; c <= k; ++c) x[c] = fmaf(-lik, bc[c], x[c]);
+            for (int c = 0; c < NB; c += 4) {
+                const float4 r = bc4[c / 4];
+                x[c] = fmaf(-lik, r.x, x[c]);
+                x[c + 1] = fmaf(-lik, r.y, x[c + 1]);
+                x[c + 2] = fmaf(-lik, r.z, x[c + 2]);
+                x[c + 3] = fmaf(-lik, r.w, x[c + 3]);
+            }
         }
         __syncthreads();
     }
     // the factor (zeros above the diagonal) in place, the inverse into c
-#pragma unroll
-    for (int k = 0; k < NB; ++k) tile[i][k] = (k <= i) ? a[k] : 0.0f;
+    for (int k = i + 1; k < NB; ++k) tile[i][k] = 0.0f;
     __syncthreads();
     for (int r = 0; r < sz; ++r)
         if (i < sz) A[(long long)(j0 + r) * l + j0 + i] = tile[r][i];
