@@ -10,6 +10,7 @@
 #include <limits>
 #include <new>
 #include <string>
+#include <array>
 #include <vector>
 
 #include "internal.h"
@@ -252,6 +253,7 @@ int refresh_l(const moara_ctx* ctx, int m, int n, int r) {
 // ------------------------------------------------------------------ refresh
 // Panel width of the fast blocked Cholesky (tensor-core trailing updates).
 constexpr int kFastPanel = 256;
+constexpr int kTriTcMin = 512;   // triangular-inverse levels from this block size run on tensor cores
 
 struct RefreshRunner {
     moara_ctx* ctx;
@@ -394,6 +396,54 @@ struct RefreshRunner {
         ks_run(g, 2);
     }
 
+    // One level of the blocked triangular inverse on tensor cores, for the
+    // pairs (module, a0, d0, dn) of block size sz:
+    //   T[D, A] = L[D, A] Linv[A, A];  Linv[D, A] = -Linv[D, D] T[D, A],
+    // both as three-plane (24-bit) split-precision products.  Each pair's
+    // operands are split into the module's P1 (A side) and P2 (B side)
+    // planes at running offsets; a level's pairs of one module cover
+    // disjoint rows, so they need at most 3 l^2 / 4 entries per side.
+    // Linv[D, A] is still zero here, so "out -= A B" gives the negated product.
+    template <class PairAt>
+    void tri_level_tc(int sz, size_t npairs, PairAt pair_at) {
+        for (int pass = 0; pass < 2; ++pass) {
+            std::vector<size_t> off_a(it.size(), 0), off_b(it.size(), 0);
+            std::vector<moara::TcSplitGemmItem> items;
+            moara::SmallBatch sa{}, sb{};
+            auto flush_splits = [&]() {
+                if (sa.count > 0) chk(moara::launch_split3(sa, 1, s, &ctx->launches));
+                if (sb.count > 0) chk(moara::launch_split3(sb, 0, s, &ctx->launches));
+                sa = moara::SmallBatch{};
+                sb = moara::SmallBatch{};
+            };
+            for (size_t q = 0; q < npairs; ++q) {
+                const std::array<int, 4> pr = pair_at(q);
+                const auto& x = it[pr[0]];
+                const long long l = x.l;
+                const int a0 = pr[1], d0 = pr[2], dn = pr[3];
+                const int K = pass == 0 ? sz : dn;
+                // A is read as K x M (the transpose of the left factor), B as K x N
+                const float* asrc = pass == 0 ? x.Cg + d0 * l + a0 : x.Linv + d0 * l + d0;
+                const float* bsrc = pass == 0 ? x.Linv + a0 * l + a0 : x.Tt + d0 * l + a0;
+                uint16_t* ap = x.P1 + off_a[pr[0]];
+                uint16_t* bp = x.P2 + off_b[pr[0]];
+                off_a[pr[0]] += 3 * (size_t)K * dn;
+                off_b[pr[0]] += 3 * (size_t)K * sz;
+                if (sa.count == moara::kMaxGroup) flush_splits();
+                const int ia = sa.count++, ib = sb.count++;
+                sa.a[ia] = const_cast<float*>(asrc); sa.h[ia] = ap; sa.rows[ia] = dn; sa.l[ia] = K; sa.ld[ia] = x.l;
+                sb.a[ib] = const_cast<float*>(bsrc); sb.h[ib] = bp; sb.rows[ib] = K; sb.l[ib] = sz; sb.ld[ib] = x.l;
+                moara::TcSplitGemmItem g{ap, bp, (size_t)K * dn, (size_t)K * sz,
+                                         pass == 0 ? x.Tt + d0 * l + a0 : x.Linv + d0 * l + a0, dn, sz, K, 0};
+                g.ldo = x.l;
+                g.sub = pass == 1 ? 1 : 0;
+                items.push_back(g);
+            }
+            flush_splits();
+            ks_run(items, 3);
+        }
+    }
+
     void tri_inverse(bool have_diag) {
         int lmax = 0;
         for (auto& x : it) {
@@ -407,6 +457,7 @@ struct RefreshRunner {
         }
         moara::GemmKind mul{moara::A_KCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE};
         moara::GemmKind neg{moara::A_KCONTIG, moara::B_NCONTIG, 0, 0, 0, 0, moara::EPI_STORE_NEG};
+        const bool tc = !it.empty() && it[0].tc && ctx->tc != nullptr;
         for (int sz = moara::kTriBase; sz < lmax; sz *= 2) {
             struct Pair { int mod, a0, d0, dn; };
             std::vector<Pair> pairs;
@@ -414,6 +465,13 @@ struct RefreshRunner {
                 const int l = it[i].l;
                 for (int a0 = 0; a0 + sz < l; a0 += 2 * sz)
                     pairs.push_back({i, a0, a0 + sz, std::min(sz, l - a0 - sz)});
+            }
+            if (tc && sz >= kTriTcMin) {
+                tri_level_tc(sz, pairs.size(), [&](size_t q) {
+                    const Pair& pr = pairs[q];
+                    return std::array<int, 4>{pr.mod, pr.a0, pr.d0, pr.dn};
+                });
+                continue;
             }
             for (int pass = 0; pass < 2; ++pass) {
                 for (size_t c0 = 0; c0 < pairs.size(); c0 += moara::kMaxGroup) {
@@ -597,14 +655,14 @@ struct RefreshRunner {
     // triangular apply as split-precision tensor-core products (fp32-accurate):
     // Xout = Win R^-1, R^T R = Win^T Win + shift.
     void ks_cholqr_pass(std::vector<float*>& Win, std::vector<float*>& Xout, const std::vector<int>& rows_l,
-                        float shift_rel, int planes) {
+                        float shift_rel, int planes, bool fast_chol = true) {
         std::vector<uint16_t*> p1(it.size()), p2(it.size());
         for (size_t i = 0; i < it.size(); ++i) { p1[i] = it[i].P1; p2[i] = it[i].P2; }
         std::vector<float*> cg(it.size());
         for (size_t i = 0; i < it.size(); ++i) cg[i] = it[i].Cg;
         split3(Win, p1, 0);                 // W (as A = W^T, MN-major, and as B)
         ks_gemm(p1, p1, cg, 0, planes);     // Gram W^T W
-        cholesky_blocked(rows_l, shift_rel, /*fast=*/true);
+        cholesky_blocked(rows_l, shift_rel, fast_chol);
         tri_inverse(/*have_diag=*/true);
         std::vector<float*> linv(it.size());
         for (size_t i = 0; i < it.size(); ++i) linv[i] = it[i].Linv;
@@ -807,11 +865,11 @@ struct RefreshRunner {
                 split3(Xa, p1, 0);
                 ks_gemm(cp, p1, Xb, 0, planes);          // W = C X
                 ks_cholqr_pass(Xb, Xa, rows_l, 2.0f * u_rnd, planes);
-                // the tensor cores accumulate long sums less tightly than
-                // fp32 FMAs: the pass that fixes the final orthonormality of
-                // X runs on the fp32 units
-                if (!last) ks_cholqr_pass(Xa, Xb, rows_l, 0.0f, planes);
-                else cholqr_pass(Xa, Xb, rows_l, 0.0f);
+                // the pass that fixes the final orthonormality of X: three
+                // planes and an fp32 Cholesky (the tensor cores' short
+                // diagonal of the Gram matrix scales the columns of X alike;
+                // P's columns are stored at unit length)
+                ks_cholqr_pass(Xa, Xb, rows_l, 0.0f, planes, /*fast_chol=*/!last);
                 std::swap(Xa, Xb);                       // X in Xa
             } else {
                 gemm(prod, [&](int i, moara::GemmProb& p) {

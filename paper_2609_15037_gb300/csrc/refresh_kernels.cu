@@ -4,6 +4,7 @@
 // inverse used by CholeskyQR, the ordering of Ritz vectors, and the final sign
 // convention.  One CTA per problem (or per diagonal block); the problems of a
 // group run side by side in one launch.
+#include <algorithm>
 #include <cuda_bf16.h>
 
 #include "internal.h"
@@ -353,6 +354,10 @@ __global__ void __launch_bounds__(256) k_split3(const __grid_constant__ SmallBat
     const long long plane = (long long)rows * cols;
     const int tr = (rows + 31) / 32, tc = (cols + 31) / 32;
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    // stores: thread (ty2, tx2) writes output rows ty2 and ty2 + 16 of the
+    // tile, columns 2 tx2 and 2 tx2 + 1, as 4-byte pairs where aligned
+    const int tx2 = threadIdx.x & 15, ty2 = threadIdx.x >> 4;
+    const int orows = transpose ? cols : rows, ocols = transpose ? rows : cols;
     for (int tile = blockIdx.x; tile < tr * tc; tile += gridDim.x) {
         const int ti = tile / tc, tj = tile - ti * tc;
         for (int r = ty; r < 32; r += 8) {
@@ -360,21 +365,44 @@ __global__ void __launch_bounds__(256) k_split3(const __grid_constant__ SmallBat
             t[r][tx] = (i < rows && j < cols) ? src[(long long)i * lds + j] : 0.0f;
         }
         __syncthreads();
-        for (int r = ty; r < 32; r += 8) {
-            int i, j, oc;
-            float x;
-            if (transpose) { i = tj * 32 + r; j = ti * 32 + tx; oc = rows; x = t[tx][r]; }   // out row i = src column
-            else           { i = ti * 32 + r; j = tj * 32 + tx; oc = cols; x = t[r][tx]; }
-            const bool in = transpose ? (i < cols && j < rows) : (i < rows && j < cols);
-            if (in) {
-                const __nv_bfloat16 h0 = __float2bfloat16_rn(x);
-                const float r1 = x - __bfloat162float(h0);
-                const __nv_bfloat16 h1 = __float2bfloat16_rn(r1);
-                const __nv_bfloat16 h2 = __float2bfloat16_rn(r1 - __bfloat162float(h1));
-                const long long o = (long long)i * oc + j;
-                dst[o] = *reinterpret_cast<const uint16_t*>(&h0);
-                dst[plane + o] = *reinterpret_cast<const uint16_t*>(&h1);
-                dst[2 * plane + o] = *reinterpret_cast<const uint16_t*>(&h2);
+        for (int rr = ty2; rr < 32; rr += 16) {
+            const int i = (transpose ? tj : ti) * 32 + rr;          // output row
+            const int j = (transpose ? ti : tj) * 32 + 2 * tx2;     // output column of the pair
+            if (i < orows && j < ocols) {
+                const float x0 = transpose ? t[2 * tx2][rr] : t[rr][2 * tx2];
+                const float x1 = transpose ? t[2 * tx2 + 1][rr] : t[rr][2 * tx2 + 1];
+                uint16_t h[3], g[3];
+                {
+                    const __nv_bfloat16 a0 = __float2bfloat16_rn(x0);
+                    const float r0 = x0 - __bfloat162float(a0);
+                    const __nv_bfloat16 a1 = __float2bfloat16_rn(r0);
+                    const __nv_bfloat16 a2 = __float2bfloat16_rn(r0 - __bfloat162float(a1));
+                    h[0] = *reinterpret_cast<const uint16_t*>(&a0);
+                    h[1] = *reinterpret_cast<const uint16_t*>(&a1);
+                    h[2] = *reinterpret_cast<const uint16_t*>(&a2);
+                }
+                {
+                    const __nv_bfloat16 a0 = __float2bfloat16_rn(x1);
+                    const float r0 = x1 - __bfloat162float(a0);
+                    const __nv_bfloat16 a1 = __float2bfloat16_rn(r0);
+                    const __nv_bfloat16 a2 = __float2bfloat16_rn(r0 - __bfloat162float(a1));
+                    g[0] = *reinterpret_cast<const uint16_t*>(&a0);
+                    g[1] = *reinterpret_cast<const uint16_t*>(&a1);
+                    g[2] = *reinterpret_cast<const uint16_t*>(&a2);
+                }
+                const long long o = (long long)i * ocols + j;
+                if (j + 1 < ocols && ((o | plane) & 1) == 0 && (reinterpret_cast<uintptr_t>(dst) & 3) == 0) {
+#pragma unroll
+                    for (int q = 0; q < 3; ++q)
+                        *reinterpret_cast<uint32_t*>(dst + q * plane + o) =
+                            static_cast<uint32_t>(h[q]) | (static_cast<uint32_t>(g[q]) << 16);
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 3; ++q) {
+                        dst[q * plane + o] = h[q];
+                        if (j + 1 < ocols) dst[q * plane + o + 1] = g[q];
+                    }
+                }
             }
         }
         __syncthreads();
@@ -383,7 +411,11 @@ __global__ void __launch_bounds__(256) k_split3(const __grid_constant__ SmallBat
 
 cudaError_t launch_split3(const SmallBatch& b, int transpose, cudaStream_t s, int64_t* launches) {
     if (b.count <= 0) return cudaSuccess;
-    k_split3<<<dim3(256, 1, b.count), 256, 0, s>>>(b, transpose);
+    // as many blocks per item as the largest item has 32 x 32 tiles (at most 256)
+    long long tiles = 1;
+    for (int q = 0; q < b.count; ++q)
+        tiles = std::max(tiles, (long long)((b.rows[q] + 31) / 32) * ((b.l[q] + 31) / 32));
+    k_split3<<<dim3(static_cast<unsigned>(std::min(256LL, tiles)), 1, b.count), 256, 0, s>>>(b, transpose);
     ++*launches;
     return cudaGetLastError();
 }
