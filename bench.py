@@ -393,6 +393,13 @@ def run_gpu(args):
     alg_bytes, alg_flops, _ = _algorithmic(mods, B, sbytes, args.proj_rule)
     total_ms = step_ms + refresh_ms / 200.0
     roof_ms = max(alg_bytes / (hbm * 1e9), alg_flops / (bf16_sus * 1e12)) * 1e3
+    # the refresh's product flops: 2q + 2 products of V (m x n) with an
+    # n x l or m x l basis, l = min(r + p, m, n), at 2 m n l flops each
+    rf_flops = 0.0
+    for md in mods:
+        lw = min(md.r + hp.oversample, md.m, md.n)
+        rf_flops += (2 * hp.power_iters + 2) * 2.0 * md.m * md.n * lw
+    rf_roof_ms = rf_flops / (bf16_sus * 1e12) * 1e3
 
     # dominant kernel
     used_tc = prof["tc_project"][1] > 0
@@ -472,6 +479,10 @@ def run_gpu(args):
         "step_ms_no_refresh": round(step_ms, 4),
         "clip_norm_ms": round(prof["clip_norm"][0] / args.steps, 4) if prof["clip_norm"][1] else None,
         "refresh_ms": round(refresh_ms, 2), "refresh_amortised_ms": round(refresh_ms / 200.0, 4),
+        "refresh_roofline": {"flops": rf_flops, "roofline_ms": round(rf_roof_ms, 2),
+                             "frac": round(rf_roof_ms / refresh_ms, 4) if refresh_ms > 0 else None,
+                             "basis": f"(2q+2)*2*m*n*(r+p) with q = {hp.power_iters}, p = {hp.oversample}, "
+                                      f"at the sustained bf16 rate"},
         "hbm_gbs_algorithmic": round(alg_bytes / (step_ms * 1e-3) / 1e9, 1),
         "step_roofline": {"alg_bytes": alg_bytes, "alg_flops": alg_flops,
                           "roofline_ms": round(roof_ms, 3),
