@@ -562,7 +562,9 @@ struct RefreshRunner {
         std::vector<moara::TcGemmItem> gram;
         for (size_t i = 0; i < it.size(); ++i) {
             const int l = it[i].l;
-            gram.push_back({Xin[i], nullptr, Xin[i], it[i].Cg, nullptr, l, l, rows[i], 0});
+            moara::TcGemmItem g{Xin[i], nullptr, Xin[i], it[i].Cg, nullptr, l, l, rows[i], 0};
+            g.lower = 1;                    // the Cholesky reads the lower triangle only
+            gram.push_back(g);
         }
         tc_gemm(0, gram);
         cholesky_blocked(rows, shift_rel, /*fast=*/true);

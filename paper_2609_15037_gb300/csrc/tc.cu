@@ -1096,6 +1096,7 @@ struct KrParams {
     int al_B, al_log2B;                // block size (a power of two) and its log2
     int M[kKrGroup], N[kKrGroup], K[kKrGroup];
     int ktri[kKrGroup];
+    int lower[kKrGroup];               // tiles above the diagonal are skipped
     int tiles_n[kKrGroup];
     int tile_start[kKrGroup + 1];
     int count;
@@ -1125,6 +1126,7 @@ __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constan
     const int M = p.M[pi], N = p.N[pi], K = p.K[pi];
     const int i0 = (local / p.tiles_n[pi]) * KR_BM;
     const int n0 = (local % p.tiles_n[pi]) * KR_BN;
+    if (p.lower[pi] && n0 >= i0 + KR_BM) return;     // whole CTA, before any barrier or TMEM
     const int nch = min(4, (N - n0 + 63) / 64);            // 64-column chunks of B in this tile
     const int halves = (M - i0) > 128 ? 2 : 1;
     const int kend = p.ktri[pi] ? min(K, n0 + KR_BN) : K;
@@ -2209,6 +2211,7 @@ static int kr_launch(TcState* st, int a_kmajor, const TcGemmItem* items, int cou
                 }
                 kp.M[q] = x.M; kp.N[q] = x.N; kp.K[q] = x.K;
                 kp.ktri[q] = x.ktri;
+                kp.lower[q] = x.lower;
                 kp.tiles_n[q] = (x.N + KR_BN - 1) / KR_BN;
                 kp.tile_start[q] = total;
                 total += ((x.M + KR_BM - 1) / KR_BM) * kp.tiles_n[q];

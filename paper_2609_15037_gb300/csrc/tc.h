@@ -49,6 +49,7 @@ struct TcGemmItem {
     int M, N, K;
     int ktri;              // B upper triangular: column j needs k <= j only
     uint16_t* out_lo;      // M x N row-major bf16 residual out - bf16(out), or null
+    int lower;             // 1: only output tiles on or below the diagonal (M = N)
 };
 
 // Grouped launch of TcGemmItems (A read K-major when a_kmajor, else
