@@ -174,21 +174,26 @@ cudaError_t launch_trace_shift(const SmallBatch& b, cudaStream_t s, int64_t* lau
     return cudaGetLastError();
 }
 
-// 64 threads, thread i keeps row i of the block in registers.  The step
-// loops stay rolled (a fully unrolled 64 x 64 factorisation is too large for
-// the instruction cache and stalls on instruction fetch): during the
-// factorisation each row is shifted left by one column per step, so the
-// column being eliminated is always a[0] and every register index is a
-// compile-time constant; the finished column j of the factor is broadcast
-// through shared memory.  The inverse then runs by forward substitution,
-// thread i holding row i of the inverse; the finished row k is broadcast
-// (its entries past k are exact zeros, so every row update may run over all
-// 64 columns).  Each step costs two barriers of two warps.  The block moves
-// between global and shared memory coalesced.
-__global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
+// 128 threads, two per row: thread (i, h) keeps columns 32 h .. 32 h + 31 of
+// row i of the block in registers (the two threads of a row are adjacent
+// lanes of one warp).  The step loops stay rolled (a fully unrolled 64 x 64
+// factorisation is too large for the instruction cache and stalls on
+// instruction fetch): during the factorisation each row is shifted left by
+// one column per step, the column crossing from the upper to the lower half
+// by a lane shuffle, so the column being eliminated is always a[0] of the
+// h = 0 thread and every register index is a compile-time constant; the
+// finished column j of the factor is broadcast through shared memory from
+// index 0, read as aligned 16-byte vectors.  The inverse then runs by
+// forward substitution, thread (i, h) holding half of row i of the inverse;
+// the finished row k is broadcast (its entries past k are exact zeros, so
+// every row update may run over all 64 columns).  Each step costs two
+// barriers of four warps.  The block moves between global and shared memory
+// coalesced.
+__global__ void __launch_bounds__(128) k_chol_diag(const __grid_constant__ SmallBatch b, int j0) {
     constexpr int NB = kTriBase;
+    constexpr int HB = NB / 2;
     __shared__ float tile[NB][NB + 1];   // the block; the factor's lower part as it is finished
-    __shared__ __align__(16) float bc[NB + 4];   // broadcast column of the factor / row of the inverse
+    __shared__ __align__(16) float bc[NB];   // broadcast column of the factor / row of the inverse
     __shared__ float piv;
     __shared__ int s_fail;
     const int pi = blockIdx.x;
@@ -198,24 +203,28 @@ __global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallB
     float* A = b.a[pi];
     float* X = b.c[pi];
     const float shift = b.b[pi][0];
-    const int i = threadIdx.x;
+    const int t = threadIdx.x;
+    const int i = t >> 1, h = t & 1, c0 = h * HB;
+    const int lane = t & 31;
     // rows and columns past sz are padded with the identity
-    for (int r = 0; r < NB; ++r)
-        tile[r][i] = (r < sz && i < sz) ? A[(long long)(j0 + r) * l + j0 + i] + (r == i ? shift : 0.0f)
-                                        : (r == i ? 1.0f : 0.0f);
-    if (i == 0) s_fail = 0;
-    bc[i] = 0.0f;
-    if (i < 4) bc[NB + i] = 0.0f;
+    for (int r = t >> 6; r < NB; r += 2) {
+        const int c = t & 63;
+        tile[r][c] = (r < sz && c < sz) ? A[(long long)(j0 + r) * l + j0 + c] + (r == c ? shift : 0.0f)
+                                        : (r == c ? 1.0f : 0.0f);
+    }
+    if (t == 0) s_fail = 0;
+    if (t < NB) bc[t] = 0.0f;
     __syncthreads();
-    float a[NB];
+    float a[HB];
 #pragma unroll
-    for (int k = 0; k < NB; ++k) a[k] = tile[i][k];
-    // right-looking factorisation; at step j, a[k] of row i holds column j + k
-    // of the updated matrix.  A pivot that is not positive and finite is
-    // replaced by 1 and marks the failure.
+    for (int k = 0; k < HB; ++k) a[k] = tile[i][c0 + k];
+    // right-looking factorisation; at step j, a[k] of thread (i, h) holds
+    // column j + 32 h + k of the updated row i.  A pivot that is not positive
+    // and finite is replaced by 1 and marks the failure.
+    const float4* col4 = reinterpret_cast<const float4*>(bc) + h * (HB / 4);
 #pragma unroll 1
     for (int j = 0; j < NB; ++j) {
-        if (i == j) {
+        if (i == j && h == 0) {
             float d = a[0];
             if (!(d > 0.0f) || !isfinite(d)) {
                 d = 1.0f;
@@ -227,41 +236,45 @@ __global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallB
         }
         __syncthreads();
         float lij = 0.0f;
-        if (i > j) {
+        if (i > j && h == 0) {
             lij = a[0] / piv;
             bc[i - j - 1] = lij;       // column j of L below the diagonal, from index 0
             tile[i][j] = lij;
         }
+        lij = __shfl_sync(0xffffffffu, lij, lane & ~1);
+        const float up = __shfl_sync(0xffffffffu, a[0], lane | 1);   // column j + 32, before its update
         __syncthreads();
         // row i -= L[i][j] * (column j of L)^T over columns j + 1 .., shifted
-        // left by one: a[k] (column j + k) takes bc[k - 1] = L[j + k][j].
-        // Past index 62 - j, bc holds earlier columns' values; they reach
-        // only slots of columns past the block or above the diagonal (and
-        // rows i <= j, which are finished), none of which is read again.
-        const float4* col4 = reinterpret_cast<const float4*>(bc);
+        // left by one: a[k] (column j + 32 h + k) takes bc[32 h + k - 1] =
+        // L[j + 32 h + k][j].  Past index 62 - j, bc holds earlier columns'
+        // values; they reach only slots of columns past the block or above
+        // the diagonal (and rows i <= j, which are finished), none of which
+        // is read again.
 #pragma unroll
-        for (int k = 1; k < NB; k += 4) {
+        for (int k = 1; k < HB; k += 4) {
             const float4 lk = col4[(k - 1) / 4];
             a[k - 1] = fmaf(-lij, lk.x, a[k]);
             a[k] = fmaf(-lij, lk.y, a[k + 1]);
             a[k + 1] = fmaf(-lij, lk.z, a[k + 2]);
-            if (k + 3 < NB) a[k + 2] = fmaf(-lij, lk.w, a[k + 3]);
+            if (k + 3 < HB) a[k + 2] = fmaf(-lij, lk.w, a[k + 3]);
         }
-        a[NB - 1] = 0.0f;
+        // the last slot: column j + 32 crosses from the upper half (h = 0
+        // takes it, updated with bc[31]); past the block for h = 1
+        a[HB - 1] = h == 0 ? fmaf(-lij, bc[HB - 1], up) : 0.0f;
     }
     // inverse by forward substitution: row k of the inverse is finished at
     // step k (divided by the pivot) and broadcast; rows below subtract
     // L[i][k] times it
-    float x[NB];
+    float x[HB];
 #pragma unroll
-    for (int c = 0; c < NB; ++c) x[c] = (c == i) ? 1.0f : 0.0f;
-    float4* bc4 = reinterpret_cast<float4*>(bc);
+    for (int c = 0; c < HB; ++c) x[c] = (c0 + c == i) ? 1.0f : 0.0f;
+    float4* bc4 = reinterpret_cast<float4*>(bc) + h * (HB / 4);
 #pragma unroll 1
     for (int k = 0; k < NB; ++k) {
         if (i == k) {
             const float inv = 1.0f / tile[k][k];
 #pragma unroll
-            for (int c = 0; c < NB; c += 4) {
+            for (int c = 0; c < HB; c += 4) {
                 x[c] *= inv; x[c + 1] *= inv; x[c + 2] *= inv; x[c + 3] *= inv;
                 bc4[c / 4] = make_float4(x[c], x[c + 1], x[c + 2], x[c + 3]);
             }
@@ -270,7 +283,7 @@ __global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallB
         if (i > k) {
             const float lik = tile[i][k];
 #pragma unroll
-            for (int c = 0; c < NB; c += 4) {
+            for (int c = 0; c < HB; c += 4) {
                 const float4 r = bc4[c / 4];
                 x[c] = fmaf(-lik, r.x, x[c]);
                 x[c + 1] = fmaf(-lik, r.y, x[c + 1]);
@@ -281,22 +294,28 @@ __global__ void __launch_bounds__(64) k_chol_diag(const __grid_constant__ SmallB
         __syncthreads();
     }
     // the factor (zeros above the diagonal) in place, the inverse into c
-    for (int k = i + 1; k < NB; ++k) tile[i][k] = 0.0f;
+#pragma unroll
+    for (int k = 0; k < HB; ++k)
+        if (c0 + k > i) tile[i][c0 + k] = 0.0f;
     __syncthreads();
-    for (int r = 0; r < sz; ++r)
-        if (i < sz) A[(long long)(j0 + r) * l + j0 + i] = tile[r][i];
+    for (int r = t >> 6; r < sz; r += 2) {
+        const int c = t & 63;
+        if (c < sz) A[(long long)(j0 + r) * l + j0 + c] = tile[r][c];
+    }
     __syncthreads();
 #pragma unroll
-    for (int k = 0; k < NB; ++k) tile[i][k] = (k <= i) ? x[k] : 0.0f;
+    for (int k = 0; k < HB; ++k) tile[i][c0 + k] = (c0 + k <= i) ? x[k] : 0.0f;
     __syncthreads();
-    for (int r = 0; r < sz; ++r)
-        if (i < sz) X[(long long)(j0 + r) * l + j0 + i] = tile[r][i];
-    if (i == 0 && s_fail && b.fail[pi] != nullptr) *b.fail[pi] = 1;
+    for (int r = t >> 6; r < sz; r += 2) {
+        const int c = t & 63;
+        if (c < sz) X[(long long)(j0 + r) * l + j0 + c] = tile[r][c];
+    }
+    if (t == 0 && s_fail && b.fail[pi] != nullptr) *b.fail[pi] = 1;
 }
 
 cudaError_t launch_chol_diag(const SmallBatch& b, int j0, cudaStream_t s, int64_t* launches) {
     if (b.count <= 0) return cudaSuccess;
-    k_chol_diag<<<b.count, 64, 0, s>>>(b, j0);
+    k_chol_diag<<<b.count, 128, 0, s>>>(b, j0);
     ++*launches;
     return cudaGetLastError();
 }
