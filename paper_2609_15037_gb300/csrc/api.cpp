@@ -401,8 +401,10 @@ struct RefreshRunner {
     //   T[D, A] = L[D, A] Linv[A, A];  Linv[D, A] = -Linv[D, D] T[D, A],
     // both as three-plane (24-bit) split-precision products.  Each pair's
     // operands are split into the module's P1 (A side) and P2 (B side)
-    // planes at running offsets; a level's pairs of one module cover
-    // disjoint rows, so they need at most 3 l^2 / 4 entries per side.
+    // planes at running offsets.  A level's pairs of one module cover
+    // disjoint row blocks D, so the A sides need at most 3 sz (l - sz) <=
+    // 3 l^2 / 4 entries; the B side of the first product, 3 sz^2 per pair
+    // over at most (l - sz) / (2 sz) + 1 pairs, stays within 3 l^2.
     // Linv[D, A] is still zero here, so "out -= A B" gives the negated product.
     template <class PairAt>
     void tri_level_tc(int sz, size_t npairs, PairAt pair_at) {
