@@ -83,11 +83,12 @@ def check_refresh(P, X, r, p, q, key, exact_bar=None, tol_angle=1e-2, rsi_slack=
     * With exact_bar: captured energy >= (1 - exact_bar) of the optimum
       sum_{i<=r} sigma_i^2 (exact TruncatedSVD).
     Returns the deficits (1 - energy / optimum) of the device and of the
-    float64 method."""
+    float64 method, k_gap, and max |P^T P - I|."""
     from oracle import rsi_ref as R
     P = np.asarray(P, dtype=np.float64)
     X = np.asarray(X, dtype=np.float64)
-    np.testing.assert_allclose(P.T @ P, np.eye(r), atol=1e-5)
+    orth = float(np.abs(P.T @ P - np.eye(r)).max())
+    assert orth <= 1e-5, orth
     U, w = top_subspace(X, r)
     k = gap_index(np.sqrt(w), r)
     if k > 0:
@@ -100,4 +101,4 @@ def check_refresh(P, X, r, p, q, key, exact_bar=None, tol_angle=1e-2, rsi_slack=
     assert e_dev >= e_rsi - (rsi_slack + rsi_frac * d_rsi) * e_opt, (d_dev, d_rsi)
     if exact_bar is not None:
         assert e_dev >= (1.0 - exact_bar) * e_opt, d_dev
-    return {"k_gap": k, "deficit": d_dev, "deficit_rsi": d_rsi}
+    return {"k_gap": k, "deficit": d_dev, "deficit_rsi": d_rsi, "orth": orth}

@@ -106,7 +106,7 @@ def test_qwen2_7b_layer_refresh_and_step(M):
         V = o.decompose(G1[i], B)[1]
         res = check_refresh(P, V, md.r, hp.oversample, hp.power_iters, R.sketch_key(hp.seed, g.ids[i], 0))
         print(f"{md.name} {md.m}x{md.n} r={md.r}: deficit {res['deficit']:.2e} "
-              f"(float64 method {res['deficit_rsi']:.2e}), k_gap {res['k_gap']}")
+              f"(float64 method {res['deficit_rsi']:.2e}), k_gap {res['k_gap']}, |P^T P - I| {res['orth']:.1e}")
         Pb.append(g.modules[i].P_bf16.view(torch.bfloat16).double().cpu().numpy())
     # the oracle fed the device's bf16 projector, refresh off
     G2 = [_grad(md, i, 2, wl) for i, md in enumerate(mods)]

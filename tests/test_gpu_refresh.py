@@ -65,7 +65,7 @@ def test_refresh_llama300m_attention_and_mlp(M, src):
         P = g.modules[i].P.double().cpu().numpy()
         X = o.decompose(grads[i][0], B)[1] if src == "V" else grads[i][0]
         res = _check(g, g.ids[i], P, X, r)
-        print(f"{m}x{n} r={r} src={src}: deficit {res['deficit']:.2e} (float64 method {res['deficit_rsi']:.2e})")
+        print(f"{m}x{n} r={r} src={src}: deficit {res['deficit']:.2e} (float64 method {res['deficit_rsi']:.2e}), |P^T P - I| {res['orth']:.1e}")
         Pb = g.modules[i].P_bf16.view(torch.bfloat16).float().cpu().numpy()
         np.testing.assert_allclose(Pb, P, rtol=2 ** -8, atol=1e-30)
     g.close()
@@ -149,7 +149,7 @@ def test_refresh_qwen2_7b_gqa_modules_with_step(M):
         P = g.modules[i].P.double().cpu().numpy()
         X = o.decompose(grads[i][0], B)[1]
         res = _check(g, g.ids[i], P, X, r)
-        print(f"{m}x{n} r={r}: deficit {res['deficit']:.2e} (float64 method {res['deficit_rsi']:.2e})")
+        print(f"{m}x{n} r={r}: deficit {res['deficit']:.2e} (float64 method {res['deficit_rsi']:.2e}), |P^T P - I| {res['orth']:.1e}")
         assert np.all(np.isfinite(g.modules[i].W.cpu().numpy()))
     g.close()
 
@@ -222,5 +222,5 @@ def test_refresh_llama2_7b_full_size_modules(M, m, n, r):
     P = g.modules[0].P.double().cpu().numpy()
     X = o.decompose(G, B)[1]
     res = _check(g, mid, P, X, r)
-    print(f"{m}x{n} r={r}: deficit {res['deficit']:.2e} (float64 method {res['deficit_rsi']:.2e}), k_gap {res['k_gap']}")
+    print(f"{m}x{n} r={r}: deficit {res['deficit']:.2e} (float64 method {res['deficit_rsi']:.2e}), k_gap {res['k_gap']}, |P^T P - I| {res['orth']:.1e}")
     g.close()
