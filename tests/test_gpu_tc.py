@@ -94,6 +94,18 @@ def test_tc_ragged_shapes(M, m, n, r, B):
     assert rel_err(out[0], refs[0].W) <= 2e-3
 
 
+def test_tc_update_chunk_layouts_in_one_group(M):
+    """One launch group mixing the two ways K2 hands an fp32 update to W: in
+    64-row x 64-column chunks through the 3-D view of W (n a multiple of 64;
+    here also n = 64, a partial last column tile of 192 columns, and rows
+    past m in the second row half of the last row tile) and in 128-row x
+    32-column chunks (n not a multiple of 64), with B = 64, three steps."""
+    shapes = [(136, 192, 64), (200, 136, 32), (64, 64, 16), (300, 448, 128), (72, 200, 24)]
+    out, refs, _ = run_tc(M, shapes, 64, 3, P_mode="random", seed=3)
+    for i in range(len(shapes)):
+        assert rel_err(out[i], refs[i].W) <= 2e-3, shapes[i]
+
+
 def test_tc_galore_mode(M):
     """Decomposition off: R = P^T G, W -= lr * alpha * P Adam(R)."""
     shapes = [(384, 256, 64), (256, 512, 128)]
