@@ -126,7 +126,9 @@ constexpr int K2_BM = 128, K2_BN = 256, K2_BK = 64;
 constexpr int K2_A_BYTES = K2_BM * K2_BK * 2;           // 16 KB: P rows, K-major
 constexpr int K2_B_BYTES = K2_BK * (K2_BN / 2) * 2;     // 16 KB: this CTA's two 64-column chunks of N
 constexpr int K2_STAGE_BYTES = K2_A_BYTES + K2_B_BYTES;
-// W moves in chunks of 128 rows x one 128-byte row (32 fp32 / 64 bf16 columns).
+// W moves in 16 KB chunks: 128 rows x one 128-byte row (32 fp32 / 64 bf16
+// columns), or for an fp32 W whose n is a multiple of 64, 64 rows x 64
+// columns through a 3-D view of W (256 contiguous bytes per row).
 // fp32 W (SB false): the epilogue writes the update dW = -lr*alpha*(Rep_B(dM)
 // (.) dV) into a staging chunk and a TMA reduce-add applies it to W in L2, so
 // W never enters the SM: two staging chunks, six operand stages.  bf16 W (SB
