@@ -446,6 +446,11 @@ def run_gpu(args):
         kernels[k] = {"ms_per_step": round(ms, 4), "launches_per_step": prof[k][1] / args.steps,
                       "share": round(prof[k][0] / max(sum(prof[x][0] for x in names), 1e-9), 4),
                       "alg_gbs": round(kbytes.get(k, 0) / (ms * 1e-3) / 1e9, 1)}
+        if k in ("tc_project", "tc_backproject"):
+            # each product kernel's algorithmic flops (half the step's) and its
+            # own bytes against the sustained bf16 rate and the copy bandwidth
+            kernels[k]["tensor_frac"] = round(alg_flops / 2 / (ms * 1e-3) / 1e12 / bf16_sus, 4)
+            kernels[k]["hbm_frac"] = round(kbytes.get(k, 0) / (ms * 1e-3) / 1e9 / hbm, 4)
     if overlap:
         # the decomposition of all but the first module part runs on the
         # library's auxiliary stream, concurrent with K1 / K2: its event time
