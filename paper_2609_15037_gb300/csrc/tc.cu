@@ -1083,7 +1083,7 @@ template <bool LO> struct KrCfg {
 constexpr int KR_WARPS = 10;                              // 0 TMA, 1 MMA, 2-9 epilogue
 constexpr int KR_THREADS = KR_WARPS * 32;
 constexpr int KR_SMEM = 1024 + 6 * KR_PLANE + 2048;
-constexpr int kKrGroup = 48;
+constexpr int kKrGroup = 64;                              // problems per launch (three maps each in the parameters)
 
 struct KrParams {
     CUtensorMap amap[kKrGroup];        // A_hi, box {64, 64}
@@ -1109,6 +1109,8 @@ struct KrParams {
     int* status;
     long long wait_limit;              // clock cycles of a bounded wait before it gives up
 };
+
+static_assert(sizeof(KrParams) <= 32764, "KR's parameter block fits the kernel parameter space");
 
 template <bool KMAJOR, bool LO, bool ALIGN = false>
 __global__ void __launch_bounds__(KR_THREADS, 1) kr_product(const __grid_constant__ KrParams p) {
@@ -1374,7 +1376,7 @@ template <int NP> struct KsCfg {
     static constexpr int STAGES = KS_RING / STAGE;
     static constexpr int PRODUCTS = NP == 3 ? 6 : 3;
 };
-constexpr int kKsGroup = 36;                              // problems per launch (six maps each in the parameters)
+constexpr int kKsGroup = 38;                              // problems per launch (six maps each in the parameters)
 
 struct KsParams {
     CUtensorMap amap[kKsGroup][3];     // A planes ({M, K}, box {64, 32})
@@ -1391,6 +1393,8 @@ struct KsParams {
     int* status;
     long long wait_limit;              // clock cycles of a bounded wait before it gives up
 };
+
+static_assert(sizeof(KsParams) <= 32764, "KS's parameter block fits the kernel parameter space");
 
 template <int NP>
 __global__ void __launch_bounds__(KR_THREADS, 1) ks_product(const __grid_constant__ KsParams p) {
